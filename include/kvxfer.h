@@ -1,0 +1,234 @@
+/*
+ * kvxfer.h -- C ABI of the paged-KV <-> pinned-host-chunk transfer library
+ * (libkvxfer.so, CUDA, sm_103a).
+ *
+ * The paper (Sec. 2, Fig. 1) runs full inference replicas, one per GPU, that
+ * share one host-memory KV tier.  Each replica keeps its KV cache as a pool of
+ * pages (Table 1: paged cache, HND layout); the shared tier holds fixed-token
+ * chunks (Table 1: 1,568-token chunks in a 256 GiB RAM pool).  Storing a
+ * prefix gathers its pages into packed chunks in pinned host memory; loading
+ * it on another replica scatters the chunks into freshly allocated pages
+ * (Sec. 3.2, "gather/scatter dependencies").  Every copy is ordered on the
+ * caller's current CUDA stream: the paper's diagnosed corruption (Sec. 3.2,
+ * Fig. 2) is a copy that omits exactly this dependency.
+ *
+ * Data layout (all sizes in bytes unless stated; row = head_dim * elem_bytes):
+ *   pool layer l   : num_blocks pages, page = [2 (K,V)][H][B][row] for
+ *                    KVX_LAYOUT_HND, [2][B][H][row] for KVX_LAYOUT_NHD.
+ *   block table    : int32 device array; entry i = page of logical block i,
+ *                    i.e. of tokens [i*B, (i+1)*B).
+ *   chunk c        : tokens [c*C, min((c+1)*C, tok_end)), packed densely as
+ *                    [layer][2 (K,V)][token][head][row]; a short last chunk
+ *                    holds fewer tokens and is not padded.  The layout does
+ *                    not depend on the page layout, so HND and NHD pools
+ *                    exchange chunks (Sec. 3.1: a wrong view of the bytes was
+ *                    the paper's first corruption).
+ *   host chunk i   : the i-th chunk of the call's range, i.e. chunk
+ *                    tok_begin/C + i; page-locked host memory, 16-byte
+ *                    aligned, at least kv_chunk_layout(...).chunk_bytes long.
+ *
+ * Threading: a kvx_ctx may be shared by host threads (calls are serialised
+ * inside).  Calls are asynchronous with respect to the host.
+ *
+ * Error behaviour: argument errors return before anything is enqueued and
+ * leave every buffer untouched.  A block-table entry outside [0, num_blocks)
+ * is found on the device: its page is skipped and the lowest such logical
+ * block index is kept for kv_get_device_error().  No call aborts the process,
+ * traps on the device, or waits without a bound.
+ */
+#ifndef KVXFER_H
+#define KVXFER_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define KVX_ABI_VERSION 1
+#define KVX_MAX_LAYERS 128 /* layers per pool description */
+
+/* Same handle as cudaStream_t; NULL is the legacy default stream. */
+typedef struct CUstream_st* kvx_stream_t;
+
+typedef enum {
+  KVX_OK = 0,
+  KVX_EINVAL = -1,     /* null pointer, non-positive size, unknown enum value   */
+  KVX_EALIGN = -2,     /* tok_begin % C, C % B, row % 16 or a pointer % 16 != 0 */
+  KVX_ERANGE = -3,     /* tok_end beyond the table, too few chunks, bad slot    */
+  KVX_ENOTPINNED = -4, /* a host buffer is not page-locked host memory          */
+  KVX_ECUDA = -5,      /* a CUDA runtime call failed (kv_last_cuda_error)       */
+  KVX_ENOMEM = -6,     /* staging or device allocation failed                   */
+  KVX_EDEVICE = -7     /* a device pointer is not device memory of ctx's GPU    */
+} kvx_status;
+
+typedef enum { KVX_LAYOUT_HND = 0, KVX_LAYOUT_NHD = 1 } kvx_layout;
+
+/* How host chunks are filled and read.  Both move exactly the same bytes. */
+typedef enum {
+  KVX_MODE_AUTO = 0,     /* library's measured default per direction          */
+  KVX_MODE_STAGED = 1,   /* pack into a device staging ring, then
+                            cudaMemcpyAsync over the host link on a side stream,
+                            pack of batch i+1 overlapping the copy of batch i  */
+  KVX_MODE_ZEROCOPY = 2  /* the kernel reads/writes the mapped pinned chunks
+                            directly over the host link; no staging            */
+} kvx_mode;
+
+/* Options flags */
+#define KVX_FLAG_TIME_KERNELS 0x1u /* record CUDA events around every kernel
+                                      launch; read with kv_ctx_stats()        */
+#define KVX_FLAG_UNORDERED 0x2u    /* NEGATIVE CONTROL ONLY: drop the wait on
+                                      the caller's stream, reproducing the
+                                      paper's missing dependency (Sec. 3.2).
+                                      Results are then undefined.             */
+
+typedef struct {
+  int32_t store_mode;         /* kvx_mode                                       */
+  int32_t load_mode;          /* kvx_mode                                       */
+  int32_t staging_slots;      /* staged ring depth (>= 2); 0 = 4                */
+  int64_t staging_slot_bytes; /* bytes per slot; 0 = 32 MiB; a slot must hold
+                                 one layer of one chunk                         */
+  int32_t max_ctas;           /* cap on CTAs per kernel launch; 0 = fill GPU    */
+  uint32_t flags;             /* KVX_FLAG_*                                     */
+} kvx_opts;
+
+/* Caller-owned description of one paged KV pool (device memory). */
+typedef struct {
+  int32_t num_layers;        /* 1 .. KVX_MAX_LAYERS                            */
+  void* const* layer_base;   /* host array [num_layers] of device pointers, each
+                                16-byte aligned, num_blocks * page_bytes long   */
+  int64_t num_blocks;        /* pages per layer                                */
+  int32_t block_tokens;      /* B: tokens per page                             */
+  int32_t num_heads;         /* H: KV heads                                    */
+  int32_t head_dim;          /* D: elements per head vector                    */
+  int32_t elem_bytes;        /* e: bytes per element (bf16 = 2, fp8 = 1, ...)  */
+  int32_t layout;            /* kvx_layout                                     */
+} kvx_pool;
+
+/* Byte geometry of one packed chunk holding tokens_in_chunk tokens. */
+typedef struct {
+  int32_t chunk_tokens;      /* C                                              */
+  int32_t tokens;            /* tokens held (<= C)                             */
+  int64_t chunk_bytes;       /* L * 2 * tokens * H * row                       */
+  int64_t layer_stride;      /* 2 * tokens * H * row                           */
+  int64_t kv_stride;         /* tokens * H * row                               */
+  int64_t token_stride;      /* H * row                                        */
+  int64_t head_stride;       /* row                                            */
+  int64_t page_bytes;        /* bytes of one pool page (2 * H * B * row)       */
+} kvx_chunk_layout;
+
+/* Counters kept by a context (see KVX_FLAG_TIME_KERNELS). */
+typedef struct {
+  int64_t kernel_launches;   /* kernels this context has launched              */
+  int64_t timed_launches;    /* launches with a recorded duration              */
+  double kernel_ms;          /* summed durations of timed launches             */
+  int64_t kernel_bytes;      /* algorithmic bytes moved by timed launches:
+                                read + written, host or device                  */
+  int64_t memcpy_calls;      /* cudaMemcpyAsync calls issued (staged mode)     */
+} kvx_stats;
+
+typedef struct kvx_ctx kvx_ctx;
+
+/*
+ * Create a context on `device`: side streams, per-slot events, the staging
+ * ring (KVX_MODE_STAGED only, allocated on first use) and a device error word.
+ * opts may be NULL (all defaults).  Returns KVX_ENOMEM if an allocation fails.
+ */
+kvx_status kv_ctx_create(int device, const kvx_opts* opts, kvx_ctx** out);
+
+/* Synchronises the context's streams, then frees everything it owns. */
+void kv_ctx_destroy(kvx_ctx* ctx);
+
+/*
+ * Geometry of a chunk (Table 1: fixed-token chunks of the shared tier).
+ * chunk_tokens must be a positive multiple of pool->block_tokens and
+ * 0 <= tokens_in_chunk <= chunk_tokens.  Pure host arithmetic.
+ */
+kvx_status kv_chunk_layout(const kvx_pool* pool, int32_t chunk_tokens, int32_t tokens_in_chunk,
+                           kvx_chunk_layout* out);
+
+/*
+ * Store (Sec. 3.2 gather; Fig. 2 lower panel ordering): pack tokens
+ * [tok_begin, tok_end) of the pages named by block_table into host_chunks.
+ *   block_table : device int32 [table_len]; pages of logical blocks 0..
+ *   tok_begin   : multiple of chunk_tokens (chunks start on aligned recovery
+ *                 boundaries, Sec. 2.2);  tok_end <= table_len * B.
+ *   host_chunks : host array [n_chunks] of pinned host pointers; chunk i gets
+ *                 chunk tok_begin/C + i; n_chunks >= ceil(tok_end/C) - tok_begin/C.
+ *   stream      : the caller's current stream.  All reads of the pool happen
+ *                 after the work already enqueued on it; work enqueued on it
+ *                 after this call runs after the chunks are written.
+ * The host must synchronise `stream` before reading the chunks (Fig. 2
+ * caption: completion must precede host consumption).  Only the first
+ * chunk_bytes of each chunk are written.
+ */
+kvx_status kv_store(kvx_ctx* ctx, const kvx_pool* pool, const int32_t* block_table, int64_t table_len,
+                    int64_t tok_begin, int64_t tok_end, int32_t chunk_tokens,
+                    void* const* host_chunks, int64_t n_chunks, kvx_stream_t stream);
+
+/*
+ * Load (Sec. 3.2 scatter into freshly allocated pages): the inverse of
+ * kv_store into the pages named by block_table.  Exactly the page rows of
+ * tokens [tok_begin, tok_end) are written; all other pool bytes (other pages,
+ * slots past tok_end in a partial last page) are left untouched.  Host chunks
+ * must not be modified or freed before `stream` has passed this call.
+ * A physical page listed twice in block_table is a caller error (the bytes
+ * written there are then unspecified).
+ */
+kvx_status kv_load(kvx_ctx* ctx, const kvx_pool* pool, const int32_t* block_table, int64_t table_len,
+                   int64_t tok_begin, int64_t tok_end, int32_t chunk_tokens,
+                   const void* const* host_chunks, int64_t n_chunks, kvx_stream_t stream);
+
+/*
+ * Device-side pack / unpack: kv_store / kv_load with chunks in device memory
+ * of ctx's GPU (16-byte aligned) instead of pinned host memory.  Same rules,
+ * one kernel pass, ordered on `stream`.
+ */
+kvx_status kv_pack(kvx_ctx* ctx, const kvx_pool* pool, const int32_t* block_table, int64_t table_len,
+                   int64_t tok_begin, int64_t tok_end, int32_t chunk_tokens,
+                   void* const* dev_chunks, int64_t n_chunks, kvx_stream_t stream);
+kvx_status kv_unpack(kvx_ctx* ctx, const kvx_pool* pool, const int32_t* block_table, int64_t table_len,
+                     int64_t tok_begin, int64_t tok_end, int32_t chunk_tokens,
+                     const void* const* dev_chunks, int64_t n_chunks, kvx_stream_t stream);
+
+/*
+ * Recurrent-state snapshot (Sec. 2.2: a recurrent page -- convolution state,
+ * recurrent state and padding -- is moved as opaque addressable bytes; a
+ * hybrid prefix is recovered only with the snapshot taken at its boundary).
+ *   layer_base : host array [num_layers] of device pointers to
+ *                [num_slots][slot_bytes] state pools.
+ *   host_obj   : pinned host buffer [num_layers][slot_bytes].
+ * kv_state_store copies slot `slot` of every layer into host_obj;
+ * kv_state_load copies host_obj into slot `slot`.  Ordered on `stream`.
+ */
+kvx_status kv_state_store(kvx_ctx* ctx, int32_t num_layers, void* const* layer_base, int64_t num_slots,
+                          int64_t slot_bytes, int64_t slot, void* host_obj, kvx_stream_t stream);
+kvx_status kv_state_load(kvx_ctx* ctx, int32_t num_layers, void* const* layer_base, int64_t num_slots,
+                         int64_t slot_bytes, int64_t slot, const void* host_obj, kvx_stream_t stream);
+
+/*
+ * Lowest logical block index whose table entry was out of range in any call
+ * completed since the last query, or -1.  Call after the caller's stream has
+ * been synchronised.  Clears the record.
+ */
+kvx_status kv_get_device_error(kvx_ctx* ctx, int64_t* first_bad_block);
+
+/* Counters of this context; waits for timed launches to finish. */
+kvx_status kv_ctx_stats(kvx_ctx* ctx, kvx_stats* out);
+kvx_status kv_ctx_reset_stats(kvx_ctx* ctx);
+
+/* The mode a context resolved for each direction (after KVX_MODE_AUTO). */
+kvx_status kv_ctx_modes(const kvx_ctx* ctx, int32_t* store_mode, int32_t* load_mode);
+
+/* The last CUDA error code seen by this thread inside the library (0 = none). */
+int kv_last_cuda_error(void);
+
+/* Static text for a status value. */
+const char* kv_status_string(kvx_status status);
+
+int kv_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* KVXFER_H */
