@@ -30,8 +30,9 @@
  * Bytes are moved with memcpy, one row at a time.  Bytes of a chunk past its
  * L*2*T_c*H*row valid bytes, and pool bytes of token slots outside
  * [t_begin, t_end), are never written.  A table entry outside
- * [0, num_blocks) is skipped (nothing copied for its tokens) and the lowest
- * offending logical block index is reported.
+ * [0, num_blocks) names no page: a store writes zero bytes for its tokens,
+ * a load writes nothing for them, and the lowest offending logical block
+ * index is reported.  (The paper does not define this case.)
  *
  * Recurrent-state snapshots (Sec. 2.2: a recurrent page is handled as opaque
  * addressable bytes) are a plain byte copy of one slot per layer.
@@ -127,6 +128,8 @@ static void* run_job(void* arg) {
           int64_t p = J->table[blk];
           if (p < 0 || p >= P->num_blocks) {
             if (J->bad < 0 || blk < J->bad) J->bad = blk;
+            if (J->to_chunk) /* the token's rows of this (layer, kv) read as zeros */
+              memset(chunk + chunk_row(P, T_c, l, kv, u, 0), 0, (size_t)(P->num_heads * row));
             continue;
           }
           for (int64_t h = 0; h < P->num_heads; ++h) {

@@ -259,7 +259,8 @@ def pin_error_codes(orc):
 
 
 def pin_bad_block(orc):
-    """An out-of-range page id skips that page's tokens and names the lowest such logical block."""
+    """An out-of-range page id names no page: a store zero-fills its tokens, a load leaves the
+    pool alone, and the lowest such logical block is reported."""
     spec = PoolSpec(1, 4, 4, 2, 8, 2, HND)
     layers = make_layers(spec, 41, avoid_poison=True)
     table = np.array([1, 4, 2, -1], dtype=np.int32)  # 4 == num_blocks: first id past the end
@@ -272,9 +273,15 @@ def pin_bad_block(orc):
     ref = good[0].reshape(2, 16, HR)
     for t in range(16):
         if t // 4 in (1, 3):
-            assert np.all(got[:, t] == POISON), t
+            assert np.all(got[:, t] == 0), t
         else:
             assert np.array_equal(got[:, t], ref[:, t]), t
+    dest = [np.full_like(layers[0], POISON)]
+    rc, bad = orc.load(spec, dest, table, 0, 16, 16, good)
+    assert rc == oracle.OK and bad == 1, (rc, bad)
+    pages = dest[0].reshape(4, spec.page_bytes)
+    assert np.all(pages[0] == POISON) and np.all(pages[3] == POISON)   # pages named by no valid entry
+    assert not np.all(pages[1] == POISON) and not np.all(pages[2] == POISON)
 
 
 def pin_threads_match_single(orc):
