@@ -32,9 +32,12 @@
  *
  * Error behaviour: argument errors return before anything is enqueued and
  * leave every buffer untouched.  A block-table entry outside [0, num_blocks)
- * is found on the device: its page is skipped and the lowest such logical
- * block index is kept for kv_get_device_error().  No call aborts the process,
- * traps on the device, or waits without a bound.
+ * is found on the device: it names no page, so a store writes zero bytes for
+ * its tokens (never stale staging bytes) and a load writes nothing for them;
+ * the lowest such logical block index is kept for kv_get_device_error().  A
+ * CUDA failure while work is being enqueued returns KVX_ECUDA after making
+ * `stream` wait for whatever was already enqueued.  No call aborts the
+ * process, traps on the device, or waits without a bound.
  */
 #ifndef KVXFER_H
 #define KVXFER_H
@@ -117,14 +120,17 @@ typedef struct {
   int64_t page_bytes;        /* bytes of one pool page (2 * H * B * row)       */
 } kvx_chunk_layout;
 
-/* Counters kept by a context (see KVX_FLAG_TIME_KERNELS). */
+/* Counters kept by a context.  Index [0] is the pack direction (kv_store,
+   kv_pack, kv_state_store), [1] the unpack direction.  Durations are kept
+   only with KVX_FLAG_TIME_KERNELS: a pair of CUDA events is recorded around
+   each kernel launch on the stream it runs on. */
 typedef struct {
   int64_t kernel_launches;   /* kernels this context has launched              */
-  int64_t timed_launches;    /* launches with a recorded duration              */
-  double kernel_ms;          /* summed durations of timed launches             */
-  int64_t kernel_bytes;      /* algorithmic bytes moved by timed launches:
-                                read + written, host or device                  */
   int64_t memcpy_calls;      /* cudaMemcpyAsync calls issued (staged mode)     */
+  int64_t timed_launches[2]; /* launches with a recorded duration              */
+  double kernel_ms[2];       /* summed durations of timed launches             */
+  int64_t kernel_bytes[2];   /* algorithmic bytes of timed launches: every byte
+                                read plus every byte written, host or device   */
 } kvx_stats;
 
 typedef struct kvx_ctx kvx_ctx;
@@ -222,6 +228,11 @@ kvx_status kv_ctx_modes(const kvx_ctx* ctx, int32_t* store_mode, int32_t* load_m
 
 /* The last CUDA error code seen by this thread inside the library (0 = none). */
 int kv_last_cuda_error(void);
+
+/* Text naming the CUDA call behind the last KVX_ECUDA of this thread ("" if
+   none).  The string belongs to the library and stays valid until the
+   thread's next failing call. */
+const char* kv_last_error_message(void);
 
 /* Static text for a status value. */
 const char* kv_status_string(kvx_status status);

@@ -1,0 +1,65 @@
+// kvx_internal.h -- declarations shared by the library's translation units.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "kvxfer.h"
+
+namespace kvx {
+
+constexpr int kMaxJobs = 64;      // chunk-side segments per kernel launch
+constexpr int kThreads = 256;     // threads per CTA of the move kernels
+constexpr int kMaxSegments = 96;  // segments per opaque-copy launch (params < 4 KiB)
+
+enum Dir : int { kPack = 0, kUnpack = 1 };
+
+// One contiguous chunk-side region: layers [l0, l0 + nl) of one chunk.
+struct Job {
+  uint8_t* chunk;       // chunk-side address of layer l0 (device, staging or mapped host)
+  int64_t first_block;  // logical block index of the chunk's first token
+  int64_t unit_end;     // exclusive prefix sum of units up to and including this job
+  int32_t tokens;       // T_c: tokens held by the chunk
+  int32_t l0;           // first layer of the region
+};
+
+// Kernel parameters of one pack/unpack launch (passed by value, < 4 KiB).
+struct MoveParams {
+  uint8_t* layer_base[KVX_MAX_LAYERS];
+  Job jobs[kMaxJobs];
+  const int32_t* table;        // device block table
+  long long* err;              // device error word (lowest bad logical block)
+  int64_t num_blocks;          // pages per layer
+  int64_t page_bytes;          // 2 * H * B * row
+  int64_t total_units;         // units of this launch
+  int32_t n_jobs;
+  int32_t blocks_per_chunk;    // C / B
+  int32_t B, H, R;             // tokens per page, heads, row bytes
+  int32_t fast;                // 1 if R/16 is a power of two <= 32
+  int32_t vpr_shift;           // log2(R / 16) when fast
+  int32_t rpi_div_h, rpi_mod_h; // (32 / (R/16)) / H and % H when fast
+};
+
+struct Segment {
+  const uint8_t* src;
+  uint8_t* dst;
+  int64_t unit_end;  // exclusive prefix sum of 32 KiB units
+  int64_t bytes;
+};
+
+struct SegmentParams {
+  Segment seg[kMaxSegments];
+  int64_t total_units;
+  int32_t n_seg;
+};
+
+// Launchers (pack_kernels.cu).  Return the cudaError_t of the launch.
+cudaError_t launch_move(int dir, int layout, const MoveParams& p, int grid, cudaStream_t s);
+cudaError_t launch_segments(const SegmentParams& p, int grid, cudaStream_t s);
+int move_ctas_per_sm(int dir, int layout);
+int segment_ctas_per_sm();
+
+// Records the last CUDA error seen by this thread (kv_last_cuda_error).
+void set_last_cuda_error(int e);
+
+}  // namespace kvx

@@ -1,0 +1,247 @@
+// pack_kernels.cu -- gather (pack) and scatter (unpack) kernels between the
+// paged KV pool and packed chunks, for sm_103a.
+//
+// Paper Sec. 3.2: storing a prefix gathers its KV pages into the host tier's
+// packed chunk, loading scatters the chunk back into freshly allocated pages.
+// This is pure byte movement bound by memory bandwidth (HBM for device chunks
+// and staging, the host link for mapped pinned chunks), so it runs on the
+// load/store units with 16-byte vectors; no tensor cores are involved.
+//
+// Work unit: one (chunk, layer, page, K|V) region, handled by one warp.  For
+// the shapes of a 27B-class model (B = 16 tokens, H = 8 heads, 256-byte rows)
+// a unit is 32 KiB: both its page side and its chunk side are contiguous
+// 32 KiB extents, the chunk side in [token][head] row order and the page side
+// in [head][token] order (HND) or [token][head] order (NHD).  Every 256-byte
+// row is read and written whole by 16 lanes, so each 128-byte line is used in
+// full on both sides.  Each lane keeps kInflight 16-byte loads in flight
+// before storing them.
+//
+// Out-of-range block-table entries skip their unit and lower a device error
+// word (atomicMin of the logical block index); nothing traps.
+
+#include "kvx_internal.h"
+
+namespace kvx {
+namespace {
+
+constexpr int kInflight = 8;  // 16-byte vectors per lane between loads and stores
+
+// Streaming (evict-first) accesses: every byte is touched exactly once.
+__device__ __forceinline__ uint4 ld16(const uint8_t* p) {
+  return __ldcs(reinterpret_cast<const uint4*>(p));
+}
+__device__ __forceinline__ void st16(uint8_t* p, const uint4& v) {
+  __stcs(reinterpret_cast<uint4*>(p), v);
+}
+
+// Move kInflight vectors: pack reads the page side, unpack reads the chunk side.
+template <int DIR>
+__device__ __forceinline__ void move_batch(uint8_t* pg, uint8_t* ck, const int64_t (&po)[kInflight],
+                                           const int64_t (&co)[kInflight]) {
+  uint4 v[kInflight];
+  if (DIR == kPack) {
+#pragma unroll
+    for (int i = 0; i < kInflight; ++i) v[i] = ld16(pg + po[i]);
+#pragma unroll
+    for (int i = 0; i < kInflight; ++i) st16(ck + co[i], v[i]);
+  } else {
+#pragma unroll
+    for (int i = 0; i < kInflight; ++i) v[i] = ld16(ck + co[i]);
+#pragma unroll
+    for (int i = 0; i < kInflight; ++i) st16(pg + po[i], v[i]);
+  }
+}
+
+template <int DIR>
+__device__ __forceinline__ void move_one(uint8_t* pg, uint8_t* ck, int64_t po, int64_t co) {
+  if (DIR == kPack)
+    st16(ck + co, ld16(pg + po));
+  else
+    st16(pg + po, ld16(ck + co));
+}
+
+// Same byte order on both sides (NHD pages, opaque segments): a flat copy of
+// nbytes (a multiple of 16).
+template <int DIR>
+__device__ __forceinline__ void move_flat(uint8_t* pg, uint8_t* ck, int64_t nbytes, int lane) {
+  int64_t off = (int64_t)lane * 16;
+  constexpr int64_t kStep = 32 * 16;
+  for (; off + (kInflight - 1) * kStep < nbytes; off += kInflight * kStep) {
+    int64_t o[kInflight];
+#pragma unroll
+    for (int i = 0; i < kInflight; ++i) o[i] = off + i * kStep;
+    move_batch<DIR>(pg, ck, o, o);
+  }
+  for (; off < nbytes; off += kStep) move_one<DIR>(pg, ck, off, off);
+}
+
+// HND page side [H][B][R] <-> chunk side [nb][H][R], nr = nb * H rows, when
+// R / 16 is a power of two no larger than 32: a warp covers 32 / (R/16) whole
+// rows per step, each lane a fixed 16-byte column, and the (token, head) pair
+// of a lane's row is advanced incrementally (no division in the loop).
+template <int DIR>
+__device__ __forceinline__ void move_hnd_fast(uint8_t* pg, uint8_t* ck, int nr, const MoveParams& p,
+                                              int lane) {
+  const int rows_per_step = 32 >> p.vpr_shift;
+  const int64_t col = (int64_t)(lane & ((1 << p.vpr_shift) - 1)) * 16;
+  const int64_t R = p.R, B = p.B;
+  const int H = p.H;
+  int r = lane >> p.vpr_shift;  // row in chunk order: r = s * H + h
+  int s = r / H;
+  int h = r - s * H;
+  while (r + (kInflight - 1) * rows_per_step < nr) {
+    int64_t po[kInflight], co[kInflight];
+#pragma unroll
+    for (int i = 0; i < kInflight; ++i) {
+      po[i] = ((int64_t)h * B + s) * R + col;
+      co[i] = (int64_t)r * R + col;
+      r += rows_per_step;
+      s += p.rpi_div_h;
+      h += p.rpi_mod_h;
+      if (h >= H) {
+        h -= H;
+        ++s;
+      }
+    }
+    move_batch<DIR>(pg, ck, po, co);
+  }
+  while (r < nr) {
+    move_one<DIR>(pg, ck, ((int64_t)h * B + s) * R + col, (int64_t)r * R + col);
+    r += rows_per_step;
+    s += p.rpi_div_h;
+    h += p.rpi_mod_h;
+    if (h >= H) {
+      h -= H;
+      ++s;
+    }
+  }
+}
+
+// HND for any row size that is a multiple of 16 bytes.
+template <int DIR>
+__device__ __forceinline__ void move_hnd_generic(uint8_t* pg, uint8_t* ck, int nr, const MoveParams& p,
+                                                 int lane) {
+  const int vpr = p.R / 16;
+  const int64_t nv = (int64_t)nr * vpr;
+  for (int64_t v = lane; v < nv; v += 32) {
+    const int64_t r = v / vpr;
+    const int64_t c = (v - r * vpr) * 16;
+    const int64_t s = r / p.H;
+    const int64_t h = r - s * p.H;
+    move_one<DIR>(pg, ck, (h * p.B + s) * p.R + c, r * p.R + c);
+  }
+}
+
+template <int DIR, int LAYOUT>
+__global__ void __launch_bounds__(kThreads) move_kernel(const __grid_constant__ MoveParams p) {
+  const int lane = threadIdx.x & 31;
+  const int64_t nwarps = ((int64_t)gridDim.x * kThreads) >> 5;
+  int64_t u = ((int64_t)blockIdx.x * kThreads + threadIdx.x) >> 5;
+  int j = 0;
+  int64_t job_begin = 0;
+  const int64_t half_page = p.page_bytes >> 1;  // K or V part of a page: H * B * R
+  const int64_t HR = (int64_t)p.H * p.R;
+  for (; u < p.total_units; u += nwarps) {
+    while (u >= p.jobs[j].unit_end) {  // warp-uniform; units ascend per warp
+      job_begin = p.jobs[j].unit_end;
+      ++j;
+    }
+    const Job& J = p.jobs[j];
+    const int64_t local = u - job_begin;
+    const int kv = (int)(local & 1);
+    const int64_t rest = local >> 1;
+    const int jb = (int)(rest % p.blocks_per_chunk);
+    const int l = J.l0 + (int)(rest / p.blocks_per_chunk);
+    const int tok0 = jb * p.B;
+    if (tok0 >= J.tokens) continue;  // past the end of a short last chunk
+    const int nb = min(p.B, J.tokens - tok0);
+    const int64_t lblk = J.first_block + jb;
+    const int32_t page = __ldg(p.table + lblk);
+    uint8_t* ck = J.chunk + ((int64_t)(l - J.l0) * 2 + kv) * J.tokens * HR + (int64_t)tok0 * HR;
+    const int nr = nb * p.H;
+    if (page < 0 || (int64_t)page >= p.num_blocks) {
+      if (lane == 0) atomicMin(p.err, (long long)lblk);
+      if (DIR == kPack) {  // the unit's chunk rows (contiguous) read as zeros
+        const uint4 z = make_uint4(0, 0, 0, 0);
+        for (int64_t off = (int64_t)lane * 16; off < (int64_t)nr * p.R; off += 32 * 16) st16(ck + off, z);
+      }
+      continue;
+    }
+    uint8_t* pg = p.layer_base[l] + (int64_t)page * p.page_bytes + kv * half_page;
+    if (LAYOUT == KVX_LAYOUT_NHD)
+      move_flat<DIR>(pg, ck, (int64_t)nr * p.R, lane);
+    else if (p.fast)
+      move_hnd_fast<DIR>(pg, ck, nr, p, lane);
+    else
+      move_hnd_generic<DIR>(pg, ck, nr, p, lane);
+  }
+}
+
+// Opaque byte segments (recurrent-state slots), 32 KiB per warp unit.
+constexpr int64_t kSegUnit = 32 * 1024;
+
+__global__ void __launch_bounds__(kThreads) segment_kernel(const __grid_constant__ SegmentParams p) {
+  const int lane = threadIdx.x & 31;
+  const int64_t nwarps = ((int64_t)gridDim.x * kThreads) >> 5;
+  int64_t u = ((int64_t)blockIdx.x * kThreads + threadIdx.x) >> 5;
+  int j = 0;
+  int64_t seg_begin = 0;
+  for (; u < p.total_units; u += nwarps) {
+    while (u >= p.seg[j].unit_end) {
+      seg_begin = p.seg[j].unit_end;
+      ++j;
+    }
+    const Segment& S = p.seg[j];
+    const int64_t off = (u - seg_begin) * kSegUnit;
+    const int64_t n = min(kSegUnit, S.bytes - off);
+    move_flat<kPack>(const_cast<uint8_t*>(S.src) + off, S.dst + off, n, lane);
+  }
+}
+
+template <int DIR, int LAYOUT>
+int occupancy_of() {
+  int n = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, move_kernel<DIR, LAYOUT>, kThreads, 0) !=
+      cudaSuccess) {
+    cudaGetLastError();
+    return 1;
+  }
+  return n > 0 ? n : 1;
+}
+
+}  // namespace
+
+cudaError_t launch_move(int dir, int layout, const MoveParams& p, int grid, cudaStream_t s) {
+  if (dir == kPack && layout == KVX_LAYOUT_HND)
+    move_kernel<kPack, KVX_LAYOUT_HND><<<grid, kThreads, 0, s>>>(p);
+  else if (dir == kPack)
+    move_kernel<kPack, KVX_LAYOUT_NHD><<<grid, kThreads, 0, s>>>(p);
+  else if (layout == KVX_LAYOUT_HND)
+    move_kernel<kUnpack, KVX_LAYOUT_HND><<<grid, kThreads, 0, s>>>(p);
+  else
+    move_kernel<kUnpack, KVX_LAYOUT_NHD><<<grid, kThreads, 0, s>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_segments(const SegmentParams& p, int grid, cudaStream_t s) {
+  segment_kernel<<<grid, kThreads, 0, s>>>(p);
+  return cudaGetLastError();
+}
+
+int move_ctas_per_sm(int dir, int layout) {
+  if (dir == kPack) return layout == KVX_LAYOUT_HND ? occupancy_of<kPack, KVX_LAYOUT_HND>()
+                                                    : occupancy_of<kPack, KVX_LAYOUT_NHD>();
+  return layout == KVX_LAYOUT_HND ? occupancy_of<kUnpack, KVX_LAYOUT_HND>()
+                                  : occupancy_of<kUnpack, KVX_LAYOUT_NHD>();
+}
+
+int segment_ctas_per_sm() {
+  int n = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, segment_kernel, kThreads, 0) != cudaSuccess) {
+    cudaGetLastError();
+    return 1;
+  }
+  return n > 0 ? n : 1;
+}
+
+}  // namespace kvx

@@ -1,0 +1,341 @@
+"""Python binding of libkvxfer.so (ctypes): argument marshalling only.
+
+Every function has the name of the C entry point it calls (``include/kvxfer.h``,
+``include/kvxfer_probe.h``); all data movement happens in the library's CUDA
+kernels and copies.  Tensors are PyTorch tensors (device memory, pinned host
+buffers, streams); a C status other than ``KVX_OK`` raises ``KvxError``.
+
+The library must have been built (``paper_2609_15021_gb300._build.build()``):
+importing this module without it raises ``ImportError`` -- there is no fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass
+from typing import Sequence
+
+_LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "_lib", "libkvxfer.so")
+
+KVX_OK, KVX_EINVAL, KVX_EALIGN, KVX_ERANGE = 0, -1, -2, -3
+KVX_ENOTPINNED, KVX_ECUDA, KVX_ENOMEM, KVX_EDEVICE = -4, -5, -6, -7
+KVX_LAYOUT_HND, KVX_LAYOUT_NHD = 0, 1
+KVX_MODE_AUTO, KVX_MODE_STAGED, KVX_MODE_ZEROCOPY = 0, 1, 2
+KVX_FLAG_TIME_KERNELS, KVX_FLAG_UNORDERED = 0x1, 0x2
+KVX_MAX_LAYERS = 128
+KVX_PROBE_RAW, KVX_PROBE_WAIT_THEN_COPY, KVX_PROBE_ASYNC_ON_STREAM = 0, 1, 2
+KVX_PROBE_MAX_CYCLES = 4_000_000_000
+
+MODE_NAMES = {KVX_MODE_AUTO: "auto", KVX_MODE_STAGED: "staged", KVX_MODE_ZEROCOPY: "zerocopy"}
+
+# Every symbol the headers declare; a test checks the library exports them all.
+EXPORTED = (
+    "kv_ctx_create", "kv_ctx_destroy", "kv_chunk_layout", "kv_store", "kv_load", "kv_pack", "kv_unpack",
+    "kv_state_store", "kv_state_load", "kv_get_device_error", "kv_ctx_stats", "kv_ctx_reset_stats",
+    "kv_ctx_modes", "kv_last_cuda_error", "kv_last_error_message", "kv_status_string", "kv_abi_version",
+    "kvx_probe_delayed_fill", "kvx_probe_delayed_copy", "kvx_probe_copy",
+)
+
+
+class KvxError(RuntimeError):
+    def __init__(self, status: int, where: str, message: str):
+        super().__init__(f"{where}: {message} (status {status})")
+        self.status = status
+
+
+class kvx_opts(ctypes.Structure):
+    _fields_ = [("store_mode", ctypes.c_int32), ("load_mode", ctypes.c_int32),
+                ("staging_slots", ctypes.c_int32), ("staging_slot_bytes", ctypes.c_int64),
+                ("max_ctas", ctypes.c_int32), ("flags", ctypes.c_uint32)]
+
+
+class kvx_pool(ctypes.Structure):
+    _fields_ = [("num_layers", ctypes.c_int32), ("layer_base", ctypes.POINTER(ctypes.c_void_p)),
+                ("num_blocks", ctypes.c_int64), ("block_tokens", ctypes.c_int32),
+                ("num_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
+                ("elem_bytes", ctypes.c_int32), ("layout", ctypes.c_int32)]
+
+
+class kvx_chunk_layout(ctypes.Structure):
+    _fields_ = [("chunk_tokens", ctypes.c_int32), ("tokens", ctypes.c_int32),
+                ("chunk_bytes", ctypes.c_int64), ("layer_stride", ctypes.c_int64),
+                ("kv_stride", ctypes.c_int64), ("token_stride", ctypes.c_int64),
+                ("head_stride", ctypes.c_int64), ("page_bytes", ctypes.c_int64)]
+
+
+class kvx_stats(ctypes.Structure):
+    _fields_ = [("kernel_launches", ctypes.c_int64), ("memcpy_calls", ctypes.c_int64),
+                ("timed_launches", ctypes.c_int64 * 2), ("kernel_ms", ctypes.c_double * 2),
+                ("kernel_bytes", ctypes.c_int64 * 2)]
+
+
+def _declare(lib):
+    P, vp, i32, i64 = ctypes.POINTER, ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64
+    st = ctypes.c_int
+    sig = {
+        "kv_ctx_create": (st, [ctypes.c_int, P(kvx_opts), P(vp)]),
+        "kv_ctx_destroy": (None, [vp]),
+        "kv_chunk_layout": (st, [P(kvx_pool), i32, i32, P(kvx_chunk_layout)]),
+        "kv_store": (st, [vp, P(kvx_pool), vp, i64, i64, i64, i32, P(vp), i64, vp]),
+        "kv_load": (st, [vp, P(kvx_pool), vp, i64, i64, i64, i32, P(vp), i64, vp]),
+        "kv_pack": (st, [vp, P(kvx_pool), vp, i64, i64, i64, i32, P(vp), i64, vp]),
+        "kv_unpack": (st, [vp, P(kvx_pool), vp, i64, i64, i64, i32, P(vp), i64, vp]),
+        "kv_state_store": (st, [vp, i32, P(vp), i64, i64, i64, vp, vp]),
+        "kv_state_load": (st, [vp, i32, P(vp), i64, i64, i64, vp, vp]),
+        "kv_get_device_error": (st, [vp, P(i64)]),
+        "kv_ctx_stats": (st, [vp, P(kvx_stats)]),
+        "kv_ctx_reset_stats": (st, [vp]),
+        "kv_ctx_modes": (st, [vp, P(i32), P(i32)]),
+        "kv_last_cuda_error": (ctypes.c_int, []),
+        "kv_last_error_message": (ctypes.c_char_p, []),
+        "kv_status_string": (ctypes.c_char_p, [ctypes.c_int]),
+        "kv_abi_version": (ctypes.c_int, []),
+        "kvx_probe_delayed_fill": (st, [vp, i64, i32, i64, vp]),
+        "kvx_probe_delayed_copy": (st, [vp, vp, i64, i64, vp]),
+        "kvx_probe_copy": (st, [vp, vp, i64, i32, vp]),
+    }
+    for name, (res, args) in sig.items():
+        f = getattr(lib, name)
+        f.restype = res
+        f.argtypes = args
+    return lib
+
+
+def load_library(path: str = _LIB_PATH):
+    if not os.path.exists(path):
+        raise ImportError(f"libkvxfer.so is not built ({path}); run paper_2609_15021_gb300._build.build()")
+    return _declare(ctypes.CDLL(path))
+
+
+_lib = load_library()
+
+
+def library_path() -> str:
+    return _LIB_PATH
+
+
+def _check(status: int, where: str):
+    if status != KVX_OK:
+        msg = _lib.kv_status_string(status).decode()
+        if status == KVX_ECUDA:
+            msg += f" (cuda error {_lib.kv_last_cuda_error()}: {_lib.kv_last_error_message().decode()})"
+        raise KvxError(status, where, msg)
+
+
+def _stream_handle(stream) -> int | None:
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream or None
+    if isinstance(stream, int):
+        return stream or None
+    return stream.cuda_stream or None
+
+
+def _ptr(x) -> int:
+    return x if isinstance(x, int) else x.data_ptr()
+
+
+# ---------------------------------------------------------------- pools
+
+
+@dataclass
+class KvPool:
+    """A paged KV pool: one contiguous device buffer per layer."""
+
+    layers: Sequence  # torch tensors (any dtype), one per layer, num_blocks * page_bytes each
+    num_blocks: int
+    block_tokens: int
+    num_heads: int
+    head_dim: int
+    elem_bytes: int
+    layout: int = KVX_LAYOUT_HND
+
+    def __post_init__(self):
+        self._bases = (ctypes.c_void_p * max(1, len(self.layers)))(*[_ptr(t) for t in self.layers])
+        self._c = kvx_pool(len(self.layers), ctypes.cast(self._bases, ctypes.POINTER(ctypes.c_void_p)),
+                           self.num_blocks, self.block_tokens, self.num_heads, self.head_dim,
+                           self.elem_bytes, self.layout)
+
+    @property
+    def row_bytes(self) -> int:
+        return self.head_dim * self.elem_bytes
+
+    @property
+    def page_bytes(self) -> int:
+        return 2 * self.num_heads * self.block_tokens * self.row_bytes
+
+    @property
+    def c(self) -> kvx_pool:
+        return self._c
+
+
+# ---------------------------------------------------------------- context
+
+
+def kv_ctx_create(device: int = 0, store_mode: int = KVX_MODE_AUTO, load_mode: int = KVX_MODE_AUTO,
+                  staging_slots: int = 0, staging_slot_bytes: int = 0, max_ctas: int = 0,
+                  flags: int = 0) -> int:
+    opts = kvx_opts(store_mode, load_mode, staging_slots, staging_slot_bytes, max_ctas, flags)
+    out = ctypes.c_void_p()
+    _check(_lib.kv_ctx_create(device, ctypes.byref(opts), ctypes.byref(out)), "kv_ctx_create")
+    return out.value
+
+
+def kv_ctx_destroy(ctx: int) -> None:
+    _lib.kv_ctx_destroy(ctx)
+
+
+def kv_chunk_layout(pool: KvPool, chunk_tokens: int, tokens_in_chunk: int) -> kvx_chunk_layout:
+    out = kvx_chunk_layout()
+    _check(_lib.kv_chunk_layout(ctypes.byref(pool.c), chunk_tokens, tokens_in_chunk, ctypes.byref(out)),
+           "kv_chunk_layout")
+    return out
+
+
+def _ptr_array(chunks):
+    return (ctypes.c_void_p * max(1, len(chunks)))(*[_ptr(c) for c in chunks])
+
+
+def _transfer(fn, name, ctx, pool, block_table, tok_begin, tok_end, chunk_tokens, chunks, stream,
+              table_len=None):
+    arr = _ptr_array(chunks)
+    n_tab = block_table.numel() if table_len is None else table_len
+    _check(fn(ctx, ctypes.byref(pool.c), _ptr(block_table), n_tab, tok_begin, tok_end, chunk_tokens,
+              arr, len(chunks), _stream_handle(stream)), name)
+
+
+def kv_store(ctx, pool: KvPool, block_table, tok_begin: int, tok_end: int, chunk_tokens: int,
+             host_chunks, stream=None, table_len: int | None = None) -> None:
+    """Gather tokens [tok_begin, tok_end) into pinned host chunks, ordered on `stream`."""
+    _transfer(_lib.kv_store, "kv_store", ctx, pool, block_table, tok_begin, tok_end, chunk_tokens,
+              host_chunks, stream, table_len)
+
+
+def kv_load(ctx, pool: KvPool, block_table, tok_begin: int, tok_end: int, chunk_tokens: int,
+            host_chunks, stream=None, table_len: int | None = None) -> None:
+    """Scatter pinned host chunks into the pages of `block_table`, ordered on `stream`."""
+    _transfer(_lib.kv_load, "kv_load", ctx, pool, block_table, tok_begin, tok_end, chunk_tokens,
+              host_chunks, stream, table_len)
+
+
+def kv_pack(ctx, pool: KvPool, block_table, tok_begin: int, tok_end: int, chunk_tokens: int,
+            dev_chunks, stream=None, table_len: int | None = None) -> None:
+    _transfer(_lib.kv_pack, "kv_pack", ctx, pool, block_table, tok_begin, tok_end, chunk_tokens,
+              dev_chunks, stream, table_len)
+
+
+def kv_unpack(ctx, pool: KvPool, block_table, tok_begin: int, tok_end: int, chunk_tokens: int,
+              dev_chunks, stream=None, table_len: int | None = None) -> None:
+    _transfer(_lib.kv_unpack, "kv_unpack", ctx, pool, block_table, tok_begin, tok_end, chunk_tokens,
+              dev_chunks, stream, table_len)
+
+
+def kv_state_store(ctx, layers, num_slots: int, slot_bytes: int, slot: int, host_obj, stream=None) -> None:
+    arr = _ptr_array(layers)
+    _check(_lib.kv_state_store(ctx, len(layers), arr, num_slots, slot_bytes, slot, _ptr(host_obj),
+                               _stream_handle(stream)), "kv_state_store")
+
+
+def kv_state_load(ctx, layers, num_slots: int, slot_bytes: int, slot: int, host_obj, stream=None) -> None:
+    arr = _ptr_array(layers)
+    _check(_lib.kv_state_load(ctx, len(layers), arr, num_slots, slot_bytes, slot, _ptr(host_obj),
+                              _stream_handle(stream)), "kv_state_load")
+
+
+def kv_get_device_error(ctx) -> int:
+    v = ctypes.c_int64(-1)
+    _check(_lib.kv_get_device_error(ctx, ctypes.byref(v)), "kv_get_device_error")
+    return v.value
+
+
+def kv_ctx_stats(ctx) -> dict:
+    s = kvx_stats()
+    _check(_lib.kv_ctx_stats(ctx, ctypes.byref(s)), "kv_ctx_stats")
+    out = {}
+    for name, _ in kvx_stats._fields_:
+        v = getattr(s, name)
+        out[name] = list(v) if isinstance(v, ctypes.Array) else v
+    return out
+
+
+def kv_ctx_reset_stats(ctx) -> None:
+    _check(_lib.kv_ctx_reset_stats(ctx), "kv_ctx_reset_stats")
+
+
+def kv_ctx_modes(ctx) -> tuple[int, int]:
+    a, b = ctypes.c_int32(), ctypes.c_int32()
+    _check(_lib.kv_ctx_modes(ctx, ctypes.byref(a), ctypes.byref(b)), "kv_ctx_modes")
+    return a.value, b.value
+
+
+def kv_abi_version() -> int:
+    return _lib.kv_abi_version()
+
+
+def kv_status_string(status: int) -> str:
+    return _lib.kv_status_string(status).decode()
+
+
+# ---------------------------------------------------------------- ordering probes
+
+
+def kvx_probe_delayed_fill(dev, nbytes: int, value: int, cycles: int, stream=None) -> None:
+    _check(_lib.kvx_probe_delayed_fill(_ptr(dev), nbytes, value, cycles, _stream_handle(stream)),
+           "kvx_probe_delayed_fill")
+
+
+def kvx_probe_delayed_copy(dst, src, nbytes: int, cycles: int, stream=None) -> None:
+    _check(_lib.kvx_probe_delayed_copy(_ptr(dst), _ptr(src), nbytes, cycles, _stream_handle(stream)),
+           "kvx_probe_delayed_copy")
+
+
+def kvx_probe_copy(dst, src, nbytes: int, how: int, stream=None) -> None:
+    _check(_lib.kvx_probe_copy(_ptr(dst), _ptr(src), nbytes, how, _stream_handle(stream)), "kvx_probe_copy")
+
+
+# ---------------------------------------------------------------- convenience
+
+
+class KvTransfer:
+    """Owns one kvx_ctx; the methods forward to the functions above."""
+
+    def __init__(self, device: int = 0, **opts):
+        self.ctx = kv_ctx_create(device, **opts)
+
+    def close(self):
+        if self.ctx:
+            kv_ctx_destroy(self.ctx)
+            self.ctx = None
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.close()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def store(self, pool, table, t0, t1, chunk_tokens, host_chunks, stream=None):
+        kv_store(self.ctx, pool, table, t0, t1, chunk_tokens, host_chunks, stream)
+
+    def load(self, pool, table, t0, t1, chunk_tokens, host_chunks, stream=None):
+        kv_load(self.ctx, pool, table, t0, t1, chunk_tokens, host_chunks, stream)
+
+    def pack(self, pool, table, t0, t1, chunk_tokens, dev_chunks, stream=None):
+        kv_pack(self.ctx, pool, table, t0, t1, chunk_tokens, dev_chunks, stream)
+
+    def unpack(self, pool, table, t0, t1, chunk_tokens, dev_chunks, stream=None):
+        kv_unpack(self.ctx, pool, table, t0, t1, chunk_tokens, dev_chunks, stream)
+
+    def device_error(self) -> int:
+        return kv_get_device_error(self.ctx)
+
+    def stats(self) -> dict:
+        return kv_ctx_stats(self.ctx)
+
+    def modes(self) -> tuple[int, int]:
+        return kv_ctx_modes(self.ctx)

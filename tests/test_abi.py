@@ -1,0 +1,110 @@
+"""The C-ABI library without a GPU: it loads, exports every declared symbol, and
+its host-only logic (chunk geometry, argument checks) behaves as documented."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import oracle
+from paper_2609_15021_gb300 import _build
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def k():
+    _build.build()
+    from paper_2609_15021_gb300 import kvxfer
+    return kvxfer
+
+
+def declared_functions():
+    names = set()
+    for h in os.listdir(os.path.join(ROOT, "include")):
+        if not h.endswith(".h"):
+            continue
+        text = open(os.path.join(ROOT, "include", h)).read()
+        text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+        for m in re.finditer(r"^\s*(?:const\s+)?[A-Za-z_][\w\s\*]*?\b([a-z]\w*)\s*\(", text, flags=re.M):
+            names.add(m.group(1))
+    return names - {"if", "while", "for", "return", "sizeof"}
+
+
+def test_exports_every_declared_symbol(k):
+    declared = declared_functions()
+    assert "kv_store" in declared and "kvx_probe_copy" in declared
+    lib = ctypes.CDLL(k.library_path())
+    missing = [n for n in sorted(declared) if not hasattr(lib, n)]
+    assert not missing, missing
+    assert set(k.EXPORTED) == declared
+
+
+def test_abi_version_and_strings(k):
+    assert k.kv_abi_version() == 1
+    assert k.kv_status_string(k.KVX_ENOTPINNED) == "host buffer is not page-locked"
+    assert k.kv_status_string(123) == "unknown status"
+
+
+def _pool(k, L=62, N=4096, B=16, H=8, D=128, e=2, layout=0):
+    return k.KvPool([0] * L, N, B, H, D, e, layout)
+
+
+@pytest.mark.parametrize("shape", [(62, 4096, 16, 8, 128, 2), (2, 64, 16, 2, 64, 2), (16, 100, 32, 4, 256, 1),
+                                   (3, 7, 4, 3, 24, 2)])
+@pytest.mark.parametrize("tokens_frac", [1.0, 0.5, 0.0])
+def test_chunk_layout_matches_oracle_geometry(k, orc, shape, tokens_frac):
+    L, N, B, H, D, e = shape
+    C = 4 * B
+    T = int(C * tokens_frac)
+    lay = k.kv_chunk_layout(_pool(k, *shape), C, T)
+    spec = oracle.PoolSpec(L, N, B, H, D, e)
+    assert lay.chunk_bytes == orc.chunk_bytes(spec, T)
+    assert lay.head_stride == D * e
+    assert lay.token_stride == H * D * e
+    assert lay.kv_stride == T * H * D * e
+    assert lay.layer_stride == 2 * T * H * D * e
+    assert lay.page_bytes == spec.page_bytes
+
+
+def test_chunk_layout_errors(k):
+    with pytest.raises(k.KvxError) as e:
+        k.kv_chunk_layout(_pool(k, B=16), 24, 24)      # C not a multiple of B
+    assert e.value.status == k.KVX_EALIGN
+    with pytest.raises(k.KvxError) as e:
+        k.kv_chunk_layout(_pool(k, D=12, e=1), 32, 32)  # 12-byte rows
+    assert e.value.status == k.KVX_EALIGN
+    with pytest.raises(k.KvxError) as e:
+        k.kv_chunk_layout(_pool(k), 256, 257)           # more tokens than the chunk
+    assert e.value.status == k.KVX_EINVAL
+    with pytest.raises(k.KvxError) as e:
+        k.kv_chunk_layout(_pool(k, L=k.KVX_MAX_LAYERS + 1), 256, 1)
+    assert e.value.status == k.KVX_EINVAL
+    with pytest.raises(k.KvxError) as e:
+        k.kv_chunk_layout(_pool(k, layout=7), 256, 1)
+    assert e.value.status == k.KVX_EINVAL
+
+
+def test_null_context_rejected_before_cuda(k):
+    pool = _pool(k)
+    arr = (ctypes.c_void_p * 1)(0)
+    for fn in (k._lib.kv_store, k._lib.kv_load, k._lib.kv_pack, k._lib.kv_unpack):
+        assert fn(None, ctypes.byref(pool.c), 0, 0, 0, 0, 256, arr, 0, None) == k.KVX_EINVAL
+    assert k._lib.kv_get_device_error(None, None) == k.KVX_EINVAL
+    assert k._lib.kv_ctx_create(0, None, None) == k.KVX_EINVAL
+
+
+def test_bad_options_rejected(k):
+    for kw in ({"store_mode": 9}, {"staging_slots": 1}, {"staging_slot_bytes": 17}, {"max_ctas": -1}):
+        with pytest.raises(k.KvxError) as e:
+            k.kv_ctx_create(0, **kw)
+        assert e.value.status == k.KVX_EINVAL
+
+
+def test_no_gpu_context_reports_cuda_error(k):
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is present")
+    with pytest.raises(k.KvxError) as e:
+        k.kv_ctx_create(0)
+    assert e.value.status in (k.KVX_ECUDA, k.KVX_EINVAL)

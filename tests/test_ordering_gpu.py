@@ -1,0 +1,180 @@
+"""Copy ordering on the caller's current stream (paper Sec. 3.2, Fig. 2, Table 2).
+
+1. The paper's byte probes: a kernel on a non-blocking stream writes 37 after
+   ~10^8 SM cycles (host->device variant: reads the old value 0 after the
+   delay) and a copy is issued (a) with no stream argument -- the raw
+   fallback -- or (b) by one of the three ordered mechanisms.  Sizes 4 KiB,
+   1 MiB, 16 MiB, both directions, delayed and undelayed, ten trials per cell.
+   Delayed raw copies must see every byte stale; ordered copies none.
+2. The same experiment through kv_store / kv_load: a delayed producer writes
+   the final KV just before kv_store on the caller's stream; a delayed
+   consumer reads pages just before kv_load overwrites them.  Both transfer
+   modes must give the final (store) / old (consumer) bytes.  The library's
+   negative control (KVX_FLAG_UNORDERED drops the wait on the caller's stream)
+   must give stale bytes in every delayed trial.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from gpu_util import POISON, device_pool, first_mismatch, host_layers, kvx, np_of, oracle_load, oracle_store
+from paper_2609_15021_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+DELAY = 10 ** 8          # SM cycles (Sec. 3.2 supplementary controls)
+TRIALS = 10              # per cell (Sec. 3.2)
+SIZES = [4096, 1 << 20, 16 << 20]
+MECHS = ["raw", "wait_then_copy", "async_on_stream", "same_stream_tensor_copy"]
+
+
+def _copy(k, how, dst, src, n, stream):
+    if how == "same_stream_tensor_copy":
+        with torch.cuda.stream(stream):
+            dst.copy_(src, non_blocking=True)
+        return
+    code = {"raw": k.KVX_PROBE_RAW, "wait_then_copy": k.KVX_PROBE_WAIT_THEN_COPY,
+            "async_on_stream": k.KVX_PROBE_ASYNC_ON_STREAM}[how]
+    k.kvx_probe_copy(dst, src, n, code, stream)
+
+
+def _d2h_mismatches(k, how, n, delay):
+    stream = torch.cuda.Stream()
+    dev = torch.zeros(n, dtype=torch.uint8, device="cuda")
+    host = torch.zeros(n, dtype=torch.uint8).pin_memory()
+    torch.cuda.synchronize()
+    k.kvx_probe_delayed_fill(dev, n, 37, delay, stream)   # producer: delayed write of 37
+    _copy(k, how, host, dev, n, stream)
+    stream.synchronize()                                   # host completion before consumption
+    return int((host != 37).sum())
+
+
+def _h2d_mismatches(k, how, n, delay):
+    stream = torch.cuda.Stream()
+    buf = torch.zeros(n, dtype=torch.uint8, device="cuda")   # old value 0
+    readout = torch.full((n,), 1, dtype=torch.uint8, device="cuda")
+    src = torch.full((n,), 53, dtype=torch.uint8).pin_memory()
+    torch.cuda.synchronize()
+    k.kvx_probe_delayed_copy(readout, buf, n, delay, stream)  # consumer: delayed read of the old value
+    _copy(k, how, buf, src, n, stream)                        # then overwrite with 53
+    stream.synchronize()
+    torch.cuda.synchronize()
+    return int((readout != 0).sum())
+
+
+def test_probe_matrix():
+    """Table 2 'Copy-ordering controls': delayed raw fails every check, ordered controls pass all."""
+    k = kvx()
+    counts = {}
+    for n in SIZES:
+        for direction, fn in (("d2h", _d2h_mismatches), ("h2d", _h2d_mismatches)):
+            for delay in (0, DELAY):
+                for how in MECHS:
+                    res = [fn(k, how, n, delay) for _ in range(TRIALS)]
+                    counts[(n, direction, delay, how)] = res
+                    if how != "raw":
+                        assert all(r == 0 for r in res), (n, direction, delay, how, res)
+                    elif delay:
+                        assert all(r == n for r in res), (n, direction, how, res)
+    delayed_raw = [c for key, c in counts.items() if key[3] == "raw" and key[2]]
+    ordered = [c for key, c in counts.items() if key[3] != "raw"]
+    assert sum(len(c) for c in delayed_raw) == 60 and sum(len(c) for c in ordered) == 360
+    undelayed_raw_pass = sum(r == 0 for key, c in counts.items() if key[3] == "raw" and not key[2] for r in c)
+    print(f"undelayed raw checks passing: {undelayed_raw_pass}/60")
+
+
+def _api_case(n_bytes):
+    """A one-layer HND pool whose single chunk holds n_bytes (rows of 256 B)."""
+    if n_bytes == 4096:
+        B, C = 8, 8
+    else:
+        B, C = 16, n_bytes // (2 * 256)
+    n_pages = C // B
+    spec = oracle.PoolSpec(1, n_pages + 3, B, 1, 128, 2, oracle.HND)
+    return spec, C, synth.permuted_table(n_pages + 3, n_pages, seed=n_bytes % 997)
+
+
+@pytest.fixture(scope="module")
+def ctxs():
+    k = kvx()
+    made = {}
+
+    def get(mode, unordered=False):
+        key = (mode, unordered)
+        if key not in made:
+            made[key] = k.kv_ctx_create(0, store_mode=mode, load_mode=mode,
+                                        flags=k.KVX_FLAG_UNORDERED if unordered else 0)
+        return made[key]
+
+    yield get
+    for c in made.values():
+        k.kv_ctx_destroy(c)
+
+
+VARIANTS = [("staged", 1, False), ("zerocopy", 2, False), ("staged_unordered", 1, True),
+            ("zerocopy_unordered", 2, True)]
+
+
+@pytest.mark.parametrize("n_bytes", SIZES)
+def test_store_after_delayed_producer(orc, ctxs, n_bytes):
+    k = kvx()
+    spec, C, table = _api_case(n_bytes)
+    stale_np = host_layers(spec, 1)
+    final_np = host_layers(spec, 2)
+    want_final, _ = oracle_store(orc, spec, final_np, table, 0, C, C)
+    want_stale, _ = oracle_store(orc, spec, stale_np, table, 0, C, C)
+    assert want_final[0].size == n_bytes
+    final_dev = torch.from_numpy(final_np[0]).cuda()
+    table_d = torch.from_numpy(table).cuda()
+    for name, mode, unordered in VARIANTS:
+        ctx = ctxs(mode, unordered)
+        for delay in (0, DELAY):
+            for trial in range(TRIALS):
+                pool = device_pool(spec, stale_np)
+                host = [torch.full((n_bytes,), POISON, dtype=torch.uint8).pin_memory()]
+                stream = torch.cuda.Stream()
+                torch.cuda.synchronize()
+                k.kvx_probe_delayed_copy(pool.layers[0], final_dev, spec.layer_bytes, delay, stream)
+                k.kv_store(ctx, pool, table_d, 0, C, C, host, stream=stream)
+                stream.synchronize()
+                got = np_of(host[0])
+                if not unordered:
+                    assert first_mismatch(got, want_final[0]) is None, (name, delay, trial)
+                elif delay:
+                    # the paper's missing dependency: every byte is the stale one
+                    assert first_mismatch(got, want_stale[0]) is None, (name, trial)
+                torch.cuda.synchronize()
+
+
+@pytest.mark.parametrize("n_bytes", SIZES)
+def test_load_after_delayed_consumer(orc, ctxs, n_bytes):
+    k = kvx()
+    spec, C, table = _api_case(n_bytes)
+    old_np = host_layers(spec, 3)
+    new_np = host_layers(spec, 4)
+    chunk_new, _ = oracle_store(orc, spec, new_np, table, 0, C, C)
+    loaded, _ = oracle_load(orc, spec, old_np, table, 0, C, C, chunk_new)
+    host = [torch.from_numpy(chunk_new[0]).pin_memory()]
+    table_d = torch.from_numpy(table).cuda()
+    for name, mode, unordered in VARIANTS:
+        ctx = ctxs(mode, unordered)
+        for delay in (0, DELAY):
+            for trial in range(TRIALS):
+                pool = device_pool(spec, old_np)
+                readout = torch.full((spec.layer_bytes,), POISON, dtype=torch.uint8, device="cuda")
+                after = torch.full((spec.layer_bytes,), POISON, dtype=torch.uint8, device="cuda")
+                stream = torch.cuda.Stream()
+                torch.cuda.synchronize()
+                k.kvx_probe_delayed_copy(readout, pool.layers[0], spec.layer_bytes, delay, stream)
+                k.kv_load(ctx, pool, table_d, 0, C, C, host, stream=stream)
+                k.kvx_probe_delayed_copy(after, pool.layers[0], spec.layer_bytes, 0, stream)
+                stream.synchronize()
+                assert first_mismatch(np_of(pool.layers[0]), loaded[0]) is None, (name, delay, trial)
+                # a consumer enqueued after kv_load sees the loaded pages
+                assert first_mismatch(np_of(after), loaded[0]) is None, (name, delay, trial)
+                if not unordered:
+                    assert first_mismatch(np_of(readout), old_np[0]) is None, (name, delay, trial)
+                elif delay:
+                    # the consumer read bytes the load had already overwritten
+                    assert first_mismatch(np_of(readout), loaded[0]) is None, (name, trial)

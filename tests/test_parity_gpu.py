@@ -1,0 +1,246 @@
+"""Bit-exact parity of the CUDA path with the CPU oracle, through the C ABI.
+
+Sizes are small enough for the oracle to finish in well under a second each,
+yet span several warp units, several kernel launches (more chunks than one
+launch carries), staging batches that split a chunk by layers, ragged last
+pages and short last chunks, a non-zero start, both page layouts, the fast
+(power-of-two row) and generic row paths, and both transfer modes.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from gpu_util import (POISON, device_chunks, device_pool, first_mismatch, host_layers, kvx, np_of,
+                      oracle_load, oracle_store, pinned_chunks, spec_of)
+from paper_2609_15021_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+HND, NHD = oracle.HND, oracle.NHD
+
+# name: (L, N, B, H, D, e, layout, n_used, C, first_chunk, t1 short by)
+CASES = {
+    "tiny_cfg_hnd": (2, 64, 16, 2, 64, 2, HND, 32, 256, 0, 0),
+    "tiny_cfg_nhd": (2, 64, 16, 2, 64, 2, NHD, 32, 256, 0, 0),
+    "ragged_tail_offset_start": (3, 40, 16, 4, 64, 2, HND, 37, 64, 1, 5),
+    "ragged_tail_nhd": (3, 40, 16, 4, 64, 2, NHD, 37, 64, 2, 9),
+    "rows_48B_generic": (2, 20, 4, 3, 24, 2, HND, 17, 8, 0, 3),
+    "rows_1KiB_generic": (2, 12, 8, 2, 256, 4, HND, 10, 16, 0, 1),
+    "rows_16B_16_heads": (1, 30, 2, 16, 16, 1, HND, 25, 4, 2, 1),
+    "fp8_1568_token_chunks": (4, 120, 32, 4, 256, 1, HND, 103, 1568, 0, 7),
+    "many_chunks_three_launches": (1, 300, 1, 1, 8, 2, HND, 300, 2, 0, 1),
+    "one_token": (2, 8, 16, 8, 128, 2, HND, 1, 256, 0, 15),
+    "27b_shape_two_chunks": (62, 48, 16, 8, 128, 2, HND, 40, 256, 0, 3),
+}
+
+MODES = {"staged": 1, "zerocopy": 2}
+
+
+def _range(case):
+    L, N, B, H, D, e, layout, n_used, C, c0, short = case
+    return c0 * C, n_used * B - short
+
+
+@pytest.fixture(scope="module")
+def ctxs():
+    k = kvx()
+    made = {}
+
+    def get(mode, slot_bytes=0):
+        key = (mode, slot_bytes)
+        if key not in made:
+            made[key] = k.kv_ctx_create(0, store_mode=mode, load_mode=mode, staging_slot_bytes=slot_bytes)
+        return made[key]
+
+    yield get
+    for c in made.values():
+        k.kv_ctx_destroy(c)
+
+
+def _run_case(orc, ctx, case, stream):
+    k = kvx()
+    L, N, B, H, D, e, layout, n_used, C, c0, short = case
+    spec = oracle.PoolSpec(L, N, B, H, D, e, layout)
+    t0, t1 = _range(case)
+    src_np = host_layers(spec, seed=hash(case) % 100000)
+    src = device_pool(spec, src_np)
+    ta = synth.permuted_table(N, n_used, seed=11)
+    tb = synth.permuted_table(N, n_used, seed=12)
+    ta_d = torch.from_numpy(ta).cuda()
+    tb_d = torch.from_numpy(tb).cuda()
+    extra = 48
+    host = pinned_chunks(orc, spec, t0, t1, C, extra=extra)
+    torch.cuda.synchronize()
+    with torch.cuda.stream(stream):
+        k.kv_store(ctx, src, ta_d, t0, t1, C, host)
+    stream.synchronize()
+    want, _ = oracle_store(orc, spec, src_np, ta, t0, t1, C)
+    assert len(want) == len(host)
+    for i, (h, w) in enumerate(zip(host, want)):
+        got = np_of(h)
+        assert first_mismatch(got[:-extra], w) is None, (i, first_mismatch(got[:-extra], w))
+        assert np.all(got[-extra:] == POISON), f"chunk {i}: bytes written past its end"
+    # load into a poisoned pool through another table
+    dst = device_pool(spec)
+    with torch.cuda.stream(stream):
+        k.kv_load(ctx, dst, tb_d, t0, t1, C, host)
+    stream.synchronize()
+    poisoned = [np.full(spec.layer_bytes, POISON, np.uint8) for _ in range(L)]
+    want_l, _ = oracle_load(orc, spec, poisoned, tb, t0, t1, C, want)
+    for l in range(L):
+        assert first_mismatch(np_of(dst.layers[l]), want_l[l]) is None, (l, first_mismatch(np_of(dst.layers[l]), want_l[l]))
+    assert k.kv_get_device_error(ctx) == -1
+
+
+@pytest.mark.parametrize("mode", list(MODES))
+@pytest.mark.parametrize("name", list(CASES))
+def test_store_load_parity(orc, ctxs, name, mode):
+    stream = torch.cuda.Stream()  # a non-blocking pool stream, as in the paper's setting
+    _run_case(orc, ctxs(MODES[mode]), CASES[name], stream)
+
+
+@pytest.mark.parametrize("name", ["ragged_tail_offset_start", "27b_shape_two_chunks", "fp8_1568_token_chunks"])
+def test_staged_one_layer_per_slot(orc, ctxs, name):
+    """Staging slots that hold exactly one layer of a full chunk: every chunk is split
+    into per-layer pieces, and the ring of slots is reused many times per call."""
+    case = CASES[name]
+    L, N, B, H, D, e, layout, n_used, C, c0, short = case
+    slot = 2 * C * H * D * e
+    _run_case(orc, ctxs(1, slot), case, torch.cuda.Stream())
+
+
+@pytest.mark.parametrize("name", ["tiny_cfg_hnd", "ragged_tail_nhd", "rows_48B_generic", "many_chunks_three_launches",
+                                  "27b_shape_two_chunks"])
+def test_device_pack_unpack_parity(orc, ctxs, name):
+    k = kvx()
+    case = CASES[name]
+    L, N, B, H, D, e, layout, n_used, C, c0, short = case
+    spec = oracle.PoolSpec(L, N, B, H, D, e, layout)
+    t0, t1 = _range(case)
+    src_np = host_layers(spec, seed=77)
+    src = device_pool(spec, src_np)
+    ta = synth.permuted_table(N, n_used, seed=21)
+    tb = synth.permuted_table(N, n_used, seed=22)
+    extra = 32
+    dev = device_chunks(orc, spec, t0, t1, C, extra=extra)
+    ctx = ctxs(1)
+    k.kv_pack(ctx, src, torch.from_numpy(ta).cuda(), t0, t1, C, dev)
+    torch.cuda.synchronize()
+    want, _ = oracle_store(orc, spec, src_np, ta, t0, t1, C)
+    for i, (d, w) in enumerate(zip(dev, want)):
+        got = np_of(d)
+        assert first_mismatch(got[:-extra], w) is None, i
+        assert np.all(got[-extra:] == POISON)
+    dst = device_pool(spec)
+    k.kv_unpack(ctx, dst, torch.from_numpy(tb).cuda(), t0, t1, C, dev)
+    torch.cuda.synchronize()
+    want_l, _ = oracle_load(orc, spec, [np.full(spec.layer_bytes, POISON, np.uint8) for _ in range(L)],
+                            tb, t0, t1, C, want)
+    for l in range(L):
+        assert first_mismatch(np_of(dst.layers[l]), want_l[l]) is None, l
+
+
+@pytest.mark.parametrize("mode", list(MODES))
+def test_out_of_range_pages_reported(orc, ctxs, mode):
+    """Entries outside [0, num_blocks) skip their page and report the lowest bad logical block;
+    every other byte still matches the oracle (which applies the same rule)."""
+    k = kvx()
+    spec = oracle.PoolSpec(2, 16, 16, 2, 64, 2, HND)
+    src_np = host_layers(spec, seed=5)
+    src = device_pool(spec, src_np)
+    table = synth.permuted_table(16, 12, seed=3)
+    table[5] = 16      # one past the last page
+    table[9] = -3
+    C, t0, t1 = 64, 0, 12 * 16
+    host = pinned_chunks(orc, spec, t0, t1, C)
+    ctx = ctxs(MODES[mode])
+    k.kv_store(ctx, src, torch.from_numpy(table).cuda(), t0, t1, C, host)
+    torch.cuda.synchronize()
+    assert k.kv_get_device_error(ctx) == 5
+    assert k.kv_get_device_error(ctx) == -1  # cleared by the query
+    want, bad = oracle_store(orc, spec, src_np, table, t0, t1, C)
+    assert bad == 5
+    for h, w in zip(host, want):
+        assert first_mismatch(np_of(h), w) is None
+
+
+@pytest.mark.parametrize("mode", list(MODES))
+def test_empty_range_is_a_no_op(orc, ctxs, mode):
+    k = kvx()
+    spec = oracle.PoolSpec(1, 4, 16, 1, 64, 2, HND)
+    src = device_pool(spec, host_layers(spec, 1))
+    host = [torch.full((4096,), POISON, dtype=torch.uint8).pin_memory()]
+    table = torch.arange(4, dtype=torch.int32, device="cuda")
+    ctx = ctxs(MODES[mode])
+    k.kv_store(ctx, src, table, 32, 32, 32, host)
+    k.kv_load(ctx, src, table, 32, 32, 32, [])
+    torch.cuda.synchronize()
+    assert np.all(np_of(host[0]) == POISON)
+
+
+def test_back_to_back_calls_reuse_slots(orc, ctxs):
+    """store A -> load B -> store B with no host synchronisation in between, through
+    one-layer staging slots: slot reuse across calls must respect every event edge."""
+    k = kvx()
+    spec = oracle.PoolSpec(4, 64, 16, 4, 64, 2, HND)
+    C, n_used = 128, 60
+    t0, t1 = 0, n_used * 16 - 3
+    src_np = host_layers(spec, 99)
+    src = device_pool(spec, src_np)
+    ta = torch.from_numpy(synth.permuted_table(64, n_used, 1)).cuda()
+    tb = torch.from_numpy(synth.permuted_table(64, n_used, 2)).cuda()
+    ctx = ctxs(1, 2 * C * 4 * 64 * 2)
+    h1 = pinned_chunks(orc, spec, t0, t1, C)
+    h2 = pinned_chunks(orc, spec, t0, t1, C)
+    dst = device_pool(spec)
+    s = torch.cuda.Stream()
+    with torch.cuda.stream(s):
+        for _ in range(3):
+            k.kv_store(ctx, src, ta, t0, t1, C, h1)
+            k.kv_load(ctx, dst, tb, t0, t1, C, h1)
+            k.kv_store(ctx, dst, tb, t0, t1, C, h2)
+    s.synchronize()
+    want, _ = oracle_store(orc, spec, src_np, ta.cpu().numpy(), t0, t1, C)
+    for a, b, w in zip(h1, h2, want):
+        assert first_mismatch(np_of(a), w) is None
+        assert first_mismatch(np_of(b), w) is None
+
+
+@pytest.mark.parametrize("which", ["legacy_default", "per_thread", "torch_default"])
+def test_special_streams(orc, ctxs, which):
+    k = kvx()
+    spec = oracle.PoolSpec(2, 32, 16, 2, 64, 2, HND)
+    src_np = host_layers(spec, 3)
+    src = device_pool(spec, src_np)
+    table = synth.permuted_table(32, 20, 4)
+    host = pinned_chunks(orc, spec, 0, 320, 64)
+    stream = {"legacy_default": 0, "per_thread": 2, "torch_default": torch.cuda.default_stream().cuda_stream}[which]
+    k.kv_store(ctxs(1), src, torch.from_numpy(table).cuda(), 0, 320, 64, host, stream=stream)
+    torch.cuda.synchronize()
+    want, _ = oracle_store(orc, spec, src_np, table, 0, 320, 64)
+    for h, w in zip(host, want):
+        assert first_mismatch(np_of(h), w) is None
+
+
+@pytest.mark.parametrize("mode", list(MODES))
+def test_state_snapshot_parity(orc, ctxs, mode):
+    """Recurrent-state snapshots: slot 3 of 5 layers out to host, then into slot 1."""
+    k = kvx()
+    L, slots, sb = 5, 4, 16 * 128 * 128 * 4 // 64
+    layers_np = [synth.splitmix64_bytes(slots * sb, 900 + l) for l in range(L)]
+    layers = [torch.from_numpy(a).cuda() for a in layers_np]
+    obj = torch.full((L * sb,), POISON, dtype=torch.uint8).pin_memory()
+    ctx = ctxs(MODES[mode])
+    k.kv_state_store(ctx, layers, slots, sb, 3, obj)
+    torch.cuda.synchronize()
+    want = np.full(L * sb, POISON, np.uint8)
+    assert orc.state_copy(layers_np, sb, 3, want, True) == 0
+    assert first_mismatch(np_of(obj), want) is None
+    dst_np = [np.full(slots * sb, POISON, np.uint8) for _ in range(L)]
+    dst = [torch.from_numpy(a).cuda() for a in dst_np]
+    k.kv_state_load(ctx, dst, slots, sb, 1, obj)
+    torch.cuda.synchronize()
+    assert orc.state_copy(dst_np, sb, 1, want, False) == 0
+    for a, b in zip(dst, dst_np):
+        assert first_mismatch(np_of(a), b) is None
