@@ -213,6 +213,40 @@ kvx_status kv_state_load(kvx_ctx* ctx, int32_t num_layers, void* const* layer_ba
                          int64_t slot_bytes, int64_t slot, const void* host_obj, kvx_stream_t stream);
 
 /*
+ * kv_store without any allocation (the paper has no counterpart: this entry
+ * point exists for callers that cannot allocate device memory).
+ *
+ * Who needs it: code running under an engine whose memory pool owns all free
+ * GPU memory and must not see allocations it does not track, or code that must
+ * not let cudaMalloc/cudaFree synchronise the device mid-pipeline.  kv_store
+ * needs a context, and a context allocates a staging ring, streams and events.
+ * This call creates nothing: it packs into a static device array of
+ * KVX_NOALLOC_SCRATCH_BYTES (64 MiB, plus 256 bytes) that every GPU loading
+ * this part of the library holds until the process exits, and copies each
+ * packed batch to the host chunks with cudaMemcpyAsync, all on `stream` and in
+ * stream order (no overlap of packing and copying, unlike kv_store).
+ *
+ * Arguments, layout, alignment, pinned-memory and range rules are those of
+ * kv_store; it runs on the calling thread's current device.  One layer of one
+ * chunk (2 * tokens * H * head_dim * elem_bytes) must fit in the array, else
+ * KVX_ERANGE (kv_last_error_message names both sizes).
+ *   dev_first_bad_block : NULL, or a device int64 that the kernel lowers by
+ *                         atomicMin to the lowest logical block whose table
+ *                         entry is out of range (initialise it, e.g. to
+ *                         INT64_MAX); such tokens are stored as zeros.
+ * Set-up: the first call on a device (with that device current) looks up the
+ * array's device address with cudaGetSymbolAddress and caches it; make that
+ * first call before any stream capture.  All calls share the one array and
+ * nothing in it needs to start at zero (every staged byte is written before it
+ * is copied).  Calls that overlap on the GPU -- on different streams without an
+ * ordering between them -- race on the array: order them.
+ */
+#define KVX_NOALLOC_SCRATCH_BYTES (64ll << 20)
+kvx_status kv_store_noalloc(const kvx_pool* pool, const int32_t* block_table, int64_t table_len,
+                            int64_t tok_begin, int64_t tok_end, int32_t chunk_tokens, void* const* host_chunks,
+                            int64_t n_chunks, int64_t* dev_first_bad_block, kvx_stream_t stream);
+
+/*
  * Lowest logical block index whose table entry was out of range in any call
  * completed since the last query, or -1.  Call after the caller's stream has
  * been synchronised.  Clears the record.

@@ -53,6 +53,30 @@ struct SegmentParams {
   int32_t n_seg;
 };
 
+// Byte geometry of a pool description.
+struct Geometry {
+  int64_t row;          // head_dim * elem_bytes
+  int64_t page_bytes;   // 2 * H * B * row
+  int64_t layer_bytes;  // num_blocks * page_bytes
+};
+
+enum Where : int { kHostChunks = 0, kDeviceChunks = 1 };
+
+// Argument checks shared by the pack/unpack entry points (kvxfer.cu): pool
+// shape and memory, token range, block table, and every chunk pointer of
+// [t0, t1) on `device`.  Fills *g and *n (chunks in the range) and, when
+// `side` is not null, side[i] = the address of chunk i that the kernel or
+// copy engine uses (mapped address for zero-copy host chunks).  Enqueues
+// nothing and allocates nothing.
+kvx_status check_transfer(int device, const kvx_pool* P, const int32_t* table, int64_t table_len, int64_t t0,
+                          int64_t t1, int32_t C, void* const* chunks, int64_t n_chunks, cudaStream_t stream,
+                          int where, int mode, Geometry* g, int64_t* n, uint8_t** side);
+void init_params(MoveParams* p, long long* err, const kvx_pool* P, const Geometry& g, const int32_t* table,
+                 int32_t C);
+void push_job(MoveParams* p, uint8_t* chunk_side, int64_t first_block, int32_t tokens, int32_t l0, int32_t nl);
+int64_t chunk_bytes(const kvx_pool* P, const Geometry& g, int64_t tokens);
+void set_error_text(const char* text);
+
 // Launchers (pack_kernels.cu).  Return the cudaError_t of the launch.
 cudaError_t launch_move(int dir, int layout, const MoveParams& p, int grid, cudaStream_t s);
 cudaError_t launch_segments(const SegmentParams& p, int grid, cudaStream_t s);

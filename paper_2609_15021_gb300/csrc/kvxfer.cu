@@ -166,12 +166,6 @@ kvx_status check_stream_device(cudaStream_t s, int device) {
   return d == device ? KVX_OK : KVX_EDEVICE;
 }
 
-struct Geometry {
-  int64_t row;         // head_dim * elem_bytes
-  int64_t page_bytes;  // 2 * H * B * row
-  int64_t layer_bytes; // num_blocks * page_bytes
-};
-
 kvx_status check_pool_shape(const kvx_pool* P, Geometry* g) {
   if (!P || !P->layer_base) return KVX_EINVAL;
   if (P->num_layers < 1 || P->num_layers > KVX_MAX_LAYERS) return KVX_EINVAL;
@@ -192,12 +186,12 @@ kvx_status check_pool_shape(const kvx_pool* P, Geometry* g) {
   return KVX_OK;
 }
 
-kvx_status check_pool_memory(const kvx_ctx* ctx, const kvx_pool* P, const Geometry& g) {
+kvx_status check_pool_memory(int device, const kvx_pool* P, const Geometry& g) {
   for (int l = 0; l < P->num_layers; ++l) {
     const void* b = P->layer_base[l];
     if (!b) return KVX_EINVAL;
     if ((uintptr_t)b & 15) return KVX_EALIGN;
-    kvx_status st = check_device_range(ctx->device, b, g.layer_bytes);
+    kvx_status st = check_device_range(device, b, g.layer_bytes);
     if (st != KVX_OK) return st;
   }
   return KVX_OK;
@@ -263,12 +257,12 @@ kvx_status launch_move_timed(kvx_ctx* ctx, int dir, int layout, const MoveParams
   return KVX_OK;
 }
 
-void init_move_params(MoveParams* p, const kvx_ctx* ctx, const kvx_pool* P, const Geometry& g,
+void init_move_params(MoveParams* p, long long* err, const kvx_pool* P, const Geometry& g,
                       const int32_t* table, int32_t C) {
   memset(p, 0, sizeof(*p));
   for (int l = 0; l < P->num_layers; ++l) p->layer_base[l] = (uint8_t*)P->layer_base[l];
   p->table = table;
-  p->err = ctx->d_err;
+  p->err = err;
   p->num_blocks = P->num_blocks;
   p->page_bytes = g.page_bytes;
   p->blocks_per_chunk = C / P->block_tokens;
@@ -340,7 +334,7 @@ struct Plan {
 // Zero-copy and device chunks: one kernel pass per batch of whole chunks.
 kvx_status enqueue_direct(kvx_ctx* ctx, const Plan& pl) {
   MoveParams p;
-  init_move_params(&p, ctx, pl.P, pl.g, pl.table, pl.C);
+  init_move_params(&p, ctx->d_err, pl.P, pl.g, pl.table, pl.C);
   int64_t bytes = 0;
   for (int64_t i = 0; i < pl.n; ++i) {
     add_job(&p, pl.side[i], (pl.first_chunk + i) * pl.bpc, pl.tokens[i], 0, pl.P->num_layers);
@@ -372,7 +366,7 @@ kvx_status enqueue_staged(kvx_ctx* ctx, const Plan& pl) {
     ctx->next_slot = (ctx->next_slot + 1) % ctx->nslots;
     uint8_t* slot = ctx->slots[k];
     MoveParams p;
-    init_move_params(&p, ctx, P, pl.g, pl.table, pl.C);
+    init_move_params(&p, ctx->d_err, P, pl.g, pl.table, pl.C);
     int64_t off = 0;
     for (const Piece& pc : batch) {
       add_job(&p, slot + off, (pl.first_chunk + pc.i) * pl.bpc, pl.tokens[pc.i], pc.l0, pc.nl);
@@ -459,35 +453,88 @@ kvx_status join_caller(kvx_ctx* ctx, cudaStream_t stream, bool copy_stream_used)
   return KVX_OK;
 }
 
-enum Where { kHostChunks = 0, kDeviceChunks = 1 };
+}  // namespace
+
+namespace kvx {
+
+void set_error_text(const char* text) { snprintf(g_last_error_text, sizeof(g_last_error_text), "%s", text); }
+
+kvx_status check_transfer(int device, const kvx_pool* P, const int32_t* table, int64_t table_len, int64_t t0,
+                          int64_t t1, int32_t C, void* const* chunks, int64_t n_chunks, cudaStream_t stream,
+                          int where, int mode, Geometry* g, int64_t* n_out, uint8_t** side) {
+  kvx_status st = check_pool_shape(P, g);
+  if (st != KVX_OK) return st;
+  int64_t n = 0;
+  st = check_range(P, table_len, t0, t1, C, n_chunks, &n);
+  if (st != KVX_OK) return st;
+  if (n > 0 && (!table || !chunks)) return KVX_EINVAL;
+  st = check_stream_device(stream, device);
+  if (st != KVX_OK) return st;
+  *n_out = n;
+  if (n == 0) return KVX_OK;  // empty range: nothing to order or move
+  st = check_pool_memory(device, P, *g);
+  if (st != KVX_OK) return st;
+  if ((uintptr_t)table & 3) return KVX_EALIGN;
+  const int64_t blocks_needed = (t1 + P->block_tokens - 1) / P->block_tokens;
+  st = check_device_range(device, table, blocks_needed * (int64_t)sizeof(int32_t));
+  if (st != KVX_OK) return st;
+  const int64_t first_chunk = t0 / C;
+  for (int64_t i = 0; i < n; ++i) {
+    const int64_t tokens = std::min<int64_t>(C, t1 - (first_chunk + i) * C);
+    const int64_t bytes = chunk_bytes_of(P, *g, tokens);
+    void* c = chunks[i];
+    if (!c) return KVX_EINVAL;
+    if ((uintptr_t)c & 15) return KVX_EALIGN;
+    uint8_t* s = (uint8_t*)c;
+    if (where == kDeviceChunks) {
+      st = check_device_range(device, c, bytes);
+      if (st != KVX_OK) return st;
+    } else {
+      uint8_t* mapped = nullptr;
+      st = check_pinned_range(c, bytes, &mapped);
+      if (st != KVX_OK) return st;
+      if (mode == KVX_MODE_ZEROCOPY) {
+        if (!mapped) return KVX_ENOTPINNED;
+        s = mapped;
+      }
+    }
+    if (side) side[i] = s;
+  }
+  return KVX_OK;
+}
+
+void init_params(MoveParams* p, long long* err, const kvx_pool* P, const Geometry& g, const int32_t* table,
+                 int32_t C) {
+  init_move_params(p, err, P, g, table, C);
+}
+
+void push_job(MoveParams* p, uint8_t* chunk_side, int64_t first_block, int32_t tokens, int32_t l0, int32_t nl) {
+  add_job(p, chunk_side, first_block, tokens, l0, nl);
+}
+
+int64_t chunk_bytes(const kvx_pool* P, const Geometry& g, int64_t tokens) { return chunk_bytes_of(P, g, tokens); }
+
+}  // namespace kvx
+
+namespace {
 
 // The shared body of kv_store / kv_load / kv_pack / kv_unpack.
 kvx_status transfer(kvx_ctx* ctx, const kvx_pool* P, const int32_t* table, int64_t table_len, int64_t t0,
                     int64_t t1, int32_t C, void* const* chunks, int64_t n_chunks, cudaStream_t stream,
                     int dir, int where) {
   if (!ctx) return KVX_EINVAL;
-  Plan pl;
-  kvx_status st = check_pool_shape(P, &pl.g);
-  if (st != KVX_OK) return st;
-  int64_t n = 0;
-  st = check_range(P, table_len, t0, t1, C, n_chunks, &n);
-  if (st != KVX_OK) return st;
-  if (n > 0 && (!table || !chunks)) return KVX_EINVAL;
-
   DeviceGuard guard(ctx->device);
   if (!guard.ok) return KVX_ECUDA;
-  st = check_stream_device(stream, ctx->device);
-  if (st != KVX_OK) return st;
-  if (n == 0) return KVX_OK;  // empty range: nothing to order or move
-  st = check_pool_memory(ctx, P, pl.g);
-  if (st != KVX_OK) return st;
-  if ((uintptr_t)table & 3) return KVX_EALIGN;
-  const int64_t blocks_needed = (t1 + P->block_tokens - 1) / P->block_tokens;
-  st = check_device_range(ctx->device, table, blocks_needed * (int64_t)sizeof(int32_t));
-  if (st != KVX_OK) return st;
-
   const int mode = (where == kDeviceChunks) ? KVX_MODE_ZEROCOPY
                                             : (dir == kPack ? ctx->store_mode : ctx->load_mode);
+  Plan pl;
+  int64_t cap = 0;  // entries the chunk arrays may need (checked below)
+  if (C > 0 && t0 >= 0 && t1 > t0) cap = std::min<int64_t>(n_chunks, (t1 + C - 1) / C - t0 / C);
+  pl.side.resize((size_t)std::max<int64_t>(cap, 0));
+  int64_t n = 0;
+  kvx_status st = check_transfer(ctx->device, P, table, table_len, t0, t1, C, chunks, n_chunks, stream, where,
+                                 mode, &pl.g, &n, pl.side.data());
+  if (st != KVX_OK || n == 0) return st;
   pl.P = P;
   pl.table = table;
   pl.C = C;
@@ -496,30 +543,8 @@ kvx_status transfer(kvx_ctx* ctx, const kvx_pool* P, const int32_t* table, int64
   pl.bpc = C / P->block_tokens;
   pl.dir = dir;
   pl.tokens.resize((size_t)n);
-  pl.side.resize((size_t)n);
-  for (int64_t i = 0; i < n; ++i) {
-    const int64_t first_tok = (pl.first_chunk + i) * C;
-    pl.tokens[i] = (int32_t)std::min<int64_t>(C, t1 - first_tok);
-    const int64_t bytes = chunk_bytes_of(P, pl.g, pl.tokens[i]);
-    void* c = chunks[i];
-    if (!c) return KVX_EINVAL;
-    if ((uintptr_t)c & 15) return KVX_EALIGN;
-    if (where == kDeviceChunks) {
-      st = check_device_range(ctx->device, c, bytes);
-      if (st != KVX_OK) return st;
-      pl.side[i] = (uint8_t*)c;
-    } else {
-      uint8_t* mapped = nullptr;
-      st = check_pinned_range(c, bytes, &mapped);
-      if (st != KVX_OK) return st;
-      if (mode == KVX_MODE_ZEROCOPY) {
-        if (!mapped) return KVX_ENOTPINNED;
-        pl.side[i] = mapped;
-      } else {
-        pl.side[i] = (uint8_t*)c;
-      }
-    }
-  }
+  for (int64_t i = 0; i < n; ++i)
+    pl.tokens[i] = (int32_t)std::min<int64_t>(C, t1 - (pl.first_chunk + i) * C);
   const bool staged = (mode == KVX_MODE_STAGED);
   const int64_t max_layer_bytes = 2ll * std::min<int64_t>(C, t1 - t0) * P->num_heads * pl.g.row;
   if (staged && max_layer_bytes > ctx->slot_bytes) return KVX_EINVAL;

@@ -1,0 +1,167 @@
+// no_alloc.cu -- kv_store_noalloc: the staged store with its staging buffer in
+// a static device array instead of memory the library allocates.
+//
+// Some callers cannot call cudaMalloc: an engine whose memory pool owns all
+// of the GPU's free memory and must not see allocations it does not track, or
+// code that must not let cudaMalloc / cudaFree synchronise the device in the
+// middle of a pipeline.  They keep inputs and outputs in their own buffers,
+// but the staged store also needs scratch memory to pack chunks before the
+// copy engines move them to the host.  This entry point takes that scratch
+// from g_scratch, a file-scope array of fixed size that every GPU which loads
+// this part of the library holds until the process exits.  It creates no
+// context, stream or event, and allocates no device, pinned or heap memory.
+//
+// In host code g_scratch is only a host-side stand-in for the symbol, not a
+// device address: it must not be passed to a kernel.  The device address is
+// obtained once per device with cudaGetSymbolAddress (first call on that
+// device, with the device current) and cached.
+
+#include <cuda_runtime.h>
+#include <stdio.h>
+
+#include <algorithm>
+#include <mutex>
+
+#include "kvx_internal.h"
+
+using namespace kvx;
+
+namespace {
+
+constexpr int64_t kSink = 256;  // head of the array: error word when the caller passes none
+constexpr int kMaxDevices = 64;
+
+static __device__ __align__(256) uint8_t g_scratch[kSink + KVX_NOALLOC_SCRATCH_BYTES];
+
+std::mutex g_mu;
+uint8_t* g_scratch_addr[kMaxDevices] = {};
+
+// Device address of g_scratch on `device` (which must be current).
+kvx_status scratch_address(int device, uint8_t** out) {
+  if (device < 0 || device >= kMaxDevices) return KVX_EINVAL;
+  std::lock_guard<std::mutex> lock(g_mu);
+  if (!g_scratch_addr[device]) {
+    void* p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_scratch);
+    if (e != cudaSuccess) {
+      set_last_cuda_error((int)e);
+      set_error_text("cudaGetSymbolAddress of the static staging array failed");
+      cudaGetLastError();
+      return KVX_ECUDA;
+    }
+    g_scratch_addr[device] = (uint8_t*)p;
+  }
+  *out = g_scratch_addr[device];
+  return KVX_OK;
+}
+
+kvx_status fail_cuda(cudaError_t e, const char* what) {
+  set_last_cuda_error((int)e);
+  set_error_text(what);
+  cudaGetLastError();
+  return KVX_ECUDA;
+}
+
+}  // namespace
+
+extern "C" kvx_status kv_store_noalloc(const kvx_pool* pool, const int32_t* block_table, int64_t table_len,
+                                       int64_t tok_begin, int64_t tok_end, int32_t chunk_tokens,
+                                       void* const* host_chunks, int64_t n_chunks, int64_t* dev_first_bad_block,
+                                       kvx_stream_t stream_handle) {
+  cudaStream_t stream = (cudaStream_t)stream_handle;
+  int device = 0;
+  cudaError_t e = cudaGetDevice(&device);
+  if (e != cudaSuccess) return fail_cuda(e, "cudaGetDevice");
+  Geometry g;
+  int64_t n = 0;
+  kvx_status st = check_transfer(device, pool, block_table, table_len, tok_begin, tok_end, chunk_tokens,
+                                 host_chunks, n_chunks, stream, kHostChunks, KVX_MODE_STAGED, &g, &n, nullptr);
+  if (st != KVX_OK || n == 0) return st;
+  const int64_t layer_bytes_max = 2ll * std::min<int64_t>(chunk_tokens, tok_end - tok_begin) * pool->num_heads * g.row;
+  if (layer_bytes_max > KVX_NOALLOC_SCRATCH_BYTES) {
+    char msg[160];
+    snprintf(msg, sizeof(msg), "one layer of one chunk needs %lld bytes; the static staging array holds %lld",
+             (long long)layer_bytes_max, (long long)KVX_NOALLOC_SCRATCH_BYTES);
+    set_error_text(msg);
+    return KVX_ERANGE;
+  }
+  if (dev_first_bad_block) {
+    if ((uintptr_t)dev_first_bad_block & 7) return KVX_EALIGN;
+    cudaPointerAttributes a;
+    if (cudaPointerGetAttributes(&a, dev_first_bad_block) != cudaSuccess) {
+      cudaGetLastError();
+      return KVX_EDEVICE;
+    }
+    if (a.type != cudaMemoryTypeDevice || a.device != device) return KVX_EDEVICE;
+  }
+  uint8_t* base = nullptr;
+  st = scratch_address(device, &base);
+  if (st != KVX_OK) return st;
+  uint8_t* staging = base + kSink;
+  long long* err = dev_first_bad_block ? (long long*)dev_first_bad_block : (long long*)base;
+  int sms = 1;
+  if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device)) != cudaSuccess)
+    return fail_cuda(e, "cudaDeviceGetAttribute");
+  const int64_t grid_cap = (int64_t)std::max(1, sms) * move_ctas_per_sm(kPack, pool->layout);
+
+  // Batches of (chunk, layer range) pieces that fit the array, each packed and
+  // then copied out on the caller's stream.  Stream order alone keeps a batch
+  // from overwriting the array before the previous batch's copies have read it.
+  const int64_t first_chunk = tok_begin / chunk_tokens;
+  const int64_t bpc = chunk_tokens / pool->block_tokens;
+  struct Piece {
+    int64_t i;
+    int32_t l0, nl;
+    int64_t bytes;
+  } batch[kMaxJobs];
+  int nb = 0;
+  int64_t used = 0;
+  auto tokens_of = [&](int64_t i) { return std::min<int64_t>(chunk_tokens, tok_end - (first_chunk + i) * chunk_tokens); };
+  auto layer_bytes = [&](int64_t i) { return 2ll * tokens_of(i) * pool->num_heads * g.row; };
+  auto flush = [&]() -> kvx_status {
+    if (nb == 0) return KVX_OK;
+    MoveParams p;
+    init_params(&p, err, pool, g, block_table, chunk_tokens);
+    int64_t off = 0;
+    for (int q = 0; q < nb; ++q) {
+      push_job(&p, staging + off, (first_chunk + batch[q].i) * bpc, (int32_t)tokens_of(batch[q].i), batch[q].l0,
+               batch[q].nl);
+      off += batch[q].bytes;
+    }
+    const int64_t grid = std::max<int64_t>(1, std::min<int64_t>((p.total_units + 7) / 8, grid_cap));
+    cudaError_t le = launch_move(kPack, pool->layout, p, (int)grid, stream);
+    if (le != cudaSuccess) return fail_cuda(le, "pack kernel launch");
+    int64_t soff = 0;
+    for (int q = 0; q < nb;) {
+      const int64_t i = batch[q].i;
+      uint8_t* h = (uint8_t*)host_chunks[i] + (int64_t)batch[q].l0 * layer_bytes(i);
+      int64_t len = 0;
+      int r = q;
+      while (r < nb && batch[r].i == i) len += batch[r++].bytes;  // one chunk = one allocation
+      cudaError_t ce = cudaMemcpyAsync(h, staging + soff, (size_t)len, cudaMemcpyDeviceToHost, stream);
+      if (ce != cudaSuccess) return fail_cuda(ce, "cudaMemcpyAsync staging -> host chunk");
+      soff += len;
+      q = r;
+    }
+    nb = 0;
+    used = 0;
+    return KVX_OK;
+  };
+  for (int64_t i = 0; i < n; ++i) {
+    const int64_t ls = layer_bytes(i);
+    int32_t l = 0;
+    while (l < pool->num_layers) {
+      const int64_t room = (KVX_NOALLOC_SCRATCH_BYTES - used) / ls;
+      if (room < 1 || nb == kMaxJobs) {
+        st = flush();
+        if (st != KVX_OK) return st;
+        continue;
+      }
+      const int32_t nl = (int32_t)std::min<int64_t>(room, pool->num_layers - l);
+      batch[nb++] = {i, l, nl, nl * ls};
+      used += nl * ls;
+      l += nl;
+    }
+  }
+  return flush();
+}

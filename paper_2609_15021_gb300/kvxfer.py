@@ -33,7 +33,7 @@ EXPORTED = (
     "kv_ctx_create", "kv_ctx_destroy", "kv_chunk_layout", "kv_store", "kv_load", "kv_pack", "kv_unpack",
     "kv_state_store", "kv_state_load", "kv_get_device_error", "kv_ctx_stats", "kv_ctx_reset_stats",
     "kv_ctx_modes", "kv_last_cuda_error", "kv_last_error_message", "kv_status_string", "kv_abi_version",
-    "kvx_probe_delayed_fill", "kvx_probe_delayed_copy", "kvx_probe_copy",
+    "kvx_probe_delayed_fill", "kvx_probe_delayed_copy", "kvx_probe_copy", "kv_store_noalloc",
 )
 
 
@@ -93,6 +93,7 @@ def _declare(lib):
         "kvx_probe_delayed_fill": (st, [vp, i64, i32, i64, vp]),
         "kvx_probe_delayed_copy": (st, [vp, vp, i64, i64, vp]),
         "kvx_probe_copy": (st, [vp, vp, i64, i32, vp]),
+        "kv_store_noalloc": (st, [P(kvx_pool), vp, i64, i64, i64, i32, P(vp), i64, vp, vp]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -119,6 +120,8 @@ def _check(status: int, where: str):
         msg = _lib.kv_status_string(status).decode()
         if status == KVX_ECUDA:
             msg += f" (cuda error {_lib.kv_last_cuda_error()}: {_lib.kv_last_error_message().decode()})"
+        elif _lib.kv_last_error_message():
+            msg += f" ({_lib.kv_last_error_message().decode()})"
         raise KvxError(status, where, msg)
 
 
@@ -228,6 +231,20 @@ def kv_unpack(ctx, pool: KvPool, block_table, tok_begin: int, tok_end: int, chun
               dev_chunks, stream=None, table_len: int | None = None) -> None:
     _transfer(_lib.kv_unpack, "kv_unpack", ctx, pool, block_table, tok_begin, tok_end, chunk_tokens,
               dev_chunks, stream, table_len)
+
+
+def kv_store_noalloc(pool: KvPool, block_table, tok_begin: int, tok_end: int, chunk_tokens: int,
+                     host_chunks, dev_first_bad_block=None, stream=None, table_len: int | None = None) -> None:
+    """kv_store for callers that cannot allocate: no context, static device staging (see kvxfer.h)."""
+    arr = _ptr_array(host_chunks)
+    n_tab = block_table.numel() if table_len is None else table_len
+    err = None if dev_first_bad_block is None else _ptr(dev_first_bad_block)
+    _check(_lib.kv_store_noalloc(ctypes.byref(pool.c), _ptr(block_table), n_tab, tok_begin, tok_end,
+                                 chunk_tokens, arr, len(host_chunks), err, _stream_handle(stream)),
+           "kv_store_noalloc")
+
+
+KVX_NOALLOC_SCRATCH_BYTES = 64 << 20
 
 
 def kv_state_store(ctx, layers, num_slots: int, slot_bytes: int, slot: int, host_obj, stream=None) -> None:
