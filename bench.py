@@ -36,6 +36,7 @@ if ROOT not in sys.path:
 METRIC = "KV store/load GB/s vs host-link & HBM peak; 128k-token context restore ms"
 SHAPE = dict(L=62, H=8, D=128, e=2, B=16, C=256)
 CONFIGS = {
+    "2k": dict(tokens=2048, pool_blocks=256),  # profiling size: 2 x 1 GB pools, 520 MB per direction
     "32k": dict(tokens=32768, pool_blocks=4096),
     "128k": dict(tokens=131072, pool_blocks=10240),
     "256k": dict(tokens=262144, pool_blocks=20480),
@@ -154,6 +155,8 @@ def parse():
     ap.add_argument("--cpu-sample-chunks", type=int, default=32)
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-hbm-roofline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
     return ap.parse_args()
 
 
@@ -367,25 +370,27 @@ def run_ours(args):
     value = 2 * X * args.steps * world / (total_ms_max * 1e-3) / GB
 
     # end to end through the public API on the host clock
-    ta_host = torch.from_numpy(ta_np).pin_memory()
-    tb_host = torch.from_numpy(tb_np).pin_memory()
-    torch.cuda.synchronize()
-    barrier(world)
-    t0 = time.perf_counter()
-    for _ in range(args.steps):
-        with torch.cuda.stream(stream):
-            ta.copy_(ta_host, non_blocking=True)
-            tb.copy_(tb_host, non_blocking=True)
-        k.kv_store(ctx, src, ta, 0, T, C, chunks, stream=stream)
-        stream.synchronize()          # the host may use the chunks only after this
-        k.kv_load(ctx, dst, tb, 0, T, C, chunks, stream=stream)
-        stream.synchronize()
-        bad = k.kv_get_device_error(ctx)  # device->host read of the step's status word
-        assert bad == -1
-    e2e_s = time.perf_counter() - t0
-    e2e_s = max_over_ranks(world, e2e_s, local)
-    e2e = {"value": 2 * X * args.steps * world / e2e_s / GB, "unit": "GB/s",
-           "h2d_bytes_per_step": X + ta_np.nbytes + tb_np.nbytes, "d2h_bytes_per_step": X + 8}
+    e2e = None
+    if not args.no_e2e:
+        ta_host = torch.from_numpy(ta_np).pin_memory()
+        tb_host = torch.from_numpy(tb_np).pin_memory()
+        torch.cuda.synchronize()
+        barrier(world)
+        t0 = time.perf_counter()
+        for _ in range(args.steps):
+            with torch.cuda.stream(stream):
+                ta.copy_(ta_host, non_blocking=True)
+                tb.copy_(tb_host, non_blocking=True)
+            k.kv_store(ctx, src, ta, 0, T, C, chunks, stream=stream)
+            stream.synchronize()          # the host may use the chunks only after this
+            k.kv_load(ctx, dst, tb, 0, T, C, chunks, stream=stream)
+            stream.synchronize()
+            bad = k.kv_get_device_error(ctx)  # device->host read of the step's status word
+            assert bad == -1
+        e2e_s = time.perf_counter() - t0
+        e2e_s = max_over_ranks(world, e2e_s, local)
+        e2e = {"value": 2 * X * args.steps * world / e2e_s / GB, "unit": "GB/s",
+               "h2d_bytes_per_step": X + ta_np.nbytes + tb_np.nbytes, "d2h_bytes_per_step": X + 8}
 
     # dominant kernel: the direction with more kernel time
     kern = {}
@@ -397,14 +402,59 @@ def run_ours(args):
             kern[name] = {"launches": nl, "avg_launch_ms": avg_ms, "bytes_per_launch": per_launch,
                           "total_ms": stats["kernel_ms"][d], "achieved_gbs": per_launch / (avg_ms * 1e-3) / GB}
     hbm_peak, peak_src = load_peaks()
+    traffic = recorded_traffic()
     roofline = None
     if kern:
         dom = max(kern, key=lambda n: kern[n]["total_ms"])
-        traffic = recorded_traffic()
-        roofline = {"bound": "hbm", "kernel": f"move_kernel<{dom},HND>", "achieved": kern[dom]["achieved_gbs"],
-                    "peak": hbm_peak, "unit": "GB/s", "frac": kern[dom]["achieved_gbs"] / hbm_peak,
-                    "traffic": traffic.get(dom) if traffic else None, "peak_source": peak_src,
-                    "algorithmic_bytes_per_launch": kern[dom]["bytes_per_launch"]}
+        zero_copy = (store_mode if dom == "pack" else load_mode) == k.KVX_MODE_ZEROCOPY
+        if zero_copy:
+            # the kernel moves each byte once over the host link: that link bounds it
+            link_bytes = kern[dom]["bytes_per_launch"] / 2
+            achieved = link_bytes / (kern[dom]["avg_launch_ms"] * 1e-3) / GB
+            peak = link["d2h" if dom == "pack" else "h2d"]
+            roofline = {"bound": "host_link", "kernel": f"move_kernel<{dom},HND> (zero-copy)", "achieved": achieved,
+                        "peak": peak, "unit": "GB/s", "frac": achieved / peak,
+                        "traffic": traffic.get(f"zerocopy_{dom}") if traffic else None,
+                        "peak_source": "pinned cudaMemcpyAsync of 1 GiB measured in this run (host link; "
+                                       "MEASURED_PEAKS.json has no host-link figure)",
+                        "algorithmic_bytes_per_launch": link_bytes}
+        else:
+            roofline = {"bound": "hbm", "kernel": f"move_kernel<{dom},HND> (staged)",
+                        "achieved": kern[dom]["achieved_gbs"], "peak": hbm_peak, "unit": "GB/s",
+                        "frac": kern[dom]["achieved_gbs"] / hbm_peak,
+                        "traffic": traffic.get(f"staged_{dom}") if traffic else None, "peak_source": peak_src,
+                        "algorithmic_bytes_per_launch": kern[dom]["bytes_per_launch"]}
+
+    # device-side pack / unpack of the same context into device chunks: the
+    # HBM-bound form of the kernels (staged mode, kv_pack / kv_unpack)
+    hbm_roofline = None
+    if not args.no_hbm_roofline:
+        dev_slab = torch.empty(n_chunks * cb, dtype=torch.uint8, device=dev)
+        dchunks = [dev_slab[i * cb:(i + 1) * cb] for i in range(n_chunks)]
+        hctx = k.kv_ctx_create(local, flags=k.KVX_FLAG_TIME_KERNELS)
+        for _ in range(2):
+            k.kv_pack(hctx, src, ta, 0, T, C, dchunks, stream=stream)
+            k.kv_unpack(hctx, dst, tb, 0, T, C, dchunks, stream=stream)
+        stream.synchronize()
+        k.kv_ctx_reset_stats(hctx)
+        for _ in range(3):
+            k.kv_pack(hctx, src, ta, 0, T, C, dchunks, stream=stream)
+            k.kv_unpack(hctx, dst, tb, 0, T, C, dchunks, stream=stream)
+        stream.synchronize()
+        hs = k.kv_ctx_stats(hctx)
+        assert k.kv_get_device_error(hctx) == -1
+        k.kv_ctx_destroy(hctx)
+        hbm_roofline = {"bound": "hbm", "peak": hbm_peak, "unit": "GB/s", "peak_source": peak_src}
+        for d, name in ((0, "pack"), (1, "unpack")):
+            nl = hs["timed_launches"][d]
+            per_launch = hs["kernel_bytes"][d] / nl
+            achieved = per_launch / (hs["kernel_ms"][d] / nl * 1e-3) / GB
+            hbm_roofline[name] = {"kernel": f"move_kernel<{name},HND> (device chunks)", "achieved": achieved,
+                                  "frac": achieved / hbm_peak, "launches": nl,
+                                  "algorithmic_bytes_per_launch": per_launch,
+                                  "avg_launch_ms": hs["kernel_ms"][d] / nl,
+                                  "traffic": traffic.get(f"device_{name}") if traffic else None}
+        del dev_slab, dchunks
 
     store_gbs = X / (statistics.median(store_ms) * 1e-3) / GB
     restore_gbs = X / (statistics.median(restore_ms) * 1e-3) / GB
@@ -451,6 +501,7 @@ def run_ours(args):
         "store_ms": {"median": statistics.median(store_ms), "min": min(store_ms), "max": max(store_ms)},
         "host_link": host_link,
         "roofline": roofline,
+        "hbm_roofline": hbm_roofline,
         "kernels": kern,
         "cpu_baseline": cpu,
         "verified_sample_vs_oracle": verified,

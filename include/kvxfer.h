@@ -69,7 +69,9 @@ typedef enum { KVX_LAYOUT_HND = 0, KVX_LAYOUT_NHD = 1 } kvx_layout;
 
 /* How host chunks are filled and read.  Both move exactly the same bytes. */
 typedef enum {
-  KVX_MODE_AUTO = 0,     /* library's measured default per direction          */
+  KVX_MODE_AUTO = 0,     /* library's measured default: ZEROCOPY both ways
+                            (GB300 + Grace: link peak every step; STAGED
+                            alternates between peak and ~25% slower steps)   */
   KVX_MODE_STAGED = 1,   /* pack into a device staging ring, then
                             cudaMemcpyAsync over the host link on a side stream,
                             pack of batch i+1 overlapping the copy of batch i  */
@@ -91,7 +93,12 @@ typedef struct {
   int32_t staging_slots;      /* staged ring depth (>= 2); 0 = 4                */
   int64_t staging_slot_bytes; /* bytes per slot; 0 = 32 MiB; a slot must hold
                                  one layer of one chunk                         */
-  int32_t max_ctas;           /* cap on CTAs per kernel launch; 0 = fill GPU    */
+  int32_t max_ctas;           /* cap on CTAs per kernel launch; 0 = default:
+                                 launches that read or write host memory
+                                 (zero-copy) use a quarter of the SMs, which
+                                 saturates the host link and leaves the rest to
+                                 the replica's compute; device-side launches
+                                 fill the GPU                                   */
   uint32_t flags;             /* KVX_FLAG_*                                     */
 } kvx_opts;
 
