@@ -326,9 +326,9 @@ def run_ours(args):
     ta = torch.from_numpy(ta_np).to(dev)
     tb = torch.from_numpy(tb_np).to(dev)
     t_pin = time.perf_counter()
-    slab = torch.empty(n_chunks * cb, dtype=torch.uint8).pin_memory()
+    host_pool = k.HostBuffer(n_chunks * cb)  # exact-size pinned, mapped pool (no power-of-two rounding)
     pin_seconds = time.perf_counter() - t_pin
-    chunks = [slab[i * cb:(i + 1) * cb] for i in range(n_chunks)]
+    chunks = [host_pool.tensor[i * cb:(i + 1) * cb] for i in range(n_chunks)]
 
     mode = {"auto": k.KVX_MODE_AUTO, "staged": k.KVX_MODE_STAGED, "zerocopy": k.KVX_MODE_ZEROCOPY}[args.mode]
     ctx = k.kv_ctx_create(local, store_mode=mode, load_mode=mode, staging_slot_bytes=args.slot_mib << 20,

@@ -254,6 +254,19 @@ kvx_status kv_store_noalloc(const kvx_pool* pool, const int32_t* block_table, in
                             int64_t n_chunks, int64_t* dev_first_bad_block, kvx_stream_t stream);
 
 /*
+ * Page-locked host memory for a shared chunk pool (Sec. 3.3: the shared tier
+ * is one full-size pinned allocation; the paper's 256 GiB + 4096 B request
+ * was rounded up to a power of two by the framework's pinned allocator and
+ * silently fell back to pageable memory).  kv_host_alloc allocates exactly
+ * `bytes` (no rounding), portable to every device and mapped for zero-copy,
+ * checks that the result is page-locked, and otherwise fails: KVX_ENOMEM when
+ * the memory is not available, never a pageable fallback.  Free with
+ * kv_host_free (NULL is ignored).
+ */
+kvx_status kv_host_alloc(int64_t bytes, void** out);
+void kv_host_free(void* host);
+
+/*
  * Lowest logical block index whose table entry was out of range in any call
  * completed since the last query, or -1.  Call after the caller's stream has
  * been synchronised.  Clears the record.

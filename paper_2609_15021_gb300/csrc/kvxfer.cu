@@ -846,6 +846,37 @@ kvx_status kv_state_load(kvx_ctx* ctx, int32_t num_layers, void* const* layer_ba
                     (cudaStream_t)stream, false);
 }
 
+kvx_status kv_host_alloc(int64_t bytes, void** out) {
+  if (!out) return KVX_EINVAL;
+  *out = nullptr;
+  if (bytes <= 0) return KVX_EINVAL;
+  void* p = nullptr;
+  // Exactly `bytes`, no rounding; portable and mapped so every context and
+  // the zero-copy kernels can use it.  No pageable fallback: a failure is an
+  // error (Sec. 3.3: a full-pool request that silently fell back to pageable
+  // memory).
+  cudaError_t e = cudaHostAlloc(&p, (size_t)bytes, cudaHostAllocPortable | cudaHostAllocMapped);
+  if (e != cudaSuccess) {
+    record_cuda_error((int)e, "cudaHostAlloc", __LINE__);
+    cudaGetLastError();
+    return e == cudaErrorMemoryAllocation ? KVX_ENOMEM : KVX_ECUDA;
+  }
+  uint8_t* mapped = nullptr;
+  if (check_pinned_range(p, bytes, &mapped) != KVX_OK) {
+    cudaFreeHost(p);
+    return KVX_ENOTPINNED;
+  }
+  *out = p;
+  return KVX_OK;
+}
+
+void kv_host_free(void* p) {
+  if (p) {
+    cudaFreeHost(p);
+    cudaGetLastError();
+  }
+}
+
 kvx_status kv_get_device_error(kvx_ctx* ctx, int64_t* first_bad_block) {
   if (!ctx || !first_bad_block) return KVX_EINVAL;
   DeviceGuard guard(ctx->device);

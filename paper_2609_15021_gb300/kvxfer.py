@@ -34,6 +34,7 @@ EXPORTED = (
     "kv_state_store", "kv_state_load", "kv_get_device_error", "kv_ctx_stats", "kv_ctx_reset_stats",
     "kv_ctx_modes", "kv_last_cuda_error", "kv_last_error_message", "kv_status_string", "kv_abi_version",
     "kvx_probe_delayed_fill", "kvx_probe_delayed_copy", "kvx_probe_copy", "kv_store_noalloc",
+    "kv_host_alloc", "kv_host_free",
 )
 
 
@@ -94,6 +95,8 @@ def _declare(lib):
         "kvx_probe_delayed_copy": (st, [vp, vp, i64, i64, vp]),
         "kvx_probe_copy": (st, [vp, vp, i64, i32, vp]),
         "kv_store_noalloc": (st, [P(kvx_pool), vp, i64, i64, i64, i32, P(vp), i64, vp, vp]),
+        "kv_host_alloc": (st, [i64, P(vp)]),
+        "kv_host_free": (None, [vp]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -245,6 +248,40 @@ def kv_store_noalloc(pool: KvPool, block_table, tok_begin: int, tok_end: int, ch
 
 
 KVX_NOALLOC_SCRATCH_BYTES = 64 << 20
+
+
+def kv_host_alloc(nbytes: int) -> int:
+    """Exact-size page-locked, mapped host allocation (raises, never falls back to pageable)."""
+    out = ctypes.c_void_p()
+    _check(_lib.kv_host_alloc(nbytes, ctypes.byref(out)), "kv_host_alloc")
+    return out.value
+
+
+def kv_host_free(ptr: int) -> None:
+    _lib.kv_host_free(ptr)
+
+
+class HostBuffer:
+    """A kv_host_alloc allocation with a uint8 CPU tensor view (``.tensor``) over it."""
+
+    def __init__(self, nbytes: int):
+        import torch
+        self.nbytes = nbytes
+        self.ptr = kv_host_alloc(nbytes)
+        raw = (ctypes.c_uint8 * nbytes).from_address(self.ptr)
+        self.tensor = torch.frombuffer(raw, dtype=torch.uint8, count=nbytes)
+
+    def close(self):
+        if self.ptr:
+            self.tensor = None
+            kv_host_free(self.ptr)
+            self.ptr = 0
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
 
 
 def kv_state_store(ctx, layers, num_slots: int, slot_bytes: int, slot: int, host_obj, stream=None) -> None:

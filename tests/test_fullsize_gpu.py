@@ -1,9 +1,18 @@
 """Full-size 27B-class workloads (62 layers, 8 KV heads, head_dim 128, bf16, 16-token
-pages, 256-token chunks) at 32k and 128k tokens, through the default context the
-benchmark uses: every chunk is hashed on the host, sampled chunks are compared
-with the oracle byte for byte, and sampled pages outside the load table must be
-untouched.  The oracle runs on a mini-pool of exactly the pages a sampled chunk
-reads (gathered from the device pool by PyTorch indexing)."""
+pages, 256-token chunks) at 32k, 128k and 256k tokens, through the default context
+the benchmark uses: sampled chunks are compared with the oracle byte for byte
+(and by SHA-256), restored pages with the oracle's restore, and sampled pages
+outside the load table must be untouched.  The oracle runs on a mini-pool of
+exactly the pages a sampled chunk reads (gathered from the device pool by
+PyTorch indexing).
+
+The 256k case also exercises the shared tier's full-pool pinned allocation
+(paper Sec. 3.3): the chunks live in one exact-size page-locked pool of the
+paper's 256 GiB + 4096 B when host memory allows, else the largest size that
+leaves 32 GiB of host memory free (recorded in the test output).
+"""
+import time
+
 import numpy as np
 import pytest
 import torch
@@ -15,9 +24,18 @@ from paper_2609_15021_gb300 import synth
 pytestmark = pytest.mark.gpu
 
 L, B, H, D, E, C = 62, 16, 8, 128, 2, 256
+PAPER_POOL_BYTES = 274_877_911_040  # 256 GiB + 4096 B (Sec. 3.3)
 
 
-@pytest.mark.parametrize("ctx_tokens,pool_blocks", [(32768, 4096), (131072, 10240)])
+def host_available() -> int:
+    with open("/proc/meminfo") as f:
+        for line in f:
+            if line.startswith("MemAvailable:"):
+                return int(line.split()[1]) * 1024
+    return 0
+
+
+@pytest.mark.parametrize("ctx_tokens,pool_blocks", [(32768, 4096), (131072, 10240), (262144, 20480)])
 def test_fullsize_store_restore_sampled(orc, ctx_tokens, pool_blocks):
     k = kvx()
     spec = oracle.PoolSpec(L, pool_blocks, B, H, D, E, oracle.HND)
@@ -25,46 +43,75 @@ def test_fullsize_store_restore_sampled(orc, ctx_tokens, pool_blocks):
     free, _ = torch.cuda.mem_get_info()
     if free < need + (4 << 30):
         pytest.skip(f"needs {need >> 30} GiB of device memory")
-    n_used = ctx_tokens // B
-    src_layers = [synth.normal_bf16_(torch.empty(spec.layer_bytes, dtype=torch.uint8, device="cuda"),
-                                     synth.SEED + l) for l in range(L)]
-    src = k.KvPool(src_layers, pool_blocks, B, H, D, E)
-    dst_layers = [torch.full((spec.layer_bytes,), POISON, dtype=torch.uint8, device="cuda") for _ in range(L)]
-    dst = k.KvPool(dst_layers, pool_blocks, B, H, D, E)
-    ta = synth.permuted_table(pool_blocks, n_used, seed=1)
-    tb = synth.permuted_table(pool_blocks, n_used, seed=2)
     n_chunks = ctx_tokens // C
     cb = orc.chunk_bytes(spec, C)
-    slab = torch.empty(n_chunks * cb, dtype=torch.uint8).pin_memory()
-    chunks = [slab[i * cb:(i + 1) * cb] for i in range(n_chunks)]
-    ctx = k.kv_ctx_create(0)
+    pool_bytes = n_chunks * cb
+    if ctx_tokens == 262144:  # the shared-tier budget
+        pool_bytes = max(pool_bytes, min(PAPER_POOL_BYTES, host_available() - (32 << 30)))
+    if pool_bytes < n_chunks * cb or host_available() < pool_bytes + (16 << 30):
+        pytest.skip("not enough host memory for the chunk pool")
+    t_pin = time.perf_counter()
+    host_pool = k.HostBuffer(pool_bytes)
+    pin_s = time.perf_counter() - t_pin
+    print(f"\npinned host pool: {pool_bytes} bytes in {pin_s:.2f} s "
+          f"({'chunks only' if ctx_tokens != 262144 else 'paper size' if pool_bytes == PAPER_POOL_BYTES else 'largest feasible budget'})")
     try:
-        stream = torch.cuda.Stream()
-        with torch.cuda.stream(stream):
-            k.kv_store(ctx, src, torch.from_numpy(ta).cuda(), 0, ctx_tokens, C, chunks)
-            k.kv_load(ctx, dst, torch.from_numpy(tb).cuda(), 0, ctx_tokens, C, chunks)
-        stream.synchronize()
-        assert k.kv_get_device_error(ctx) == -1
+        chunks = [host_pool.tensor[i * cb:(i + 1) * cb] for i in range(n_chunks)]
+        src_layers = [synth.normal_bf16_(torch.empty(spec.layer_bytes, dtype=torch.uint8, device="cuda"),
+                                         synth.SEED + l) for l in range(L)]
+        src = k.KvPool(src_layers, pool_blocks, B, H, D, E)
+        dst_layers = [torch.full((spec.layer_bytes,), POISON, dtype=torch.uint8, device="cuda") for _ in range(L)]
+        dst = k.KvPool(dst_layers, pool_blocks, B, H, D, E)
+        ta = synth.permuted_table(pool_blocks, ctx_tokens // B, seed=1)
+        tb = synth.permuted_table(pool_blocks, ctx_tokens // B, seed=2)
+        ctx = k.kv_ctx_create(0)
+        try:
+            stream = torch.cuda.Stream()
+            with torch.cuda.stream(stream):
+                k.kv_store(ctx, src, torch.from_numpy(ta).cuda(), 0, ctx_tokens, C, chunks)
+                k.kv_load(ctx, dst, torch.from_numpy(tb).cuda(), 0, ctx_tokens, C, chunks)
+            stream.synchronize()
+            assert k.kv_get_device_error(ctx) == -1
+        finally:
+            k.kv_ctx_destroy(ctx)
+        bpc = C // B
+        r = synth.rng(ctx_tokens)
+        sample = sorted({0, 1, n_chunks // 2, n_chunks - 1, *map(int, r.integers(0, n_chunks, 3))})
+        mini = oracle.PoolSpec(L, bpc, B, H, D, E, oracle.HND)
+        ident = np.arange(bpc, dtype=np.int32)
+        for c in sample:
+            pool_np = [gather_pages(t, spec.page_bytes, ta[c * bpc:(c + 1) * bpc]) for t in src_layers]
+            want = [np.full(cb, POISON, np.uint8)]
+            assert orc.store(mini, pool_np, ident, 0, C, C, want, n_threads=8)[0] == 0
+            got = np_of(chunks[c])
+            assert sha(got) == sha(want[0]), (c, first_mismatch(got, want[0]))
+            loaded = [np.full(mini.layer_bytes, POISON, np.uint8) for _ in range(L)]
+            assert orc.load(mini, loaded, ident, 0, C, C, want, n_threads=8)[0] == 0
+            for l in (0, 1, L // 2, L - 1):
+                got_pages = gather_pages(dst_layers[l], spec.page_bytes, tb[c * bpc:(c + 1) * bpc])
+                assert first_mismatch(got_pages, loaded[l]) is None, (c, l)
+        unused = np.setdiff1d(np.arange(pool_blocks), tb)
+        probe = synth.rng(7).choice(unused, size=min(8, unused.size), replace=False)
+        for l in (0, L - 1):
+            assert np.all(gather_pages(dst_layers[l], spec.page_bytes, probe) == POISON)
+        del src_layers, dst_layers, src, dst, chunks
+        torch.cuda.empty_cache()
     finally:
-        k.kv_ctx_destroy(ctx)
-    bpc = C // B
-    r = synth.rng(ctx_tokens)
-    sample = sorted({0, 1, n_chunks // 2, n_chunks - 1, *map(int, r.integers(0, n_chunks, 3))})
-    mini = oracle.PoolSpec(L, bpc, B, H, D, E, oracle.HND)
-    ident = np.arange(bpc, dtype=np.int32)
-    for c in sample:
-        pages_a = ta[c * bpc:(c + 1) * bpc]
-        pool_np = [gather_pages(t, spec.page_bytes, pages_a) for t in src_layers]
-        want = [np.full(cb, POISON, np.uint8)]
-        assert orc.store(mini, pool_np, ident, 0, C, C, want, n_threads=8)[0] == 0
-        got = np_of(chunks[c])
-        assert sha(got) == sha(want[0]), (c, first_mismatch(got, want[0]))
-        pages_b = tb[c * bpc:(c + 1) * bpc]
-        loaded = [np.full(mini.layer_bytes, POISON, np.uint8) for _ in range(L)]
-        assert orc.load(mini, loaded, ident, 0, C, C, want, n_threads=8)[0] == 0
-        for l in (0, 1, L // 2, L - 1):
-            assert first_mismatch(gather_pages(dst_layers[l], spec.page_bytes, pages_b), loaded[l]) is None, (c, l)
-    unused = np.setdiff1d(np.arange(pool_blocks), tb)
-    probe = synth.rng(7).choice(unused, size=min(8, unused.size), replace=False)
-    for l in (0, L - 1):
-        assert np.all(gather_pages(dst_layers[l], spec.page_bytes, probe) == POISON)
+        host_pool.close()
+
+
+def test_host_alloc_exact_and_pinned():
+    """kv_host_alloc returns exactly the requested, page-locked, mapped size (no rounding)."""
+    k = kvx()
+    n = (1 << 30) + 4096  # a size a power-of-two rounding allocator would double
+    buf = k.HostBuffer(n)
+    try:
+        assert buf.tensor.numel() == n
+        buf.tensor[-1] = 7
+        assert int(buf.tensor[-1]) == 7
+        d = torch.zeros(4096, dtype=torch.uint8, device="cuda")
+        d.copy_(buf.tensor[-4096:], non_blocking=True)
+        torch.cuda.synchronize()
+        assert int(d[-1]) == 7
+    finally:
+        buf.close()
