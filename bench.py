@@ -34,26 +34,33 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 METRIC = "KV store/load GB/s vs host-link & HBM peak; 128k-token context restore ms"
-SHAPE = dict(L=62, H=8, D=128, e=2, B=16, C=256)
+# 27B-class attention KV of the benchmark configurations
+SHAPE_27B = dict(L=62, H=8, D=128, e=2, B=16, C=256, name="27B-class paged KV (62 layers x 8 KV heads x "
+                 "head_dim 128, bf16, 16-token pages)", dtype="bf16")
+# the paper's own attention KV (Table 1, Sec. 3.1): 16 full-attention layers x 4 KV heads x
+# head_dim 256 in FP8, 32-token kernel pages, 1,568-token chunks of 49 pages
+SHAPE_PAPER = dict(L=16, H=4, D=256, e=1, B=32, C=1568, name="the paper's FP8 attention KV (16 layers x 4 KV "
+                   "heads x head_dim 256, 1 byte, 32-token pages)", dtype="fp8 bytes")
 CONFIGS = {
-    "2k": dict(tokens=2048, pool_blocks=256),  # profiling size: 2 x 1 GB pools, 520 MB per direction
-    "32k": dict(tokens=32768, pool_blocks=4096),
-    "128k": dict(tokens=131072, pool_blocks=10240),
-    "256k": dict(tokens=262144, pool_blocks=20480),
+    "2k": dict(tokens=2048, pool_blocks=256, shape=SHAPE_27B),  # profiling size: 2 x 1 GB pools
+    "32k": dict(tokens=32768, pool_blocks=4096, shape=SHAPE_27B),
+    "128k": dict(tokens=131072, pool_blocks=10240, shape=SHAPE_27B),
+    "256k": dict(tokens=262144, pool_blocks=20480, shape=SHAPE_27B),
+    # the paper's 128k cross-replica hit: 127,008 tokens = 81 chunks (Sec. 3.2)
+    "paper127k": dict(tokens=127008, pool_blocks=16384, shape=SHAPE_PAPER),
 }
 FALLBACK_HBM_GBS = 6800.0
 GB = 1e9
 
 
 def workload_name(cfg):
-    t, n = cfg["tokens"], cfg["pool_blocks"]
-    return (f"27B-class paged KV (62 layers x 8 KV heads x head_dim 128, bf16, 16-token pages), "
-            f"{t // 1024}k-token context = {t // 16} of {n} pages by seeded permutation, 256-token chunks: "
-            f"full store to pinned host chunks, then restore into a cold pool")
+    t, n, s = cfg["tokens"], cfg["pool_blocks"], cfg["shape"]
+    return (f"{s['name']}, {t}-token context = {t // s['B']} of {n} pages by seeded permutation, "
+            f"{s['C']}-token chunks: full store to pinned host chunks, then restore into a cold pool")
 
 
 def bytes_per_direction(cfg):
-    s = SHAPE
+    s = cfg["shape"]
     return cfg["tokens"] * s["L"] * 2 * s["H"] * s["D"] * s["e"]
 
 
@@ -73,8 +80,27 @@ def kernel_source_hash():
         return hashlib.sha256(f.read()).hexdigest()[:16]
 
 
-def recorded_traffic():
-    """Per-launch DRAM bytes from a committed ncu summary, if taken on this kernel source."""
+def shape_key(s):
+    return f"L{s['L']} H{s['H']} D{s['D']} e{s['e']} B{s['B']} C{s['C']}"
+
+
+class Traffic:
+    """DRAM bytes per launch from a committed ncu capture of this kernel source and
+    shape, scaled to a launch of a given size by its algorithmic bytes (the capture
+    is taken on a smaller launch of the same kernel)."""
+
+    def __init__(self, record):
+        self.captured = record["captured"] if record else {}
+
+    def get(self, name, alg_bytes):
+        if name not in self.captured:
+            return None
+        traffic, captured_alg = self.captured[name]
+        return traffic * alg_bytes / captured_alg
+
+
+def recorded_traffic(shape):
+    """Traffic record from profiles/ for this kernel source and KV shape, else None."""
     pdir = os.path.join(ROOT, "profiles")
     want = kernel_source_hash()
     if not os.path.isdir(pdir):
@@ -87,9 +113,9 @@ def recorded_traffic():
                 m = re.match(r"\s*bench-traffic:\s*(\{.*\})\s*$", line)
                 if m:
                     d = json.loads(m.group(1))
-                    if d.get("kernel_sha256") == want:
-                        return d
-    return None
+                    if d.get("kernel_sha256") == want and d.get("shape") == shape_key(shape):
+                        return Traffic(d)
+    return Traffic(None)
 
 
 class ClockSampler:
@@ -200,7 +226,7 @@ def oracle_sample(cfg, n_chunks_sample, pool_pages_np=None):
 
     import oracle
     from paper_2609_15021_gb300 import synth
-    s = SHAPE
+    s = cfg["shape"]
     bpc = s["C"] // s["B"]
     spec = oracle.PoolSpec(s["L"], n_chunks_sample * bpc, s["B"], s["H"], s["D"], s["e"], oracle.HND)
     if pool_pages_np is None:
@@ -209,13 +235,12 @@ def oracle_sample(cfg, n_chunks_sample, pool_pages_np=None):
     return spec, pool_pages_np, ident
 
 
-def time_oracle(spec, layers, ident, n_chunks_sample, min_seconds, threads):
+def time_oracle(spec, layers, ident, n_chunks_sample, min_seconds, threads, C):
     """Store then load of the sample, repeated until min_seconds have passed."""
     import numpy as np
 
     import oracle
     orc = oracle.c_oracle()
-    C = SHAPE["C"]
     t1 = n_chunks_sample * C
     cb = orc.chunk_bytes(spec, C)
     chunks = [np.empty(cb, np.uint8) for _ in range(n_chunks_sample)]
@@ -247,12 +272,12 @@ def run_reference(args):
     moved = None
     for i in range(args.warmup + args.steps):
         t0 = time.perf_counter()
-        reps, el, _, moved = time_oracle(spec, layers, ident, S, 0.0, threads)
+        reps, el, _, moved = time_oracle(spec, layers, ident, S, 0.0, threads, cfg["shape"]["C"])
         if i >= args.warmup:
             step_times.append(time.perf_counter() - t0)
     total = sum(step_times)
     value = moved * len(step_times) / total / GB
-    sample = (f"{S} of {cfg['tokens'] // SHAPE['C']} chunks of the workload per step "
+    sample = (f"{S} of {cfg['tokens'] // cfg['shape']['C']} chunks of the workload per step "
               f"({moved // 2} bytes per direction), store then load, {threads} threads")
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world,
@@ -305,13 +330,13 @@ def run_ours(args):
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
     cfg = CONFIGS[args.config]
-    s = SHAPE
+    s = cfg["shape"]
     L, B, H, D, e, C = s["L"], s["B"], s["H"], s["D"], s["e"], s["C"]
     N, T = cfg["pool_blocks"], cfg["tokens"]
     page = 2 * H * B * D * e
     layer_bytes = N * page
     X = bytes_per_direction(cfg)
-    n_chunks = T // C
+    n_chunks = -(-T // C)
     cb = L * 2 * C * H * D * e
 
     link = host_link_peak(torch, dev)
@@ -402,7 +427,7 @@ def run_ours(args):
             kern[name] = {"launches": nl, "avg_launch_ms": avg_ms, "bytes_per_launch": per_launch,
                           "total_ms": stats["kernel_ms"][d], "achieved_gbs": per_launch / (avg_ms * 1e-3) / GB}
     hbm_peak, peak_src = load_peaks()
-    traffic = recorded_traffic()
+    traffic = recorded_traffic(s)
     roofline = None
     if kern:
         dom = max(kern, key=lambda n: kern[n]["total_ms"])
@@ -414,7 +439,7 @@ def run_ours(args):
             peak = link["d2h" if dom == "pack" else "h2d"]
             roofline = {"bound": "host_link", "kernel": f"move_kernel<{dom},HND> (zero-copy)", "achieved": achieved,
                         "peak": peak, "unit": "GB/s", "frac": achieved / peak,
-                        "traffic": traffic.get(f"zerocopy_{dom}") if traffic else None,
+                        "traffic": traffic.get(f"zerocopy_{dom}", link_bytes),
                         "peak_source": "pinned cudaMemcpyAsync of 1 GiB measured in this run (host link; "
                                        "MEASURED_PEAKS.json has no host-link figure)",
                         "algorithmic_bytes_per_launch": link_bytes}
@@ -422,7 +447,7 @@ def run_ours(args):
             roofline = {"bound": "hbm", "kernel": f"move_kernel<{dom},HND> (staged)",
                         "achieved": kern[dom]["achieved_gbs"], "peak": hbm_peak, "unit": "GB/s",
                         "frac": kern[dom]["achieved_gbs"] / hbm_peak,
-                        "traffic": traffic.get(f"staged_{dom}") if traffic else None, "peak_source": peak_src,
+                        "traffic": traffic.get(f"staged_{dom}", kern[dom]["bytes_per_launch"]), "peak_source": peak_src,
                         "algorithmic_bytes_per_launch": kern[dom]["bytes_per_launch"]}
 
     # device-side pack / unpack of the same context into device chunks: the
@@ -453,7 +478,7 @@ def run_ours(args):
                                   "frac": achieved / hbm_peak, "launches": nl,
                                   "algorithmic_bytes_per_launch": per_launch,
                                   "avg_launch_ms": hs["kernel_ms"][d] / nl,
-                                  "traffic": traffic.get(f"device_{name}") if traffic else None}
+                                  "traffic": traffic.get(f"device_{name}", per_launch)}
         del dev_slab, dchunks
 
     store_gbs = X / (statistics.median(store_ms) * 1e-3) / GB
@@ -476,7 +501,7 @@ def run_ours(args):
         pool_np = [t.view(-1, page).index_select(0, idx).cpu().numpy().reshape(-1) for t in src_layers]
         spec, layers_np, ident = oracle_sample(cfg, S, pool_np)
         threads = os.cpu_count() or 1
-        reps, el, want, moved = time_oracle(spec, layers_np, ident, S, args.cpu_seconds, threads)
+        reps, el, want, moved = time_oracle(spec, layers_np, ident, S, args.cpu_seconds, threads, C)
         cpu = {"value": moved * reps / el / GB, "unit": "GB/s", "cores": min(threads, S), "kind": "oracle",
                "sample": f"{S} of {n_chunks} chunks (evenly spaced), store then load, repeated {reps}x "
                          f"in {el:.1f} s on {threads} host threads"}
@@ -491,7 +516,7 @@ def run_ours(args):
         "scaling": "weak", "vs_baseline": None, "dtype": "u8",
         "data": "synthetic: bf16 ~N(0,1) KV from a fixed seed; seeded random-permutation block tables",
         "config": {"workload": workload_name(cfg), "context_tokens": T, "layers": L, "kv_heads": H,
-                   "head_dim": D, "kv_dtype": "bf16", "block_tokens": B, "chunk_tokens": C, "pool_blocks": N,
+                   "head_dim": D, "kv_dtype": s["dtype"], "block_tokens": B, "chunk_tokens": C, "pool_blocks": N,
                    "bytes_per_direction": X, "l2": f"inputs larger than L2 ({X} bytes per direction), no flush",
                    "store_mode": k.MODE_NAMES[store_mode], "load_mode": k.MODE_NAMES[load_mode],
                    "parallelism": f"replicas x{world}", "pinned_host_bytes": n_chunks * cb,
