@@ -50,6 +50,7 @@ class PoolSpec:
     head_dim: int
     elem_bytes: int
     layout: int = HND
+    pages_per_block: int = 1  # pages per logical block named by the table
 
     @property
     def row_bytes(self) -> int:
@@ -73,6 +74,7 @@ class _OrPool(ctypes.Structure):
         ("head_dim", ctypes.c_int32),
         ("elem_bytes", ctypes.c_int32),
         ("layout", ctypes.c_int32),
+        ("pages_per_block", ctypes.c_int32),
     ]
 
 
@@ -109,7 +111,7 @@ class COracle:
     @staticmethod
     def _pool(spec: PoolSpec) -> _OrPool:
         return _OrPool(spec.num_layers, spec.num_blocks, spec.block_tokens, spec.num_heads,
-                       spec.head_dim, spec.elem_bytes, spec.layout)
+                       spec.head_dim, spec.elem_bytes, spec.layout, spec.pages_per_block)
 
     @staticmethod
     def _ptrs(arrays) -> ctypes.Array:

@@ -17,7 +17,11 @@
  *       NHD: [block_tokens][num_heads][row]
  *   where a row is head_dim * elem_bytes bytes (one head vector of one token).
  *
- *   token t lives in page p = table[t / B] at slot s = t % B.
+ *   The block table names logical blocks of P = pages_per_block packed
+ *   pages (Sec. 3.1: a 1,568-token logical block spans 49 pages of 32
+ *   tokens); logical block b holds pages b*P .. b*P + P-1 of the pool.
+ *   Token t lies in kernel page k = t / B at slot s = t % B; its page is
+ *       p = table[k / P] * P + k % P          (P = 1: p = table[t / B]).
  *
  *   chunk c covers tokens [c*C, min((c+1)*C, t_end)); it is laid out
  *       [layer][kv][u][head][row],  u = t - c*C,  T_c tokens per chunk,
@@ -60,7 +64,10 @@ typedef struct {
   int32_t head_dim;     /* D */
   int32_t elem_bytes;   /* e */
   int32_t layout;       /* OR_HND or OR_NHD */
+  int32_t pages_per_block; /* P: pages per logical block of the table (0 means 1) */
 } or_pool;
+
+static int64_t ppb_of(const or_pool* P) { return P->pages_per_block > 1 ? P->pages_per_block : 1; }
 
 static int64_t row_bytes(const or_pool* P) { return (int64_t)P->head_dim * P->elem_bytes; }
 
@@ -85,10 +92,12 @@ static int check_args(const or_pool* P, int64_t table_len, int64_t t_begin, int6
       P->head_dim < 1 || P->elem_bytes < 1 || (P->layout != OR_HND && P->layout != OR_NHD) ||
       C < 1 || table_len < 0 || n_chunks < 0)
     return OR_EINVAL;
+  if (P->pages_per_block < 0) return OR_EINVAL;
+  if (P->num_blocks % ppb_of(P) != 0) return OR_EALIGN;
   if (t_begin < 0 || t_end < t_begin) return OR_ERANGE;
   if (C % P->block_tokens != 0) return OR_EALIGN;
   if (t_begin % C != 0) return OR_EALIGN;
-  if (t_end > table_len * (int64_t)P->block_tokens) return OR_ERANGE;
+  if (t_end > table_len * ppb_of(P) * (int64_t)P->block_tokens) return OR_ERANGE;
   {
     int64_t first = t_begin / C;
     int64_t last = (t_end + C - 1) / C; /* one past the last chunk */
@@ -112,7 +121,7 @@ typedef struct {
 static void* run_job(void* arg) {
   or_job* J = (or_job*)arg;
   const or_pool* P = J->P;
-  int64_t B = P->block_tokens, C = J->C, row = row_bytes(P);
+  int64_t B = P->block_tokens, C = J->C, row = row_bytes(P), ppb = ppb_of(P);
   int64_t c0 = J->t_begin / C;
   for (int64_t i = J->c_lo; i < J->c_hi; ++i) {
     int64_t c = c0 + i;
@@ -123,10 +132,12 @@ static void* run_job(void* arg) {
       for (int64_t kv = 0; kv < 2; ++kv)
         for (int64_t u = 0; u < T_c; ++u) {
           int64_t t = first + u;
-          int64_t blk = t / B;
+          int64_t kpage = t / B;            /* kernel page of the token */
+          int64_t blk = kpage / ppb;        /* logical block in the table */
           int64_t s = t % B;
-          int64_t p = J->table[blk];
-          if (p < 0 || p >= P->num_blocks) {
+          int64_t entry = J->table[blk];
+          int64_t p = entry * ppb + kpage % ppb;
+          if (entry < 0 || entry >= P->num_blocks / ppb) {
             if (J->bad < 0 || blk < J->bad) J->bad = blk;
             if (J->to_chunk) /* the token's rows of this (layer, kv) read as zeros */
               memset(chunk + chunk_row(P, T_c, l, kv, u, 0), 0, (size_t)(P->num_heads * row));

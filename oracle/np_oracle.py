@@ -25,9 +25,13 @@ def _view(layer: np.ndarray, spec) -> np.ndarray:
     return layer.reshape(shape)
 
 
-def _token_coords(table, t_begin, t_end, block_tokens):
+def _token_coords(table, t_begin, t_end, block_tokens, pages_per_block=1):
+    """Page and slot of every token: the table names logical blocks of
+    pages_per_block consecutive pages (Sec. 3.1's packed sub-pages)."""
     t = np.arange(t_begin, t_end, dtype=np.int64)
-    pages = np.asarray(table, dtype=np.int64)[t // block_tokens]
+    kernel_page = t // block_tokens
+    logical = np.asarray(table, dtype=np.int64)[kernel_page // pages_per_block]
+    pages = logical * pages_per_block + kernel_page % pages_per_block
     slots = t % block_tokens
     return pages, slots
 
@@ -47,7 +51,7 @@ def _gather_layer(view, spec, pages, slots) -> np.ndarray:
 
 def np_store(spec, layers, table, t_begin, t_end, chunk_tokens):
     """Return the list of packed chunks (uint8 arrays) for tokens [t_begin, t_end)."""
-    pages, slots = _token_coords(table, t_begin, t_end, spec.block_tokens)
+    pages, slots = _token_coords(table, t_begin, t_end, spec.block_tokens, max(1, spec.pages_per_block))
     per_layer = [_gather_layer(_view(layers[l], spec), spec, pages, slots)
                  for l in range(spec.num_layers)]
     allk = np.stack(per_layer)                # [L][kv][T][H][row]
@@ -63,7 +67,7 @@ def np_store(spec, layers, table, t_begin, t_end, chunk_tokens):
 
 def np_load(spec, layers, table, t_begin, t_end, chunk_tokens, chunks):
     """Scatter ``chunks`` into copies of ``layers``; returns the new layers."""
-    pages, slots = _token_coords(table, t_begin, t_end, spec.block_tokens)
+    pages, slots = _token_coords(table, t_begin, t_end, spec.block_tokens, max(1, spec.pages_per_block))
     H, R, L = spec.num_heads, spec.row_bytes, spec.num_layers
     parts = []
     start, i = t_begin, 0

@@ -311,7 +311,47 @@ def pin_state_copy(orc):
     assert orc.state_copy(dest, sb, 5, obj, False) == oracle.ERANGE
 
 
+def pin_logical_block_nhd_identity(orc):
+    """Logical blocks of P packed pages (Sec. 3.1: 49 pages of 32 tokens per 1,568-token
+    block), NHD, identity table, chunk = one logical block: the chunk is the block's P
+    pages with the page axis moved inside the K/V axis (np.transpose of [P][2][rest])."""
+    for P in (2, 3):
+        spec = PoolSpec(1, 4 * P, 4, 3, 8, 2, NHD, P)
+        layers = make_layers(spec, 61 + P)
+        C = P * spec.block_tokens
+        chunks = do_store(orc, spec, layers, np.arange(4, dtype=np.int32), 0, 4 * C, C)
+        lb_bytes = P * spec.page_bytes
+        for c, ch in enumerate(chunks):
+            block = layers[0][c * lb_bytes:(c + 1) * lb_bytes].reshape(P, 2, -1)
+            assert np.array_equal(ch, np.transpose(block, (1, 0, 2)).reshape(-1)), (P, c)
+
+
+def pin_logical_block_table_is_take(orc):
+    """Through logical blocks, the table acts as np.take over [blocks][P pages]."""
+    for layout in (HND, NHD):
+        P = 3
+        spec = PoolSpec(2, 6 * P, 4, 2, 8, 2, layout, P)
+        layers = make_layers(spec, 67)
+        table = synth.permuted_table(6, 5, seed=8)
+        C = 2 * spec.block_tokens  # chunks that end inside a logical block
+        t1 = 5 * P * spec.block_tokens - 5
+        got = do_store(orc, spec, layers, table, 0, t1, C)
+        taken = [np.take(l.reshape(6, P * spec.page_bytes), table, axis=0).reshape(-1) for l in layers]
+        spec5 = PoolSpec(2, 5 * P, 4, 2, 8, 2, layout, P)
+        want = do_store(orc, spec5, taken, np.arange(5, dtype=np.int32), 0, t1, C)
+        for a, b in zip(got, want):
+            assert np.array_equal(a, b), layout
+        # a table of logical blocks covers P pages per entry, no more
+        ch = poisoned_chunks(orc, spec, 0, 6 * P * 4, C)  # full-size chunks, more than enough
+        assert orc.store(spec, layers, table, 0, 5 * P * 4, C, ch)[0] == oracle.OK
+        assert orc.store(spec, layers, table, 0, 5 * P * 4 + 1, C, ch)[0] == oracle.ERANGE
+        bad = PoolSpec(2, 6 * P + 1, 4, 2, 8, 2, layout, P)  # pool not a whole number of blocks
+        assert orc.store(bad, [np.zeros(bad.layer_bytes, np.uint8)] * 2, table, 0, 8, C, ch)[0] == oracle.EALIGN
+
+
 PINS = [
+    pin_logical_block_nhd_identity,
+    pin_logical_block_table_is_take,
     pin_nhd_identity_is_page_bytes,
     pin_hnd_identity_is_transpose,
     pin_table_is_take,

@@ -28,14 +28,20 @@ MUTATIONS = {
     "chunk_kv_dropped": ("(((l * 2 + kv) * T_c + u) * H + h)", "(((l * 2 + 0) * T_c + u) * H + h)"),
     "chunk_token_head_transposed": ("(((l * 2 + kv) * T_c + u) * H + h)", "(((l * 2 + kv) * H + h) * T_c + u)"),
     "chunk_padded_tail": ("chunk_row(P, T_c, l, kv, u, h)", "chunk_row(P, C, l, kv, u, h)"),
-    "block_from_local_token": ("int64_t blk = t / B;", "int64_t blk = u / B;"),
+    "block_from_local_token": ("int64_t kpage = t / B;", "int64_t kpage = u / B;"),
     "tail_length_ignored": ("int64_t T_c = (J->t_end - first < C) ? (J->t_end - first) : C;", "int64_t T_c = C;"),
     "load_copies_backwards": ("memcpy(p_ptr, c_ptr, (size_t)row);", "memcpy(c_ptr, p_ptr, (size_t)row);"),
     "chunk_index_ignores_start": ("int64_t c = c0 + i;", "int64_t c = i;"),
-    "capacity_off_by_one": ("if (t_end > table_len * (int64_t)P->block_tokens) return OR_ERANGE;",
-                            "if (t_end >= table_len * (int64_t)P->block_tokens) return OR_ERANGE;"),
+    "capacity_off_by_one": ("if (t_end > table_len * ppb_of(P) * (int64_t)P->block_tokens) return OR_ERANGE;",
+                            "if (t_end >= table_len * ppb_of(P) * (int64_t)P->block_tokens) return OR_ERANGE;"),
+    "capacity_ignores_logical_blocks": ("if (t_end > table_len * ppb_of(P) * (int64_t)P->block_tokens)",
+                                        "if (t_end > table_len * (int64_t)P->block_tokens)"),
     "start_alignment_unchecked": ("if (t_begin % C != 0) return OR_EALIGN;", ""),
-    "page_bound_off_by_one": ("if (p < 0 || p >= P->num_blocks) {", "if (p < 0 || p > P->num_blocks) {"),
+    "page_bound_off_by_one": ("if (entry < 0 || entry >= P->num_blocks / ppb) {",
+                              "if (entry < 0 || entry > P->num_blocks / ppb) {"),
+    "logical_block_not_scaled": ("int64_t p = entry * ppb + kpage % ppb;", "int64_t p = entry + kpage % ppb;"),
+    "subpage_dropped": ("int64_t p = entry * ppb + kpage % ppb;", "int64_t p = entry * ppb;"),
+    "subpage_from_slot": ("int64_t p = entry * ppb + kpage % ppb;", "int64_t p = entry * ppb + s % ppb;"),
     "row_ignores_elem_bytes": ("return (int64_t)P->head_dim * P->elem_bytes;", "return (int64_t)P->head_dim;"),
     "state_slot_offset_dropped": ("uint8_t* s = layers[l] + slot * slot_bytes;", "uint8_t* s = layers[l] + slot_bytes;"),
 }
