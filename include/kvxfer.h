@@ -15,8 +15,9 @@
  * Data layout (all sizes in bytes unless stated; row = head_dim * elem_bytes):
  *   pool layer l   : num_blocks pages, page = [2 (K,V)][H][B][row] for
  *                    KVX_LAYOUT_HND, [2][B][H][row] for KVX_LAYOUT_NHD.
- *   block table    : int32 device array; entry i = page of logical block i,
- *                    i.e. of tokens [i*B, (i+1)*B).
+ *   block table    : int32 device array; entry i names logical block i, i.e.
+ *                    the pages of tokens [i*P*B, (i+1)*P*B) (P =
+ *                    kvx_pool.pages_per_block, 1 unless pages are packed).
  *   chunk c        : tokens [c*C, min((c+1)*C, tok_end)), packed densely as
  *                    [layer][2 (K,V)][token][head][row]; a short last chunk
  *                    holds fewer tokens and is not padded.  The layout does
@@ -48,7 +49,7 @@
 extern "C" {
 #endif
 
-#define KVX_ABI_VERSION 1
+#define KVX_ABI_VERSION 2
 #define KVX_MAX_LAYERS 128 /* layers per pool description */
 
 /* Same handle as cudaStream_t; NULL is the legacy default stream. */
@@ -113,6 +114,13 @@ typedef struct {
   int32_t head_dim;          /* D: elements per head vector                    */
   int32_t elem_bytes;        /* e: bytes per element (bf16 = 2, fp8 = 1, ...)  */
   int32_t layout;            /* kvx_layout                                     */
+  int32_t pages_per_block;   /* P: pages per logical block named by the block
+                                table (0 or 1: the table names pages).  Sec.
+                                3.1: a 1,568-token logical block packs 49 pages
+                                of 32 tokens; logical block b is pages
+                                b*P .. b*P+P-1, so token t lies in page
+                                table[(t/B)/P]*P + (t/B)%P.  num_blocks (pages)
+                                must be a multiple of P.                        */
 } kvx_pool;
 
 /* Byte geometry of one packed chunk holding tokens_in_chunk tokens. */
@@ -159,6 +167,25 @@ void kv_ctx_destroy(kvx_ctx* ctx);
  */
 kvx_status kv_chunk_layout(const kvx_pool* pool, int32_t chunk_tokens, int32_t tokens_in_chunk,
                            kvx_chunk_layout* out);
+
+/*
+ * Check that a framework's view of one pool layer -- its shape and byte
+ * strides, outermost dimension first -- is the layout `pool` declares.
+ * Sec. 3.1: the paper's first corruption came from reading the same bytes
+ * with a different logical shape; its NHD attempt failed a divisibility check
+ * because the transfer patch's view and the attention backend's shape and
+ * strides disagreed.  A mismatch must be rejected, never silently mis-copied.
+ * Accepted views (element strides, C-contiguous, times elem_bytes in bytes):
+ *   HND: [num_blocks, 2, H, B, D]       or packed [num_blocks/P, P, 2, H, B, D]
+ *   NHD: [num_blocks, 2, B, H, D]       or packed [num_blocks/P, P, 2, B, H, D]
+ * (P = pool->pages_per_block).  Pure host check; pool->layer_base is not read.
+ * Returns KVX_OK, or KVX_EINVAL with kv_last_error_message naming the first
+ * dimension or stride that disagrees.  A view whose H and B are equal and
+ * whose layout differs cannot be told apart by shape; its strides still must
+ * be the declared layout's.
+ */
+kvx_status kv_pool_view_check(const kvx_pool* pool, int32_t ndim, const int64_t* shape,
+                              const int64_t* strides_bytes);
 
 /*
  * Store (Sec. 3.2 gather; Fig. 2 lower panel ordering): pack tokens

@@ -33,7 +33,8 @@ struct MoveParams {
   int64_t page_bytes;          // 2 * H * B * row
   int64_t total_units;         // units of this launch
   int32_t n_jobs;
-  int32_t blocks_per_chunk;    // C / B
+  int32_t blocks_per_chunk;    // C / B: kernel pages per chunk
+  int32_t ppb;                 // pages per logical block named by the table (>= 1)
   int32_t B, H, R;             // tokens per page, heads, row bytes
   int32_t fast;                // 1 if R/16 is a power of two <= 32
   int32_t vpr_shift;           // log2(R / 16) when fast

@@ -111,6 +111,8 @@ struct DeviceGuard {
   }
 };
 
+int32_t pages_per_block(const kvx_pool* P) { return P->pages_per_block > 1 ? P->pages_per_block : 1; }
+
 bool mul_ok(int64_t a, int64_t b, int64_t* out) {
   if (a < 0 || b < 0) return false;
   if (a != 0 && b > INT64_MAX / a) return false;
@@ -175,6 +177,8 @@ kvx_status check_pool_shape(const kvx_pool* P, Geometry* g) {
     return KVX_EINVAL;
   if (P->layout != KVX_LAYOUT_HND && P->layout != KVX_LAYOUT_NHD) return KVX_EINVAL;
   if ((int64_t)P->block_tokens * P->num_heads > (1ll << 30)) return KVX_EINVAL;
+  if (P->pages_per_block < 0) return KVX_EINVAL;
+  if (P->num_blocks % pages_per_block(P) != 0) return KVX_EALIGN;
   int64_t row, hb, page, layer;
   if (!mul_ok(P->head_dim, P->elem_bytes, &row) || row > (1ll << 30)) return KVX_EINVAL;
   if (!mul_ok((int64_t)P->num_heads * P->block_tokens, 2 * row, &page)) return KVX_EINVAL;
@@ -209,7 +213,7 @@ kvx_status check_range(const kvx_pool* P, int64_t table_len, int64_t t0, int64_t
   if (C % P->block_tokens != 0) return KVX_EALIGN;
   if (t0 % C != 0) return KVX_EALIGN;
   int64_t cap;
-  if (!mul_ok(table_len, P->block_tokens, &cap)) return KVX_EINVAL;
+  if (!mul_ok(table_len, (int64_t)P->block_tokens * pages_per_block(P), &cap)) return KVX_EINVAL;
   if (t1 > cap) return KVX_ERANGE;
   const int64_t need = (t1 == t0) ? 0 : (t1 + C - 1) / C - t0 / C;
   if (need > n_chunks) return KVX_ERANGE;
@@ -272,6 +276,7 @@ void init_move_params(MoveParams* p, long long* err, const kvx_pool* P, const Ge
   p->num_blocks = P->num_blocks;
   p->page_bytes = g.page_bytes;
   p->blocks_per_chunk = C / P->block_tokens;
+  p->ppb = pages_per_block(P);
   p->B = P->block_tokens;
   p->H = P->num_heads;
   p->R = (int32_t)g.row;
@@ -482,7 +487,8 @@ kvx_status check_transfer(int device, const kvx_pool* P, const int32_t* table, i
   st = check_pool_memory(device, P, *g);
   if (st != KVX_OK) return st;
   if ((uintptr_t)table & 3) return KVX_EALIGN;
-  const int64_t blocks_needed = (t1 + P->block_tokens - 1) / P->block_tokens;
+  const int64_t block_span = (int64_t)P->block_tokens * pages_per_block(P);
+  const int64_t blocks_needed = (t1 + block_span - 1) / block_span;
   st = check_device_range(device, table, blocks_needed * (int64_t)sizeof(int32_t));
   if (st != KVX_OK) return st;
   const int64_t first_chunk = t0 / C;
@@ -844,6 +850,56 @@ kvx_status kv_state_load(kvx_ctx* ctx, int32_t num_layers, void* const* layer_ba
                          int64_t slot_bytes, int64_t slot, const void* host_obj, kvx_stream_t stream) {
   return state_copy(ctx, num_layers, layer_base, num_slots, slot_bytes, slot, const_cast<void*>(host_obj),
                     (cudaStream_t)stream, false);
+}
+
+kvx_status kv_pool_view_check(const kvx_pool* pool, int32_t ndim, const int64_t* shape,
+                              const int64_t* strides_bytes) {
+  if (!pool || !shape || !strides_bytes) return KVX_EINVAL;
+  Geometry g;
+  kvx_pool p = *pool;
+  static void* const dummy[1] = {nullptr};
+  if (!p.layer_base) p.layer_base = dummy;
+  kvx_status st = check_pool_shape(&p, &g);
+  if (st != KVX_OK) return st;
+  const int64_t P = pages_per_block(pool);
+  const int64_t H = pool->num_heads, B = pool->block_tokens, D = pool->head_dim;
+  int64_t want[6];
+  int nd = 0;
+  if (ndim == 6) {
+    want[nd++] = pool->num_blocks / P;
+    want[nd++] = P;
+  } else if (ndim == 5) {
+    want[nd++] = pool->num_blocks;
+  } else {
+    set_error_text("a pool layer view has 5 dimensions, or 6 with packed pages");
+    return KVX_EINVAL;
+  }
+  want[nd++] = 2;
+  want[nd++] = pool->layout == KVX_LAYOUT_HND ? H : B;
+  want[nd++] = pool->layout == KVX_LAYOUT_HND ? B : H;
+  want[nd++] = D;
+  static const char* const names_hnd[] = {"pages", "K/V", "heads", "tokens per page", "head_dim"};
+  static const char* const names_nhd[] = {"pages", "K/V", "tokens per page", "heads", "head_dim"};
+  const char* const* names = pool->layout == KVX_LAYOUT_HND ? names_hnd : names_nhd;
+  int64_t stride = pool->elem_bytes;
+  for (int d = ndim - 1; d >= 0; --d) {
+    const char* name = d >= ndim - 5 ? names[d - (ndim - 5)] : "logical blocks";
+    char msg[192];
+    if (shape[d] != want[d]) {
+      snprintf(msg, sizeof(msg), "dimension %d (%s) is %lld, the %s pool description needs %lld", d, name,
+               (long long)shape[d], pool->layout == KVX_LAYOUT_HND ? "HND" : "NHD", (long long)want[d]);
+      set_error_text(msg);
+      return KVX_EINVAL;
+    }
+    if (shape[d] > 1 && strides_bytes[d] != stride) {
+      snprintf(msg, sizeof(msg), "dimension %d (%s) has stride %lld bytes, the %s layout needs %lld", d, name,
+               (long long)strides_bytes[d], pool->layout == KVX_LAYOUT_HND ? "HND" : "NHD", (long long)stride);
+      set_error_text(msg);
+      return KVX_EINVAL;
+    }
+    stride *= shape[d];
+  }
+  return KVX_OK;
 }
 
 kvx_status kv_host_alloc(int64_t bytes, void** out) {

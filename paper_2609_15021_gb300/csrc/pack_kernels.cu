@@ -132,8 +132,9 @@ __device__ __forceinline__ void move_hnd_generic(uint8_t* pg, uint8_t* ck, int n
   }
 }
 
+// At most 64 registers (4 CTAs of 256 threads per SM); no variant spills.
 template <int DIR, int LAYOUT>
-__global__ void __launch_bounds__(kThreads) move_kernel(const __grid_constant__ MoveParams p) {
+__global__ void __launch_bounds__(kThreads, 4) move_kernel(const __grid_constant__ MoveParams p) {
   const int lane = threadIdx.x & 31;
   const int64_t nwarps = ((int64_t)gridDim.x * kThreads) >> 5;
   int64_t u = ((int64_t)blockIdx.x * kThreads + threadIdx.x) >> 5;
@@ -155,11 +156,14 @@ __global__ void __launch_bounds__(kThreads) move_kernel(const __grid_constant__ 
     const int tok0 = jb * p.B;
     if (tok0 >= J.tokens) continue;  // past the end of a short last chunk
     const int nb = min(p.B, J.tokens - tok0);
-    const int64_t lblk = J.first_block + jb;
-    const int32_t page = __ldg(p.table + lblk);
+    // kernel page of the unit, the logical block naming it, and the pool page
+    const int64_t kpage = J.first_block + jb;
+    const int64_t lblk = kpage / p.ppb;
+    const int32_t entry = __ldg(p.table + lblk);
+    const int64_t page = (int64_t)entry * p.ppb + (kpage - lblk * p.ppb);
     uint8_t* ck = J.chunk + ((int64_t)(l - J.l0) * 2 + kv) * J.tokens * HR + (int64_t)tok0 * HR;
     const int nr = nb * p.H;
-    if (page < 0 || (int64_t)page >= p.num_blocks) {
+    if (entry < 0 || (int64_t)entry >= p.num_blocks / p.ppb) {
       if (lane == 0) atomicMin(p.err, (long long)lblk);
       if (DIR == kPack) {  // the unit's chunk rows (contiguous) read as zeros
         const uint4 z = make_uint4(0, 0, 0, 0);

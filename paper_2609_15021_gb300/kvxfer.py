@@ -34,7 +34,7 @@ EXPORTED = (
     "kv_state_store", "kv_state_load", "kv_get_device_error", "kv_ctx_stats", "kv_ctx_reset_stats",
     "kv_ctx_modes", "kv_last_cuda_error", "kv_last_error_message", "kv_status_string", "kv_abi_version",
     "kvx_probe_delayed_fill", "kvx_probe_delayed_copy", "kvx_probe_copy", "kv_store_noalloc",
-    "kv_host_alloc", "kv_host_free",
+    "kv_host_alloc", "kv_host_free", "kv_pool_view_check",
 )
 
 
@@ -54,7 +54,8 @@ class kvx_pool(ctypes.Structure):
     _fields_ = [("num_layers", ctypes.c_int32), ("layer_base", ctypes.POINTER(ctypes.c_void_p)),
                 ("num_blocks", ctypes.c_int64), ("block_tokens", ctypes.c_int32),
                 ("num_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
-                ("elem_bytes", ctypes.c_int32), ("layout", ctypes.c_int32)]
+                ("elem_bytes", ctypes.c_int32), ("layout", ctypes.c_int32),
+                ("pages_per_block", ctypes.c_int32)]
 
 
 class kvx_chunk_layout(ctypes.Structure):
@@ -97,6 +98,7 @@ def _declare(lib):
         "kv_store_noalloc": (st, [P(kvx_pool), vp, i64, i64, i64, i32, P(vp), i64, vp, vp]),
         "kv_host_alloc": (st, [i64, P(vp)]),
         "kv_host_free": (None, [vp]),
+        "kv_pool_view_check": (st, [P(kvx_pool), i32, P(i64), P(i64)]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -155,12 +157,28 @@ class KvPool:
     head_dim: int
     elem_bytes: int
     layout: int = KVX_LAYOUT_HND
+    pages_per_block: int = 1  # pages per logical block named by the block table
 
     def __post_init__(self):
         self._bases = (ctypes.c_void_p * max(1, len(self.layers)))(*[_ptr(t) for t in self.layers])
         self._c = kvx_pool(len(self.layers), ctypes.cast(self._bases, ctypes.POINTER(ctypes.c_void_p)),
                            self.num_blocks, self.block_tokens, self.num_heads, self.head_dim,
-                           self.elem_bytes, self.layout)
+                           self.elem_bytes, self.layout, self.pages_per_block)
+
+    @classmethod
+    def from_tensors(cls, layers, num_heads: int, block_tokens: int, layout: int = KVX_LAYOUT_HND,
+                     pages_per_block: int = 1) -> "KvPool":
+        """Describe a pool from per-layer tensors shaped [pages, 2, H, B, D] (HND) or
+        [pages, 2, B, H, D] (NHD), or packed [blocks, P, 2, ...]; every tensor's view
+        is checked against the declared layout (kv_pool_view_check)."""
+        t = layers[0]
+        head_dim = int(t.shape[-1])
+        pages = t.numel() // (2 * num_heads * block_tokens * head_dim)
+        pool = cls(list(layers), pages, block_tokens, num_heads, head_dim, t.element_size(), layout,
+                   pages_per_block)
+        for x in layers:
+            kv_pool_view_check(pool, x)
+        return pool
 
     @property
     def row_bytes(self) -> int:
@@ -196,6 +214,14 @@ def kv_chunk_layout(pool: KvPool, chunk_tokens: int, tokens_in_chunk: int) -> kv
     _check(_lib.kv_chunk_layout(ctypes.byref(pool.c), chunk_tokens, tokens_in_chunk, ctypes.byref(out)),
            "kv_chunk_layout")
     return out
+
+
+def kv_pool_view_check(pool: KvPool, tensor) -> None:
+    """Raise KvxError unless `tensor`'s shape and strides are the layout `pool` declares."""
+    nd = tensor.dim()
+    shape = (ctypes.c_int64 * nd)(*tensor.shape)
+    strides = (ctypes.c_int64 * nd)(*[s * tensor.element_size() for s in tensor.stride()])
+    _check(_lib.kv_pool_view_check(ctypes.byref(pool.c), nd, shape, strides), "kv_pool_view_check")
 
 
 def _ptr_array(chunks):

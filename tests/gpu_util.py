@@ -33,7 +33,7 @@ def device_pool(spec: oracle.PoolSpec, host_layers=None, fill=POISON):
     else:
         layers = [torch.from_numpy(h).to("cuda") for h in host_layers]
     return k.KvPool(layers, spec.num_blocks, spec.block_tokens, spec.num_heads, spec.head_dim,
-                    spec.elem_bytes, spec.layout)
+                    spec.elem_bytes, spec.layout, spec.pages_per_block)
 
 
 def host_layers(spec: oracle.PoolSpec, seed: int):

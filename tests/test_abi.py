@@ -41,7 +41,7 @@ def test_exports_every_declared_symbol(k):
 
 
 def test_abi_version_and_strings(k):
-    assert k.kv_abi_version() == 1
+    assert k.kv_abi_version() == 2
     assert k.kv_status_string(k.KVX_ENOTPINNED) == "host buffer is not page-locked"
     assert k.kv_status_string(123) == "unknown status"
 
@@ -83,6 +83,31 @@ def test_chunk_layout_errors(k):
     with pytest.raises(k.KvxError) as e:
         k.kv_chunk_layout(_pool(k, layout=7), 256, 1)
     assert e.value.status == k.KVX_EINVAL
+
+
+def test_pool_view_check(k):
+    """Layout views are checked against the declaration (paper Sec. 3.1: an NHD/HND
+    mismatch must be rejected, not silently mis-copied)."""
+    import torch
+    N, H, B, D = 12, 8, 16, 128
+    hnd = torch.empty(N, 2, H, B, D, dtype=torch.bfloat16)
+    nhd = torch.empty(N, 2, B, H, D, dtype=torch.bfloat16)
+    pool = k.KvPool.from_tensors([hnd, hnd], H, B, k.KVX_LAYOUT_HND)
+    assert (pool.num_blocks, pool.head_dim, pool.elem_bytes) == (N, D, 2)
+    k.KvPool.from_tensors([nhd], H, B, k.KVX_LAYOUT_NHD)
+    with pytest.raises(k.KvxError) as e:                  # NHD bytes declared HND
+        k.KvPool.from_tensors([nhd], H, B, k.KVX_LAYOUT_HND)
+    assert e.value.status == k.KVX_EINVAL and "dimension 3 (tokens per page) is 8" in str(e.value)
+    with pytest.raises(k.KvxError) as e:                  # an NHD tensor viewed with HND's shape
+        k.KvPool.from_tensors([nhd.transpose(2, 3)], H, B, k.KVX_LAYOUT_HND)
+    assert "stride" in str(e.value)
+    packed = torch.empty(N // 3, 3, 2, H, B, D, dtype=torch.bfloat16)   # 3 pages per logical block
+    k.KvPool.from_tensors([packed], H, B, k.KVX_LAYOUT_HND, pages_per_block=3)
+    with pytest.raises(k.KvxError) as e:
+        k.KvPool.from_tensors([packed], H, B, k.KVX_LAYOUT_HND, pages_per_block=4)
+    assert e.value.status in (k.KVX_EINVAL, k.KVX_EALIGN)
+    with pytest.raises(k.KvxError):
+        k.kv_pool_view_check(pool, torch.empty(N, 2, H, B * D, dtype=torch.bfloat16))
 
 
 def test_null_context_rejected_before_cuda(k):

@@ -32,14 +32,23 @@ CASES = {
     "many_chunks_three_launches": (1, 300, 1, 1, 8, 2, HND, 300, 2, 0, 1),
     "one_token": (2, 8, 16, 8, 128, 2, HND, 1, 256, 0, 15),
     "27b_shape_two_chunks": (62, 48, 16, 8, 128, 2, HND, 40, 256, 0, 3),
+    # logical blocks of packed pages (Sec. 3.1): 49 pages of 32 tokens per 1,568-token block;
+    # n_used counts logical blocks, N pages
+    "paper_logical_blocks_49": (4, 49 * 6, 32, 4, 256, 1, HND, 5, 1568, 1, 100, 49),
+    "logical_blocks_4_nhd_ragged": (3, 4 * 20, 16, 2, 64, 2, NHD, 17, 96, 2, 7, 4),
 }
 
 MODES = {"staged": 1, "zerocopy": 2}
 
 
+def _unpack(case):
+    """(L, N, B, H, D, e, layout, n_used, C, c0, short, pages per logical block)"""
+    return tuple(case) + (1,) * (12 - len(case))
+
+
 def _range(case):
-    L, N, B, H, D, e, layout, n_used, C, c0, short = case
-    return c0 * C, n_used * B - short
+    L, N, B, H, D, e, layout, n_used, C, c0, short, ppb = _unpack(case)
+    return c0 * C, n_used * ppb * B - short
 
 
 @pytest.fixture(scope="module")
@@ -60,13 +69,13 @@ def ctxs():
 
 def _run_case(orc, ctx, case, stream):
     k = kvx()
-    L, N, B, H, D, e, layout, n_used, C, c0, short = case
-    spec = oracle.PoolSpec(L, N, B, H, D, e, layout)
+    L, N, B, H, D, e, layout, n_used, C, c0, short, ppb = _unpack(case)
+    spec = oracle.PoolSpec(L, N, B, H, D, e, layout, ppb)
     t0, t1 = _range(case)
     src_np = host_layers(spec, seed=hash(case) % 100000)
     src = device_pool(spec, src_np)
-    ta = synth.permuted_table(N, n_used, seed=11)
-    tb = synth.permuted_table(N, n_used, seed=12)
+    ta = synth.permuted_table(N // ppb, n_used, seed=11)
+    tb = synth.permuted_table(N // ppb, n_used, seed=12)
     ta_d = torch.from_numpy(ta).cuda()
     tb_d = torch.from_numpy(tb).cuda()
     extra = 48
