@@ -33,8 +33,17 @@ class HybridShape:
     kv_heads: int = 8
     head_dim: int = 128
     elem_bytes: int = 2            # bf16 K/V
-    state_bytes: int = 16 * 128 * 128 * 4  # fp32 state: 16 heads x 128 x 128
+    recurrent_bytes: int = 16 * 128 * 128 * 4   # fp32 recurrent state: 16 heads x 128 x 128
+    conv_bytes: int = 3 * 8192 * 2              # convolution window: 3 past steps x 8192 channels, bf16
+    slot_align: int = 4096                      # the page is padded to a multiple of this
     chunk_tokens: int = 256
+
+    @property
+    def state_bytes(self) -> int:
+        """One recurrent page (Sec. 2.2): recurrent state, convolution state and padding,
+        moved as opaque bytes."""
+        raw = self.recurrent_bytes + self.conv_bytes
+        return -(-raw // self.slot_align) * self.slot_align
 
     @property
     def page_bytes(self) -> int:

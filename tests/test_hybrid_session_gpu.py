@@ -1,8 +1,10 @@
 """Hybrid six-turn session across two replicas on one GPU (paper Sec. 2.2, Sec. 4.2).
 
 64 layers of which every 4th is full attention (16 paged bf16 layers, 8 KV
-heads, head_dim 128, 16-token pages) and 48 hold an fp32 recurrent state of
-16 heads x 128 x 128 (1 MiB per layer).  Replica A prefills a 32k-token
+heads, head_dim 128, 16-token pages) and 48 hold a recurrent page: an fp32
+recurrent state of 16 heads x 128 x 128 plus a bf16 convolution window,
+padded to 4 KiB (1,097,728 bytes per layer, moved as opaque bytes as the
+paper's patch does, Sec. 2.2).  Replica A prefills a 32k-token
 context and stores it with the state snapshot at 32,768; each later turn the
 other replica restores the chunks it lacks plus the snapshot at the current
 boundary, appends 2,048 tokens (new pages and a new state), and stores the new
