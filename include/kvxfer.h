@@ -63,7 +63,9 @@ typedef enum {
   KVX_ENOTPINNED = -4, /* a host buffer is not page-locked host memory          */
   KVX_ECUDA = -5,      /* a CUDA runtime call failed (kv_last_cuda_error)       */
   KVX_ENOMEM = -6,     /* staging or device allocation failed                   */
-  KVX_EDEVICE = -7     /* a device pointer is not device memory of ctx's GPU    */
+  KVX_EDEVICE = -7,    /* a device pointer is not device memory of ctx's GPU    */
+  KVX_ENOENT = -8,     /* tier: no committed entry for the key                  */
+  KVX_EBUSY = -9       /* tier: the entry is still in use and cannot be rewritten */
 } kvx_status;
 
 typedef enum { KVX_LAYOUT_HND = 0, KVX_LAYOUT_NHD = 1 } kvx_layout;
@@ -292,6 +294,66 @@ kvx_status kv_store_noalloc(const kvx_pool* pool, const int32_t* block_table, in
  */
 kvx_status kv_host_alloc(int64_t bytes, void** out);
 void kv_host_free(void* host);
+
+/* ------------------------------------------------------------------------
+ * Shared host tier (Table 1: one pinned RAM pool of fixed-token chunks with
+ * LRU eviction).  A tier is n_slots fixed-size slots in one pool, each slot
+ * holding one chunk under a 64-bit key.  Entries follow the ordering rule of
+ * Sec. 3.2: a writer reserves a slot, enqueues kv_store into it, then commits
+ * on its stream (an event is recorded there); a reader acquires with its own
+ * stream, which is made to wait for that event, enqueues kv_load, then
+ * releases on its stream.  A slot is never handed out again while it is
+ * pinned or while the GPU may still be writing or reading it (commit and
+ * release events not yet complete): the premature reuse of asynchronous-copy
+ * buffers the paper cites is ruled out.  All tier calls are host-thread safe.
+ * Pass KVX_NO_STREAM when the caller has already synchronised (no event).
+ * ------------------------------------------------------------------------ */
+#define KVX_NO_STREAM ((kvx_stream_t)(intptr_t)-1)
+
+typedef struct kvx_tier kvx_tier;
+
+typedef struct {
+  int64_t slots, slot_bytes, entries, pinned;
+  int64_t hits, misses, evictions;
+} kvx_tier_stats;
+
+/*
+ * Keys of the chunks of a token sequence: key c depends on the salt, on every
+ * token of chunks 0..c and on chunk c's length, so a chunk is found only after
+ * the same prefix (KV depends on everything before it).  The salt separates
+ * namespaces (Sec. 3.2: a new cache salt forces a cold computation; Sec. 4.4:
+ * a reused namespace produced spurious hits).  keys must hold
+ * ceil(n_tokens / chunk_tokens) entries.  SplitMix64 finaliser as the mixer.
+ */
+kvx_status kv_chunk_keys(const int32_t* tokens, int64_t n_tokens, int32_t chunk_tokens, uint64_t salt,
+                         uint64_t* keys, int64_t n_keys);
+
+/* A tier over one new exact-size pinned pool (kv_host_alloc) of
+   slot_bytes * n_slots; slot_bytes a multiple of 16. */
+kvx_status kv_tier_create(int64_t slot_bytes, int64_t n_slots, kvx_tier** out);
+/* A tier over caller-owned memory (16-byte aligned, slot_bytes * n_slots
+   long), not freed by kv_tier_destroy. */
+kvx_status kv_tier_create_on(void* base, int64_t slot_bytes, int64_t n_slots, kvx_tier** out);
+/* Frees the tier (and its pool if kv_tier_create made it); the caller first
+   synchronises every stream that uses it. */
+void kv_tier_destroy(kvx_tier* tier);
+
+/* Slot for writing `key` (a free slot, or the least recently used entry that
+   is neither pinned nor in use by the GPU).  Pins it until kv_tier_commit.
+   KVX_ENOMEM if every slot is pinned or busy; KVX_EBUSY if `key` itself is. */
+kvx_status kv_tier_reserve(kvx_tier* tier, uint64_t key, void** slot);
+/* Marks a reserved entry readable once the work already enqueued on
+   `stream` (the store into it) completes; unpins it. */
+kvx_status kv_tier_commit(kvx_tier* tier, uint64_t key, kvx_stream_t stream);
+/* Slot of a committed entry; `stream` is made to wait for its commit event.
+   Pins it until kv_tier_release.  KVX_ENOENT if absent or not committed. */
+kvx_status kv_tier_acquire(kvx_tier* tier, uint64_t key, kvx_stream_t stream, void** slot);
+/* Unpins; the slot stays in use until the work already enqueued on `stream`
+   (the load from it) completes. */
+kvx_status kv_tier_release(kvx_tier* tier, uint64_t key, kvx_stream_t stream);
+/* Number of leading keys with committed entries (the cached prefix). */
+kvx_status kv_tier_prefix_hits(kvx_tier* tier, const uint64_t* keys, int64_t n, int64_t* hits);
+kvx_status kv_tier_stats(kvx_tier* tier, kvx_tier_stats* out);
 
 /*
  * Lowest logical block index whose table entry was out of range in any call

@@ -13,7 +13,7 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "_lib", "libkvxfer.so")
 
-SOURCES = ["pack_kernels.cu", "kvxfer.cu", "probe.cu", "no_alloc.cu"]
+SOURCES = ["pack_kernels.cu", "kvxfer.cu", "probe.cu", "no_alloc.cu", "tier.cpp"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC,-O2", f"-I{INCLUDE}"]
 
@@ -49,7 +49,7 @@ def build(force: bool = False, verbose: bool = False, ptxas_report: str | None =
     extra = ["-Xptxas", "-v"] if ptxas_report else []
 
     def compile_one(src: str):
-        obj = os.path.join(BUILD, src.replace(".cu", ".o"))
+        obj = os.path.join(BUILD, os.path.splitext(src)[0] + ".o")
         cmd = [nvcc, *ARCH, *FLAGS, *extra, "-c", os.path.join(CSRC, src), "-o", obj]
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:

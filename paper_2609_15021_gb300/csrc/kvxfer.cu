@@ -716,6 +716,8 @@ const char* kv_status_string(kvx_status s) {
     case KVX_ECUDA: return "CUDA runtime error";
     case KVX_ENOMEM: return "out of memory";
     case KVX_EDEVICE: return "pointer is not device memory of the context's GPU";
+    case KVX_ENOENT: return "no committed tier entry for the key";
+    case KVX_EBUSY: return "tier entry still in use";
   }
   return "unknown status";
 }

@@ -35,7 +35,11 @@ EXPORTED = (
     "kv_ctx_modes", "kv_last_cuda_error", "kv_last_error_message", "kv_status_string", "kv_abi_version",
     "kvx_probe_delayed_fill", "kvx_probe_delayed_copy", "kvx_probe_copy", "kv_store_noalloc",
     "kv_host_alloc", "kv_host_free", "kv_pool_view_check",
+    "kv_chunk_keys", "kv_tier_create", "kv_tier_create_on", "kv_tier_destroy", "kv_tier_reserve", "kv_tier_commit",
+    "kv_tier_acquire", "kv_tier_release", "kv_tier_prefix_hits", "kv_tier_stats",
 )
+KVX_ENOENT, KVX_EBUSY = -8, -9
+KVX_NO_STREAM = -1  # the handle value of KVX_NO_STREAM
 
 
 class KvxError(RuntimeError):
@@ -71,6 +75,11 @@ class kvx_stats(ctypes.Structure):
                 ("kernel_bytes", ctypes.c_int64 * 2)]
 
 
+class kvx_tier_stats(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int64) for n in ("slots", "slot_bytes", "entries", "pinned", "hits", "misses",
+                                                 "evictions")]
+
+
 def _declare(lib):
     P, vp, i32, i64 = ctypes.POINTER, ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64
     st = ctypes.c_int
@@ -99,6 +108,16 @@ def _declare(lib):
         "kv_host_alloc": (st, [i64, P(vp)]),
         "kv_host_free": (None, [vp]),
         "kv_pool_view_check": (st, [P(kvx_pool), i32, P(i64), P(i64)]),
+        "kv_chunk_keys": (st, [P(i32), i64, i32, ctypes.c_uint64, P(ctypes.c_uint64), i64]),
+        "kv_tier_create": (st, [i64, i64, P(vp)]),
+        "kv_tier_create_on": (st, [vp, i64, i64, P(vp)]),
+        "kv_tier_destroy": (None, [vp]),
+        "kv_tier_reserve": (st, [vp, ctypes.c_uint64, P(vp)]),
+        "kv_tier_commit": (st, [vp, ctypes.c_uint64, vp]),
+        "kv_tier_acquire": (st, [vp, ctypes.c_uint64, vp, P(vp)]),
+        "kv_tier_release": (st, [vp, ctypes.c_uint64, vp]),
+        "kv_tier_prefix_hits": (st, [vp, P(ctypes.c_uint64), i64, P(i64)]),
+        "kv_tier_stats": (st, [vp, P(kvx_tier_stats)]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -374,6 +393,80 @@ def kvx_probe_copy(dst, src, nbytes: int, how: int, stream=None) -> None:
 
 
 # ---------------------------------------------------------------- convenience
+
+
+def kv_chunk_keys(tokens, chunk_tokens: int, salt: int = 0) -> list[int]:
+    """Prefix-chained keys of the chunks of a token sequence (a sequence of ints)."""
+    import numpy as np
+    t = np.ascontiguousarray(np.asarray(tokens, dtype=np.int32))
+    n = -(-len(t) // chunk_tokens) if len(t) else 0
+    keys = (ctypes.c_uint64 * max(1, n))()
+    _check(_lib.kv_chunk_keys(t.ctypes.data_as(ctypes.POINTER(ctypes.c_int32)), len(t), chunk_tokens,
+                              salt & (2**64 - 1), keys, n), "kv_chunk_keys")
+    return list(keys[:n])
+
+
+class KvTier:
+    """The shared host tier (see kvxfer.h): fixed chunk slots in one pinned pool, LRU."""
+
+    def __init__(self, slot_bytes: int, n_slots: int, base: int | None = None):
+        out = ctypes.c_void_p()
+        if base is None:
+            _check(_lib.kv_tier_create(slot_bytes, n_slots, ctypes.byref(out)), "kv_tier_create")
+        else:
+            _check(_lib.kv_tier_create_on(base, slot_bytes, n_slots, ctypes.byref(out)), "kv_tier_create_on")
+        self.handle = out.value
+        self.slot_bytes = slot_bytes
+
+    def close(self):
+        if self.handle:
+            _lib.kv_tier_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def _slot_tensor(self, ptr: int):
+        import torch
+        raw = (ctypes.c_uint8 * self.slot_bytes).from_address(ptr)
+        return torch.frombuffer(raw, dtype=torch.uint8, count=self.slot_bytes)
+
+    @staticmethod
+    def _stream(stream):
+        if stream == KVX_NO_STREAM:
+            return ctypes.c_void_p(KVX_NO_STREAM & (2**64 - 1))
+        return _stream_handle(stream)
+
+    def reserve(self, key: int):
+        """Host tensor view of the slot to write `key` into (pinned until commit)."""
+        out = ctypes.c_void_p()
+        _check(_lib.kv_tier_reserve(self.handle, key, ctypes.byref(out)), "kv_tier_reserve")
+        return self._slot_tensor(out.value)
+
+    def commit(self, key: int, stream=None):
+        _check(_lib.kv_tier_commit(self.handle, key, self._stream(stream)), "kv_tier_commit")
+
+    def acquire(self, key: int, stream=None):
+        out = ctypes.c_void_p()
+        _check(_lib.kv_tier_acquire(self.handle, key, self._stream(stream), ctypes.byref(out)), "kv_tier_acquire")
+        return self._slot_tensor(out.value)
+
+    def release(self, key: int, stream=None):
+        _check(_lib.kv_tier_release(self.handle, key, self._stream(stream)), "kv_tier_release")
+
+    def prefix_hits(self, keys) -> int:
+        arr = (ctypes.c_uint64 * max(1, len(keys)))(*keys)
+        out = ctypes.c_int64()
+        _check(_lib.kv_tier_prefix_hits(self.handle, arr, len(keys), ctypes.byref(out)), "kv_tier_prefix_hits")
+        return out.value
+
+    def stats(self) -> dict:
+        s = kvx_tier_stats()
+        _check(_lib.kv_tier_stats(self.handle, ctypes.byref(s)), "kv_tier_stats")
+        return {n: getattr(s, n) for n, _ in kvx_tier_stats._fields_}
 
 
 class KvTransfer:

@@ -1,0 +1,102 @@
+"""The shared host tier's bookkeeping on CPU: chunk keys, LRU eviction, pinning.
+
+Runs over caller-owned host memory with KVX_NO_STREAM (no CUDA call is made).
+"""
+import numpy as np
+import pytest
+
+from paper_2609_15021_gb300 import _build
+
+
+@pytest.fixture(scope="module")
+def k():
+    _build.build()
+    from paper_2609_15021_gb300 import kvxfer
+    return kvxfer
+
+
+NO = -1  # KVX_NO_STREAM
+
+
+def test_chunk_keys_chain_over_the_prefix(k):
+    toks = np.arange(1000, dtype=np.int32) * 7 % 5003
+    keys = k.kv_chunk_keys(toks, 256, salt=1)
+    assert len(keys) == 4 and len(set(keys)) == 4
+    assert keys == k.kv_chunk_keys(toks, 256, salt=1)                 # deterministic
+    assert all(a != b for a, b in zip(keys, k.kv_chunk_keys(toks, 256, salt=2)))  # salt = namespace
+    t2 = toks.copy()
+    t2[600] += 1                                                      # a token of chunk 2
+    k2 = k.kv_chunk_keys(t2, 256, salt=1)
+    assert k2[:2] == keys[:2] and all(a != b for a, b in zip(k2[2:], keys[2:]))
+    t3 = toks.copy()
+    t3[0] += 1                                                        # the first token: every key
+    assert all(a != b for a, b in zip(k.kv_chunk_keys(t3, 256, salt=1), keys))
+    assert k.kv_chunk_keys(toks[:999], 256, salt=1)[:3] == keys[:3]
+    assert k.kv_chunk_keys(toks[:999], 256, salt=1)[3] != keys[3]     # a shorter last chunk differs
+    # the same chunk tokens after a different prefix get a different key
+    a = np.concatenate([np.full(256, 5, np.int32), np.full(256, 9, np.int32)])
+    b = np.concatenate([np.full(256, 6, np.int32), np.full(256, 9, np.int32)])
+    assert k.kv_chunk_keys(a, 256)[1] != k.kv_chunk_keys(b, 256)[1]
+
+
+def _tier(k, slots, slot_bytes=64):
+    buf = np.zeros(slots * slot_bytes + 16, np.uint8)
+    off = (-buf.ctypes.data) % 16
+    return k.KvTier(slot_bytes, slots, base=buf.ctypes.data + off), buf
+
+
+def test_lru_eviction_and_prefix_hits(k):
+    tier, buf = _tier(k, 3)
+    for key in (11, 12, 13):
+        s = tier.reserve(key)
+        s.fill_(key)
+        tier.commit(key, NO)
+    assert tier.prefix_hits([11, 12, 13, 14]) == 3
+    s = tier.acquire(11, NO)                 # 11 becomes most recently used
+    assert int(s[0]) == 11
+    tier.release(11, NO)
+    tier.reserve(14).fill_(14)                # evicts the least recently used: 12
+    tier.commit(14, NO)
+    assert tier.prefix_hits([11, 12, 13]) == 1
+    assert tier.prefix_hits([11, 13, 14]) == 3
+    with pytest.raises(k.KvxError) as e:
+        tier.acquire(12, NO)
+    assert e.value.status == k.KVX_ENOENT
+    st = tier.stats()
+    assert st["entries"] == 3 and st["evictions"] == 1 and st["hits"] == 1 and st["misses"] == 1
+    assert int(tier.acquire(14, NO)[5]) == 14
+    tier.release(14, NO)
+    tier.close()
+
+
+def test_pinned_entries_are_never_evicted(k):
+    tier, buf = _tier(k, 2)
+    for key in (1, 2):
+        tier.reserve(key)
+        tier.commit(key, NO)
+    tier.acquire(1, NO)                       # pinned by a reader
+    tier.reserve(3)                           # evicts 2, not the pinned 1
+    assert tier.prefix_hits([1]) == 1
+    with pytest.raises(k.KvxError) as e:      # 1 is read, 3 is being written: nothing to evict
+        tier.reserve(4)
+    assert e.value.status == k.KVX_ENOMEM
+    with pytest.raises(k.KvxError) as e:      # a pinned key cannot be rewritten
+        tier.reserve(1)
+    assert e.value.status == k.KVX_EBUSY
+    assert tier.prefix_hits([3]) == 0         # reserved but not committed: not readable
+    tier.commit(3, NO)
+    tier.release(1, NO)
+    tier.reserve(4)                           # now the least recently used (1) goes
+    tier.commit(4, NO)
+    assert tier.prefix_hits([1]) == 0 and tier.prefix_hits([3, 4]) == 2
+    with pytest.raises(k.KvxError) as e:      # releasing more than acquired
+        tier.release(4, NO)
+    assert e.value.status == k.KVX_EINVAL
+    tier.close()
+
+
+def test_bad_tier_arguments(k):
+    with pytest.raises(k.KvxError):
+        k.KvTier(17, 4, base=16 * 1000)       # slot size not a multiple of 16
+    with pytest.raises(k.KvxError):
+        k.KvTier(64, 0, base=16 * 1000)
