@@ -183,6 +183,8 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-hbm-roofline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--device-engine", choices=["lsu", "tma"], default="lsu",
+                    help="kernel of the device-side (HBM) pack/unpack leg")
     return ap.parse_args()
 
 
@@ -456,7 +458,8 @@ def run_ours(args):
     if not args.no_hbm_roofline:
         dev_slab = torch.empty(n_chunks * cb, dtype=torch.uint8, device=dev)
         dchunks = [dev_slab[i * cb:(i + 1) * cb] for i in range(n_chunks)]
-        hctx = k.kv_ctx_create(local, flags=k.KVX_FLAG_TIME_KERNELS)
+        tma = args.device_engine == "tma"
+        hctx = k.kv_ctx_create(local, flags=k.KVX_FLAG_TIME_KERNELS | (k.KVX_FLAG_DEVICE_TMA if tma else 0))
         for _ in range(2):
             k.kv_pack(hctx, src, ta, 0, T, C, dchunks, stream=stream)
             k.kv_unpack(hctx, dst, tb, 0, T, C, dchunks, stream=stream)
@@ -469,7 +472,8 @@ def run_ours(args):
         hs = k.kv_ctx_stats(hctx)
         assert k.kv_get_device_error(hctx) == -1
         k.kv_ctx_destroy(hctx)
-        hbm_roofline = {"bound": "hbm", "peak": hbm_peak, "unit": "GB/s", "peak_source": peak_src}
+        hbm_roofline = {"bound": "hbm", "peak": hbm_peak, "unit": "GB/s", "peak_source": peak_src,
+                        "engine": "tma bulk copies (tma_move_kernel)" if tma else "16-byte loads/stores (move_kernel)"}
         for d, name in ((0, "pack"), (1, "unpack")):
             nl = hs["timed_launches"][d]
             per_launch = hs["kernel_bytes"][d] / nl

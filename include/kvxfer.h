@@ -65,7 +65,9 @@ typedef enum {
   KVX_ENOMEM = -6,     /* staging or device allocation failed                   */
   KVX_EDEVICE = -7,    /* a device pointer is not device memory of ctx's GPU    */
   KVX_ENOENT = -8,     /* tier: no committed entry for the key                  */
-  KVX_EBUSY = -9       /* tier: the entry is still in use and cannot be rewritten */
+  KVX_EBUSY = -9,      /* tier: the entry is still in use and cannot be rewritten */
+  KVX_ETIMEOUT = -10   /* a bounded wait inside a kernel expired; the kernel
+                          returned early and its output is incomplete          */
 } kvx_status;
 
 typedef enum { KVX_LAYOUT_HND = 0, KVX_LAYOUT_NHD = 1 } kvx_layout;
@@ -89,6 +91,12 @@ typedef enum {
                                       the caller's stream, reproducing the
                                       paper's missing dependency (Sec. 3.2).
                                       Results are then undefined.             */
+#define KVX_FLAG_DEVICE_TMA 0x4u   /* device-side moves (kv_pack, kv_unpack,
+                                      staged mode) use TMA bulk copies staged
+                                      through shared memory instead of 16-byte
+                                      loads/stores (same bytes); pages of more
+                                      than 48 KiB per K or V half keep the
+                                      load/store kernel                       */
 
 typedef struct {
   int32_t store_mode;         /* kvx_mode                                       */

@@ -81,6 +81,11 @@ void set_error_text(const char* text);
 // Launchers (pack_kernels.cu).  Return the cudaError_t of the launch.
 cudaError_t launch_move(int dir, int layout, const MoveParams& p, int grid, cudaStream_t s);
 cudaError_t launch_segments(const SegmentParams& p, int grid, cudaStream_t s);
+// Bulk-copy (TMA) variant for chunks in device memory (tma_kernels.cu): one
+// warp per CTA, `stages` shared-memory stages of stage_bytes each; sets
+// *timeout (device int) if a bounded wait expires.
+cudaError_t launch_move_tma(int dir, int layout, const MoveParams& p, int grid, int stage_bytes, int stages,
+                            int* timeout, cudaStream_t s);
 int move_ctas_per_sm(int dir, int layout);
 int segment_ctas_per_sm();
 

@@ -81,7 +81,8 @@ struct kvx_ctx {
   std::vector<cudaEvent_t> ev_ready;  // slot written (by pack or by an H2D copy)
   std::vector<cudaEvent_t> ev_free;   // slot consumed (by a D2H copy or by unpack)
   int32_t next_slot = 0;
-  long long* d_err = nullptr;
+  long long* d_err = nullptr;  // 16-byte allocation: error word, then the timeout flag
+  int* d_timeout = nullptr;
   std::mutex mu;
   int64_t launches = 0, memcpys = 0;
   int64_t timed[2] = {0, 0}, timed_bytes[2] = {0, 0};
@@ -241,9 +242,23 @@ cudaEvent_t take_timing_event(kvx_ctx* ctx) {
 // not HBM, bounds it and a fraction of the SMs saturates it.
 kvx_status launch_move_timed(kvx_ctx* ctx, int dir, int layout, const MoveParams& p, int64_t bytes,
                              cudaStream_t s, bool over_link) {
-  const int64_t warps_per_cta = kThreads / 32;
-  int64_t grid = (p.total_units + warps_per_cta - 1) / warps_per_cta;
-  int64_t cap = (int64_t)ctx->num_sms * ctx->move_occ[dir][layout];
+  // TMA bulk-copy variant: device-side chunks only, and a K or V half page
+  // (the largest unit) of at most 48 KiB so that 3-4 stages fit in shared memory
+  const int64_t unit_bytes = (int64_t)p.B * p.H * p.R;
+  const bool tma = !over_link && (ctx->opts.flags & KVX_FLAG_DEVICE_TMA) && unit_bytes <= (48 << 10);
+  int stage_bytes = 0, stages = 0;
+  int64_t grid, cap;
+  if (tma) {
+    stage_bytes = (int)((unit_bytes + 127) / 128 * 128);
+    stages = stage_bytes <= (32 << 10) ? 3 : 2;        // 2 CTAs of one warp per SM
+    const int per_sm = std::max(1, (int)((224 << 10) / ((int64_t)stage_bytes * stages + 1024)));
+    grid = p.total_units;
+    cap = (int64_t)ctx->num_sms * per_sm;
+  } else {
+    const int64_t warps_per_cta = kThreads / 32;
+    grid = (p.total_units + warps_per_cta - 1) / warps_per_cta;
+    cap = (int64_t)ctx->num_sms * ctx->move_occ[dir][layout];
+  }
   if (ctx->opts.max_ctas > 0)
     cap = std::min<int64_t>(cap, ctx->opts.max_ctas);
   else if (over_link)
@@ -258,7 +273,10 @@ kvx_status launch_move_timed(kvx_ctx* ctx, int dir, int layout, const MoveParams
       KVX_CUDA(cudaEventRecord(a, s));
     }
   }
-  KVX_CUDA(launch_move(dir, layout, p, (int)grid, s));
+  if (tma)
+    KVX_CUDA(launch_move_tma(dir, layout, p, (int)grid, stage_bytes, stages, ctx->d_timeout, s));
+  else
+    KVX_CUDA(launch_move(dir, layout, p, (int)grid, s));
   ctx->launches++;
   if (timing && a && b) {
     KVX_CUDA(cudaEventRecord(b, s));
@@ -718,6 +736,7 @@ const char* kv_status_string(kvx_status s) {
     case KVX_EDEVICE: return "pointer is not device memory of the context's GPU";
     case KVX_ENOENT: return "no committed tier entry for the key";
     case KVX_EBUSY: return "tier entry still in use";
+    case KVX_ETIMEOUT: return "a bounded wait in a kernel expired";
   }
   return "unknown status";
 }
@@ -771,9 +790,10 @@ kvx_status kv_ctx_create(int device, const kvx_opts* opts, kvx_ctx** out) {
     if ((e = cudaEventCreateWithFlags(&b, cudaEventDisableTiming)) != cudaSuccess) return fail(e);
     ctx->ev_free.push_back(b);
   }
-  if ((e = cudaMalloc(&ctx->d_err, sizeof(long long))) != cudaSuccess) return fail(e);
-  const long long none = kNoError;
-  if ((e = cudaMemcpy(ctx->d_err, &none, sizeof(none), cudaMemcpyHostToDevice)) != cudaSuccess) return fail(e);
+  if ((e = cudaMalloc(&ctx->d_err, 16)) != cudaSuccess) return fail(e);
+  ctx->d_timeout = reinterpret_cast<int*>(ctx->d_err + 1);
+  const long long init[2] = {kNoError, 0};
+  if ((e = cudaMemcpy(ctx->d_err, init, sizeof(init), cudaMemcpyHostToDevice)) != cudaSuccess) return fail(e);
   for (int d = 0; d < 2; ++d)
     for (int l = 0; l < 2; ++l) ctx->move_occ[d][l] = move_ctas_per_sm(d, l);
   ctx->seg_occ = segment_ctas_per_sm();
@@ -940,14 +960,14 @@ kvx_status kv_get_device_error(kvx_ctx* ctx, int64_t* first_bad_block) {
   DeviceGuard guard(ctx->device);
   if (!guard.ok) return KVX_ECUDA;
   std::lock_guard<std::mutex> lock(ctx->mu);
-  long long v = kNoError;
-  const long long none = kNoError;
-  KVX_CUDA(cudaMemcpyAsync(&v, ctx->d_err, sizeof(v), cudaMemcpyDeviceToHost, ctx->s_aux));
+  long long v[2] = {kNoError, 0};
+  const long long none[2] = {kNoError, 0};
+  KVX_CUDA(cudaMemcpyAsync(v, ctx->d_err, sizeof(v), cudaMemcpyDeviceToHost, ctx->s_aux));
   KVX_CUDA(cudaStreamSynchronize(ctx->s_aux));
-  KVX_CUDA(cudaMemcpyAsync(ctx->d_err, &none, sizeof(none), cudaMemcpyHostToDevice, ctx->s_aux));
+  KVX_CUDA(cudaMemcpyAsync(ctx->d_err, none, sizeof(none), cudaMemcpyHostToDevice, ctx->s_aux));
   KVX_CUDA(cudaStreamSynchronize(ctx->s_aux));
-  *first_bad_block = (v == kNoError) ? -1 : (int64_t)v;
-  return KVX_OK;
+  *first_bad_block = (v[0] == kNoError) ? -1 : (int64_t)v[0];
+  return (int)v[1] != 0 ? KVX_ETIMEOUT : KVX_OK;
 }
 
 kvx_status kv_ctx_stats(kvx_ctx* ctx, kvx_stats* out) {

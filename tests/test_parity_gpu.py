@@ -56,10 +56,11 @@ def ctxs():
     k = kvx()
     made = {}
 
-    def get(mode, slot_bytes=0):
-        key = (mode, slot_bytes)
+    def get(mode, slot_bytes=0, flags=0):
+        key = (mode, slot_bytes, flags)
         if key not in made:
-            made[key] = k.kv_ctx_create(0, store_mode=mode, load_mode=mode, staging_slot_bytes=slot_bytes)
+            made[key] = k.kv_ctx_create(0, store_mode=mode, load_mode=mode, staging_slot_bytes=slot_bytes,
+                                        flags=flags)
         return made[key]
 
     yield get
@@ -109,6 +110,12 @@ def test_store_load_parity(orc, ctxs, name, mode):
     _run_case(orc, ctxs(MODES[mode]), CASES[name], stream)
 
 
+@pytest.mark.parametrize("name", list(CASES))
+def test_store_load_parity_staged_tma(orc, ctxs, name):
+    """Staged mode with the TMA bulk-copy kernel packing into / unpacking from the ring."""
+    _run_case(orc, ctxs(1, 0, kvx().KVX_FLAG_DEVICE_TMA), CASES[name], torch.cuda.Stream())
+
+
 @pytest.mark.parametrize("name", ["ragged_tail_offset_start", "27b_shape_two_chunks", "fp8_1568_token_chunks"])
 def test_staged_one_layer_per_slot(orc, ctxs, name):
     """Staging slots that hold exactly one layer of a full chunk: every chunk is split
@@ -119,23 +126,26 @@ def test_staged_one_layer_per_slot(orc, ctxs, name):
     _run_case(orc, ctxs(1, slot), case, torch.cuda.Stream())
 
 
+@pytest.mark.parametrize("engine", ["lsu", "tma"])
 @pytest.mark.parametrize("name", ["tiny_cfg_hnd", "ragged_tail_nhd", "rows_48B_generic", "many_chunks_three_launches",
-                                  "27b_shape_two_chunks"])
-def test_device_pack_unpack_parity(orc, ctxs, name):
+                                  "27b_shape_two_chunks", "paper_logical_blocks_49", "logical_blocks_4_nhd_ragged",
+                                  "rows_16B_16_heads", "one_token"])
+def test_device_pack_unpack_parity(orc, ctxs, name, engine):
     k = kvx()
     case = CASES[name]
-    L, N, B, H, D, e, layout, n_used, C, c0, short = case
-    spec = oracle.PoolSpec(L, N, B, H, D, e, layout)
+    L, N, B, H, D, e, layout, n_used, C, c0, short, ppb = _unpack(case)
+    spec = oracle.PoolSpec(L, N, B, H, D, e, layout, ppb)
     t0, t1 = _range(case)
     src_np = host_layers(spec, seed=77)
     src = device_pool(spec, src_np)
-    ta = synth.permuted_table(N, n_used, seed=21)
-    tb = synth.permuted_table(N, n_used, seed=22)
+    ta = synth.permuted_table(N // ppb, n_used, seed=21)
+    tb = synth.permuted_table(N // ppb, n_used, seed=22)
     extra = 32
     dev = device_chunks(orc, spec, t0, t1, C, extra=extra)
-    ctx = ctxs(1)
+    ctx = ctxs(1, 0, k.KVX_FLAG_DEVICE_TMA if engine == "tma" else 0)
     k.kv_pack(ctx, src, torch.from_numpy(ta).cuda(), t0, t1, C, dev)
     torch.cuda.synchronize()
+    assert k.kv_get_device_error(ctx) == -1   # no bad entry, no expired wait (KVX_ETIMEOUT raises)
     want, _ = oracle_store(orc, spec, src_np, ta, t0, t1, C)
     for i, (d, w) in enumerate(zip(dev, want)):
         got = np_of(d)
@@ -148,6 +158,36 @@ def test_device_pack_unpack_parity(orc, ctxs, name):
                             tb, t0, t1, C, want)
     for l in range(L):
         assert first_mismatch(np_of(dst.layers[l]), want_l[l]) is None, l
+    assert k.kv_get_device_error(ctx) == -1
+
+
+def test_tma_out_of_range_pages(orc, ctxs):
+    """The TMA engine applies the same bad-entry rule (zeros on pack, skip on unpack)."""
+    k = kvx()
+    spec = oracle.PoolSpec(2, 16, 16, 2, 64, 2, HND)
+    src_np = host_layers(spec, seed=15)
+    src = device_pool(spec, src_np)
+    table = synth.permuted_table(16, 12, seed=13)
+    table[3] = 16
+    table[10] = -1
+    C, t0, t1 = 64, 0, 12 * 16
+    dev = device_chunks(orc, spec, t0, t1, C)
+    ctx = ctxs(1, 0, k.KVX_FLAG_DEVICE_TMA)
+    k.kv_pack(ctx, src, torch.from_numpy(table).cuda(), t0, t1, C, dev)
+    torch.cuda.synchronize()
+    assert k.kv_get_device_error(ctx) == 3
+    want, bad = oracle_store(orc, spec, src_np, table, t0, t1, C)
+    assert bad == 3
+    for d, w in zip(dev, want):
+        assert first_mismatch(np_of(d), w) is None
+    dst = device_pool(spec)
+    k.kv_unpack(ctx, dst, torch.from_numpy(table).cuda(), t0, t1, C, dev)
+    torch.cuda.synchronize()
+    assert k.kv_get_device_error(ctx) == 3
+    want_l, _ = oracle_load(orc, spec, [np.full(spec.layer_bytes, POISON, np.uint8) for _ in range(2)],
+                            table, t0, t1, C, want)
+    for l in range(2):
+        assert first_mismatch(np_of(dst.layers[l]), want_l[l]) is None
 
 
 @pytest.mark.parametrize("mode", list(MODES))
