@@ -21,9 +21,20 @@
 #include <new>
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "kvx_internal.h"
 
 using namespace kvx;
+
+namespace {
+// NVTX range around an entry point: a profiler timeline shows each call's
+// host-side checks and enqueue (free when no tool is attached).
+struct TraceRange {
+  explicit TraceRange(const char* name) { nvtxRangePushA(name); }
+  ~TraceRange() { nvtxRangePop(); }
+};
+}  // namespace
 
 namespace kvx {
 thread_local int g_last_cuda_error = 0;
@@ -837,6 +848,7 @@ kvx_status kv_chunk_layout(const kvx_pool* pool, int32_t chunk_tokens, int32_t t
 kvx_status kv_store(kvx_ctx* ctx, const kvx_pool* pool, const int32_t* block_table, int64_t table_len,
                     int64_t tok_begin, int64_t tok_end, int32_t chunk_tokens, void* const* host_chunks,
                     int64_t n_chunks, kvx_stream_t stream) {
+  TraceRange trace("kv_store");
   return transfer(ctx, pool, block_table, table_len, tok_begin, tok_end, chunk_tokens, host_chunks, n_chunks,
                   (cudaStream_t)stream, kPack, kHostChunks);
 }
@@ -844,6 +856,7 @@ kvx_status kv_store(kvx_ctx* ctx, const kvx_pool* pool, const int32_t* block_tab
 kvx_status kv_load(kvx_ctx* ctx, const kvx_pool* pool, const int32_t* block_table, int64_t table_len,
                    int64_t tok_begin, int64_t tok_end, int32_t chunk_tokens, const void* const* host_chunks,
                    int64_t n_chunks, kvx_stream_t stream) {
+  TraceRange trace("kv_load");
   return transfer(ctx, pool, block_table, table_len, tok_begin, tok_end, chunk_tokens,
                   const_cast<void* const*>(host_chunks), n_chunks, (cudaStream_t)stream, kUnpack, kHostChunks);
 }
@@ -851,6 +864,7 @@ kvx_status kv_load(kvx_ctx* ctx, const kvx_pool* pool, const int32_t* block_tabl
 kvx_status kv_pack(kvx_ctx* ctx, const kvx_pool* pool, const int32_t* block_table, int64_t table_len,
                    int64_t tok_begin, int64_t tok_end, int32_t chunk_tokens, void* const* dev_chunks,
                    int64_t n_chunks, kvx_stream_t stream) {
+  TraceRange trace("kv_pack");
   return transfer(ctx, pool, block_table, table_len, tok_begin, tok_end, chunk_tokens, dev_chunks, n_chunks,
                   (cudaStream_t)stream, kPack, kDeviceChunks);
 }
@@ -858,18 +872,21 @@ kvx_status kv_pack(kvx_ctx* ctx, const kvx_pool* pool, const int32_t* block_tabl
 kvx_status kv_unpack(kvx_ctx* ctx, const kvx_pool* pool, const int32_t* block_table, int64_t table_len,
                      int64_t tok_begin, int64_t tok_end, int32_t chunk_tokens, const void* const* dev_chunks,
                      int64_t n_chunks, kvx_stream_t stream) {
+  TraceRange trace("kv_unpack");
   return transfer(ctx, pool, block_table, table_len, tok_begin, tok_end, chunk_tokens,
                   const_cast<void* const*>(dev_chunks), n_chunks, (cudaStream_t)stream, kUnpack, kDeviceChunks);
 }
 
 kvx_status kv_state_store(kvx_ctx* ctx, int32_t num_layers, void* const* layer_base, int64_t num_slots,
                           int64_t slot_bytes, int64_t slot, void* host_obj, kvx_stream_t stream) {
+  TraceRange trace("kv_state_store");
   return state_copy(ctx, num_layers, layer_base, num_slots, slot_bytes, slot, host_obj, (cudaStream_t)stream,
                     true);
 }
 
 kvx_status kv_state_load(kvx_ctx* ctx, int32_t num_layers, void* const* layer_base, int64_t num_slots,
                          int64_t slot_bytes, int64_t slot, const void* host_obj, kvx_stream_t stream) {
+  TraceRange trace("kv_state_load");
   return state_copy(ctx, num_layers, layer_base, num_slots, slot_bytes, slot, const_cast<void*>(host_obj),
                     (cudaStream_t)stream, false);
 }
