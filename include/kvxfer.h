@@ -385,6 +385,17 @@ int kv_last_cuda_error(void);
    thread's next failing call. */
 const char* kv_last_error_message(void);
 
+/*
+ * Host-side fault injection for testing error handling without faulting a
+ * GPU: the (after_calls + 1)-th next CUDA call at `point` in this process
+ * fails with cudaErrorUnknown (cudaErrorMemoryAllocation for "host_alloc")
+ * instead of being made.  Points: "launch" (kernel launches), "memcpy"
+ * (staged-mode copies), "event" (the ordering event recorded on the caller's
+ * stream), "host_alloc" (kv_host_alloc).  One point is armed at a time;
+ * point NULL or "" disarms.  KVX_EINVAL for an unknown point.
+ */
+kvx_status kv_fault_inject(const char* point, int32_t after_calls);
+
 /* Static text for a status value. */
 const char* kv_status_string(kvx_status status);
 

@@ -47,15 +47,33 @@ void record_cuda_error(int e, const char* call, int line) {
 }
 }  // namespace kvx
 
-#define KVX_CUDA(call)                              \
-  do {                                              \
-    cudaError_t e_ = (call);                        \
-    if (e_ != cudaSuccess) {                        \
-      record_cuda_error((int)e_, #call, __LINE__);  \
-      cudaGetLastError();                           \
-      return KVX_ECUDA;                             \
-    }                                               \
+// Host-side fault injection (kv_fault_inject): the armed point fails its
+// n-th next call with cudaErrorUnknown instead of calling CUDA.
+namespace {
+std::mutex g_fault_mu;
+char g_fault_point[32] = "";
+int g_fault_countdown = -1;
+
+bool fault_now(const char* point) {
+  if (g_fault_countdown < 0) return false;  // unarmed (racy read is benign: re-checked under the lock)
+  std::lock_guard<std::mutex> lock(g_fault_mu);
+  if (g_fault_countdown < 0 || strcmp(point, g_fault_point) != 0) return false;
+  if (g_fault_countdown-- > 0) return false;
+  g_fault_point[0] = 0;
+  return true;
+}
+}  // namespace
+
+#define KVX_CUDA_AT(point, call)                                                   \
+  do {                                                                             \
+    cudaError_t e_ = fault_now(point) ? cudaErrorUnknown : (call);                 \
+    if (e_ != cudaSuccess) {                                                       \
+      record_cuda_error((int)e_, #call, __LINE__);                                 \
+      cudaGetLastError();                                                          \
+      return KVX_ECUDA;                                                            \
+    }                                                                              \
   } while (0)
+#define KVX_CUDA(call) KVX_CUDA_AT("", call)
 
 namespace {
 
@@ -285,9 +303,9 @@ kvx_status launch_move_timed(kvx_ctx* ctx, int dir, int layout, const MoveParams
     }
   }
   if (tma)
-    KVX_CUDA(launch_move_tma(dir, layout, p, (int)grid, stage_bytes, stages, ctx->d_timeout, s));
+    KVX_CUDA_AT("launch", launch_move_tma(dir, layout, p, (int)grid, stage_bytes, stages, ctx->d_timeout, s));
   else
-    KVX_CUDA(launch_move(dir, layout, p, (int)grid, s));
+    KVX_CUDA_AT("launch", launch_move(dir, layout, p, (int)grid, s));
   ctx->launches++;
   if (timing && a && b) {
     KVX_CUDA(cudaEventRecord(b, s));
@@ -430,9 +448,9 @@ kvx_status enqueue_staged(kvx_ctx* ctx, const Plan& pl) {
           ++r;
         }
         if (to_host)
-          KVX_CUDA(cudaMemcpyAsync(h, slot + soff, (size_t)len, cudaMemcpyDeviceToHost, ctx->s_copy));
+          KVX_CUDA_AT("memcpy", cudaMemcpyAsync(h, slot + soff, (size_t)len, cudaMemcpyDeviceToHost, ctx->s_copy));
         else
-          KVX_CUDA(cudaMemcpyAsync(slot + soff, h, (size_t)len, cudaMemcpyHostToDevice, ctx->s_copy));
+          KVX_CUDA_AT("memcpy", cudaMemcpyAsync(slot + soff, h, (size_t)len, cudaMemcpyHostToDevice, ctx->s_copy));
         ctx->memcpys++;
         soff += len;
         q = r;
@@ -597,7 +615,7 @@ kvx_status transfer(kvx_ctx* ctx, const kvx_pool* P, const int32_t* table, int64
     st = ensure_staging(ctx);
     if (st != KVX_OK) return st;
   }
-  KVX_CUDA(cudaEventRecord(ctx->ev_in, stream));
+  KVX_CUDA_AT("event", cudaEventRecord(ctx->ev_in, stream));
   if ((ctx->opts.flags & KVX_FLAG_UNORDERED) == 0) {
     KVX_CUDA(cudaStreamWaitEvent(ctx->s_kern, ctx->ev_in, 0));
     if (staged) KVX_CUDA(cudaStreamWaitEvent(ctx->s_copy, ctx->ev_in, 0));
@@ -891,6 +909,22 @@ kvx_status kv_state_load(kvx_ctx* ctx, int32_t num_layers, void* const* layer_ba
                     (cudaStream_t)stream, false);
 }
 
+kvx_status kv_fault_inject(const char* point, int32_t after_calls) {
+  static const char* const points[] = {"launch", "memcpy", "event", "host_alloc"};
+  std::lock_guard<std::mutex> lock(g_fault_mu);
+  if (!point || !point[0]) {
+    g_fault_point[0] = 0;
+    g_fault_countdown = -1;
+    return KVX_OK;
+  }
+  bool known = false;
+  for (const char* q : points) known |= strcmp(q, point) == 0;
+  if (!known || after_calls < 0) return KVX_EINVAL;
+  snprintf(g_fault_point, sizeof(g_fault_point), "%s", point);
+  g_fault_countdown = after_calls;
+  return KVX_OK;
+}
+
 kvx_status kv_pool_view_check(const kvx_pool* pool, int32_t ndim, const int64_t* shape,
                               const int64_t* strides_bytes) {
   if (!pool || !shape || !strides_bytes) return KVX_EINVAL;
@@ -950,7 +984,9 @@ kvx_status kv_host_alloc(int64_t bytes, void** out) {
   // the zero-copy kernels can use it.  No pageable fallback: a failure is an
   // error (Sec. 3.3: a full-pool request that silently fell back to pageable
   // memory).
-  cudaError_t e = cudaHostAlloc(&p, (size_t)bytes, cudaHostAllocPortable | cudaHostAllocMapped);
+  cudaError_t e = fault_now("host_alloc")
+                      ? cudaErrorMemoryAllocation
+                      : cudaHostAlloc(&p, (size_t)bytes, cudaHostAllocPortable | cudaHostAllocMapped);
   if (e != cudaSuccess) {
     record_cuda_error((int)e, "cudaHostAlloc", __LINE__);
     cudaGetLastError();

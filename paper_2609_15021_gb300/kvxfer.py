@@ -37,7 +37,7 @@ EXPORTED = (
     "kvx_probe_delayed_fill", "kvx_probe_delayed_copy", "kvx_probe_copy", "kv_store_noalloc",
     "kv_host_alloc", "kv_host_free", "kv_pool_view_check",
     "kv_chunk_keys", "kv_tier_create", "kv_tier_create_on", "kv_tier_destroy", "kv_tier_reserve", "kv_tier_commit",
-    "kv_tier_acquire", "kv_tier_release", "kv_tier_prefix_hits", "kv_tier_stats",
+    "kv_tier_acquire", "kv_tier_release", "kv_tier_prefix_hits", "kv_tier_stats", "kv_fault_inject",
 )
 KVX_ENOENT, KVX_EBUSY = -8, -9
 KVX_NO_STREAM = -1  # the handle value of KVX_NO_STREAM
@@ -119,6 +119,7 @@ def _declare(lib):
         "kv_tier_release": (st, [vp, ctypes.c_uint64, vp]),
         "kv_tier_prefix_hits": (st, [vp, P(ctypes.c_uint64), i64, P(i64)]),
         "kv_tier_stats": (st, [vp, P(kvx_tier_stats)]),
+        "kv_fault_inject": (st, [ctypes.c_char_p, i32]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -394,6 +395,11 @@ def kvx_probe_copy(dst, src, nbytes: int, how: int, stream=None) -> None:
 
 
 # ---------------------------------------------------------------- convenience
+
+
+def kv_fault_inject(point: str | None, after_calls: int = 0) -> None:
+    """Make the (after_calls+1)-th next CUDA call at `point` fail (host side); None disarms."""
+    _check(_lib.kv_fault_inject(point.encode() if point else None, after_calls), "kv_fault_inject")
 
 
 def kv_chunk_keys(tokens, chunk_tokens: int, salt: int = 0) -> list[int]:
