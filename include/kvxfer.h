@@ -342,13 +342,35 @@ kvx_status kv_tier_create(int64_t slot_bytes, int64_t n_slots, kvx_tier** out);
 /* A tier over caller-owned memory (16-byte aligned, slot_bytes * n_slots
    long), not freed by kv_tier_destroy. */
 kvx_status kv_tier_create_on(void* base, int64_t slot_bytes, int64_t n_slots, kvx_tier** out);
-/* Frees the tier (and its pool if kv_tier_create made it); the caller first
-   synchronises every stream that uses it. */
+/*
+ * A tier shared by the processes of one host (Fig. 1: complete replicas, each
+ * its own process, share one pinned RAM pool).  `name` is a POSIX shared-memory
+ * name ("/..."); with KVX_TIER_CREATE the region (slot table, a process-shared
+ * robust mutex, and slot_bytes * n_slots of data) is created, otherwise an
+ * existing one is opened and slot_bytes / n_slots are ignored.  Each process
+ * registers the data as pinned, mapped memory (cudaHostRegister) unless
+ * KVX_TIER_NO_PIN (bookkeeping only, no transfers).  An entry committed on a
+ * stream becomes readable by other processes only once the writer's process
+ * has seen that work complete (any tier call or kv_tier_poll in that process);
+ * in the writer's own process it is readable at once, the reader's stream
+ * waiting on the writer's event.  The creator's kv_tier_destroy removes the
+ * name; mappings in other processes stay valid.
+ */
+#define KVX_TIER_CREATE 0x1u
+#define KVX_TIER_NO_PIN 0x2u
+kvx_status kv_tier_open_shared(const char* name, int64_t slot_bytes, int64_t n_slots, uint32_t flags,
+                               kvx_tier** out);
+/* Settle this process's completed work on the tier: entries it committed
+   become readable everywhere, pins held for its queued reads are dropped. */
+kvx_status kv_tier_poll(kvx_tier* tier);
+/* Waits for this process's pending work on the tier, then frees the tier (and
+   its pool if kv_tier_create made it). */
 void kv_tier_destroy(kvx_tier* tier);
 
-/* Slot for writing `key` (a free slot, or the least recently used entry that
-   is neither pinned nor in use by the GPU).  Pins it until kv_tier_commit.
-   KVX_ENOMEM if every slot is pinned or busy; KVX_EBUSY if `key` itself is. */
+/* Slot for writing `key` (a free slot, or the least recently used committed
+   entry that is neither pinned nor in use by queued GPU work).  Pins it until
+   kv_tier_commit (or kv_tier_release to give it up).  KVX_ENOMEM if every
+   slot is pinned or busy; KVX_EBUSY if `key` itself is. */
 kvx_status kv_tier_reserve(kvx_tier* tier, uint64_t key, void** slot);
 /* Marks a reserved entry readable once the work already enqueued on
    `stream` (the store into it) completes; unpins it. */

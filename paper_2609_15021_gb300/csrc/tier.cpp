@@ -1,20 +1,38 @@
 // tier.cpp -- the shared host tier: fixed-size chunk slots in one pinned pool,
 // keyed by prefix-chained chunk keys, evicted least-recently-used.
 //
-// Paper Table 1: the shared tier is one pinned RAM pool holding fixed-token
-// chunks with LRU eviction.  Sec. 3.2: a copy must be ordered on the current
-// stream, and the related reports it cites concern asynchronous-copy buffers
-// reused too early.  So an entry written by an asynchronous store becomes
-// readable only through an event recorded on the writer's stream (a reader's
-// stream waits on it), and a slot is never handed out again while work that
-// reads or writes it may still be running: pinned entries, and entries whose
-// release event has not completed, are not evicted.  Sec. 3.2 / Sec. 4.4: a
-// cache salt forces a cold path and namespaces must not collide, so keys
-// include a caller salt.
+// Paper Table 1 / Fig. 1: complete replicas share one pinned RAM pool holding
+// fixed-token chunks with LRU eviction.  Sec. 3.2: a copy must be ordered on
+// the current stream, and the related reports it cites concern asynchronous-
+// copy buffers reused too early.  Sec. 3.2 / Sec. 4.4: a cache salt forces a
+// cold path and namespaces must not collide, so keys include a caller salt.
+//
+// A tier is either private to one process or shared by several (POSIX shared
+// memory holding the slot table, a process-shared robust mutex and the data,
+// which every process registers as pinned, mapped memory).  Entry states:
+//   WRITING    reserved by a writer, not readable
+//   COMMITTING committed on the writer's stream, GPU work still pending:
+//              readable in the writer's process (the reader's stream waits on
+//              the writer's event), invisible to other processes
+//   READY      the data is complete: readable everywhere
+// The writer's process turns COMMITTING into READY when its event completes
+// (checked at every tier call of that process and by kv_tier_poll), which is
+// the paper's completion-before-consumption rule applied across processes.
+// Readers pin entries; a release on a stream keeps the pin until the work on
+// that stream completes, so a slot in use by queued GPU work is never evicted.
 
 #include <cuda_runtime.h>
+#include <errno.h>
+#include <fcntl.h>
+#include <pthread.h>
 #include <stdint.h>
 #include <stdio.h>
+#include <stdlib.h>
+#include <string.h>
+#include <sys/mman.h>
+#include <sys/stat.h>
+#include <time.h>
+#include <unistd.h>
 
 #include <mutex>
 #include <new>
@@ -27,17 +45,26 @@ using namespace kvx;
 
 namespace {
 
-enum SlotState : int { kFree = 0, kWriting = 1, kReady = 2 };
+constexpr uint64_t kMagic = 0x3152454954584B56ull;  // "VKXTIER1"
+constexpr int64_t kDataAlign = 2ll << 20;
 
-struct Slot {
-  uint64_t key = 0;
-  int state = kFree;
-  int64_t pins = 0;             // outstanding reserve/acquire without release
-  uint64_t tick = 0;            // last use, for LRU
-  cudaEvent_t ready = nullptr;  // recorded by commit on the writer's stream
-  bool ready_recorded = false;
-  cudaEvent_t done = nullptr;   // recorded by release on the user's stream
-  bool done_recorded = false;
+enum SlotState : int32_t { kFree = 0, kWriting = 1, kCommitting = 2, kReady = 3 };
+
+struct Header {
+  uint64_t magic;
+  int64_t slot_bytes, n_slots, data_offset, total_bytes;
+  pthread_mutex_t mu;
+  uint64_t clock;
+  int64_t hits, misses, evictions;
+  volatile int32_t initialised;
+};
+
+struct SlotMeta {
+  uint64_t key;
+  int32_t state;
+  int32_t writer_pid;  // process whose event decides COMMITTING -> READY
+  int64_t pins;        // outstanding acquires/reserves, and releases whose GPU work is pending
+  uint64_t tick;       // last use, for LRU
 };
 
 // SplitMix64 finaliser (Steele, Lea & Flood 2014) as the mixing step.
@@ -57,74 +84,172 @@ kvx_status cuda_fail(cudaError_t e, const char* what) {
   return KVX_ECUDA;
 }
 
+struct PendingEvent {
+  int64_t slot;
+  cudaEvent_t ev;
+};
+
 }  // namespace
 
 struct kvx_tier {
-  uint8_t* base = nullptr;
-  bool owns = false;
-  int64_t slot_bytes = 0;
-  std::vector<Slot> slots;
-  std::unordered_map<uint64_t, int64_t> index;  // key -> slot
-  uint64_t clock = 0;
-  int64_t hits = 0, misses = 0, evictions = 0;
-  std::mutex mu;
+  // the slot table and counters: in shared memory for a shared tier
+  Header* hdr = nullptr;
+  SlotMeta* meta = nullptr;
+  uint8_t* data = nullptr;
+  // ownership
+  void* mapping = nullptr;   // shared: the whole mmap; private: the metadata allocation
+  int64_t mapping_bytes = 0;
+  bool shared = false;
+  bool creator = false;
+  bool registered = false;   // data registered with cudaHostRegister by this process
+  bool owns_data = false;    // private tier whose pool came from kv_host_alloc
+  char name[128] = "";
+  int32_t pid = 0;
+  // this process's pending GPU work on slots
+  std::vector<PendingEvent> commits;   // COMMITTING entries written by this process
+  std::vector<PendingEvent> releases;  // pins held until queued work completes
+  std::unordered_map<int64_t, cudaEvent_t> commit_event;  // slot -> event readers here may wait on
+  std::vector<cudaEvent_t> spare;
+  std::mutex local;          // guards the members above
+  std::unordered_map<uint64_t, int64_t> index;  // private tier: key -> slot
 };
 
 namespace {
 
-// An entry may be evicted when nothing pins it and the work that wrote it
-// (commit event) and the work that last used it (release event) have
-// completed on the GPU.
-bool evictable(Slot& s) {
-  if (s.pins > 0) return false;
-  if (s.ready_recorded) {
-    const cudaError_t q = cudaEventQuery(s.ready);
-    if (q == cudaErrorNotReady) return false;
-    cudaGetLastError();
+// Process-shared lock over the slot table (robust: a holder that died leaves it usable).
+struct TierLock {
+  kvx_tier* t;
+  explicit TierLock(kvx_tier* tier) : t(tier) {
+    t->local.lock();
+    int r = pthread_mutex_lock(&t->hdr->mu);
+    if (r == EOWNERDEAD) pthread_mutex_consistent(&t->hdr->mu);
   }
-  if (s.done_recorded) {
-    const cudaError_t q = cudaEventQuery(s.done);
-    if (q == cudaErrorNotReady) return false;
-    cudaGetLastError();
-    s.done_recorded = false;
+  ~TierLock() {
+    pthread_mutex_unlock(&t->hdr->mu);
+    t->local.unlock();
   }
-  return true;
+};
+
+cudaEvent_t take_event(kvx_tier* t) {
+  if (!t->spare.empty()) {
+    cudaEvent_t e = t->spare.back();
+    t->spare.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  if (cudaEventCreateWithFlags(&e, cudaEventDisableTiming) != cudaSuccess) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  return e;
 }
 
-// Free slot, else the least recently used evictable one; -1 if none.
+// Settle this process's completed GPU work: COMMITTING -> READY, pins dropped.
+void poll_locked(kvx_tier* t, bool wait) {
+  auto done = [&](cudaEvent_t e) {
+    cudaError_t q = wait ? cudaEventSynchronize(e) : cudaEventQuery(e);
+    if (q == cudaErrorNotReady) return false;
+    cudaGetLastError();
+    return true;
+  };
+  for (size_t i = 0; i < t->commits.size();) {
+    PendingEvent& p = t->commits[i];
+    if (!done(p.ev)) {
+      ++i;
+      continue;
+    }
+    SlotMeta& m = t->meta[p.slot];
+    if (m.state == kCommitting && m.writer_pid == t->pid) m.state = kReady;
+    auto it = t->commit_event.find(p.slot);
+    if (it != t->commit_event.end() && it->second == p.ev) t->commit_event.erase(it);
+    t->spare.push_back(p.ev);
+    t->commits[i] = t->commits.back();
+    t->commits.pop_back();
+  }
+  for (size_t i = 0; i < t->releases.size();) {
+    PendingEvent& p = t->releases[i];
+    if (!done(p.ev)) {
+      ++i;
+      continue;
+    }
+    if (t->meta[p.slot].pins > 0) t->meta[p.slot].pins--;
+    t->spare.push_back(p.ev);
+    t->releases[i] = t->releases.back();
+    t->releases.pop_back();
+  }
+}
+
+int64_t find_slot(kvx_tier* t, uint64_t key) {
+  if (!t->shared) {
+    auto it = t->index.find(key);
+    return it == t->index.end() ? -1 : it->second;
+  }
+  for (int64_t i = 0; i < t->hdr->n_slots; ++i)
+    if (t->meta[i].state != kFree && t->meta[i].key == key) return i;
+  return -1;
+}
+
+// Free slot, else the least recently used slot that is READY and unpinned; -1 if none.
 int64_t pick_slot(kvx_tier* t) {
   int64_t best = -1;
-  for (int64_t i = 0; i < (int64_t)t->slots.size(); ++i) {
-    Slot& s = t->slots[i];
-    if (s.state == kFree) return i;
-  }
-  for (int64_t i = 0; i < (int64_t)t->slots.size(); ++i) {
-    Slot& s = t->slots[i];
-    if (!evictable(s)) continue;
-    if (best < 0 || s.tick < t->slots[best].tick) best = i;
+  for (int64_t i = 0; i < t->hdr->n_slots; ++i) {
+    const SlotMeta& m = t->meta[i];
+    if (m.state == kFree) return i;
+    if (m.state != kReady || m.pins > 0) continue;
+    if (best < 0 || m.tick < t->meta[best].tick) best = i;
   }
   return best;
 }
 
-kvx_status ensure_event(cudaEvent_t* e) {
-  if (*e) return KVX_OK;
-  const cudaError_t r = cudaEventCreateWithFlags(e, cudaEventDisableTiming);
-  if (r != cudaSuccess) {
-    *e = nullptr;
-    return cuda_fail(r, "cudaEventCreateWithFlags for a tier entry");
-  }
-  return KVX_OK;
-}
-
 void destroy_tier(kvx_tier* t) {
   if (!t) return;
-  for (Slot& s : t->slots) {
-    if (s.ready) cudaEventDestroy(s.ready);
-    if (s.done) cudaEventDestroy(s.done);
+  {
+    std::lock_guard<std::mutex> g(t->local);
+    if (t->hdr) {
+      int r = pthread_mutex_lock(&t->hdr->mu);
+      if (r == EOWNERDEAD) pthread_mutex_consistent(&t->hdr->mu);
+      poll_locked(t, true);  // settle this process's pending work
+      pthread_mutex_unlock(&t->hdr->mu);
+    }
+    for (cudaEvent_t e : t->spare) cudaEventDestroy(e);
+    cudaGetLastError();
   }
-  cudaGetLastError();
-  if (t->owns) kv_host_free(t->base);
+  if (t->registered) {
+    cudaHostUnregister(t->data);
+    cudaGetLastError();
+  }
+  if (t->shared) {
+    munmap(t->mapping, (size_t)t->mapping_bytes);
+    if (t->creator) shm_unlink(t->name);
+  } else {
+    free(t->mapping);
+    if (t->owns_data) kv_host_free(t->data);
+  }
   delete t;
+}
+
+kvx_status init_private(void* base, int64_t slot_bytes, int64_t n_slots, kvx_tier** out) {
+  kvx_tier* t = new (std::nothrow) kvx_tier;
+  if (!t) return KVX_ENOMEM;
+  const int64_t meta_bytes = (int64_t)sizeof(Header) + n_slots * (int64_t)sizeof(SlotMeta);
+  void* m = calloc(1, (size_t)meta_bytes);
+  if (!m) {
+    delete t;
+    return KVX_ENOMEM;
+  }
+  t->mapping = m;
+  t->hdr = (Header*)m;
+  t->meta = (SlotMeta*)((uint8_t*)m + sizeof(Header));
+  t->data = (uint8_t*)base;
+  t->pid = (int32_t)getpid();
+  Header* h = t->hdr;
+  h->magic = kMagic;
+  h->slot_bytes = slot_bytes;
+  h->n_slots = n_slots;
+  pthread_mutex_init(&h->mu, nullptr);
+  h->initialised = 1;
+  *out = t;
+  return KVX_OK;
 }
 
 }  // namespace
@@ -152,13 +277,7 @@ kvx_status kv_tier_create_on(void* base, int64_t slot_bytes, int64_t n_slots, kv
   *out = nullptr;
   if (!base || slot_bytes < 16 || slot_bytes % 16 != 0 || n_slots < 1) return KVX_EINVAL;
   if ((uintptr_t)base & 15) return KVX_EALIGN;
-  kvx_tier* t = new (std::nothrow) kvx_tier;
-  if (!t) return KVX_ENOMEM;
-  t->base = (uint8_t*)base;
-  t->slot_bytes = slot_bytes;
-  t->slots.resize((size_t)n_slots);
-  *out = t;
-  return KVX_OK;
+  return init_private(base, slot_bytes, n_slots, out);
 }
 
 kvx_status kv_tier_create(int64_t slot_bytes, int64_t n_slots, kvx_tier** out) {
@@ -169,114 +288,252 @@ kvx_status kv_tier_create(int64_t slot_bytes, int64_t n_slots, kvx_tier** out) {
   void* p = nullptr;
   kvx_status st = kv_host_alloc(slot_bytes * n_slots, &p);
   if (st != KVX_OK) return st;
-  st = kv_tier_create_on(p, slot_bytes, n_slots, out);
+  st = init_private(p, slot_bytes, n_slots, out);
   if (st != KVX_OK) {
     kv_host_free(p);
     return st;
   }
-  (*out)->owns = true;
+  (*out)->owns_data = true;
+  return KVX_OK;
+}
+
+kvx_status kv_tier_open_shared(const char* name, int64_t slot_bytes, int64_t n_slots, uint32_t flags,
+                               kvx_tier** out) {
+  if (!out || !name || name[0] != '/' || strlen(name) >= 120) return KVX_EINVAL;
+  *out = nullptr;
+  const bool create = (flags & KVX_TIER_CREATE) != 0;
+  if (create && (slot_bytes < 16 || slot_bytes % 16 != 0 || n_slots < 1)) return KVX_EINVAL;
+  const int fd = shm_open(name, create ? (O_CREAT | O_EXCL | O_RDWR) : O_RDWR, 0600);
+  if (fd < 0) {
+    set_error_text(create ? "shm_open: the name exists or cannot be created" : "shm_open: no such tier");
+    return create ? KVX_EINVAL : KVX_ENOENT;
+  }
+  int64_t total = 0, data_offset = 0;
+  if (create) {
+    const int64_t meta_bytes = (int64_t)sizeof(Header) + n_slots * (int64_t)sizeof(SlotMeta);
+    data_offset = (meta_bytes + kDataAlign - 1) / kDataAlign * kDataAlign;
+    if (n_slots > (INT64_MAX - data_offset) / slot_bytes) {
+      close(fd);
+      shm_unlink(name);
+      return KVX_EINVAL;
+    }
+    total = data_offset + slot_bytes * n_slots;
+    if (ftruncate(fd, (off_t)total) != 0) {
+      close(fd);
+      shm_unlink(name);
+      set_error_text("ftruncate of the shared tier failed");
+      return KVX_ENOMEM;
+    }
+  } else {
+    struct stat sb;
+    // wait (bounded) for the creator to size and initialise the region
+    for (int i = 0; i < 5000; ++i) {
+      if (fstat(fd, &sb) == 0 && sb.st_size >= (off_t)sizeof(Header)) break;
+      usleep(1000);
+    }
+    if (fstat(fd, &sb) != 0 || sb.st_size < (off_t)sizeof(Header)) {
+      close(fd);
+      return KVX_ENOENT;
+    }
+    total = (int64_t)sb.st_size;
+  }
+  void* map = mmap(nullptr, (size_t)total, PROT_READ | PROT_WRITE, MAP_SHARED, fd, 0);
+  close(fd);
+  if (map == MAP_FAILED) {
+    if (create) shm_unlink(name);
+    return KVX_ENOMEM;
+  }
+  kvx_tier* t = new (std::nothrow) kvx_tier;
+  if (!t) {
+    munmap(map, (size_t)total);
+    if (create) shm_unlink(name);
+    return KVX_ENOMEM;
+  }
+  t->shared = true;
+  t->creator = create;
+  t->mapping = map;
+  t->mapping_bytes = total;
+  t->pid = (int32_t)getpid();
+  snprintf(t->name, sizeof(t->name), "%s", name);
+  t->hdr = (Header*)map;
+  t->meta = (SlotMeta*)((uint8_t*)map + sizeof(Header));
+  Header* h = t->hdr;
+  if (create) {
+    h->magic = kMagic;
+    h->slot_bytes = slot_bytes;
+    h->n_slots = n_slots;
+    h->data_offset = data_offset;
+    h->total_bytes = total;
+    pthread_mutexattr_t a;
+    pthread_mutexattr_init(&a);
+    pthread_mutexattr_setpshared(&a, PTHREAD_PROCESS_SHARED);
+    pthread_mutexattr_setrobust(&a, PTHREAD_MUTEX_ROBUST);
+    pthread_mutex_init(&h->mu, &a);
+    pthread_mutexattr_destroy(&a);
+    __atomic_store_n(&h->initialised, 1, __ATOMIC_RELEASE);
+  } else {
+    int i = 0;
+    while (__atomic_load_n(&h->initialised, __ATOMIC_ACQUIRE) != 1 && i++ < 5000) usleep(1000);
+    if (h->initialised != 1 || h->magic != kMagic || h->total_bytes != total) {
+      munmap(map, (size_t)total);
+      delete t;
+      set_error_text("the shared tier is not initialised or does not match");
+      return KVX_EINVAL;
+    }
+  }
+  t->data = (uint8_t*)map + h->data_offset;
+  if (!(flags & KVX_TIER_NO_PIN)) {
+    const cudaError_t e = cudaHostRegister(t->data, (size_t)(h->slot_bytes * h->n_slots),
+                                           cudaHostRegisterPortable | cudaHostRegisterMapped);
+    if (e != cudaSuccess) {
+      kvx_status st = cuda_fail(e, "cudaHostRegister of the shared tier");
+      t->creator = create;
+      destroy_tier(t);
+      return st;
+    }
+    t->registered = true;
+  }
+  *out = t;
   return KVX_OK;
 }
 
 void kv_tier_destroy(kvx_tier* t) { destroy_tier(t); }
 
+kvx_status kv_tier_poll(kvx_tier* t) {
+  if (!t) return KVX_EINVAL;
+  TierLock lock(t);
+  poll_locked(t, false);
+  return KVX_OK;
+}
+
 kvx_status kv_tier_reserve(kvx_tier* t, uint64_t key, void** slot) {
   if (!t || !slot) return KVX_EINVAL;
-  std::lock_guard<std::mutex> lock(t->mu);
-  auto it = t->index.find(key);
-  int64_t i;
-  if (it != t->index.end()) {
-    i = it->second;
-    Slot& s = t->slots[i];
-    if (s.pins > 0 || !evictable(s)) return KVX_EBUSY;  // in use: cannot be rewritten now
+  TierLock lock(t);
+  poll_locked(t, false);
+  int64_t i = find_slot(t, key);
+  if (i >= 0) {
+    SlotMeta& m = t->meta[i];
+    if (m.pins > 0 || m.state != kReady) return KVX_EBUSY;  // in use: cannot be rewritten now
   } else {
     i = pick_slot(t);
     if (i < 0) {
-      set_error_text("every tier slot is pinned or still in use by the GPU");
+      set_error_text("every tier slot is pinned, being written, or still in use by the GPU");
       return KVX_ENOMEM;
     }
-    Slot& s = t->slots[i];
-    if (s.state != kFree) {
-      t->index.erase(s.key);
-      t->evictions++;
+    SlotMeta& m = t->meta[i];
+    if (m.state != kFree) {
+      if (!t->shared) t->index.erase(m.key);
+      t->hdr->evictions++;
     }
-    t->index[key] = i;
+    if (!t->shared) t->index[key] = i;
   }
-  Slot& s = t->slots[i];
-  s.key = key;
-  s.state = kWriting;
-  s.ready_recorded = false;
-  s.pins = 1;
-  s.tick = ++t->clock;
-  *slot = t->base + i * t->slot_bytes;
+  SlotMeta& m = t->meta[i];
+  m.key = key;
+  m.state = kWriting;
+  m.writer_pid = t->pid;
+  m.pins = 1;
+  m.tick = ++t->hdr->clock;
+  *slot = t->data + i * t->hdr->slot_bytes;
   return KVX_OK;
 }
 
 kvx_status kv_tier_commit(kvx_tier* t, uint64_t key, kvx_stream_t stream) {
   if (!t) return KVX_EINVAL;
-  std::lock_guard<std::mutex> lock(t->mu);
-  auto it = t->index.find(key);
-  if (it == t->index.end()) return KVX_ENOENT;
-  Slot& s = t->slots[it->second];
-  if (s.state != kWriting) return KVX_EINVAL;
-  if (!no_stream(stream)) {
-    kvx_status st = ensure_event(&s.ready);
-    if (st != KVX_OK) return st;
-    const cudaError_t e = cudaEventRecord(s.ready, (cudaStream_t)stream);
-    if (e != cudaSuccess) return cuda_fail(e, "cudaEventRecord (tier commit)");
-    s.ready_recorded = true;
+  TierLock lock(t);
+  poll_locked(t, false);
+  const int64_t i = find_slot(t, key);
+  if (i < 0) return KVX_ENOENT;
+  SlotMeta& m = t->meta[i];
+  if (m.state != kWriting || m.writer_pid != t->pid) return KVX_EINVAL;
+  if (no_stream(stream)) {
+    m.state = kReady;
+  } else {
+    cudaEvent_t e = take_event(t);
+    if (!e) return cuda_fail(cudaErrorMemoryAllocation, "cudaEventCreate (tier commit)");
+    const cudaError_t r = cudaEventRecord(e, (cudaStream_t)stream);
+    if (r != cudaSuccess) {
+      t->spare.push_back(e);
+      return cuda_fail(r, "cudaEventRecord (tier commit)");
+    }
+    m.state = kCommitting;
+    t->commits.push_back({i, e});
+    t->commit_event[i] = e;
   }
-  s.state = kReady;
-  s.pins = s.pins > 0 ? s.pins - 1 : 0;
-  s.tick = ++t->clock;
+  m.pins = m.pins > 0 ? m.pins - 1 : 0;
+  m.tick = ++t->hdr->clock;
   return KVX_OK;
 }
 
 kvx_status kv_tier_acquire(kvx_tier* t, uint64_t key, kvx_stream_t stream, void** slot) {
   if (!t || !slot) return KVX_EINVAL;
-  std::lock_guard<std::mutex> lock(t->mu);
-  auto it = t->index.find(key);
-  if (it == t->index.end() || t->slots[it->second].state != kReady) {
-    t->misses++;
+  TierLock lock(t);
+  poll_locked(t, false);
+  const int64_t i = find_slot(t, key);
+  bool ok = i >= 0 && t->meta[i].state == kReady;
+  cudaEvent_t wait_on = nullptr;
+  if (i >= 0 && t->meta[i].state == kCommitting && t->meta[i].writer_pid == t->pid) {
+    auto it = t->commit_event.find(i);  // written here: order the reader on the writer's event
+    if (it != t->commit_event.end()) {
+      wait_on = it->second;
+      ok = true;
+    }
+  }
+  if (!ok) {
+    t->hdr->misses++;
     return KVX_ENOENT;
   }
-  Slot& s = t->slots[it->second];
-  if (s.ready_recorded && !no_stream(stream)) {
-    const cudaError_t e = cudaStreamWaitEvent((cudaStream_t)stream, s.ready, 0);
-    if (e != cudaSuccess) return cuda_fail(e, "cudaStreamWaitEvent (tier acquire)");
+  if (wait_on) {
+    if (no_stream(stream)) {
+      const cudaError_t r = cudaEventSynchronize(wait_on);
+      if (r != cudaSuccess) return cuda_fail(r, "cudaEventSynchronize (tier acquire)");
+    } else {
+      const cudaError_t r = cudaStreamWaitEvent((cudaStream_t)stream, wait_on, 0);
+      if (r != cudaSuccess) return cuda_fail(r, "cudaStreamWaitEvent (tier acquire)");
+    }
   }
-  s.pins++;
-  s.tick = ++t->clock;
-  t->hits++;
-  *slot = t->base + it->second * t->slot_bytes;
+  SlotMeta& m = t->meta[i];
+  m.pins++;
+  m.tick = ++t->hdr->clock;
+  t->hdr->hits++;
+  *slot = t->data + i * t->hdr->slot_bytes;
   return KVX_OK;
 }
 
 kvx_status kv_tier_release(kvx_tier* t, uint64_t key, kvx_stream_t stream) {
   if (!t) return KVX_EINVAL;
-  std::lock_guard<std::mutex> lock(t->mu);
-  auto it = t->index.find(key);
-  if (it == t->index.end()) return KVX_ENOENT;
-  Slot& s = t->slots[it->second];
-  if (s.pins < 1) return KVX_EINVAL;
-  if (!no_stream(stream)) {
-    kvx_status st = ensure_event(&s.done);
-    if (st != KVX_OK) return st;
-    const cudaError_t e = cudaEventRecord(s.done, (cudaStream_t)stream);
-    if (e != cudaSuccess) return cuda_fail(e, "cudaEventRecord (tier release)");
-    s.done_recorded = true;
+  TierLock lock(t);
+  poll_locked(t, false);
+  const int64_t i = find_slot(t, key);
+  if (i < 0) return KVX_ENOENT;
+  SlotMeta& m = t->meta[i];
+  if (m.pins < 1) return KVX_EINVAL;
+  if (no_stream(stream)) {
+    m.pins--;
+    if (m.state == kWriting && m.pins == 0) m.state = kFree;  // a writer giving up its reservation
+    return KVX_OK;
   }
-  s.pins--;
+  cudaEvent_t e = take_event(t);
+  if (!e) return cuda_fail(cudaErrorMemoryAllocation, "cudaEventCreate (tier release)");
+  const cudaError_t r = cudaEventRecord(e, (cudaStream_t)stream);
+  if (r != cudaSuccess) {
+    t->spare.push_back(e);
+    return cuda_fail(r, "cudaEventRecord (tier release)");
+  }
+  t->releases.push_back({i, e});  // the pin stays until the queued work completes
   return KVX_OK;
 }
 
 kvx_status kv_tier_prefix_hits(kvx_tier* t, const uint64_t* keys, int64_t n, int64_t* hits) {
   if (!t || !hits || n < 0 || (n > 0 && !keys)) return KVX_EINVAL;
-  std::lock_guard<std::mutex> lock(t->mu);
+  TierLock lock(t);
+  poll_locked(t, false);
   int64_t h = 0;
   while (h < n) {
-    auto it = t->index.find(keys[h]);
-    if (it == t->index.end() || t->slots[it->second].state != kReady) break;
+    const int64_t i = find_slot(t, keys[h]);
+    if (i < 0) break;
+    const SlotMeta& m = t->meta[i];
+    const bool visible = m.state == kReady || (m.state == kCommitting && m.writer_pid == t->pid);
+    if (!visible) break;
     ++h;
   }
   *hits = h;
@@ -285,19 +542,20 @@ kvx_status kv_tier_prefix_hits(kvx_tier* t, const uint64_t* keys, int64_t n, int
 
 kvx_status kv_tier_stats(kvx_tier* t, kvx_tier_stats* out) {
   if (!t || !out) return KVX_EINVAL;
-  std::lock_guard<std::mutex> lock(t->mu);
-  out->slots = (int64_t)t->slots.size();
-  out->slot_bytes = t->slot_bytes;
+  TierLock lock(t);
+  poll_locked(t, false);
+  out->slots = t->hdr->n_slots;
+  out->slot_bytes = t->hdr->slot_bytes;
   int64_t used = 0, pinned = 0;
-  for (const Slot& s : t->slots) {
-    used += s.state != kFree;
-    pinned += s.pins > 0;
+  for (int64_t i = 0; i < t->hdr->n_slots; ++i) {
+    used += t->meta[i].state != kFree;
+    pinned += t->meta[i].pins > 0;
   }
   out->entries = used;
   out->pinned = pinned;
-  out->hits = t->hits;
-  out->misses = t->misses;
-  out->evictions = t->evictions;
+  out->hits = t->hdr->hits;
+  out->misses = t->hdr->misses;
+  out->evictions = t->hdr->evictions;
   return KVX_OK;
 }
 

@@ -38,8 +38,10 @@ EXPORTED = (
     "kv_host_alloc", "kv_host_free", "kv_pool_view_check",
     "kv_chunk_keys", "kv_tier_create", "kv_tier_create_on", "kv_tier_destroy", "kv_tier_reserve", "kv_tier_commit",
     "kv_tier_acquire", "kv_tier_release", "kv_tier_prefix_hits", "kv_tier_stats", "kv_fault_inject",
+    "kv_tier_open_shared", "kv_tier_poll",
 )
 KVX_ENOENT, KVX_EBUSY = -8, -9
+KVX_TIER_CREATE, KVX_TIER_NO_PIN = 0x1, 0x2
 KVX_NO_STREAM = -1  # the handle value of KVX_NO_STREAM
 
 
@@ -112,6 +114,8 @@ def _declare(lib):
         "kv_chunk_keys": (st, [P(i32), i64, i32, ctypes.c_uint64, P(ctypes.c_uint64), i64]),
         "kv_tier_create": (st, [i64, i64, P(vp)]),
         "kv_tier_create_on": (st, [vp, i64, i64, P(vp)]),
+        "kv_tier_open_shared": (st, [ctypes.c_char_p, i64, i64, ctypes.c_uint32, P(vp)]),
+        "kv_tier_poll": (st, [vp]),
         "kv_tier_destroy": (None, [vp]),
         "kv_tier_reserve": (st, [vp, ctypes.c_uint64, P(vp)]),
         "kv_tier_commit": (st, [vp, ctypes.c_uint64, vp]),
@@ -416,14 +420,26 @@ def kv_chunk_keys(tokens, chunk_tokens: int, salt: int = 0) -> list[int]:
 class KvTier:
     """The shared host tier (see kvxfer.h): fixed chunk slots in one pinned pool, LRU."""
 
-    def __init__(self, slot_bytes: int, n_slots: int, base: int | None = None):
+    def __init__(self, slot_bytes: int = 0, n_slots: int = 0, base: int | None = None,
+                 shared_name: str | None = None, create: bool = False, pin: bool = True):
+        """Private tier over a new pinned pool (or over `base`), or, with shared_name, a tier
+        shared by the processes of this host (create it, or open an existing one)."""
         out = ctypes.c_void_p()
-        if base is None:
+        if shared_name is not None:
+            flags = (KVX_TIER_CREATE if create else 0) | (0 if pin else KVX_TIER_NO_PIN)
+            _check(_lib.kv_tier_open_shared(shared_name.encode(), slot_bytes, n_slots, flags, ctypes.byref(out)),
+                   "kv_tier_open_shared")
+        elif base is None:
             _check(_lib.kv_tier_create(slot_bytes, n_slots, ctypes.byref(out)), "kv_tier_create")
         else:
             _check(_lib.kv_tier_create_on(base, slot_bytes, n_slots, ctypes.byref(out)), "kv_tier_create_on")
         self.handle = out.value
+        if not slot_bytes:
+            slot_bytes = self.stats()["slot_bytes"]
         self.slot_bytes = slot_bytes
+
+    def poll(self):
+        _check(_lib.kv_tier_poll(self.handle), "kv_tier_poll")
 
     def close(self):
         if self.handle:

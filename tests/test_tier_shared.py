@@ -1,0 +1,177 @@
+"""A host tier shared by two processes (paper Fig. 1: each replica is its own
+process; both use one pinned RAM pool).
+
+CPU test: the bookkeeping only (KVX_TIER_NO_PIN): entries written and
+committed by one process are found, read and pinned by the other; LRU and
+pinning hold across processes.
+
+GPU test: process A stores chunks of a pool into the shared pool on its
+stream, behind a ~10^8-cycle delayed producer; process B must not see them
+before A has observed its GPU work complete, then restores them into its own
+pool on the same GPU and checks every byte against the oracle.  The
+processes synchronise on the host only (no kernel waits on another process).
+"""
+import multiprocessing as mp
+import os
+import sys
+
+import numpy as np
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _name(tag):
+    return f"/kvx_{tag}_{os.getpid()}"
+
+
+def _child_cpu(name, q_in, q_out):
+    sys.path.insert(0, ROOT)
+    from paper_2609_15021_gb300 import kvxfer as k
+    NO = -1
+    t = k.KvTier(shared_name=name, pin=False)
+    assert q_in.get() == "written"
+    assert t.prefix_hits([1, 2, 3]) == 2
+    s = t.acquire(1, NO)
+    q_out.put(int(s[0]))                 # the byte the other process wrote
+    s2 = t.reserve(7)                    # write an entry of our own
+    s2.fill_(77)
+    t.commit(7, NO)
+    q_out.put("pinned 1, wrote 7")
+    assert q_in.get() == "check"
+    q_out.put(t.prefix_hits([1, 7]))
+    t.release(1, NO)
+    q_out.put("released")
+    assert q_in.get() == "bye"
+    t.close()
+
+
+def test_shared_tier_bookkeeping_across_processes():
+    sys.path.insert(0, ROOT)
+    from paper_2609_15021_gb300 import _build
+    _build.build()
+    from paper_2609_15021_gb300 import kvxfer as k
+    NO = -1
+    name = _name("cpu")
+    t = k.KvTier(64, 3, shared_name=name, create=True, pin=False)
+    ctx = mp.get_context("spawn")
+    q_in, q_out = ctx.Queue(), ctx.Queue()
+    p = ctx.Process(target=_child_cpu, args=(name, q_in, q_out))
+    p.start()
+    try:
+        for key in (1, 2):
+            s = t.reserve(key)
+            s.fill_(10 + key)
+            t.commit(key, NO)
+        q_in.put("written")
+        assert q_out.get(timeout=60) == 11
+        assert q_out.get(timeout=60) == "pinned 1, wrote 7"
+        assert t.prefix_hits([7]) == 1
+        assert int(t.acquire(7, NO)[3]) == 77
+        t.release(7, NO)
+        # 3 slots: 1 (pinned by the child), 2, 7; a new key may evict 2 or 7, never 1
+        t.reserve(8)
+        t.commit(8, NO)
+        t.reserve(9)
+        t.commit(9, NO)
+        q_in.put("check")
+        assert q_out.get(timeout=60) == 1      # child still sees 1; 7 was evicted (least recent)
+        assert q_out.get(timeout=60) == "released"
+        st = t.stats()
+        assert st["entries"] == 3 and st["evictions"] == 2
+        assert t.prefix_hits([1]) == 1
+        q_in.put("bye")
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    finally:
+        if p.is_alive():
+            p.kill()
+        t.close()
+
+
+def _child_gpu(name, q_in, q_out):
+    sys.path.insert(0, ROOT)
+    sys.path.insert(0, os.path.join(ROOT, "tests"))
+    import torch
+
+    import oracle
+    from gpu_util import POISON, device_pool, first_mismatch, host_layers, np_of, oracle_load, oracle_store
+    from paper_2609_15021_gb300 import kvxfer as k
+    from paper_2609_15021_gb300 import synth
+    spec = oracle.PoolSpec(4, 64, 16, 8, 128, 2, oracle.HND)
+    C, n_used = 256, 32
+    t = k.KvTier(shared_name=name)
+    keys = q_in.get()
+    q_out.put(t.prefix_hits(keys))                 # A's GPU work is still delayed: nothing visible
+    assert q_in.get() == "committed"
+    q_out.put(t.prefix_hits(keys))
+    final_np = host_layers(spec, 2)
+    ta = synth.permuted_table(64, n_used, 3)
+    tb = synth.permuted_table(64, n_used, 4)
+    dst = device_pool(spec)
+    ctx = k.kv_ctx_create(0)
+    s = torch.cuda.Stream()
+    tb_d = torch.from_numpy(tb).cuda()
+    for c, key in enumerate(keys):
+        slot = t.acquire(key, stream=s)
+        k.kv_load(ctx, dst, tb_d, c * C, (c + 1) * C, C, [slot], stream=s)
+        t.release(key, stream=s)
+    s.synchronize()
+    orc = oracle.c_oracle()
+    want, _ = oracle_store(orc, spec, final_np, ta, 0, n_used * 16, C)
+    loaded, _ = oracle_load(orc, spec, [np.full(spec.layer_bytes, POISON, np.uint8)] * 4, tb, 0, n_used * 16, C, want)
+    ok = all(first_mismatch(np_of(dst.layers[l]), loaded[l]) is None for l in range(4))
+    k.kv_ctx_destroy(ctx)
+    t.close()
+    q_out.put(ok)
+
+
+@pytest.mark.gpu
+def test_shared_tier_store_in_one_process_restore_in_another():
+    sys.path.insert(0, ROOT)
+    sys.path.insert(0, os.path.join(ROOT, "tests"))
+    import torch
+
+    import oracle
+    from gpu_util import device_pool, host_layers
+    from paper_2609_15021_gb300 import kvxfer as k
+    from paper_2609_15021_gb300 import synth
+    spec = oracle.PoolSpec(4, 64, 16, 8, 128, 2, oracle.HND)
+    C, n_used = 256, 32
+    T = n_used * 16
+    orc = oracle.c_oracle()
+    name = _name("gpu")
+    tier = k.KvTier(orc.chunk_bytes(spec, C), 4, shared_name=name, create=True)
+    ctx_mp = mp.get_context("spawn")
+    q_in, q_out = ctx_mp.Queue(), ctx_mp.Queue()
+    p = ctx_mp.Process(target=_child_gpu, args=(name, q_in, q_out))
+    p.start()
+    ctx = k.kv_ctx_create(0)
+    try:
+        stale_np, final_np = host_layers(spec, 1), host_layers(spec, 2)
+        pool = device_pool(spec, stale_np)
+        final_dev = [torch.from_numpy(a).cuda() for a in final_np]
+        ta_d = torch.from_numpy(synth.permuted_table(64, n_used, 3)).cuda()
+        keys = k.kv_chunk_keys(synth.rng(11).integers(0, 150000, size=T).astype(np.int32), C, salt=1)
+        s = torch.cuda.Stream()
+        torch.cuda.synchronize()
+        for l in range(4):   # the producer finishes writing the KV ~10^8 cycles later
+            k.kvx_probe_delayed_copy(pool.layers[l], final_dev[l], spec.layer_bytes, 10 ** 8 if l == 0 else 0, s)
+        for c, key in enumerate(keys):
+            slot = tier.reserve(key)
+            k.kv_store(ctx, pool, ta_d, c * C, (c + 1) * C, C, [slot], stream=s)
+            tier.commit(key, stream=s)
+        q_in.put(keys)
+        assert q_out.get(timeout=120) == 0      # still in flight on our stream: invisible elsewhere
+        s.synchronize()
+        tier.poll()                             # we observed completion: entries become READY
+        q_in.put("committed")
+        assert q_out.get(timeout=120) == len(keys)
+        assert q_out.get(timeout=300) is True   # the other process restored every byte
+        p.join(timeout=120)
+        assert p.exitcode == 0
+    finally:
+        if p.is_alive():
+            p.kill()
+        k.kv_ctx_destroy(ctx)
+        tier.close()
