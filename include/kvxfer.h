@@ -31,6 +31,13 @@
  * Threading: a kvx_ctx may be shared by host threads (calls are serialised
  * inside).  Calls are asynchronous with respect to the host.
  *
+ * CUDA graphs: kv_store, kv_load, kv_pack and kv_unpack allocate nothing per
+ * call (the staging ring of KVX_MODE_STAGED is made by kv_ctx_create) and
+ * order their side-stream work with an event on `stream` and a join back to
+ * it, so they may be captured from a capturing `stream` and replayed (the
+ * buffers and ranges of the capture are replayed).  While `stream` is
+ * capturing, its device is not checked (the query would end the capture).
+ *
  * Error behaviour: argument errors return before anything is enqueued and
  * leave every buffer untouched.  A block-table entry outside [0, num_blocks)
  * is found on the device: it names no page, so a store writes zero bytes for

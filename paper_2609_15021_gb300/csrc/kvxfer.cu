@@ -191,6 +191,14 @@ kvx_status check_pinned_range(const void* p, int64_t bytes, uint8_t** mapped) {
 
 kvx_status check_stream_device(cudaStream_t s, int device) {
   if (s == nullptr || s == cudaStreamLegacy || s == cudaStreamPerThread) return KVX_OK;
+  // cudaStreamGetDevice is not permitted on a capturing stream (it would
+  // invalidate the capture): a stream being captured into a graph is taken as is.
+  cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(s, &cap) != cudaSuccess) {
+    cudaGetLastError();
+    return KVX_EINVAL;
+  }
+  if (cap != cudaStreamCaptureStatusNone) return KVX_OK;
   int d = -1;
   if (cudaStreamGetDevice(s, &d) != cudaSuccess) {
     cudaGetLastError();

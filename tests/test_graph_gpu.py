@@ -1,0 +1,59 @@
+"""kv_store + kv_load captured into a CUDA graph and replayed.
+
+The calls order their side-stream work with an event on the caller's stream
+and a join back to it, which stream capture turns into graph edges; the
+zero-copy mode allocates nothing per call.  A captured store/restore is
+replayed twice with new KV written between the replays and each replay is
+checked against the oracle.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from gpu_util import POISON, device_pool, first_mismatch, host_layers, kvx, np_of, oracle_load, oracle_store, pinned_chunks
+from paper_2609_15021_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+
+def test_store_restore_replayed_from_a_cuda_graph(orc):
+    k = kvx()
+    spec = oracle.PoolSpec(4, 64, 16, 8, 128, 2, oracle.HND)
+    C, n_used = 256, 40
+    T = n_used * 16 - 7
+    src = device_pool(spec, host_layers(spec, 1))
+    dst = device_pool(spec)
+    ta = synth.permuted_table(64, n_used, 2)
+    tb = synth.permuted_table(64, n_used, 3)
+    ta_d, tb_d = torch.from_numpy(ta).cuda(), torch.from_numpy(tb).cuda()
+    host = pinned_chunks(orc, spec, 0, T, C)
+    ctx = k.kv_ctx_create(0)
+    try:
+        s = torch.cuda.Stream()
+        with torch.cuda.stream(s):  # warm up outside the capture
+            k.kv_store(ctx, src, ta_d, 0, T, C, host)
+            k.kv_load(ctx, dst, tb_d, 0, T, C, host)
+        s.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=s, capture_error_mode="thread_local"):
+            k.kv_store(ctx, src, ta_d, 0, T, C, host)
+            k.kv_load(ctx, dst, tb_d, 0, T, C, host)
+        for seed in (10, 11):
+            new = host_layers(spec, seed)
+            for l, a in enumerate(new):
+                src.layers[l].copy_(torch.from_numpy(a))
+            for t in dst.layers:
+                t.fill_(POISON)
+            torch.cuda.synchronize()
+            g.replay()
+            torch.cuda.synchronize()
+            want, _ = oracle_store(orc, spec, new, ta, 0, T, C)
+            for h, w in zip(host, want):
+                assert first_mismatch(np_of(h), w) is None, seed
+            loaded, _ = oracle_load(orc, spec, [np.full(spec.layer_bytes, POISON, np.uint8)] * 4, tb, 0, T, C, want)
+            for l in range(4):
+                assert first_mismatch(np_of(dst.layers[l]), loaded[l]) is None, (seed, l)
+        assert k.kv_get_device_error(ctx) == -1
+    finally:
+        k.kv_ctx_destroy(ctx)
