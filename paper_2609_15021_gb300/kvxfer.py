@@ -313,13 +313,17 @@ def kv_host_free(ptr: int) -> None:
 
 
 class HostBuffer:
-    """A kv_host_alloc allocation with a uint8 CPU tensor view (``.tensor``) over it."""
+    """A kv_host_alloc allocation with a uint8 CPU tensor view (``.tensor``) over it.
+
+    Views of ``.tensor`` keep the allocation alive; ``close()`` frees it at once
+    and must only be called when no view is used any more."""
 
     def __init__(self, nbytes: int):
         import torch
         self.nbytes = nbytes
         self.ptr = kv_host_alloc(nbytes)
         raw = (ctypes.c_uint8 * nbytes).from_address(self.ptr)
+        raw._owner = self  # the tensor holds `raw`, `raw` holds this buffer
         self.tensor = torch.frombuffer(raw, dtype=torch.uint8, count=nbytes)
 
     def close(self):
@@ -455,6 +459,7 @@ class KvTier:
     def _slot_tensor(self, ptr: int):
         import torch
         raw = (ctypes.c_uint8 * self.slot_bytes).from_address(ptr)
+        raw._owner = self  # a slot view keeps the tier (and its pool) alive
         return torch.frombuffer(raw, dtype=torch.uint8, count=self.slot_bytes)
 
     @staticmethod
