@@ -74,8 +74,8 @@ def load_peaks():
         return FALLBACK_HBM_GBS, "fallback (6.8 TB/s, no MEASURED_PEAKS.json)"
 
 
-def kernel_source_hash():
-    p = os.path.join(ROOT, "paper_2609_15021_gb300", "csrc", "pack_kernels.cu")
+def kernel_source_hash(source="pack_kernels.cu"):
+    p = os.path.join(ROOT, "paper_2609_15021_gb300", "csrc", source)
     with open(p, "rb") as f:
         return hashlib.sha256(f.read()).hexdigest()[:16]
 
@@ -99,10 +99,11 @@ class Traffic:
         return traffic * alg_bytes / captured_alg
 
 
-def recorded_traffic(shape):
-    """Traffic record from profiles/ for this kernel source and KV shape, else None."""
+def recorded_traffic(shape, source="pack_kernels.cu"):
+    """Traffic record from profiles/ for this kernel source file (as it is now)
+    and KV shape; a record with no entries if none matches."""
     pdir = os.path.join(ROOT, "profiles")
-    want = kernel_source_hash()
+    want = kernel_source_hash(source)
     if not os.path.isdir(pdir):
         return None
     for name in sorted(os.listdir(pdir)):
@@ -113,7 +114,8 @@ def recorded_traffic(shape):
                 m = re.match(r"\s*bench-traffic:\s*(\{.*\})\s*$", line)
                 if m:
                     d = json.loads(m.group(1))
-                    if d.get("kernel_sha256") == want and d.get("shape") == shape_key(shape):
+                    if (d.get("kernel_sha256") == want and d.get("source", "pack_kernels.cu") == source
+                            and d.get("shape") == shape_key(shape)):
                         return Traffic(d)
     return Traffic(None)
 
@@ -183,7 +185,7 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-hbm-roofline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--device-engine", choices=["lsu", "tma"], default="lsu",
+    ap.add_argument("--device-engine", choices=["lsu", "tma"], default="tma",
                     help="kernel of the device-side (HBM) pack/unpack leg")
     return ap.parse_args()
 
@@ -459,7 +461,7 @@ def run_ours(args):
         dev_slab = torch.empty(n_chunks * cb, dtype=torch.uint8, device=dev)
         dchunks = [dev_slab[i * cb:(i + 1) * cb] for i in range(n_chunks)]
         tma = args.device_engine == "tma"
-        hctx = k.kv_ctx_create(local, flags=k.KVX_FLAG_TIME_KERNELS | (k.KVX_FLAG_DEVICE_TMA if tma else 0))
+        hctx = k.kv_ctx_create(local, flags=k.KVX_FLAG_TIME_KERNELS | (0 if tma else k.KVX_FLAG_DEVICE_LSU))
         for _ in range(2):
             k.kv_pack(hctx, src, ta, 0, T, C, dchunks, stream=stream)
             k.kv_unpack(hctx, dst, tb, 0, T, C, dchunks, stream=stream)
@@ -472,17 +474,20 @@ def run_ours(args):
         hs = k.kv_ctx_stats(hctx)
         assert k.kv_get_device_error(hctx) == -1
         k.kv_ctx_destroy(hctx)
+        dev_traffic = recorded_traffic(s, "tma_kernels.cu") if tma else traffic
         hbm_roofline = {"bound": "hbm", "peak": hbm_peak, "unit": "GB/s", "peak_source": peak_src,
-                        "engine": "tma bulk copies (tma_move_kernel)" if tma else "16-byte loads/stores (move_kernel)"}
+                        "engine": "TMA tensor-map boxes (tmap_move_kernel)" if tma else
+                                  "16-byte loads/stores (move_kernel)"}
         for d, name in ((0, "pack"), (1, "unpack")):
             nl = hs["timed_launches"][d]
             per_launch = hs["kernel_bytes"][d] / nl
             achieved = per_launch / (hs["kernel_ms"][d] / nl * 1e-3) / GB
-            hbm_roofline[name] = {"kernel": f"move_kernel<{name},HND> (device chunks)", "achieved": achieved,
+            kname = f"tmap_move_kernel<{name}>" if tma else f"move_kernel<{name},HND>"
+            hbm_roofline[name] = {"kernel": f"{kname} (device chunks)", "achieved": achieved,
                                   "frac": achieved / hbm_peak, "launches": nl,
                                   "algorithmic_bytes_per_launch": per_launch,
                                   "avg_launch_ms": hs["kernel_ms"][d] / nl,
-                                  "traffic": traffic.get(f"device_{name}", per_launch)}
+                                  "traffic": dev_traffic.get(f"device_{name}", per_launch)}
         del dev_slab, dchunks
 
     store_gbs = X / (statistics.median(store_ms) * 1e-3) / GB

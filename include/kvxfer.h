@@ -98,12 +98,14 @@ typedef enum {
                                       the caller's stream, reproducing the
                                       paper's missing dependency (Sec. 3.2).
                                       Results are then undefined.             */
-#define KVX_FLAG_DEVICE_TMA 0x4u   /* device-side moves (kv_pack, kv_unpack,
-                                      staged mode) use TMA bulk copies staged
-                                      through shared memory instead of 16-byte
-                                      loads/stores (same bytes); pages of more
-                                      than 48 KiB per K or V half keep the
-                                      load/store kernel                       */
+/* Device-side moves (kv_pack, kv_unpack, staged mode) use, by default, the
+   TMA tensor-map kernel for HND pools whose K or V page half is at most
+   48 KiB (one TMA box per page half, staged through shared memory: the same
+   HBM throughput as the load/store kernel with two warps per SM), and the
+   16-byte load/store kernel otherwise.  The flags below force one of them.  */
+#define KVX_FLAG_DEVICE_TMA 0x4u   /* TMA everywhere it fits, with one bulk
+                                      copy per row where no tensor map does  */
+#define KVX_FLAG_DEVICE_LSU 0x8u   /* the 16-byte load/store kernel always   */
 
 typedef struct {
   int32_t store_mode;         /* kvx_mode                                       */

@@ -86,6 +86,16 @@ cudaError_t launch_segments(const SegmentParams& p, int grid, cudaStream_t s);
 // *timeout (device int) if a bounded wait expires.
 cudaError_t launch_move_tma(int dir, int layout, const MoveParams& p, int grid, int stage_bytes, int stages,
                             int* timeout, cudaStream_t s);
+// Sets the TMA kernels' shared-memory limit for the current device (once per
+// context creation; never on the launch path).
+cudaError_t prepare_tma_kernels();
+// Tensor-map variant for HND pools: one TMA box per full page half.
+constexpr int kTensorMapBytes = 128;
+// Encodes one tensor map per layer of P (kTensorMapBytes each) into `out`;
+// false if the pool's shape cannot be described (the row-copy variant is used).
+bool encode_tensor_maps(const kvx_pool* P, int64_t row_bytes, void* out);
+cudaError_t launch_move_tmap(int dir, const MoveParams& p, const void* maps, int num_layers, int grid,
+                             int stage_bytes, int stages, int* timeout, cudaStream_t s);
 int move_ctas_per_sm(int dir, int layout);
 int segment_ctas_per_sm();
 

@@ -118,6 +118,11 @@ struct kvx_ctx {
   double timed_ms[2] = {0.0, 0.0};
   std::vector<TimedLaunch> pending;
   std::vector<cudaEvent_t> spare_events;
+  // tensor maps of the last HND pool moved by the tensor-map engine
+  std::vector<uint8_t> tmaps;
+  std::vector<const void*> tmap_bases;
+  int64_t tmap_shape[6] = {0, 0, 0, 0, 0, 0};
+  bool tmap_ok = false;
 };
 
 namespace {
@@ -274,33 +279,57 @@ cudaEvent_t take_timing_event(kvx_ctx* ctx) {
   return e;
 }
 
+// 64-byte aligned start of the context's tensor-map storage (CUtensorMap alignment).
+void* tensor_map_storage(kvx_ctx* ctx) {
+  uintptr_t p = (uintptr_t)ctx->tmaps.data();
+  return (void*)((p + 63) & ~(uintptr_t)63);
+}
+
+// Tensor maps of pool P (cached per pool in the context); null if P cannot be described.
+const void* tensor_maps_of(kvx_ctx* ctx, const kvx_pool* P, int64_t row) {
+  const int64_t shape[6] = {P->num_layers, P->num_blocks, P->block_tokens, P->num_heads, row, P->layout};
+  bool same = ctx->tmap_bases.size() == (size_t)P->num_layers && memcmp(shape, ctx->tmap_shape, sizeof(shape)) == 0;
+  for (int l = 0; same && l < P->num_layers; ++l) same = ctx->tmap_bases[l] == P->layer_base[l];
+  if (!same) {
+    ctx->tmaps.assign((size_t)P->num_layers * kTensorMapBytes + 64, 0);
+    ctx->tmap_ok = encode_tensor_maps(P, row, tensor_map_storage(ctx));
+    ctx->tmap_bases.assign(P->layer_base, P->layer_base + P->num_layers);
+    memcpy(ctx->tmap_shape, shape, sizeof(shape));
+  }
+  return ctx->tmap_ok ? tensor_map_storage(ctx) : nullptr;
+}
+
 // Launch one pack/unpack kernel with optional timing events around it.
 // over_link: the launch reads or writes mapped host memory, so the host link,
 // not HBM, bounds it and a fraction of the SMs saturates it.
-kvx_status launch_move_timed(kvx_ctx* ctx, int dir, int layout, const MoveParams& p, int64_t bytes,
-                             cudaStream_t s, bool over_link) {
-  // TMA bulk-copy variant: device-side chunks only, and a K or V half page
-  // (the largest unit) of at most 48 KiB so that 3-4 stages fit in shared memory
+kvx_status launch_move_timed(kvx_ctx* ctx, const kvx_pool* P, int dir, int layout, const MoveParams& p,
+                             int64_t bytes, cudaStream_t s, bool over_link) {
+  // TMA variants: device-side chunks only, and a K or V half page (the
+  // largest unit) of at most 48 KiB so that 2-3 stages fit in shared memory.
+  // Default: tensor maps where the pool can be described, else load/store.
   const int64_t unit_bytes = (int64_t)p.B * p.H * p.R;
-  const bool tma = !over_link && (ctx->opts.flags & KVX_FLAG_DEVICE_TMA) && unit_bytes <= (48 << 10);
-  int stage_bytes = 0, stages = 0;
-  int64_t grid, cap;
-  if (tma) {
-    stage_bytes = (int)((unit_bytes + 127) / 128 * 128);
-    stages = stage_bytes <= (32 << 10) ? 3 : 2;        // 2 CTAs of one warp per SM
-    const int per_sm = std::max(1, (int)((224 << 10) / ((int64_t)stage_bytes * stages + 1024)));
-    grid = p.total_units;
-    cap = (int64_t)ctx->num_sms * per_sm;
-  } else {
-    const int64_t warps_per_cta = kThreads / 32;
-    grid = (p.total_units + warps_per_cta - 1) / warps_per_cta;
-    cap = (int64_t)ctx->num_sms * ctx->move_occ[dir][layout];
-  }
+  const uint32_t f = ctx->opts.flags;
+  const bool fits = !over_link && unit_bytes <= (48 << 10) && !(f & KVX_FLAG_DEVICE_LSU);
+  const void* maps = fits && layout == KVX_LAYOUT_HND ? tensor_maps_of(ctx, P, p.R) : nullptr;
+  const bool tma = fits && (maps || (f & KVX_FLAG_DEVICE_TMA));
+  // Grid: HBM-bound launches give every unit its own warp (LSU) or CTA (TMA)
+  // and let the block scheduler spread them; measured on GB300 this keeps
+  // DRAM busier than a persistent grid walking the units in lockstep.
+  // Launches over the host link, or capped by the caller (max_ctas), are
+  // persistent: each warp or CTA strides over many units.
+  int64_t grid = tma ? p.total_units : (p.total_units + (kThreads / 32) - 1) / (kThreads / 32);
+  int64_t cap = grid;
   if (ctx->opts.max_ctas > 0)
-    cap = std::min<int64_t>(cap, ctx->opts.max_ctas);
+    cap = ctx->opts.max_ctas;
   else if (over_link)
-    cap = std::min<int64_t>(cap, ctx->link_ctas);
+    cap = std::min<int64_t>(ctx->link_ctas, (int64_t)ctx->num_sms * ctx->move_occ[dir][layout]);
   grid = std::max<int64_t>(1, std::min(grid, cap));
+  int stage_bytes = 0, stages = 0;
+  if (tma) {
+    // one stage when each CTA moves one unit; else a ring of 3 (2 above 32 KiB)
+    stage_bytes = (int)((unit_bytes + 127) / 128 * 128);
+    stages = grid >= p.total_units ? 1 : stage_bytes <= (32 << 10) ? 3 : 2;
+  }
   cudaEvent_t a = nullptr, b = nullptr;
   const bool timing = (ctx->opts.flags & KVX_FLAG_TIME_KERNELS) != 0;
   if (timing) {
@@ -310,7 +339,10 @@ kvx_status launch_move_timed(kvx_ctx* ctx, int dir, int layout, const MoveParams
       KVX_CUDA(cudaEventRecord(a, s));
     }
   }
-  if (tma)
+  if (maps)
+    KVX_CUDA_AT("launch", launch_move_tmap(dir, p, maps, P->num_layers, (int)grid, stage_bytes, stages,
+                                           ctx->d_timeout, s));
+  else if (tma)
     KVX_CUDA_AT("launch", launch_move_tma(dir, layout, p, (int)grid, stage_bytes, stages, ctx->d_timeout, s));
   else
     KVX_CUDA_AT("launch", launch_move(dir, layout, p, (int)grid, s));
@@ -407,7 +439,7 @@ kvx_status enqueue_direct(kvx_ctx* ctx, const Plan& pl) {
     add_job(&p, pl.side[i], (pl.first_chunk + i) * pl.bpc, pl.tokens[i], 0, pl.P->num_layers);
     bytes += chunk_bytes_of(pl.P, pl.g, pl.tokens[i]);
     if (p.n_jobs == kMaxJobs || i == pl.n - 1) {
-      kvx_status st = launch_move_timed(ctx, pl.dir, pl.P->layout, p, bytes, ctx->s_kern, pl.over_link);
+      kvx_status st = launch_move_timed(ctx, pl.P, pl.dir, pl.P->layout, p, bytes, ctx->s_kern, pl.over_link);
       if (st != KVX_OK) return st;
       p.n_jobs = 0;
       p.total_units = 0;
@@ -468,7 +500,7 @@ kvx_status enqueue_staged(kvx_ctx* ctx, const Plan& pl) {
     kvx_status st;
     if (pl.dir == kPack) {
       KVX_CUDA(cudaStreamWaitEvent(ctx->s_kern, ctx->ev_free[k], 0));
-      st = launch_move_timed(ctx, kPack, P->layout, p, bytes, ctx->s_kern, false);
+      st = launch_move_timed(ctx, P, kPack, P->layout, p, bytes, ctx->s_kern, false);
       if (st != KVX_OK) return st;
       KVX_CUDA(cudaEventRecord(ctx->ev_ready[k], ctx->s_kern));
       KVX_CUDA(cudaStreamWaitEvent(ctx->s_copy, ctx->ev_ready[k], 0));
@@ -481,7 +513,7 @@ kvx_status enqueue_staged(kvx_ctx* ctx, const Plan& pl) {
       if (st != KVX_OK) return st;
       KVX_CUDA(cudaEventRecord(ctx->ev_ready[k], ctx->s_copy));
       KVX_CUDA(cudaStreamWaitEvent(ctx->s_kern, ctx->ev_ready[k], 0));
-      st = launch_move_timed(ctx, kUnpack, P->layout, p, bytes, ctx->s_kern, false);
+      st = launch_move_timed(ctx, P, kUnpack, P->layout, p, bytes, ctx->s_kern, false);
       if (st != KVX_OK) return st;
       KVX_CUDA(cudaEventRecord(ctx->ev_free[k], ctx->s_kern));
     }
@@ -834,6 +866,7 @@ kvx_status kv_ctx_create(int device, const kvx_opts* opts, kvx_ctx** out) {
   for (int d = 0; d < 2; ++d)
     for (int l = 0; l < 2; ++l) ctx->move_occ[d][l] = move_ctas_per_sm(d, l);
   ctx->seg_occ = segment_ctas_per_sm();
+  if ((e = prepare_tma_kernels()) != cudaSuccess) return fail(e);
   if (ctx->store_mode == KVX_MODE_STAGED || ctx->load_mode == KVX_MODE_STAGED) {
     kvx_status st = ensure_staging(ctx);
     if (st != KVX_OK) {

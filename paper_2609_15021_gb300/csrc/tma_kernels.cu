@@ -1,20 +1,32 @@
 // tma_kernels.cu -- device-side pack / unpack with the Tensor Memory
-// Accelerator's bulk copies (cp.async.bulk) staged through shared memory.
+// Accelerator (TMA), staged through shared memory.
 //
 // Same work units and byte mapping as move_kernel (pack_kernels.cu): one
 // (chunk, layer, page, K|V) unit at a time, here per CTA of one warp.  A unit
-// is copied global -> shared by bulk copies that complete on an mbarrier, then
-// shared -> global by bulk copies tracked as bulk groups.  The page side
-// moves one 256-byte (row-sized) bulk copy per (head, token) row, landing in
-// or leaving from shared memory in the chunk's [token][head] order; the chunk
-// side moves as one contiguous bulk copy.  A ring of kStages shared-memory
-// stages keeps the loads of the next units in flight while the current unit
-// is stored.  Registers never hold the data.
+// is copied global -> shared with completion on an mbarrier, then shared ->
+// global tracked as a bulk group; registers never hold the data.  By default
+// every unit gets its own CTA with a single stage (six 32 KiB CTAs fit an SM,
+// and the block scheduler keeps DRAM busy as CTAs finish); a grid capped by
+// the caller strides each CTA over many units through a ring of stages, so
+// the loads of the next units overlap the store of the current one.
 //
-// Only for chunks in device memory (kv_pack / kv_unpack / staged mode): the
-// zero-copy path keeps the load/store kernel.  Every mbarrier wait is bounded
-// by a clock limit; on expiry the kernel sets a timeout flag, drains its own
-// bulk stores and returns instead of waiting forever.
+// Two ways to move the page side of an HND unit (its [head][token][row]
+// bytes, which the chunk holds in [token][head][row] order):
+//  * tensor maps (TMAP): each pool layer is described to the TMA unit as a
+//    5-D tensor (row bytes, head, token, K|V, page) whose head and token
+//    dimensions carry each other's strides, so one box copy of a whole page
+//    half lands in -- or leaves from -- shared memory already in chunk order;
+//  * row copies: one 1-D bulk copy per (head, token) row.
+// The chunk side is always one contiguous bulk copy.  Units that cover only
+// part of a page (the end of a range) use row copies, so no byte past the
+// range is read into a chunk or written to a page.
+//
+// Only for chunks in device memory (kv_pack / kv_unpack / staged mode).  Every
+// mbarrier wait is bounded by a clock limit; on expiry the kernel sets a
+// timeout flag, drains its own bulk stores and returns.
+
+#include <cuda.h>
+#include <string.h>
 
 #include "kvx_internal.h"
 
@@ -23,6 +35,11 @@ namespace {
 
 constexpr int kStagesMax = 4;
 constexpr long long kWaitCycles = 4000000000ll;  // about 2 s at the maximum SM clock
+
+struct TensorMaps {
+  CUtensorMap m[KVX_MAX_LAYERS];
+};
+static_assert(sizeof(CUtensorMap) == kTensorMapBytes, "tensor map size");
 
 __device__ __forceinline__ uint32_t smem_addr(const void* p) {
   return (uint32_t)__cvta_generic_to_shared(p);
@@ -62,7 +79,22 @@ __device__ __forceinline__ void bulk_store(void* gdst, const void* ssrc, uint32_
                "r"(bytes)
                : "memory");
 }
+// One box of a 5-D tensor map at (0, 0, 0, kv, page): a whole K or V page half.
+__device__ __forceinline__ void box_load(void* sdst, const CUtensorMap* map, int kv, int page, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.5d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4, %5, "
+      "%6}], [%7];" ::"r"(smem_addr(sdst)),
+      "l"(map), "r"(0), "r"(0), "r"(0), "r"(kv), "r"(page), "r"(smem_addr(bar))
+      : "memory");
+}
+__device__ __forceinline__ void box_store(const CUtensorMap* map, int kv, int page, const void* ssrc) {
+  asm volatile("cp.async.bulk.tensor.5d.global.shared::cta.tile.bulk_group [%0, {%1, %2, %3, %4, %5}], [%6];" ::"l"(
+                   map),
+               "r"(0), "r"(0), "r"(0), "r"(kv), "r"(page), "r"(smem_addr(ssrc))
+               : "memory");
+}
 __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read_0() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_read_1() { asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
@@ -72,13 +104,17 @@ struct Unit {
   uint8_t* ck;   // chunk side
   int nr;        // rows (tokens x heads)
   int move;      // 0: nothing to move (past a short chunk's end, or a bad page)
+  int full;      // the unit covers the whole page half (all B tokens)
+  int layer, kv;
+  int page;
 };
 
 // Same decode as move_kernel; a bad table entry zero-fills the chunk rows
-// (pack) with ordinary stores and reports the logical block.
+// (pack) with ordinary stores and reports the logical block.  lane < 0: a
+// second decode of the same unit (store side), which repeats no side effect.
 template <int DIR>
 __device__ __forceinline__ Unit decode(const MoveParams& p, int64_t u, int& j, int64_t& job_begin, int lane) {
-  Unit r{nullptr, nullptr, 0, 0};
+  Unit r{nullptr, nullptr, 0, 0, 0, 0, 0, 0};
   while (u >= p.jobs[j].unit_end) {
     job_begin = p.jobs[j].unit_end;
     ++j;
@@ -100,7 +136,6 @@ __device__ __forceinline__ Unit decode(const MoveParams& p, int64_t u, int& j, i
   r.ck = J.chunk + ((int64_t)(l - J.l0) * 2 + kv) * J.tokens * HR + (int64_t)tok0 * HR;
   r.nr = nb * p.H;
   if (entry < 0 || (int64_t)entry >= p.num_blocks / p.ppb) {
-    // lane < 0: a second decode of the same unit (store side), which must not repeat these writes
     if (lane == 0) atomicMin(p.err, (long long)lblk);
     if (DIR == kPack && lane >= 0) {
       const uint4 z = make_uint4(0, 0, 0, 0);
@@ -111,20 +146,26 @@ __device__ __forceinline__ Unit decode(const MoveParams& p, int64_t u, int& j, i
   }
   r.pg = p.layer_base[l] + page * p.page_bytes + kv * (p.page_bytes >> 1);
   r.move = 1;
+  r.full = nb == p.B;
+  r.layer = l;
+  r.kv = kv;
+  r.page = (int)page;
   return r;
 }
 
 // Issue the global -> shared copies of one unit into `stage`.
-template <int DIR, int LAYOUT>
-__device__ __forceinline__ void issue_loads(const MoveParams& p, const Unit& w, uint8_t* stage, uint64_t* bar,
-                                            int lane) {
-  const uint32_t bytes = w.move ? (uint32_t)(w.nr * p.R) : 0u;
+template <int DIR, int LAYOUT, bool TMAP>
+__device__ __forceinline__ void issue_loads(const MoveParams& p, const TensorMaps* maps, const Unit& w,
+                                            uint8_t* stage, uint64_t* bar, int lane) {
+  const uint32_t bytes = w.move ? (uint32_t)((TMAP && DIR == kPack && w.full ? p.B * p.H : w.nr) * p.R) : 0u;
   if (lane == 0) mbar_expect_tx(bar, bytes);
   __syncwarp();
   if (!w.move) return;
   if (DIR == kUnpack || LAYOUT == KVX_LAYOUT_NHD) {
     // chunk side (unpack) or an NHD page (pack): one contiguous run
     if (lane == 0) bulk_load(stage, DIR == kUnpack ? w.ck : w.pg, bytes, bar);
+  } else if (TMAP && w.full) {
+    if (lane == 0) box_load(stage, &maps->m[w.layer], w.kv, w.page, bar);
   } else {
     // HND page rows (h, s) land at the chunk's row r = s * H + h
     for (int r = lane; r < w.nr; r += 32) {
@@ -135,12 +176,15 @@ __device__ __forceinline__ void issue_loads(const MoveParams& p, const Unit& w, 
 }
 
 // Issue the shared -> global copies of one unit from `stage`.
-template <int DIR, int LAYOUT>
-__device__ __forceinline__ void issue_stores(const MoveParams& p, const Unit& w, const uint8_t* stage, int lane) {
+template <int DIR, int LAYOUT, bool TMAP>
+__device__ __forceinline__ void issue_stores(const MoveParams& p, const TensorMaps* maps, const Unit& w,
+                                             const uint8_t* stage, int lane) {
   if (w.move) {
     const uint32_t bytes = (uint32_t)(w.nr * p.R);
     if (DIR == kPack || LAYOUT == KVX_LAYOUT_NHD) {
       if (lane == 0) bulk_store(DIR == kPack ? w.ck : w.pg, stage, bytes);
+    } else if (TMAP && w.full) {
+      if (lane == 0) box_store(&maps->m[w.layer], w.kv, w.page, stage);
     } else {
       for (int r = lane; r < w.nr; r += 32) {
         const int s = r / p.H, h = r - s * p.H;
@@ -151,11 +195,13 @@ __device__ __forceinline__ void issue_stores(const MoveParams& p, const Unit& w,
   bulk_commit();
 }
 
-template <int DIR, int LAYOUT>
-__global__ void __launch_bounds__(32) tma_move_kernel(const __grid_constant__ MoveParams p, int stage_bytes,
-                                                      int stages, int* timeout) {
-  extern __shared__ __align__(128) uint8_t smem[];
+template <int DIR, int LAYOUT, bool TMAP>
+__device__ __forceinline__ void tma_move_body(const MoveParams& p, const TensorMaps* maps, int stage_bytes,
+                                              int stages, int* timeout) {
+  extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t bars[kStagesMax];
+  // 128-byte aligned stages (tensor copies need it)
+  uint8_t* smem = smem_raw + ((128 - (smem_addr(smem_raw) & 127)) & 127);
   const int lane = threadIdx.x;
   if (lane == 0) {
     for (int k = 0; k < stages; ++k) mbar_init(&bars[k], 1);
@@ -164,43 +210,140 @@ __global__ void __launch_bounds__(32) tma_move_kernel(const __grid_constant__ Mo
   __syncwarp();
   const int64_t first = blockIdx.x, step = gridDim.x;
   const int64_t n = p.total_units > first ? (p.total_units - first + step - 1) / step : 0;
-  // decode cursors: one for loads (runs ahead), one for stores
-  int jl = 0, js = 0;
+  int jl = 0, js = 0;  // decode cursors: loads run ahead of stores
   int64_t bl = 0, bs = 0;
-  const int64_t pro = n < stages - 1 ? n : stages - 1;
+  // Loads run `ahead` units ahead of stores: stages - 1 with a ring, and one
+  // with a single stage (the next unit's load then waits for the store to
+  // have read the stage).
+  const int ahead = stages > 1 ? stages - 1 : 1;
+  const int64_t pro = n < ahead ? n : ahead;
   for (int64_t it = 0; it < pro; ++it) {
     const Unit w = decode<DIR>(p, first + it * step, jl, bl, lane);
-    issue_loads<DIR, LAYOUT>(p, w, smem + it * stage_bytes, &bars[it], lane);
+    issue_loads<DIR, LAYOUT, TMAP>(p, maps, w, smem + it * stage_bytes, &bars[it], lane);
   }
   bool ok = true;
   for (int64_t it = 0; it < n && ok; ++it) {
     const int k = (int)(it % stages);
-    const Unit w = decode<DIR>(p, first + it * step, js, bs, -1);  // lane -1: no side effects
+    const Unit w = decode<DIR>(p, first + it * step, js, bs, -1);
     if (lane == 0) ok = mbar_wait(&bars[k], (uint32_t)((it / stages) & 1));
     ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
     if (!ok) break;
-    issue_stores<DIR, LAYOUT>(p, w, smem + (int64_t)k * stage_bytes, lane);
-    const int64_t nxt = it + stages - 1;
+    issue_stores<DIR, LAYOUT, TMAP>(p, maps, w, smem + (int64_t)k * stage_bytes, lane);
+    const int64_t nxt = it + ahead;
     if (nxt < n) {
-      bulk_wait_read_1();  // the store issued from this stage one turn ago has read it
+      // the store last issued from the next load's stage has read it: one turn
+      // ago with a ring, just now with a single stage
+      if (stages > 1)
+        bulk_wait_read_1();
+      else
+        bulk_wait_read_0();
       __syncwarp();
       const int kn = (int)(nxt % stages);
       const Unit wn = decode<DIR>(p, first + nxt * step, jl, bl, lane);
-      issue_loads<DIR, LAYOUT>(p, wn, smem + (int64_t)kn * stage_bytes, &bars[kn], lane);
+      issue_loads<DIR, LAYOUT, TMAP>(p, maps, wn, smem + (int64_t)kn * stage_bytes, &bars[kn], lane);
     }
   }
   if (!ok && lane == 0) atomicExch(timeout, 1);
   bulk_wait_all();
 }
 
+template <int DIR, int LAYOUT>
+__global__ void __launch_bounds__(32) tma_move_kernel(const __grid_constant__ MoveParams p, int stage_bytes,
+                                                      int stages, int* timeout) {
+  tma_move_body<DIR, LAYOUT, false>(p, nullptr, stage_bytes, stages, timeout);
+}
+
+template <int DIR>
+__global__ void __launch_bounds__(32) tmap_move_kernel(const __grid_constant__ MoveParams p,
+                                                       const __grid_constant__ TensorMaps maps, int stage_bytes,
+                                                       int stages, int* timeout) {
+  tma_move_body<DIR, KVX_LAYOUT_HND, true>(p, &maps, stage_bytes, stages, timeout);
+}
+
+// Largest dynamic shared memory a TMA launch uses: 96 KiB of stages (three of
+// at most 32 KiB or two of at most 48 KiB) plus 128 bytes of alignment slack.
+constexpr int kTmaSmemMax = (96 << 10) + 128;
+
+template <typename K>
+cudaError_t set_smem(K kernel) {
+  return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kTmaSmemMax);
+}
+
+using EncodeFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                              const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                              CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeFn encoder() {
+  static EncodeFn fn = [] {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) !=
+            cudaSuccess ||
+        q != cudaDriverEntryPointSuccess) {
+      cudaGetLastError();
+      f = nullptr;
+    }
+    return (EncodeFn)f;
+  }();
+  return fn;
+}
+
 }  // namespace
+
+bool encode_tensor_maps(const kvx_pool* P, int64_t row_bytes, void* out) {
+  if (P->layout != KVX_LAYOUT_HND) return false;
+  EncodeFn enc = encoder();
+  if (!enc) return false;
+  // element type: the widest of 1/2/4/8 bytes that keeps a row within a 256-element box dimension
+  int esz = 1;
+  while (esz < 8 && row_bytes / esz > 256) esz *= 2;
+  if (row_bytes % esz != 0 || row_bytes / esz > 256 || P->num_heads > 256 || P->block_tokens > 256) return false;
+  if (P->num_blocks > INT32_MAX) return false;
+  const CUtensorMapDataType type = esz == 1   ? CU_TENSOR_MAP_DATA_TYPE_UINT8
+                                   : esz == 2 ? CU_TENSOR_MAP_DATA_TYPE_UINT16
+                                   : esz == 4 ? CU_TENSOR_MAP_DATA_TYPE_UINT32
+                                              : CU_TENSOR_MAP_DATA_TYPE_INT64;
+  const cuuint64_t R = (cuuint64_t)row_bytes, H = P->num_heads, B = P->block_tokens;
+  // dimensions innermost first: row elements, head, token, K|V, page; head and
+  // token carry each other's strides, so a box lands in [token][head][row] order
+  const cuuint64_t dims[5] = {R / esz, H, B, 2, (cuuint64_t)P->num_blocks};
+  const cuuint64_t strides[4] = {B * R, R, H * B * R, 2 * H * B * R};
+  const cuuint32_t box[5] = {(cuuint32_t)(R / esz), (cuuint32_t)H, (cuuint32_t)B, 1, 1};
+  const cuuint32_t elem_strides[5] = {1, 1, 1, 1, 1};
+  CUtensorMap* maps = reinterpret_cast<CUtensorMap*>(out);
+  for (int l = 0; l < P->num_layers; ++l) {
+    if (enc(&maps[l], type, 5, P->layer_base[l], dims, strides, box, elem_strides, CU_TENSOR_MAP_INTERLEAVE_NONE,
+            CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return false;
+  }
+  return true;
+}
+
+// Raise the dynamic shared-memory limit of every TMA kernel once for the
+// current device, when a context is created, so that the launch path makes no
+// driver attribute calls.
+cudaError_t prepare_tma_kernels() {
+  cudaError_t e = cudaSuccess;
+  for (cudaError_t r : {set_smem(tma_move_kernel<kPack, KVX_LAYOUT_HND>), set_smem(tma_move_kernel<kPack, KVX_LAYOUT_NHD>),
+                        set_smem(tma_move_kernel<kUnpack, KVX_LAYOUT_HND>),
+                        set_smem(tma_move_kernel<kUnpack, KVX_LAYOUT_NHD>), set_smem(tmap_move_kernel<kPack>),
+                        set_smem(tmap_move_kernel<kUnpack>)})
+    if (r != cudaSuccess && e == cudaSuccess) e = r;
+  return e;
+}
+
+// Stage count and shared memory within what the kernels were prepared for.
+bool stages_ok(int stage_bytes, int stages) {
+  return stages >= 1 && stages <= kStagesMax && stage_bytes > 0 && stage_bytes % 128 == 0 &&
+         (int64_t)stage_bytes * stages + 128 <= kTmaSmemMax;
+}
 
 cudaError_t launch_move_tma(int dir, int layout, const MoveParams& p, int grid, int stage_bytes, int stages,
                             int* timeout, cudaStream_t s) {
-  const size_t smem = (size_t)stage_bytes * stages;
+  if (!stages_ok(stage_bytes, stages)) return cudaErrorInvalidValue;
+  const size_t smem = (size_t)stage_bytes * stages + 128;
   auto go = [&](auto kernel) {
-    cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
     kernel<<<grid, 32, smem, s>>>(p, stage_bytes, stages, timeout);
     return cudaGetLastError();
   };
@@ -209,6 +352,19 @@ cudaError_t launch_move_tma(int dir, int layout, const MoveParams& p, int grid, 
                                     : go(tma_move_kernel<kPack, KVX_LAYOUT_NHD>);
   return layout == KVX_LAYOUT_HND ? go(tma_move_kernel<kUnpack, KVX_LAYOUT_HND>)
                                   : go(tma_move_kernel<kUnpack, KVX_LAYOUT_NHD>);
+}
+
+cudaError_t launch_move_tmap(int dir, const MoveParams& p, const void* maps, int num_layers, int grid,
+                             int stage_bytes, int stages, int* timeout, cudaStream_t s) {
+  if (!stages_ok(stage_bytes, stages) || num_layers < 1 || num_layers > KVX_MAX_LAYERS) return cudaErrorInvalidValue;
+  TensorMaps m;
+  memcpy(m.m, maps, (size_t)num_layers * sizeof(CUtensorMap));
+  const size_t smem = (size_t)stage_bytes * stages + 128;
+  auto go = [&](auto kernel) {
+    kernel<<<grid, 32, smem, s>>>(p, m, stage_bytes, stages, timeout);
+    return cudaGetLastError();
+  };
+  return dir == kPack ? go(tmap_move_kernel<kPack>) : go(tmap_move_kernel<kUnpack>);
 }
 
 }  // namespace kvx

@@ -100,11 +100,11 @@ def ctxs():
     k = kvx()
     made = {}
 
-    def get(mode, unordered=False):
-        key = (mode, unordered)
+    def get(mode, unordered=False, lsu=False):
+        key = (mode, unordered, lsu)
         if key not in made:
-            made[key] = k.kv_ctx_create(0, store_mode=mode, load_mode=mode,
-                                        flags=k.KVX_FLAG_UNORDERED if unordered else 0)
+            flags = (k.KVX_FLAG_UNORDERED if unordered else 0) | (k.KVX_FLAG_DEVICE_LSU if lsu else 0)
+            made[key] = k.kv_ctx_create(0, store_mode=mode, load_mode=mode, flags=flags)
         return made[key]
 
     yield get
@@ -112,8 +112,14 @@ def ctxs():
         k.kv_ctx_destroy(c)
 
 
-VARIANTS = [("staged", 1, False), ("zerocopy", 2, False), ("staged_unordered", 1, True),
-            ("zerocopy_unordered", 2, True)]
+# (name, mode, unordered, force the load/store device engine).  The staged
+# negative control packs with the load/store engine: the TMA engine's kernels
+# ask for ~96 KiB of shared memory per CTA, and an SM whose shared-memory
+# carveout was configured for the (shared-memory-free) spinning producer cannot
+# take them until the producer leaves it, which hides the missing dependency
+# behind a hardware reconfiguration rather than exposing it.
+VARIANTS = [("staged", 1, False, False), ("staged_lsu", 1, False, True), ("zerocopy", 2, False, False),
+            ("staged_unordered", 1, True, True), ("zerocopy_unordered", 2, True, False)]
 
 
 @pytest.mark.parametrize("n_bytes", SIZES)
@@ -127,8 +133,8 @@ def test_store_after_delayed_producer(orc, ctxs, n_bytes):
     assert want_final[0].size == n_bytes
     final_dev = torch.from_numpy(final_np[0]).cuda()
     table_d = torch.from_numpy(table).cuda()
-    for name, mode, unordered in VARIANTS:
-        ctx = ctxs(mode, unordered)
+    for name, mode, unordered, lsu in VARIANTS:
+        ctx = ctxs(mode, unordered, lsu)
         for delay in (0, DELAY):
             for trial in range(TRIALS):
                 pool = device_pool(spec, stale_np)
@@ -157,8 +163,8 @@ def test_load_after_delayed_consumer(orc, ctxs, n_bytes):
     loaded, _ = oracle_load(orc, spec, old_np, table, 0, C, C, chunk_new)
     host = [torch.from_numpy(chunk_new[0]).pin_memory()]
     table_d = torch.from_numpy(table).cuda()
-    for name, mode, unordered in VARIANTS:
-        ctx = ctxs(mode, unordered)
+    for name, mode, unordered, lsu in VARIANTS:
+        ctx = ctxs(mode, unordered, lsu)
         for delay in (0, DELAY):
             for trial in range(TRIALS):
                 pool = device_pool(spec, old_np)

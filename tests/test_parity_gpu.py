@@ -56,11 +56,11 @@ def ctxs():
     k = kvx()
     made = {}
 
-    def get(mode, slot_bytes=0, flags=0):
-        key = (mode, slot_bytes, flags)
+    def get(mode, slot_bytes=0, flags=0, max_ctas=0):
+        key = (mode, slot_bytes, flags, max_ctas)
         if key not in made:
             made[key] = k.kv_ctx_create(0, store_mode=mode, load_mode=mode, staging_slot_bytes=slot_bytes,
-                                        flags=flags)
+                                        flags=flags, max_ctas=max_ctas)
         return made[key]
 
     yield get
@@ -126,7 +126,15 @@ def test_staged_one_layer_per_slot(orc, ctxs, name):
     _run_case(orc, ctxs(1, slot), case, torch.cuda.Stream())
 
 
-@pytest.mark.parametrize("engine", ["lsu", "tma"])
+# Engines of the device-side launches: by default one warp (LSU) or CTA (TMA)
+# per unit; "_capped" grids of 7 CTAs make every warp or CTA stride over many
+# units (the TMA kernel then runs its ring of shared-memory stages).
+ENGINES = {"lsu": ("KVX_FLAG_DEVICE_LSU", 0), "default": (None, 0), "tma": ("KVX_FLAG_DEVICE_TMA", 0),
+           "lsu_capped": ("KVX_FLAG_DEVICE_LSU", 7), "default_capped": (None, 7),
+           "tma_capped": ("KVX_FLAG_DEVICE_TMA", 7)}
+
+
+@pytest.mark.parametrize("engine", list(ENGINES))
 @pytest.mark.parametrize("name", ["tiny_cfg_hnd", "ragged_tail_nhd", "rows_48B_generic", "many_chunks_three_launches",
                                   "27b_shape_two_chunks", "paper_logical_blocks_49", "logical_blocks_4_nhd_ragged",
                                   "rows_16B_16_heads", "one_token"])
@@ -142,7 +150,8 @@ def test_device_pack_unpack_parity(orc, ctxs, name, engine):
     tb = synth.permuted_table(N // ppb, n_used, seed=22)
     extra = 32
     dev = device_chunks(orc, spec, t0, t1, C, extra=extra)
-    ctx = ctxs(1, 0, k.KVX_FLAG_DEVICE_TMA if engine == "tma" else 0)
+    flag, max_ctas = ENGINES[engine]
+    ctx = ctxs(1, 0, getattr(k, flag) if flag else 0, max_ctas)
     k.kv_pack(ctx, src, torch.from_numpy(ta).cuda(), t0, t1, C, dev)
     torch.cuda.synchronize()
     assert k.kv_get_device_error(ctx) == -1   # no bad entry, no expired wait (KVX_ETIMEOUT raises)
