@@ -100,9 +100,10 @@ typedef enum {
                                       Results are then undefined.             */
 /* Device-side moves (kv_pack, kv_unpack, staged mode) use, by default, the
    TMA tensor-map kernel for HND pools whose K or V page half is at most
-   48 KiB (one TMA box per page half, staged through shared memory: the same
-   HBM throughput as the load/store kernel with two warps per SM), and the
-   16-byte load/store kernel otherwise.  The flags below force one of them.  */
+   48 KiB (one TMA box per page half, staged through shared memory; measured
+   faster than the load/store kernel on GB300), and the 16-byte load/store
+   kernel otherwise.  Zero-copy moves always use the load/store kernel.  The
+   flags below force one of them for device-side moves.                      */
 #define KVX_FLAG_DEVICE_TMA 0x4u   /* TMA everywhere it fits, with one bulk
                                       copy per row where no tensor map does  */
 #define KVX_FLAG_DEVICE_LSU 0x8u   /* the 16-byte load/store kernel always   */
@@ -118,7 +119,9 @@ typedef struct {
                                  (zero-copy) use a quarter of the SMs, which
                                  saturates the host link and leaves the rest to
                                  the replica's compute; device-side launches
-                                 fill the GPU                                   */
+                                 give every 32 KiB unit its own warp or CTA.
+                                 With a cap, each warp or CTA strides over
+                                 many units                                     */
   uint32_t flags;             /* KVX_FLAG_*                                     */
 } kvx_opts;
 
