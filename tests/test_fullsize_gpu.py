@@ -65,6 +65,7 @@ def test_fullsize_store_restore_sampled(orc, ctx_tokens, pool_blocks):
         ta = synth.permuted_table(pool_blocks, ctx_tokens // B, seed=1)
         tb = synth.permuted_table(pool_blocks, ctx_tokens // B, seed=2)
         ctx = k.kv_ctx_create(0)
+        torch.cuda.synchronize()  # pools generated on the default stream before the side stream reads them
         try:
             stream = torch.cuda.Stream()
             with torch.cuda.stream(stream):
@@ -74,30 +75,78 @@ def test_fullsize_store_restore_sampled(orc, ctx_tokens, pool_blocks):
             assert k.kv_get_device_error(ctx) == -1
         finally:
             k.kv_ctx_destroy(ctx)
-        bpc = C // B
-        r = synth.rng(ctx_tokens)
-        sample = sorted({0, 1, n_chunks // 2, n_chunks - 1, *map(int, r.integers(0, n_chunks, 3))})
-        mini = oracle.PoolSpec(L, bpc, B, H, D, E, oracle.HND)
-        ident = np.arange(bpc, dtype=np.int32)
-        for c in sample:
-            pool_np = [gather_pages(t, spec.page_bytes, ta[c * bpc:(c + 1) * bpc]) for t in src_layers]
-            want = [np.full(cb, POISON, np.uint8)]
-            assert orc.store(mini, pool_np, ident, 0, C, C, want, n_threads=8)[0] == 0
-            got = np_of(chunks[c])
-            assert sha(got) == sha(want[0]), (c, first_mismatch(got, want[0]))
-            loaded = [np.full(mini.layer_bytes, POISON, np.uint8) for _ in range(L)]
-            assert orc.load(mini, loaded, ident, 0, C, C, want, n_threads=8)[0] == 0
-            for l in (0, 1, L // 2, L - 1):
-                got_pages = gather_pages(dst_layers[l], spec.page_bytes, tb[c * bpc:(c + 1) * bpc])
-                assert first_mismatch(got_pages, loaded[l]) is None, (c, l)
-        unused = np.setdiff1d(np.arange(pool_blocks), tb)
-        probe = synth.rng(7).choice(unused, size=min(8, unused.size), replace=False)
-        for l in (0, L - 1):
-            assert np.all(gather_pages(dst_layers[l], spec.page_bytes, probe) == POISON)
+        _check_sampled(orc, spec, ctx_tokens, src_layers, dst_layers, ta, tb, chunks)
         del src_layers, dst_layers, src, dst, chunks
         torch.cuda.empty_cache()
     finally:
         host_pool.close()
+
+
+def _check_sampled(orc, spec, ctx_tokens, src_layers, dst_layers, ta, tb, chunks):
+    """Sampled chunks against the oracle (SHA-256 and bytes), the restored pages of
+    those chunks against the oracle's restore, and sampled pages outside the load
+    table untouched."""
+    n_chunks = len(chunks)
+    cb = orc.chunk_bytes(spec, C)
+    bpc = C // B
+    r = synth.rng(ctx_tokens)
+    sample = sorted({0, 1, n_chunks // 2, n_chunks - 1, *map(int, r.integers(0, n_chunks, 3))})
+    mini = oracle.PoolSpec(L, bpc, B, H, D, E, oracle.HND)
+    ident = np.arange(bpc, dtype=np.int32)
+    for c in sample:
+        pool_np = [gather_pages(t, spec.page_bytes, ta[c * bpc:(c + 1) * bpc]) for t in src_layers]
+        want = [np.full(cb, POISON, np.uint8)]
+        assert orc.store(mini, pool_np, ident, 0, C, C, want, n_threads=8)[0] == 0
+        got = np_of(chunks[c])
+        assert sha(got) == sha(want[0]), (c, first_mismatch(got, want[0]))
+        loaded = [np.full(mini.layer_bytes, POISON, np.uint8) for _ in range(L)]
+        assert orc.load(mini, loaded, ident, 0, C, C, want, n_threads=8)[0] == 0
+        for l in (0, 1, L // 2, L - 1):
+            got_pages = gather_pages(dst_layers[l], spec.page_bytes, tb[c * bpc:(c + 1) * bpc])
+            assert first_mismatch(got_pages, loaded[l]) is None, (c, l)
+    unused = np.setdiff1d(np.arange(spec.num_blocks), tb)
+    probe = synth.rng(7).choice(unused, size=min(8, unused.size), replace=False)
+    for l in (0, L - 1):
+        assert np.all(gather_pages(dst_layers[l], spec.page_bytes, probe) == POISON)
+
+
+@pytest.mark.parametrize("engine", ["default", "lsu"])
+def test_fullsize_device_pack_unpack_sampled(orc, engine):
+    """The benchmark's HBM leg at 128k tokens: kv_pack into device chunks and
+    kv_unpack into a poisoned pool, in the launch configuration bench.py times
+    (64 chunks per launch, one CTA or warp per 32 KiB unit)."""
+    k = kvx()
+    ctx_tokens, pool_blocks = 131072, 10240
+    spec = oracle.PoolSpec(L, pool_blocks, B, H, D, E, oracle.HND)
+    n_chunks = ctx_tokens // C
+    cb = orc.chunk_bytes(spec, C)
+    need = 2 * L * spec.layer_bytes + n_chunks * cb
+    free, _ = torch.cuda.mem_get_info()
+    if free < need + (4 << 30):
+        pytest.skip(f"needs {need >> 30} GiB of device memory")
+    src_layers = [synth.normal_bf16_(torch.empty(spec.layer_bytes, dtype=torch.uint8, device="cuda"),
+                                     synth.SEED + l) for l in range(L)]
+    dst_layers = [torch.full((spec.layer_bytes,), POISON, dtype=torch.uint8, device="cuda") for _ in range(L)]
+    src = k.KvPool(src_layers, pool_blocks, B, H, D, E)
+    dst = k.KvPool(dst_layers, pool_blocks, B, H, D, E)
+    slab = torch.full((n_chunks * cb,), POISON, dtype=torch.uint8, device="cuda")
+    chunks = [slab[i * cb:(i + 1) * cb] for i in range(n_chunks)]
+    ta = synth.permuted_table(pool_blocks, ctx_tokens // B, seed=1)
+    tb = synth.permuted_table(pool_blocks, ctx_tokens // B, seed=2)
+    ta_d, tb_d = torch.from_numpy(ta).cuda(), torch.from_numpy(tb).cuda()
+    torch.cuda.synchronize()  # tables and poisoned buffers complete before the side stream uses them
+    ctx = k.kv_ctx_create(0, flags=k.KVX_FLAG_DEVICE_LSU if engine == "lsu" else 0)
+    try:
+        stream = torch.cuda.Stream()
+        k.kv_pack(ctx, src, ta_d, 0, ctx_tokens, C, chunks, stream=stream)
+        k.kv_unpack(ctx, dst, tb_d, 0, ctx_tokens, C, chunks, stream=stream)
+        stream.synchronize()
+        assert k.kv_get_device_error(ctx) == -1
+    finally:
+        k.kv_ctx_destroy(ctx)
+    _check_sampled(orc, spec, ctx_tokens, src_layers, dst_layers, ta, tb, chunks)
+    del src_layers, dst_layers, src, dst, chunks, slab
+    torch.cuda.empty_cache()
 
 
 def test_host_alloc_exact_and_pinned():
