@@ -66,3 +66,28 @@ def splitmix64_bytes(n: int, seed: int) -> np.ndarray:
         z = (z ^ (z >> np.uint64(27))) * np.uint64(0x94D049BB133111EB)
         z = z ^ (z >> np.uint64(31))
     return z.astype("<u8").view(np.uint8)[:n].copy()
+
+
+def normal_bf16_bytes(n_elems: int, seed: int) -> np.ndarray:
+    """Bytes of n_elems bf16 values distributed approximately N(0, 1), portably.
+
+    Each value is an Irwin-Hall sum: 12 uniforms on (0, 1) from the SplitMix64
+    stream (16 bits each, u -> (u + 1/2) / 2^16), minus 6, which has mean 0 and
+    variance 1.  The sum is an integer over 2^16, exact in float32, and is
+    rounded to bf16 (round to nearest, ties to even) with integer operations,
+    so the bytes are the same on every machine and library version.
+    """
+    u = splitmix64_bytes(n_elems * 24, seed).view("<u2").reshape(n_elems, 12).astype(np.int64)
+    k = u.sum(axis=1) - 393210          # sum of (u + 1/2) minus 6 * 2^16, over 2^16
+    f32 = (k.astype(np.float32) / np.float32(65536.0)).view(np.uint32).astype(np.uint64)
+    bf16 = ((f32 + 0x7FFF + ((f32 >> 16) & 1)) >> 16).astype("<u2")
+    return bf16.view(np.uint8).copy()
+
+
+def portable_table(num_blocks: int, n_used: int, seed: int) -> np.ndarray:
+    """Like permuted_table, but fixed by the SplitMix64 definition: page ids in the
+    order of num_blocks SplitMix64 words (stable sort), first n_used (int32)."""
+    if n_used > num_blocks:
+        raise ValueError("table longer than the pool")
+    keys = splitmix64_bytes(8 * num_blocks, seed).view("<u8")
+    return np.argsort(keys, kind="stable")[:n_used].astype(np.int32)

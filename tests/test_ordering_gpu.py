@@ -113,11 +113,11 @@ def ctxs():
 
 
 # (name, mode, unordered, force the load/store device engine).  The staged
-# negative control packs with the load/store engine: the TMA engine's kernels
-# ask for ~96 KiB of shared memory per CTA, and an SM whose shared-memory
-# carveout was configured for the (shared-memory-free) spinning producer cannot
-# take them until the producer leaves it, which hides the missing dependency
-# behind a hardware reconfiguration rather than exposing it.
+# negative control packs with the load/store engine.  With the TMA engine the
+# unordered pack did not see stale bytes: its CTAs ask for 32-96 KiB of shared
+# memory, and (the likely cause) an SM whose carveout is set for the spinning
+# producer, which uses none, takes them only after the producer leaves, so the
+# pack runs after it and the missing dependency stays hidden.
 VARIANTS = [("staged", 1, False, False), ("staged_lsu", 1, False, True), ("zerocopy", 2, False, False),
             ("staged_unordered", 1, True, True), ("zerocopy_unordered", 2, True, False)]
 
