@@ -185,6 +185,8 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-hbm-roofline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-concurrent", action="store_true",
+                    help="skip the two-replica leg (one stores while the other restores)")
     ap.add_argument("--device-engine", choices=["lsu", "tma"], default="tma",
                     help="kernel of the device-side (HBM) pack/unpack leg")
     return ap.parse_args()
@@ -317,8 +319,52 @@ def host_link_peak(torch, dev):
                 ms = a.elapsed_time(b)
                 best = ms if best is None else min(best, ms)
         out[name] = n / (best * 1e-3) / GB
-    del h, d
+    # both directions at once, one copy per stream (two replicas sharing the link)
+    h2 = torch.empty(n, dtype=torch.uint8).pin_memory()
+    d2 = torch.empty(n, dtype=torch.uint8, device=dev)
+    s1, s2 = torch.cuda.Stream(device=dev), torch.cuda.Stream(device=dev)
+    best = None
+    for i in range(7):
+        a, b1, b2 = (torch.cuda.Event(enable_timing=True) for _ in range(3))
+        torch.cuda.synchronize()
+        a.record(s1)
+        s2.wait_event(a)
+        with torch.cuda.stream(s1):
+            h.copy_(d, non_blocking=True)
+        with torch.cuda.stream(s2):
+            d2.copy_(h2, non_blocking=True)
+        b1.record(s1)
+        b2.record(s2)
+        torch.cuda.synchronize()
+        if i >= 2:
+            ms = max(a.elapsed_time(b1), a.elapsed_time(b2))
+            best = ms if best is None else min(best, ms)
+    out["bidir"] = 2 * n / (best * 1e-3) / GB
+    del h, d, h2, d2
     return out
+
+
+def host_mem_available() -> int:
+    try:
+        with open("/proc/meminfo") as f:
+            for line in f:
+                if line.startswith("MemAvailable:"):
+                    return int(line.split()[1]) * 1024
+    except OSError:
+        pass
+    return 0
+
+
+def cpu_model() -> str:
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.startswith("Model name:"):
+                return line.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    import platform
+    return platform.processor() or platform.machine()
 
 
 def run_ours(args):
@@ -493,9 +539,49 @@ def run_ours(args):
     store_gbs = X / (statistics.median(store_ms) * 1e-3) / GB
     restore_gbs = X / (statistics.median(restore_ms) * 1e-3) / GB
     host_link = {"store_gbs": store_gbs, "restore_gbs": restore_gbs, "peak_d2h_gbs": link["d2h"],
-                 "peak_h2d_gbs": link["h2d"], "store_frac": store_gbs / link["d2h"],
+                 "peak_h2d_gbs": link["h2d"], "peak_bidir_gbs": link["bidir"], "store_frac": store_gbs / link["d2h"],
                  "restore_frac": restore_gbs / link["h2d"],
                  "peak_source": "pinned cudaMemcpyAsync of 1 GiB, best of 5, measured in this run"}
+
+    # Two replicas at once, each with its own context and stream: replica A stores
+    # the context into a second chunk set while replica B restores the chunks the
+    # timed steps wrote.  The host link then carries both directions.
+    concurrent = None
+    if not args.no_concurrent and world == 1 and host_mem_available() > n_chunks * cb + (32 << 30):
+        host_pool2 = k.HostBuffer(n_chunks * cb)
+        chunks2 = [host_pool2.tensor[i * cb:(i + 1) * cb] for i in range(n_chunks)]
+        ctx_b = k.kv_ctx_create(local, store_mode=mode, load_mode=mode, staging_slot_bytes=args.slot_mib << 20)
+        s_b = torch.cuda.Stream(device=dev)
+        st_ms, ld_ms, span_ms = [], [], []
+        for i in range(2 + 5):
+            a, ea, eb = (torch.cuda.Event(enable_timing=True) for _ in range(3))
+            torch.cuda.synchronize()
+            a.record(stream)
+            s_b.wait_event(a)
+            k.kv_store(ctx, src, ta, 0, T, C, chunks2, stream=stream)
+            ea.record(stream)
+            k.kv_load(ctx_b, dst, tb, 0, T, C, chunks, stream=s_b)
+            eb.record(s_b)
+            torch.cuda.synchronize()
+            if i >= 2:
+                st_ms.append(a.elapsed_time(ea))
+                ld_ms.append(a.elapsed_time(eb))
+                span_ms.append(max(st_ms[-1], ld_ms[-1]))
+        assert k.kv_get_device_error(ctx) == -1 and k.kv_get_device_error(ctx_b) == -1
+        picks = sorted({0, n_chunks // 3, n_chunks // 2, n_chunks - 1})
+        same = all(torch.equal(chunks2[c], chunks[c]) for c in picks)
+        k.kv_ctx_destroy(ctx_b)
+        del chunks2
+        host_pool2.close()
+        span = statistics.median(span_ms)
+        agg = 2 * X / (span * 1e-3) / GB
+        concurrent = {"store_ms": statistics.median(st_ms), "restore_ms": statistics.median(ld_ms),
+                      "span_ms": span, "aggregate_gbs": agg, "peak_bidir_gbs": link["bidir"],
+                      "frac": agg / link["bidir"], "reps": len(span_ms),
+                      "second_store_equals_first_on_sampled_chunks": same,
+                      "what": "replica A kv_store of the context into a second pinned chunk set while replica B "
+                              "kv_load of the timed steps' chunks into its pool, own context and stream each; "
+                              "peak = pinned cudaMemcpyAsync of 1 GiB each way at once"}
 
     cpu = None
     verified = None
@@ -511,9 +597,11 @@ def run_ours(args):
         spec, layers_np, ident = oracle_sample(cfg, S, pool_np)
         threads = os.cpu_count() or 1
         reps, el, want, moved = time_oracle(spec, layers_np, ident, S, args.cpu_seconds, threads, C)
+        reps1, el1, _, _ = time_oracle(spec, layers_np, ident, S, args.cpu_seconds / 2, 1, C)
         cpu = {"value": moved * reps / el / GB, "unit": "GB/s", "cores": min(threads, S), "kind": "oracle",
                "sample": f"{S} of {n_chunks} chunks (evenly spaced), store then load, repeated {reps}x "
-                         f"in {el:.1f} s on {threads} host threads"}
+                         f"in {el:.1f} s on {threads} host threads",
+               "single_thread_value": moved * reps1 / el1 / GB, "cpu_model": cpu_model()}
         verified = all(np.array_equal(chunks[c].numpy(), w) for c, w in zip(picks, want))
 
     k.kv_ctx_destroy(ctx)
@@ -539,6 +627,7 @@ def run_ours(args):
         "kernels": kern,
         "cpu_baseline": cpu,
         "verified_sample_vs_oracle": verified,
+        "concurrent_replicas": concurrent,
         "e2e": e2e,
         "gpu_launches": stats["kernel_launches"],
         "memcpy_calls": stats["memcpy_calls"],
