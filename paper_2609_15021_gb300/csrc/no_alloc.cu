@@ -99,10 +99,6 @@ extern "C" kvx_status kv_store_noalloc(const kvx_pool* pool, const int32_t* bloc
   if (st != KVX_OK) return st;
   uint8_t* staging = base + kSink;
   long long* err = dev_first_bad_block ? (long long*)dev_first_bad_block : (long long*)base;
-  int sms = 1;
-  if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device)) != cudaSuccess)
-    return fail_cuda(e, "cudaDeviceGetAttribute");
-  const int64_t grid_cap = (int64_t)std::max(1, sms) * move_ctas_per_sm(kPack, pool->layout);
 
   // Batches of (chunk, layer range) pieces that fit the array, each packed and
   // then copied out on the caller's stream.  Stream order alone keeps a batch
@@ -128,7 +124,8 @@ extern "C" kvx_status kv_store_noalloc(const kvx_pool* pool, const int32_t* bloc
                batch[q].nl);
       off += batch[q].bytes;
     }
-    const int64_t grid = std::max<int64_t>(1, std::min<int64_t>((p.total_units + 7) / 8, grid_cap));
+    // one warp per unit, as for the library's other HBM-bound launches
+    const int64_t grid = std::max<int64_t>(1, (p.total_units + kThreads / 32 - 1) / (kThreads / 32));
     cudaError_t le = launch_move(kPack, pool->layout, p, (int)grid, stream);
     if (le != cudaSuccess) return fail_cuda(le, "pack kernel launch");
     int64_t soff = 0;
