@@ -107,6 +107,9 @@ typedef enum {
 #define KVX_FLAG_DEVICE_TMA 0x4u   /* TMA everywhere it fits, with one bulk
                                       copy per row where no tensor map does  */
 #define KVX_FLAG_DEVICE_LSU 0x8u   /* the 16-byte load/store kernel always   */
+/* Every defined flag.  kv_ctx_create rejects (KVX_EINVAL) other bits, and
+   KVX_FLAG_DEVICE_TMA together with KVX_FLAG_DEVICE_LSU.                     */
+#define KVX_FLAGS_ALL 0xFu
 
 typedef struct {
   int32_t store_mode;         /* kvx_mode                                       */
@@ -116,12 +119,12 @@ typedef struct {
                                  one layer of one chunk                         */
   int32_t max_ctas;           /* cap on CTAs per kernel launch; 0 = default:
                                  launches that read or write host memory
-                                 (zero-copy) use a quarter of the SMs, which
-                                 saturates the host link and leaves the rest to
-                                 the replica's compute; device-side launches
-                                 give every 32 KiB unit its own warp or CTA.
-                                 With a cap, each warp or CTA strides over
-                                 many units                                     */
+                                 (zero-copy) run one 8-warp CTA per two SMs,
+                                 which saturates the host link even beside the
+                                 replica's compute and leaves most of each SM
+                                 to it; device-side launches give every
+                                 32 KiB unit its own warp or CTA.  With a cap,
+                                 each warp or CTA strides over many units       */
   uint32_t flags;             /* KVX_FLAG_*                                     */
 } kvx_opts;
 

@@ -821,6 +821,8 @@ kvx_status kv_ctx_create(int device, const kvx_opts* opts, kvx_ctx** out) {
   if (o.staging_slots > 64) return KVX_EINVAL;
   if (o.staging_slot_bytes < 0 || o.staging_slot_bytes % 16 != 0) return KVX_EINVAL;
   if (o.max_ctas < 0) return KVX_EINVAL;
+  if (o.flags & ~KVX_FLAGS_ALL) return KVX_EINVAL;
+  if ((o.flags & KVX_FLAG_DEVICE_TMA) && (o.flags & KVX_FLAG_DEVICE_LSU)) return KVX_EINVAL;
   int count = 0;
   if (cudaGetDeviceCount(&count) != cudaSuccess) {
     g_last_cuda_error = (int)cudaGetLastError();
@@ -846,7 +848,10 @@ kvx_status kv_ctx_create(int device, const kvx_opts* opts, kvx_ctx** out) {
   cudaError_t e;
   if ((e = cudaDeviceGetAttribute(&ctx->num_sms, cudaDevAttrMultiProcessorCount, device)) != cudaSuccess)
     return fail(e);
-  ctx->link_ctas = std::max(1, (ctx->num_sms + 3) / 4);
+  // Host-link launches: half the SMs.  A quarter already saturates the link on
+  // an idle GPU; half keeps it within 2-4 % of that while a full-GPU GEMM runs
+  // beside the transfer (a quarter then loses 16-21 %), for 1-2 % more GEMM time.
+  ctx->link_ctas = std::max(1, (ctx->num_sms + 1) / 2);
   if ((e = cudaStreamCreateWithFlags(&ctx->s_kern, cudaStreamNonBlocking)) != cudaSuccess) return fail(e);
   if ((e = cudaStreamCreateWithFlags(&ctx->s_copy, cudaStreamNonBlocking)) != cudaSuccess) return fail(e);
   if ((e = cudaStreamCreateWithFlags(&ctx->s_aux, cudaStreamNonBlocking)) != cudaSuccess) return fail(e);

@@ -40,6 +40,35 @@ def test_exports_every_declared_symbol(k):
     assert set(k.EXPORTED) == declared
 
 
+def declared_constants():
+    """{name: value} of every numeric #define and enum member KVX_* in include/*.h."""
+    out = {}
+    for h in os.listdir(os.path.join(ROOT, "include")):
+        if not h.endswith(".h"):
+            continue
+        text = re.sub(r"/\*.*?\*/", "", open(os.path.join(ROOT, "include", h)).read(), flags=re.S)
+        for m in re.finditer(r"#define\s+(KVX_\w+)\s+\(?(-?(?:0x[0-9A-Fa-f]+|\d+))(?:u|ll|LL)?\b(?:\s*<<\s*(\d+))?",
+                             text):
+            v = int(m.group(2), 0)
+            out[m.group(1)] = v << int(m.group(3)) if m.group(3) else v
+        for m in re.finditer(r"\b(KVX_[A-Z0-9_]+)\s*=\s*(-?\d+)", text):
+            out[m.group(1)] = int(m.group(2))
+    return out
+
+
+def test_binding_constants_match_headers(k):
+    declared = declared_constants()
+    for name in ("KVX_OK", "KVX_ETIMEOUT", "KVX_FLAG_DEVICE_LSU", "KVX_FLAGS_ALL", "KVX_PROBE_MAX_CYCLES",
+                 "KVX_NOALLOC_SCRATCH_BYTES", "KVX_TIER_NO_PIN", "KVX_MODE_ZEROCOPY"):
+        assert name in declared, name
+    mismatched = {n: (v, getattr(k, n)) for n, v in declared.items() if hasattr(k, n) and getattr(k, n) != v}
+    assert not mismatched, mismatched
+    missing = sorted(n for n in declared if not hasattr(k, n) and n not in ("KVX_ABI_VERSION",))
+    assert not missing, missing
+    flags = [v for n, v in declared.items() if n.startswith("KVX_FLAG_")]
+    assert declared["KVX_FLAGS_ALL"] == sum(flags) and all(v & (v - 1) == 0 for v in flags)
+
+
 def test_abi_version_and_strings(k):
     assert k.kv_abi_version() == 2
     assert k.kv_status_string(k.KVX_ENOTPINNED) == "host buffer is not page-locked"
@@ -120,7 +149,8 @@ def test_null_context_rejected_before_cuda(k):
 
 
 def test_bad_options_rejected(k):
-    for kw in ({"store_mode": 9}, {"staging_slots": 1}, {"staging_slot_bytes": 17}, {"max_ctas": -1}):
+    for kw in ({"store_mode": 9}, {"staging_slots": 1}, {"staging_slot_bytes": 17}, {"max_ctas": -1},
+               {"flags": 0x100}, {"flags": k.KVX_FLAG_DEVICE_TMA | k.KVX_FLAG_DEVICE_LSU}):
         with pytest.raises(k.KvxError) as e:
             k.kv_ctx_create(0, **kw)
         assert e.value.status == k.KVX_EINVAL
