@@ -396,6 +396,14 @@ kvx_status kv_tier_acquire(kvx_tier* tier, uint64_t key, kvx_stream_t stream, vo
 /* Unpins; the slot stays in use until the work already enqueued on `stream`
    (the load from it) completes. */
 kvx_status kv_tier_release(kvx_tier* tier, uint64_t key, kvx_stream_t stream);
+/* Shared tier: drops the pins held by processes that no longer exist and
+   frees the entries they were writing or committing (their bytes may be
+   incomplete).  *reclaimed (may be null) receives the number of slots changed.
+   kv_tier_reserve does the same by itself when it finds no usable slot.
+   Liveness is judged by process id within this host's pid namespace; a
+   private tier has nothing to reclaim.  An entry can be pinned by at most 8
+   processes at once (KVX_EBUSY beyond). */
+kvx_status kv_tier_reclaim(kvx_tier* tier, int64_t* reclaimed);
 /* Number of leading keys with committed entries (the cached prefix). */
 kvx_status kv_tier_prefix_hits(kvx_tier* tier, const uint64_t* keys, int64_t n, int64_t* hits);
 kvx_status kv_tier_stats(kvx_tier* tier, kvx_tier_stats* out);

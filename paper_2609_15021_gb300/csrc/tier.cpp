@@ -20,11 +20,16 @@
 // the paper's completion-before-consumption rule applied across processes.
 // Readers pin entries; a release on a stream keeps the pin until the work on
 // that stream completes, so a slot in use by queued GPU work is never evicted.
+// Pins are kept per process: when a process sharing the tier dies, its pins
+// and the entries it was writing are reclaimed (kv_tier_reclaim, and by
+// kv_tier_reserve when it finds no slot), so a crashed replica cannot hold
+// slots forever.
 
 #include <cuda_runtime.h>
 #include <errno.h>
 #include <fcntl.h>
 #include <pthread.h>
+#include <signal.h>
 #include <stdint.h>
 #include <stdio.h>
 #include <stdlib.h>
@@ -45,8 +50,9 @@ using namespace kvx;
 
 namespace {
 
-constexpr uint64_t kMagic = 0x3152454954584B56ull;  // "VKXTIER1"
+constexpr uint64_t kMagic = 0x3252454954584B56ull;  // "VKXTIER2"
 constexpr int64_t kDataAlign = 2ll << 20;
+constexpr int kHolders = 8;  // processes that may pin one entry at the same time
 
 enum SlotState : int32_t { kFree = 0, kWriting = 1, kCommitting = 2, kReady = 3 };
 
@@ -65,7 +71,42 @@ struct SlotMeta {
   int32_t writer_pid;  // process whose event decides COMMITTING -> READY
   int64_t pins;        // outstanding acquires/reserves, and releases whose GPU work is pending
   uint64_t tick;       // last use, for LRU
+  // the pins by process, so that a process that died can be dropped from them
+  int32_t holder_pid[kHolders];
+  int32_t holder_pins[kHolders];
 };
+
+// Adds n (may be negative) to pid's pins of m; false if pid holds none and
+// every holder place is taken.
+bool add_pins(SlotMeta& m, int32_t pid, int32_t n) {
+  int free_at = -1;
+  for (int h = 0; h < kHolders; ++h) {
+    if (m.holder_pins[h] > 0 && m.holder_pid[h] == pid) {
+      const int32_t d = n < -m.holder_pins[h] ? -m.holder_pins[h] : n;
+      m.holder_pins[h] += d;
+      m.pins = m.pins + d > 0 ? m.pins + d : 0;
+      return true;
+    }
+    if (m.holder_pins[h] <= 0 && free_at < 0) free_at = h;
+  }
+  if (n <= 0) return true;  // nothing held by pid: nothing to drop
+  if (free_at < 0) return false;
+  m.holder_pid[free_at] = pid;
+  m.holder_pins[free_at] = n;
+  m.pins += n;
+  return true;
+}
+
+void clear_pins(SlotMeta& m) {
+  m.pins = 0;
+  for (int h = 0; h < kHolders; ++h) m.holder_pins[h] = 0;
+}
+
+// A process of this host (pid namespace) that no longer exists.
+bool process_gone(int32_t pid) {
+  if (pid <= 0) return false;
+  return kill(pid, 0) != 0 && errno == ESRCH;
+}
 
 // SplitMix64 finaliser (Steele, Lea & Flood 2014) as the mixing step.
 uint64_t mix64(uint64_t z) {
@@ -172,7 +213,7 @@ void poll_locked(kvx_tier* t, bool wait) {
       ++i;
       continue;
     }
-    if (t->meta[p.slot].pins > 0) t->meta[p.slot].pins--;
+    add_pins(t->meta[p.slot], t->pid, -1);
     t->spare.push_back(p.ev);
     t->releases[i] = t->releases.back();
     t->releases.pop_back();
@@ -182,7 +223,9 @@ void poll_locked(kvx_tier* t, bool wait) {
 int64_t find_slot(kvx_tier* t, uint64_t key) {
   if (!t->shared) {
     auto it = t->index.find(key);
-    return it == t->index.end() ? -1 : it->second;
+    if (it == t->index.end()) return -1;
+    const SlotMeta& m = t->meta[it->second];
+    return m.state != kFree && m.key == key ? it->second : -1;
   }
   for (int64_t i = 0; i < t->hdr->n_slots; ++i)
     if (t->meta[i].state != kFree && t->meta[i].key == key) return i;
@@ -199,6 +242,54 @@ int64_t pick_slot(kvx_tier* t) {
     if (best < 0 || m.tick < t->meta[best].tick) best = i;
   }
   return best;
+}
+
+// Pins of this process on `slot` whose release is queued behind GPU work.
+int64_t queued_releases(const kvx_tier* t, int64_t slot) {
+  int64_t n = 0;
+  for (const PendingEvent& p : t->releases) n += p.slot == slot;
+  return n;
+}
+
+int32_t pins_of(const SlotMeta& m, int32_t pid) {
+  for (int h = 0; h < kHolders; ++h)
+    if (m.holder_pins[h] > 0 && m.holder_pid[h] == pid) return m.holder_pins[h];
+  return 0;
+}
+
+// Shared tier: drop the pins of processes that no longer exist, and free the
+// entries they were writing or committing (their bytes may be incomplete; the
+// work of a process that died ended with it).  Returns the slots changed.
+int64_t reclaim_locked(kvx_tier* t) {
+  if (!t->shared) return 0;
+  std::unordered_map<int32_t, bool> gone;  // liveness, once per process per scan
+  auto is_gone = [&](int32_t pid) {
+    auto it = gone.find(pid);
+    if (it != gone.end()) return it->second;
+    const bool g = pid != t->pid && process_gone(pid);
+    gone[pid] = g;
+    return g;
+  };
+  int64_t changed = 0;
+  for (int64_t i = 0; i < t->hdr->n_slots; ++i) {
+    SlotMeta& m = t->meta[i];
+    if (m.state == kFree) continue;
+    bool c = false;
+    if ((m.state == kWriting || m.state == kCommitting) && is_gone(m.writer_pid)) {
+      m.state = kFree;
+      clear_pins(m);
+      c = true;
+    }
+    for (int h = 0; h < kHolders; ++h) {
+      if (m.holder_pins[h] > 0 && is_gone(m.holder_pid[h])) {
+        m.pins = m.pins > m.holder_pins[h] ? m.pins - m.holder_pins[h] : 0;
+        m.holder_pins[h] = 0;
+        c = true;
+      }
+    }
+    changed += c;
+  }
+  return changed;
 }
 
 void destroy_tier(kvx_tier* t) {
@@ -410,28 +501,42 @@ kvx_status kv_tier_reserve(kvx_tier* t, uint64_t key, void** slot) {
   if (!t || !slot) return KVX_EINVAL;
   TierLock lock(t);
   poll_locked(t, false);
-  int64_t i = find_slot(t, key);
-  if (i >= 0) {
-    SlotMeta& m = t->meta[i];
-    if (m.pins > 0 || m.state != kReady) return KVX_EBUSY;  // in use: cannot be rewritten now
-  } else {
+  int64_t i = -1;
+  // a second pass after reclaiming what processes that died left behind
+  for (int pass = 0; pass < 2; ++pass) {
+    if (pass == 1 && reclaim_locked(t) == 0) break;
+    i = find_slot(t, key);
+    if (i >= 0) {
+      const SlotMeta& m = t->meta[i];
+      if (m.pins == 0 && m.state == kReady) break;
+      i = -2;  // in use: cannot be rewritten now
+      continue;
+    }
     i = pick_slot(t);
-    if (i < 0) {
-      set_error_text("every tier slot is pinned, being written, or still in use by the GPU");
-      return KVX_ENOMEM;
+    if (i >= 0) {
+      SlotMeta& m = t->meta[i];
+      if (m.state != kFree) {
+        if (!t->shared) t->index.erase(m.key);
+        t->hdr->evictions++;
+      }
+      if (!t->shared) t->index[key] = i;
+      break;
     }
-    SlotMeta& m = t->meta[i];
-    if (m.state != kFree) {
-      if (!t->shared) t->index.erase(m.key);
-      t->hdr->evictions++;
-    }
-    if (!t->shared) t->index[key] = i;
+  }
+  if (i == -2) {
+    set_error_text("the entry is pinned, being written, or still in use by the GPU");
+    return KVX_EBUSY;
+  }
+  if (i < 0) {
+    set_error_text("every tier slot is pinned, being written, or still in use by the GPU");
+    return KVX_ENOMEM;
   }
   SlotMeta& m = t->meta[i];
   m.key = key;
   m.state = kWriting;
   m.writer_pid = t->pid;
-  m.pins = 1;
+  clear_pins(m);
+  add_pins(m, t->pid, 1);
   m.tick = ++t->hdr->clock;
   *slot = t->data + i * t->hdr->slot_bytes;
   return KVX_OK;
@@ -459,7 +564,7 @@ kvx_status kv_tier_commit(kvx_tier* t, uint64_t key, kvx_stream_t stream) {
     t->commits.push_back({i, e});
     t->commit_event[i] = e;
   }
-  m.pins = m.pins > 0 ? m.pins - 1 : 0;
+  add_pins(m, t->pid, -1);
   m.tick = ++t->hdr->clock;
   return KVX_OK;
 }
@@ -492,7 +597,10 @@ kvx_status kv_tier_acquire(kvx_tier* t, uint64_t key, kvx_stream_t stream, void*
     }
   }
   SlotMeta& m = t->meta[i];
-  m.pins++;
+  if (!add_pins(m, t->pid, 1)) {
+    set_error_text("the entry is pinned by as many processes as it can track");
+    return KVX_EBUSY;
+  }
   m.tick = ++t->hdr->clock;
   t->hdr->hits++;
   *slot = t->data + i * t->hdr->slot_bytes;
@@ -506,10 +614,16 @@ kvx_status kv_tier_release(kvx_tier* t, uint64_t key, kvx_stream_t stream) {
   const int64_t i = find_slot(t, key);
   if (i < 0) return KVX_ENOENT;
   SlotMeta& m = t->meta[i];
-  if (m.pins < 1) return KVX_EINVAL;
+  if (pins_of(m, t->pid) - queued_releases(t, i) < 1) {
+    set_error_text("this process holds no pin on the entry");
+    return KVX_EINVAL;
+  }
   if (no_stream(stream)) {
-    m.pins--;
-    if (m.state == kWriting && m.pins == 0) m.state = kFree;  // a writer giving up its reservation
+    add_pins(m, t->pid, -1);
+    if (m.state == kWriting && m.pins == 0) {  // a writer giving up its reservation
+      m.state = kFree;
+      if (!t->shared) t->index.erase(m.key);
+    }
     return KVX_OK;
   }
   cudaEvent_t e = take_event(t);
@@ -520,6 +634,15 @@ kvx_status kv_tier_release(kvx_tier* t, uint64_t key, kvx_stream_t stream) {
     return cuda_fail(r, "cudaEventRecord (tier release)");
   }
   t->releases.push_back({i, e});  // the pin stays until the queued work completes
+  return KVX_OK;
+}
+
+kvx_status kv_tier_reclaim(kvx_tier* t, int64_t* reclaimed) {
+  if (!t) return KVX_EINVAL;
+  TierLock lock(t);
+  poll_locked(t, false);
+  const int64_t n = reclaim_locked(t);
+  if (reclaimed) *reclaimed = n;
   return KVX_OK;
 }
 

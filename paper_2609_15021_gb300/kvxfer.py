@@ -39,7 +39,7 @@ EXPORTED = (
     "kv_host_alloc", "kv_host_free", "kv_pool_view_check",
     "kv_chunk_keys", "kv_tier_create", "kv_tier_create_on", "kv_tier_destroy", "kv_tier_reserve", "kv_tier_commit",
     "kv_tier_acquire", "kv_tier_release", "kv_tier_prefix_hits", "kv_tier_stats", "kv_fault_inject",
-    "kv_tier_open_shared", "kv_tier_poll",
+    "kv_tier_open_shared", "kv_tier_poll", "kv_tier_reclaim",
 )
 KVX_ENOENT, KVX_EBUSY = -8, -9
 KVX_TIER_CREATE, KVX_TIER_NO_PIN = 0x1, 0x2
@@ -117,6 +117,7 @@ def _declare(lib):
         "kv_tier_create_on": (st, [vp, i64, i64, P(vp)]),
         "kv_tier_open_shared": (st, [ctypes.c_char_p, i64, i64, ctypes.c_uint32, P(vp)]),
         "kv_tier_poll": (st, [vp]),
+        "kv_tier_reclaim": (st, [vp, P(i64)]),
         "kv_tier_destroy": (None, [vp]),
         "kv_tier_reserve": (st, [vp, ctypes.c_uint64, P(vp)]),
         "kv_tier_commit": (st, [vp, ctypes.c_uint64, vp]),
@@ -490,6 +491,12 @@ class KvTier:
         arr = (ctypes.c_uint64 * max(1, len(keys)))(*keys)
         out = ctypes.c_int64()
         _check(_lib.kv_tier_prefix_hits(self.handle, arr, len(keys), ctypes.byref(out)), "kv_tier_prefix_hits")
+        return out.value
+
+    def reclaim(self) -> int:
+        """Drop what processes that no longer exist left pinned or half written; slots changed."""
+        out = ctypes.c_int64(0)
+        _check(_lib.kv_tier_reclaim(self.handle, ctypes.byref(out)), "kv_tier_reclaim")
         return out.value
 
     def stats(self) -> dict:

@@ -100,3 +100,25 @@ def test_bad_tier_arguments(k):
         k.KvTier(17, 4, base=16 * 1000)       # slot size not a multiple of 16
     with pytest.raises(k.KvxError):
         k.KvTier(64, 0, base=16 * 1000)
+
+
+def test_abandoned_reservation_frees_its_key(k):
+    """A writer that releases its reservation without committing gives the slot back:
+    the key can be reserved again, and once the slot holds another key the abandoned
+    key is not found (no stale mapping to the reused slot)."""
+    tier, buf = _tier(k, 1)
+    s = tier.reserve(21)
+    s.fill_(21)
+    tier.release(21, NO)                      # give up before committing
+    assert tier.stats()["entries"] == 0
+    assert tier.prefix_hits([21]) == 0
+    s = tier.reserve(21)                      # the same key again
+    tier.release(21, NO)
+    s = tier.reserve(22)                      # the only slot now holds 22
+    s.fill_(22)
+    tier.commit(22, NO)
+    with pytest.raises(k.KvxError) as e:
+        tier.acquire(21, NO)
+    assert e.value.status == k.KVX_ENOENT
+    assert int(tier.acquire(22, NO)[0]) == 22
+    tier.release(22, NO)

@@ -89,6 +89,86 @@ def test_shared_tier_bookkeeping_across_processes():
         t.close()
 
 
+def _child_dies(name, q_out):
+    """Pins an entry, reserves another, then the process ends without releasing
+    or committing either (a replica that crashed)."""
+    sys.path.insert(0, ROOT)
+    from paper_2609_15021_gb300 import kvxfer as k
+    NO = -1
+    t = k.KvTier(shared_name=name, pin=False)
+    t.acquire(1, NO)
+    t.reserve(5).fill_(55)
+    q_out.put("holding")
+    q_out.close()
+    q_out.join_thread()             # the message is out before the process ends
+    os._exit(0)                     # no release, no commit, no close
+
+
+def test_dead_process_pins_and_writes_are_reclaimed():
+    """Failure detection on the host: a process that dies holding a pin and a
+    half-written entry does not keep either slot forever."""
+    sys.path.insert(0, ROOT)
+    from paper_2609_15021_gb300 import _build
+    _build.build()
+    from paper_2609_15021_gb300 import kvxfer as k
+    NO = -1
+    name = _name("dead")
+    t = k.KvTier(64, 2, shared_name=name, create=True, pin=False)
+    try:
+        t.reserve(1).fill_(11)
+        t.commit(1, NO)
+        ctx = mp.get_context("spawn")
+        q_out = ctx.Queue()
+        p = ctx.Process(target=_child_dies, args=(name, q_out))
+        p.start()
+        assert q_out.get(timeout=60) == "holding"
+        p.join(timeout=60)
+        assert p.exitcode == 0
+        st = t.stats()
+        assert st["entries"] == 2 and st["pinned"] == 2      # 1 pinned by the dead reader, 5 reserved
+        assert t.prefix_hits([5]) == 0                       # never committed: not visible
+        # both slots are held: a reservation reclaims what the dead process left, then succeeds
+        s = t.reserve(6)
+        s.fill_(66)
+        t.commit(6, NO)
+        assert t.prefix_hits([1]) == 1 and int(t.acquire(1, NO)[0]) == 11   # the committed entry survives
+        t.release(1, NO)
+        assert t.prefix_hits([5]) == 0 and t.prefix_hits([6]) == 1
+        st = t.stats()
+        assert st["pinned"] == 0 and st["entries"] == 2
+        assert t.reclaim() == 0                              # nothing left to reclaim
+    finally:
+        t.close()
+
+
+def test_reclaim_leaves_live_processes_alone():
+    sys.path.insert(0, ROOT)
+    from paper_2609_15021_gb300 import _build
+    _build.build()
+    from paper_2609_15021_gb300 import kvxfer as k
+    NO = -1
+    name = _name("live")
+    t = k.KvTier(64, 2, shared_name=name, create=True, pin=False)
+    try:
+        t.reserve(1)
+        t.commit(1, NO)
+        t.acquire(1, NO)
+        t.reserve(2)                                         # this process is alive: nothing reclaimed
+        assert t.reclaim() == 0
+        assert t.stats()["pinned"] == 2
+        with pytest.raises(k.KvxError) as e:
+            t.reserve(3)
+        assert e.value.status == k.KVX_ENOMEM
+        t.release(1, NO)
+        with pytest.raises(k.KvxError) as e:
+            t.release(1, NO)                                 # no pin left to drop
+        assert e.value.status == k.KVX_EINVAL
+        t.release(2, NO)                                     # give the reservation up
+        assert t.stats()["entries"] == 1
+    finally:
+        t.close()
+
+
 def _child_gpu(name, q_in, q_out):
     sys.path.insert(0, ROOT)
     sys.path.insert(0, os.path.join(ROOT, "tests"))
