@@ -170,6 +170,21 @@ def _ptr(x) -> int:
     return x if isinstance(x, int) else x.data_ptr()
 
 
+def _nbytes(x) -> int:
+    return x.numel() * x.element_size()
+
+
+def _check_tensor(x, what: str, need_bytes: int | None = None) -> None:
+    """Binding-side checks of a tensor argument that the C ABI (raw pointers) cannot make:
+    contiguity and, where known, its size.  Plain integers are taken as raw pointers."""
+    if isinstance(x, int):
+        return
+    if not x.is_contiguous():
+        raise ValueError(f"{what} must be contiguous")
+    if need_bytes is not None and _nbytes(x) < need_bytes:
+        raise ValueError(f"{what} holds {_nbytes(x)} bytes, needs {need_bytes}")
+
+
 # ---------------------------------------------------------------- pools
 
 
@@ -187,6 +202,8 @@ class KvPool:
     pages_per_block: int = 1  # pages per logical block named by the block table
 
     def __post_init__(self):
+        for i, t in enumerate(self.layers):
+            _check_tensor(t, f"layer {i}", self.num_blocks * self.page_bytes)
         self._bases = (ctypes.c_void_p * max(1, len(self.layers)))(*[_ptr(t) for t in self.layers])
         self._c = kvx_pool(len(self.layers), ctypes.cast(self._bases, ctypes.POINTER(ctypes.c_void_p)),
                            self.num_blocks, self.block_tokens, self.num_heads, self.head_dim,
@@ -201,11 +218,12 @@ class KvPool:
         t = layers[0]
         head_dim = int(t.shape[-1])
         pages = t.numel() // (2 * num_heads * block_tokens * head_dim)
-        pool = cls(list(layers), pages, block_tokens, num_heads, head_dim, t.element_size(), layout,
+        shape_only = kvx_pool(len(layers), None, pages, block_tokens, num_heads, head_dim, t.element_size(),
+                              layout, pages_per_block)
+        for x in layers:  # layout first: a wrong view is named by what is wrong with it
+            _view_check(shape_only, x)
+        return cls(list(layers), pages, block_tokens, num_heads, head_dim, t.element_size(), layout,
                    pages_per_block)
-        for x in layers:
-            kv_pool_view_check(pool, x)
-        return pool
 
     @property
     def row_bytes(self) -> int:
@@ -243,20 +261,44 @@ def kv_chunk_layout(pool: KvPool, chunk_tokens: int, tokens_in_chunk: int) -> kv
     return out
 
 
-def kv_pool_view_check(pool: KvPool, tensor) -> None:
-    """Raise KvxError unless `tensor`'s shape and strides are the layout `pool` declares."""
+def _view_check(cpool: kvx_pool, tensor) -> None:
     nd = tensor.dim()
     shape = (ctypes.c_int64 * nd)(*tensor.shape)
     strides = (ctypes.c_int64 * nd)(*[s * tensor.element_size() for s in tensor.stride()])
-    _check(_lib.kv_pool_view_check(ctypes.byref(pool.c), nd, shape, strides), "kv_pool_view_check")
+    _check(_lib.kv_pool_view_check(ctypes.byref(cpool), nd, shape, strides), "kv_pool_view_check")
+
+
+def kv_pool_view_check(pool: KvPool, tensor) -> None:
+    """Raise KvxError unless `tensor`'s shape and strides are the layout `pool` declares."""
+    _view_check(pool.c, tensor)
 
 
 def _ptr_array(chunks):
     return (ctypes.c_void_p * max(1, len(chunks)))(*[_ptr(c) for c in chunks])
 
 
+def _check_transfer_tensors(pool: KvPool, block_table, tok_begin, tok_end, chunk_tokens, chunks) -> None:
+    """The table is int32 and every chunk the range uses holds its bytes: a chunk
+    smaller than that would be written past its end by the kernels."""
+    if not isinstance(block_table, int):
+        import torch
+        if block_table.dtype != torch.int32:
+            raise TypeError(f"block table must be int32, not {block_table.dtype}")
+        _check_tensor(block_table, "block table")
+    if chunk_tokens < 1 or tok_end <= tok_begin:
+        return
+    first = tok_begin // chunk_tokens
+    per_token = pool.c.num_layers * 2 * pool.num_heads * pool.row_bytes
+    for i, c in enumerate(chunks):
+        start = (first + i) * chunk_tokens
+        if start >= tok_end:
+            break
+        _check_tensor(c, f"chunk {i}", per_token * min(chunk_tokens, tok_end - start))
+
+
 def _transfer(fn, name, ctx, pool, block_table, tok_begin, tok_end, chunk_tokens, chunks, stream,
               table_len=None):
+    _check_transfer_tensors(pool, block_table, tok_begin, tok_end, chunk_tokens, chunks)
     arr = _ptr_array(chunks)
     n_tab = block_table.numel() if table_len is None else table_len
     _check(fn(ctx, ctypes.byref(pool.c), _ptr(block_table), n_tab, tok_begin, tok_end, chunk_tokens,
@@ -292,6 +334,7 @@ def kv_unpack(ctx, pool: KvPool, block_table, tok_begin: int, tok_end: int, chun
 def kv_store_noalloc(pool: KvPool, block_table, tok_begin: int, tok_end: int, chunk_tokens: int,
                      host_chunks, dev_first_bad_block=None, stream=None, table_len: int | None = None) -> None:
     """kv_store for callers that cannot allocate: no context, static device staging (see kvxfer.h)."""
+    _check_transfer_tensors(pool, block_table, tok_begin, tok_end, chunk_tokens, host_chunks)
     arr = _ptr_array(host_chunks)
     n_tab = block_table.numel() if table_len is None else table_len
     err = None if dev_first_bad_block is None else _ptr(dev_first_bad_block)

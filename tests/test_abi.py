@@ -163,3 +163,29 @@ def test_no_gpu_context_reports_cuda_error(k):
     with pytest.raises(k.KvxError) as e:
         k.kv_ctx_create(0)
     assert e.value.status in (k.KVX_ECUDA, k.KVX_EINVAL)
+
+
+def test_binding_rejects_what_raw_pointers_cannot_show(k):
+    """The C ABI takes raw pointers; the binding checks what only the tensors know:
+    the table's dtype, contiguity, and that each chunk and layer holds its bytes."""
+    import torch
+    L, N, B, H, D, e, C = 2, 8, 16, 2, 64, 2, 32
+    page = 2 * H * B * D * e
+    with pytest.raises(ValueError, match="layer 1 holds"):
+        k.KvPool([torch.empty(N * page, dtype=torch.uint8), torch.empty(N * page - 16, dtype=torch.uint8)],
+                 N, B, H, D, e)
+    pool = k.KvPool([torch.empty(N * page, dtype=torch.uint8) for _ in range(L)], N, B, H, D, e)
+    cb = L * 2 * C * H * D * e
+    chunks = [torch.empty(cb, dtype=torch.uint8) for _ in range(2)]
+    with pytest.raises(TypeError, match="int32"):
+        k.kv_store(0, pool, torch.zeros(4, dtype=torch.int64), 0, 64, C, chunks)
+    table = torch.zeros(4, dtype=torch.int32)
+    with pytest.raises(ValueError, match="chunk 1 holds"):
+        k.kv_load(0, pool, table, 0, 64, C, [chunks[0], chunks[1][:-16]])
+    with pytest.raises(ValueError, match="contiguous"):
+        k.kv_pack(0, pool, table, 0, 64, C, [chunks[0], torch.empty(2, cb, dtype=torch.uint8)[:, 0]])
+    # a short last chunk only needs its own tokens' bytes
+    short = torch.empty(L * 2 * 10 * H * D * e, dtype=torch.uint8)
+    k._check_transfer_tensors(pool, table, 0, 42, C, [chunks[0], short])
+    with pytest.raises(ValueError, match="chunk 1 holds"):
+        k._check_transfer_tensors(pool, table, 0, 43, C, [chunks[0], short])
