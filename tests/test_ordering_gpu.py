@@ -4,8 +4,9 @@
    ~10^8 SM cycles (host->device variant: reads the old value 0 after the
    delay) and a copy is issued (a) with no stream argument -- the raw
    fallback -- or (b) by one of the three ordered mechanisms.  Sizes 4 KiB,
-   1 MiB, 16 MiB, both directions, delayed and undelayed, ten trials per cell.
-   Delayed raw copies must see every byte stale; ordered copies none.
+   1 MiB, 16 MiB, both directions, delayed and undelayed, ten trials per cell,
+   in two independent processes.  Delayed raw copies must see every byte
+   stale (120 checks); ordered copies none (720 checks).
 2. The same experiment through kv_store / kv_load: a delayed producer writes
    the final KV just before kv_store on the caller's stream; a delayed
    consumer reads pages just before kv_load overwrites them.  Both transfer
@@ -13,6 +14,8 @@
    negative control (KVX_FLAG_UNORDERED drops the wait on the caller's stream)
    must give stale bytes in every delayed trial.
 """
+import multiprocessing as mp
+
 import numpy as np
 import pytest
 import torch
@@ -63,25 +66,58 @@ def _h2d_mismatches(k, how, n, delay):
     return int((readout != 0).sum())
 
 
-def test_probe_matrix():
-    """Table 2 'Copy-ordering controls': delayed raw fails every check, ordered controls pass all."""
+PROCESSES = 2  # Sec. 3.2: two independent processes run the matrix on one GPU
+
+
+def _matrix():
     k = kvx()
     counts = {}
     for n in SIZES:
         for direction, fn in (("d2h", _d2h_mismatches), ("h2d", _h2d_mismatches)):
             for delay in (0, DELAY):
                 for how in MECHS:
-                    res = [fn(k, how, n, delay) for _ in range(TRIALS)]
-                    counts[(n, direction, delay, how)] = res
-                    if how != "raw":
-                        assert all(r == 0 for r in res), (n, direction, delay, how, res)
-                    elif delay:
-                        assert all(r == n for r in res), (n, direction, how, res)
-    delayed_raw = [c for key, c in counts.items() if key[3] == "raw" and key[2]]
-    ordered = [c for key, c in counts.items() if key[3] != "raw"]
-    assert sum(len(c) for c in delayed_raw) == 60 and sum(len(c) for c in ordered) == 360
-    undelayed_raw_pass = sum(r == 0 for key, c in counts.items() if key[3] == "raw" and not key[2] for r in c)
-    print(f"undelayed raw checks passing: {undelayed_raw_pass}/60")
+                    counts[(n, direction, delay, how)] = [fn(k, how, n, delay) for _ in range(TRIALS)]
+    return counts
+
+
+def _matrix_child(q):
+    try:
+        q.put(("ok", list(_matrix().items())))
+    except Exception as e:  # reported to the parent, which fails the test
+        q.put(("error", repr(e)))
+
+
+def test_probe_matrix():
+    """Table 2 'Copy-ordering controls', as the paper ran them: two independent
+    processes, 3 sizes x 2 directions x 2 delays, ten trials per cell.  Delayed raw
+    copies fail all 120 checks with every byte stale; the three ordered controls
+    pass all 720."""
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    procs = [ctx.Process(target=_matrix_child, args=(q,)) for _ in range(PROCESSES)]
+    for p in procs:
+        p.start()
+    try:
+        results = [q.get(timeout=900) for _ in procs]
+    finally:
+        for p in procs:
+            p.join(timeout=60)
+            if p.is_alive():
+                p.kill()
+    errors = [r for tag, r in results if tag != "ok"]
+    assert not errors, errors
+    counts = {}
+    for _, items in results:
+        for key, res in items:
+            counts.setdefault(tuple(key), []).extend(res)
+    delayed_raw = [(key, r) for key, c in counts.items() if key[3] == "raw" and key[2] for r in c]
+    ordered = [(key, r) for key, c in counts.items() if key[3] != "raw" for r in c]
+    undelayed_raw = [r for key, c in counts.items() if key[3] == "raw" and not key[2] for r in c]
+    assert len(delayed_raw) == 120 and len(ordered) == 720 and len(undelayed_raw) == 120
+    assert all(r == key[0] for key, r in delayed_raw), "a delayed raw copy saw final bytes"
+    assert all(r == 0 for _, r in ordered), "an ordered copy saw stale bytes"
+    print(f"delayed raw checks failing: {len(delayed_raw)}/120; ordered checks passing: {len(ordered)}/720; "
+          f"undelayed raw checks passing: {sum(r == 0 for r in undelayed_raw)}/120")
 
 
 def _api_case(n_bytes):
