@@ -305,7 +305,8 @@ const void* tensor_maps_of(kvx_ctx* ctx, const kvx_pool* P, int64_t row) {
 kvx_status launch_move_timed(kvx_ctx* ctx, const kvx_pool* P, int dir, int layout, const MoveParams& p,
                              int64_t bytes, cudaStream_t s, bool over_link) {
   // TMA variants: device-side chunks only, and a K or V half page (the
-  // largest unit) of at most 48 KiB so that 2-3 stages fit in shared memory.
+  // largest unit) of at most 48 KiB: one shared-memory stage per unit, or a
+  // ring of 2-3 when a capped grid strides over units.
   // Default: tensor maps where the pool can be described, else load/store.
   const int64_t unit_bytes = (int64_t)p.B * p.H * p.R;
   const uint32_t f = ctx->opts.flags;
@@ -323,7 +324,7 @@ kvx_status launch_move_timed(kvx_ctx* ctx, const kvx_pool* P, int dir, int layou
     cap = ctx->opts.max_ctas;
   else if (over_link)
     cap = std::min<int64_t>(ctx->link_ctas, (int64_t)ctx->num_sms * ctx->move_occ[dir][layout]);
-  grid = std::max<int64_t>(1, std::min(grid, cap));
+  grid = std::max<int64_t>(1, std::min(std::min(grid, cap), (int64_t)INT_MAX));  // grid.x limit
   int stage_bytes = 0, stages = 0;
   if (tma) {
     // one stage when each CTA moves one unit; else a ring of 3 (2 above 32 KiB)

@@ -21,7 +21,8 @@ import pytest
 import torch
 
 import oracle
-from gpu_util import POISON, device_pool, first_mismatch, host_layers, kvx, np_of, oracle_load, oracle_store
+from gpu_util import (POISON, device_pool, first_mismatch, gather_pages, host_layers, kvx, np_of, oracle_load,
+                      oracle_store)
 from paper_2609_15021_gb300 import synth
 
 pytestmark = pytest.mark.gpu
@@ -220,3 +221,58 @@ def test_load_after_delayed_consumer(orc, ctxs, n_bytes):
                 elif delay:
                     # the consumer read bytes the load had already overwritten
                     assert first_mismatch(np_of(readout), loaded[0]) is None, (name, trial)
+
+
+def test_injected_delay_at_full_32k_size(orc):
+    """The injected-delay experiment on the full 32k-token 27B-class workload (62
+    layers x 8 KV heads x head_dim 128 bf16, 2,048 of 4,096 pages, 128 chunks): a
+    producer on the caller's stream rewrites every layer of the pool, the first
+    after ~10^8 cycles, just before kv_store.  The stored chunks must hold the
+    final bytes; with KVX_FLAG_UNORDERED the first chunk holds the stale ones."""
+    k = kvx()
+    L, N, B, H, D, E, C, T = 62, 4096, 16, 8, 128, 2, 256, 32768
+    spec = oracle.PoolSpec(L, N, B, H, D, E, oracle.HND)
+    free, _ = torch.cuda.mem_get_info()
+    if free < 2 * L * spec.layer_bytes + (4 << 30):
+        pytest.skip("needs two 27B-class pools of device memory")
+    final = [synth.normal_bf16_(torch.empty(spec.layer_bytes, dtype=torch.uint8, device="cuda"), synth.SEED + l)
+             for l in range(L)]
+    pool_layers = [torch.empty(spec.layer_bytes, dtype=torch.uint8, device="cuda") for _ in range(L)]
+    pool = k.KvPool(pool_layers, N, B, H, D, E)
+    table = synth.permuted_table(N, T // B, seed=5)
+    table_d = torch.from_numpy(table).cuda()
+    n_chunks, bpc = T // C, C // B
+    cb = orc.chunk_bytes(spec, C)
+    host = k.HostBuffer(n_chunks * cb)
+    chunks = [host.tensor[i * cb:(i + 1) * cb] for i in range(n_chunks)]
+    mini = oracle.PoolSpec(L, bpc, B, H, D, E, oracle.HND)
+    ident = np.arange(bpc, dtype=np.int32)
+    try:
+        for unordered in (False, True):
+            for t in pool_layers:
+                t.fill_(0x11)                                  # the stale KV
+            ctx = k.kv_ctx_create(0, flags=k.KVX_FLAG_UNORDERED if unordered else 0)
+            try:
+                stream = torch.cuda.Stream()
+                torch.cuda.synchronize()
+                for l in range(L):
+                    k.kvx_probe_delayed_copy(pool_layers[l], final[l], spec.layer_bytes, DELAY if l == 0 else 0,
+                                             stream)
+                k.kv_store(ctx, pool, table_d, 0, T, C, chunks, stream=stream)
+                stream.synchronize()
+                torch.cuda.synchronize()
+                assert k.kv_get_device_error(ctx) == -1
+            finally:
+                k.kv_ctx_destroy(ctx)
+            if unordered:
+                got = np_of(chunks[0])
+                assert np.all(got == 0x11), "the unordered store of the first chunk saw final bytes"
+                continue
+            for c in (0, 1, n_chunks // 2, n_chunks - 1):
+                pages_np = [gather_pages(t, spec.page_bytes, table[c * bpc:(c + 1) * bpc]) for t in final]
+                want = [np.full(cb, POISON, np.uint8)]
+                assert orc.store(mini, pages_np, ident, 0, C, C, want, n_threads=8)[0] == 0
+                assert first_mismatch(np_of(chunks[c]), want[0]) is None, c
+    finally:
+        del chunks
+        host.close()
