@@ -164,3 +164,81 @@ def test_host_alloc_exact_and_pinned():
         assert int(d[-1]) == 7
     finally:
         buf.close()
+
+
+def _torch_chunk(layers, table_d, c, T, N, H, R):
+    """Chunk c as torch's own gather computes it (the paper's same-stream tensor-copy
+    control): pages of the chunk by index_select, [page][kv][head][token][row] ->
+    [kv][token][head][row] per layer, layers concatenated."""
+    bpc = C // B
+    pages = table_d[c * bpc:(c + 1) * bpc].long()
+    tc = min(C, T - c * C)
+    parts = []
+    for t in layers:
+        v = t.view(N, 2, H, B, R).index_select(0, pages)          # [bpc][2][H][B][R]
+        v = v.permute(1, 0, 3, 2, 4).reshape(2, bpc * B, H, R)     # [2][tokens][H][R]
+        parts.append(v[:, :tc].reshape(-1))
+    return torch.cat(parts)
+
+
+@pytest.mark.parametrize("mode", ["zerocopy", "staged", "device"])
+def test_fullsize_every_chunk_and_page_vs_torch(mode):
+    """Every chunk and every page of the 128k-token workload, not a sample: the
+    stored chunks equal torch's gather of the source pages, the restored pages
+    under the load table equal the source pages under the store table, and every
+    other page of the destination pool is still poisoned."""
+    k = kvx()
+    ctx_tokens, N = 131072, 10240
+    R = D * E
+    page = 2 * H * B * R
+    n_chunks = ctx_tokens // C
+    cb = L * 2 * C * H * R
+    free, _ = torch.cuda.mem_get_info()
+    need = 2 * L * N * page + (n_chunks * cb if mode == "device" else 0)
+    if free < need + (8 << 30):
+        pytest.skip(f"needs {need >> 30} GiB of device memory")
+    src_layers = [synth.normal_bf16_(torch.empty(N * page, dtype=torch.uint8, device="cuda"), synth.SEED + l)
+                  for l in range(L)]
+    dst_layers = [torch.full((N * page,), POISON, dtype=torch.uint8, device="cuda") for _ in range(L)]
+    src = k.KvPool(src_layers, N, B, H, D, E)
+    dst = k.KvPool(dst_layers, N, B, H, D, E)
+    ta_d = torch.from_numpy(synth.permuted_table(N, ctx_tokens // B, seed=11)).cuda()
+    tb_d = torch.from_numpy(synth.permuted_table(N, ctx_tokens // B, seed=12)).cuda()
+    host = None
+    if mode == "device":
+        slab = torch.full((n_chunks * cb,), POISON, dtype=torch.uint8, device="cuda")
+    else:
+        host = k.HostBuffer(n_chunks * cb)
+        slab = host.tensor
+    chunks = [slab[i * cb:(i + 1) * cb] for i in range(n_chunks)]
+    torch.cuda.synchronize()
+    m = {"zerocopy": k.KVX_MODE_ZEROCOPY, "staged": k.KVX_MODE_STAGED, "device": k.KVX_MODE_AUTO}[mode]
+    ctx = k.kv_ctx_create(0, store_mode=m, load_mode=m)
+    try:
+        stream = torch.cuda.Stream()
+        if mode == "device":
+            k.kv_pack(ctx, src, ta_d, 0, ctx_tokens, C, chunks, stream=stream)
+            k.kv_unpack(ctx, dst, tb_d, 0, ctx_tokens, C, chunks, stream=stream)
+        else:
+            k.kv_store(ctx, src, ta_d, 0, ctx_tokens, C, chunks, stream=stream)
+            k.kv_load(ctx, dst, tb_d, 0, ctx_tokens, C, chunks, stream=stream)
+        stream.synchronize()
+        assert k.kv_get_device_error(ctx) == -1
+    finally:
+        k.kv_ctx_destroy(ctx)
+    try:
+        bad = [c for c in range(n_chunks)
+               if not torch.equal(chunks[c].to("cuda", non_blocking=False),
+                                  _torch_chunk(src_layers, ta_d, c, ctx_tokens, N, H, R))]
+        assert not bad, f"{len(bad)} chunks differ, first {bad[0]}"
+        unused = torch.from_numpy(np.setdiff1d(np.arange(N), tb_d.cpu().numpy())).cuda()
+        for l in range(L):
+            got = dst_layers[l].view(N, page)
+            assert torch.equal(got.index_select(0, tb_d.long()), src_layers[l].view(N, page).index_select(0, ta_d.long())), l
+            assert bool((got.index_select(0, unused) == POISON).all()), l
+    finally:
+        del chunks, slab
+        if host is not None:
+            host.close()
+        del src_layers, dst_layers, src, dst
+        torch.cuda.empty_cache()
