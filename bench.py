@@ -185,6 +185,9 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-hbm-roofline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--host-alloc", choices=["cuda", "numa"], default="cuda",
+                    help="pinned pool from kv_host_alloc (cudaHostAlloc) or kv_host_alloc_numa on the "
+                         "host node nearest the GPU")
     ap.add_argument("--no-concurrent", action="store_true",
                     help="skip the two-replica leg (one stores while the other restores)")
     ap.add_argument("--device-engine", choices=["lsu", "tma"], default="tma",
@@ -401,7 +404,8 @@ def run_ours(args):
     ta = torch.from_numpy(ta_np).to(dev)
     tb = torch.from_numpy(tb_np).to(dev)
     t_pin = time.perf_counter()
-    host_pool = k.HostBuffer(n_chunks * cb)  # exact-size pinned, mapped pool (no power-of-two rounding)
+    # exact-size pinned, mapped pool (no power-of-two rounding)
+    host_pool = k.HostBuffer(n_chunks * cb, numa_node=k.KVX_NUMA_NEAREST if args.host_alloc == "numa" else None)
     pin_seconds = time.perf_counter() - t_pin
     chunks = [host_pool.tensor[i * cb:(i + 1) * cb] for i in range(n_chunks)]
 
@@ -617,6 +621,8 @@ def run_ours(args):
                    "bytes_per_direction": X, "l2": f"inputs larger than L2 ({X} bytes per direction), no flush",
                    "store_mode": k.MODE_NAMES[store_mode], "load_mode": k.MODE_NAMES[load_mode],
                    "parallelism": f"replicas x{world}", "pinned_host_bytes": n_chunks * cb,
+                   "host_alloc": args.host_alloc if host_pool.numa_node is None
+                   else f"numa node {host_pool.numa_node}",
                    "pin_seconds": pin_seconds},
         "restore_ms": {"median": statistics.median(restore_ms), "min": min(restore_ms), "max": max(restore_ms),
                        "n": len(restore_ms)},

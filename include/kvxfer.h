@@ -316,6 +316,22 @@ kvx_status kv_store_noalloc(const kvx_pool* pool, const int32_t* block_table, in
  * kv_host_free (NULL is ignored).
  */
 kvx_status kv_host_alloc(int64_t bytes, void** out);
+/*
+ * kv_host_alloc placed on one host NUMA node.  On a host with several memory
+ * nodes the pool belongs on the node next to the GPU that uses it, or every
+ * zero-copy access also crosses the link between sockets.  numa_node >= 0
+ * names the node; KVX_NUMA_NEAREST asks for the node CUDA reports as closest
+ * to the current device (no placement if it reports none).  The memory is
+ * anonymous memory with a preferred-node policy (mbind), registered
+ * page-locked, portable and mapped, exactly `bytes` long as seen by callers.
+ * KVX_EINVAL for a node that does not exist, KVX_ENOMEM if the node has less
+ * free memory than `bytes` or the memory cannot be pinned (never a pageable
+ * fallback).  *numa_out (may be NULL) receives the node of the first page,
+ * or -1 if unknown.  Free with kv_host_free.
+ */
+#define KVX_NUMA_NEAREST (-1)
+kvx_status kv_host_alloc_numa(int32_t numa_node, int64_t bytes, void** out, int32_t* numa_out);
+/* Frees kv_host_alloc and kv_host_alloc_numa memory; NULL is ignored. */
 void kv_host_free(void* host);
 
 /* ------------------------------------------------------------------------

@@ -1049,7 +1049,7 @@ kvx_status kv_host_alloc(int64_t bytes, void** out) {
 }
 
 void kv_host_free(void* p) {
-  if (p) {
+  if (p && !free_numa_allocation(p)) {
     cudaFreeHost(p);
     cudaGetLastError();
   }

@@ -39,7 +39,7 @@ EXPORTED = (
     "kv_host_alloc", "kv_host_free", "kv_pool_view_check",
     "kv_chunk_keys", "kv_tier_create", "kv_tier_create_on", "kv_tier_destroy", "kv_tier_reserve", "kv_tier_commit",
     "kv_tier_acquire", "kv_tier_release", "kv_tier_prefix_hits", "kv_tier_stats", "kv_fault_inject",
-    "kv_tier_open_shared", "kv_tier_poll", "kv_tier_reclaim",
+    "kv_tier_open_shared", "kv_tier_poll", "kv_tier_reclaim", "kv_host_alloc_numa",
 )
 KVX_ENOENT, KVX_EBUSY = -8, -9
 KVX_TIER_CREATE, KVX_TIER_NO_PIN = 0x1, 0x2
@@ -111,6 +111,7 @@ def _declare(lib):
         "kv_store_noalloc": (st, [P(kvx_pool), vp, i64, i64, i64, i32, P(vp), i64, vp, vp]),
         "kv_host_alloc": (st, [i64, P(vp)]),
         "kv_host_free": (None, [vp]),
+        "kv_host_alloc_numa": (st, [i32, i64, P(vp), P(i32)]),
         "kv_pool_view_check": (st, [P(kvx_pool), i32, P(i64), P(i64)]),
         "kv_chunk_keys": (st, [P(i32), i64, i32, ctypes.c_uint64, P(ctypes.c_uint64), i64]),
         "kv_tier_create": (st, [i64, i64, P(vp)]),
@@ -353,6 +354,18 @@ def kv_host_alloc(nbytes: int) -> int:
     return out.value
 
 
+KVX_NUMA_NEAREST = -1
+
+
+def kv_host_alloc_numa(nbytes: int, numa_node: int = KVX_NUMA_NEAREST) -> tuple[int, int]:
+    """kv_host_alloc on one host NUMA node (default: the one nearest the current GPU).
+    Returns (pointer, node of the first page or -1)."""
+    out = ctypes.c_void_p()
+    node = ctypes.c_int32(-1)
+    _check(_lib.kv_host_alloc_numa(numa_node, nbytes, ctypes.byref(out), ctypes.byref(node)), "kv_host_alloc_numa")
+    return out.value, node.value
+
+
 def kv_host_free(ptr: int) -> None:
     _lib.kv_host_free(ptr)
 
@@ -363,10 +376,16 @@ class HostBuffer:
     Views of ``.tensor`` keep the allocation alive; ``close()`` frees it at once
     and must only be called when no view is used any more."""
 
-    def __init__(self, nbytes: int):
+    def __init__(self, nbytes: int, numa_node: int | None = None):
+        """numa_node: None for kv_host_alloc, else kv_host_alloc_numa on that node
+        (KVX_NUMA_NEAREST: the node nearest the current GPU); see .numa_node."""
         import torch
         self.nbytes = nbytes
-        self.ptr = kv_host_alloc(nbytes)
+        self.numa_node = None
+        if numa_node is None:
+            self.ptr = kv_host_alloc(nbytes)
+        else:
+            self.ptr, self.numa_node = kv_host_alloc_numa(nbytes, numa_node)
         raw = (ctypes.c_uint8 * nbytes).from_address(self.ptr)
         raw._owner = self  # the tensor holds `raw`, `raw` holds this buffer
         self.tensor = torch.frombuffer(raw, dtype=torch.uint8, count=nbytes)

@@ -189,3 +189,17 @@ def test_binding_rejects_what_raw_pointers_cannot_show(k):
     k._check_transfer_tensors(pool, table, 0, 42, C, [chunks[0], short])
     with pytest.raises(ValueError, match="chunk 1 holds"):
         k._check_transfer_tensors(pool, table, 0, 43, C, [chunks[0], short])
+
+
+def test_host_alloc_numa_arguments(k):
+    import torch
+    out = ctypes.c_void_p()
+    node = ctypes.c_int32(5)
+    for numa, n in ((0, 0), (-2, 4096), (1 << 20, 4096)):
+        assert k._lib.kv_host_alloc_numa(numa, n, ctypes.byref(out), ctypes.byref(node)) == k.KVX_EINVAL
+    assert k._lib.kv_host_alloc_numa(0, 4096, None, None) == k.KVX_EINVAL
+    assert k._lib.kv_host_alloc_numa(1000, 4096, ctypes.byref(out), None) == k.KVX_EINVAL   # no such node
+    assert out.value is None and node.value == -1
+    if not torch.cuda.is_available():                   # node 0 exists; pinning needs a GPU
+        assert k._lib.kv_host_alloc_numa(0, 4096, ctypes.byref(out), None) == k.KVX_ECUDA
+        assert out.value is None

@@ -18,7 +18,8 @@ import pytest
 import torch
 
 import oracle
-from gpu_util import POISON, first_mismatch, gather_pages, kvx, np_of, sha
+from gpu_util import (POISON, device_pool, first_mismatch, gather_pages, host_layers, kvx, np_of, oracle_load,
+                      oracle_store, sha)
 from paper_2609_15021_gb300 import synth
 
 pytestmark = pytest.mark.gpu
@@ -162,6 +163,48 @@ def test_host_alloc_exact_and_pinned():
         d.copy_(buf.tensor[-4096:], non_blocking=True)
         torch.cuda.synchronize()
         assert int(d[-1]) == 7
+    finally:
+        buf.close()
+
+
+@pytest.mark.parametrize("node", ["nearest", 0])
+def test_host_alloc_numa_round_trip(orc, node):
+    """kv_host_alloc_numa: a pinned, mapped pool on a host NUMA node (the node
+    nearest the GPU, or node 0), used as the chunks of a zero-copy store and
+    restore that must match the oracle."""
+    k = kvx()
+    spec = oracle.PoolSpec(4, 64, 16, 8, 128, 2, oracle.HND)
+    Cs, n_used = 256, 40
+    T = n_used * 16 - 5
+    cb = orc.chunk_bytes(spec, Cs)
+    n_chunks = -(-T // Cs)
+    want_node = k.KVX_NUMA_NEAREST if node == "nearest" else node
+    buf = k.HostBuffer(n_chunks * cb, numa_node=want_node)
+    try:
+        if node == 0:
+            assert buf.numa_node == 0
+        print(f"\nhost pool on NUMA node {buf.numa_node} (asked: {node})")
+        chunks = [buf.tensor[i * cb:(i + 1) * cb] for i in range(n_chunks)]
+        src_np = host_layers(spec, 61)
+        src, dst = device_pool(spec, src_np), device_pool(spec)
+        ta, tb = synth.permuted_table(64, n_used, 61), synth.permuted_table(64, n_used, 62)
+        ta_d, tb_d = torch.from_numpy(ta).cuda(), torch.from_numpy(tb).cuda()
+        ctx = k.kv_ctx_create(0, store_mode=k.KVX_MODE_ZEROCOPY, load_mode=k.KVX_MODE_ZEROCOPY)
+        try:
+            s = torch.cuda.Stream()
+            k.kv_store(ctx, src, ta_d, 0, T, Cs, chunks, stream=s)
+            k.kv_load(ctx, dst, tb_d, 0, T, Cs, chunks, stream=s)
+            s.synchronize()
+            assert k.kv_get_device_error(ctx) == -1
+        finally:
+            k.kv_ctx_destroy(ctx)
+        want, _ = oracle_store(orc, spec, src_np, ta, 0, T, Cs)
+        for i, w in enumerate(want):
+            assert first_mismatch(np_of(chunks[i])[:w.size], w) is None, i
+        loaded, _ = oracle_load(orc, spec, [np.full(spec.layer_bytes, POISON, np.uint8)] * 4, tb, 0, T, Cs, want)
+        for l in range(4):
+            assert first_mismatch(np_of(dst.layers[l]), loaded[l]) is None, l
+        del chunks
     finally:
         buf.close()
 
