@@ -31,12 +31,18 @@
  * Threading: a kvx_ctx may be shared by host threads (calls are serialised
  * inside).  Calls are asynchronous with respect to the host.
  *
+ * Ordering: zero-copy and device-chunk moves and state copies are enqueued on
+ * `stream` itself, so stream order makes them follow the work already there
+ * and precede what comes after.  The staged pipeline runs on two side streams
+ * that wait on an event recorded on `stream`, and `stream` then waits on
+ * events recorded after its last piece of work.
+ *
  * CUDA graphs: kv_store, kv_load, kv_pack and kv_unpack allocate nothing per
- * call (the staging ring of KVX_MODE_STAGED is made by kv_ctx_create) and
- * order their side-stream work with an event on `stream` and a join back to
- * it, so they may be captured from a capturing `stream` and replayed (the
- * buffers and ranges of the capture are replayed).  While `stream` is
- * capturing, its device is not checked (the query would end the capture).
+ * call (the staging ring of KVX_MODE_STAGED is made by kv_ctx_create), and
+ * what they enqueue is joined to `stream`.  They may therefore be captured
+ * from a capturing `stream` and replayed; the buffers and ranges of the
+ * capture are replayed.  While `stream` is capturing, its device is not
+ * checked (the query would end the capture).
  *
  * Error behaviour: argument errors return before anything is enqueued and
  * leave every buffer untouched.  A block-table entry outside [0, num_blocks)
@@ -451,8 +457,8 @@ const char* kv_last_error_message(void);
  * GPU: the (after_calls + 1)-th next CUDA call at `point` in this process
  * fails with cudaErrorUnknown (cudaErrorMemoryAllocation for "host_alloc")
  * instead of being made.  Points: "launch" (kernel launches), "memcpy"
- * (staged-mode copies), "event" (the ordering event recorded on the caller's
- * stream), "host_alloc" (kv_host_alloc).  One point is armed at a time;
+ * (staged-mode copies), "event" (the staged pipeline's ordering event
+ * recorded on the caller's stream), "host_alloc" (kv_host_alloc).  One point is armed at a time;
  * point NULL or "" disarms.  KVX_EINVAL for an unknown point.
  */
 kvx_status kv_fault_inject(const char* point, int32_t after_calls);

@@ -41,15 +41,20 @@ struct MoveParams {
   int32_t rpi_div_h, rpi_mod_h; // (32 / (R/16)) / H and % H when fast
 };
 
+// One contiguous byte range of an opaque copy (a recurrent-state slot).
 struct Segment {
   const uint8_t* src;
   uint8_t* dst;
-  int64_t unit_end;  // exclusive prefix sum of 32 KiB units
-  int64_t bytes;
+  int64_t byte_end;  // exclusive prefix sum of segment bytes
 };
 
+// The segments of one launch are treated as one byte stream cut into units of
+// unit_bytes (a multiple of 512; the last unit may be shorter) that may span
+// segment ends, so every warp gets the same share of bytes.
 struct SegmentParams {
   Segment seg[kMaxSegments];
+  int64_t total_bytes;
+  int64_t unit_bytes;
   int64_t total_units;
   int32_t n_seg;
 };

@@ -4,12 +4,15 @@
 // Ordering contract (paper Sec. 3.2 and Fig. 2): the paper's corruption came
 // from a host<->device copy issued with no dependency on the caller's current
 // stream, which in PyTorch is a non-blocking stream and therefore not covered
-// by legacy default-stream synchronisation.  Here every call records an event
-// on the caller's stream after the work already enqueued there; the side
-// streams that do the work wait on it; the caller's stream then waits on an
-// event recorded after the last piece of work.  Staging slots are reused only
-// after an event shows their previous consumer finished (the premature-reuse
-// hazard the paper cites among related reports, Sec. 3.2).
+// by legacy default-stream synchronisation.  Here kernel-only moves (zero-copy
+// and device chunks) and state copies are enqueued on the caller's stream
+// itself, so stream order is the dependency (the paper's same-stream
+// control).  The staged pipeline overlaps packing and copying on two side
+// streams: the call records an event on the caller's stream after the work
+// already enqueued there, both side streams wait on it, and the caller's
+// stream then waits on events recorded after the last piece of work.  Staging
+// slots are reused only after an event shows their previous consumer finished
+// (the premature-reuse hazard the paper cites among related reports, Sec. 3.2).
 
 #include <cuda_runtime.h>
 #include <limits.h>
@@ -431,8 +434,9 @@ struct Plan {
   std::vector<uint8_t*> side;   // chunk i as the kernel (mapped/device) or copy engine sees it
 };
 
-// Zero-copy and device chunks: one kernel pass per batch of whole chunks.
-kvx_status enqueue_direct(kvx_ctx* ctx, const Plan& pl) {
+// Zero-copy and device chunks: one kernel pass per batch of whole chunks, on
+// stream s.
+kvx_status enqueue_direct(kvx_ctx* ctx, const Plan& pl, cudaStream_t s) {
   MoveParams p;
   init_move_params(&p, ctx->d_err, pl.P, pl.g, pl.table, pl.C);
   int64_t bytes = 0;
@@ -440,7 +444,7 @@ kvx_status enqueue_direct(kvx_ctx* ctx, const Plan& pl) {
     add_job(&p, pl.side[i], (pl.first_chunk + i) * pl.bpc, pl.tokens[i], 0, pl.P->num_layers);
     bytes += chunk_bytes_of(pl.P, pl.g, pl.tokens[i]);
     if (p.n_jobs == kMaxJobs || i == pl.n - 1) {
-      kvx_status st = launch_move_timed(ctx, pl.P, pl.dir, pl.P->layout, p, bytes, ctx->s_kern, pl.over_link);
+      kvx_status st = launch_move_timed(ctx, pl.P, pl.dir, pl.P->layout, p, bytes, s, pl.over_link);
       if (st != KVX_OK) return st;
       p.n_jobs = 0;
       p.total_units = 0;
@@ -652,16 +656,24 @@ kvx_status transfer(kvx_ctx* ctx, const kvx_pool* P, const int32_t* table, int64
   if (staged && max_layer_bytes > ctx->slot_bytes) return KVX_EINVAL;
 
   std::lock_guard<std::mutex> lock(ctx->mu);
+  const bool ordered = (ctx->opts.flags & KVX_FLAG_UNORDERED) == 0;
+  // Kernel-only moves (zero-copy or device chunks) run on the caller's stream
+  // itself: stream order is the dependency, with no event hop in between.
+  if (!staged && ordered) return enqueue_direct(ctx, pl, stream);
   if (staged) {
     st = ensure_staging(ctx);
     if (st != KVX_OK) return st;
   }
+  // The staged pipeline overlaps packing and copying on two side streams
+  // that wait on an event recorded on the caller's stream.  Without that wait
+  // (KVX_FLAG_UNORDERED, the negative control) kernel-only moves also run on
+  // a side stream, which is the paper's missing dependency.
   KVX_CUDA_AT("event", cudaEventRecord(ctx->ev_in, stream));
-  if ((ctx->opts.flags & KVX_FLAG_UNORDERED) == 0) {
+  if (ordered) {
     KVX_CUDA(cudaStreamWaitEvent(ctx->s_kern, ctx->ev_in, 0));
-    if (staged) KVX_CUDA(cudaStreamWaitEvent(ctx->s_copy, ctx->ev_in, 0));
+    KVX_CUDA(cudaStreamWaitEvent(ctx->s_copy, ctx->ev_in, 0));
   }
-  st = staged ? enqueue_staged(ctx, pl) : enqueue_direct(ctx, pl);
+  st = staged ? enqueue_staged(ctx, pl) : enqueue_direct(ctx, pl, ctx->s_kern);
   const kvx_status joined = join_caller(ctx, stream, staged);
   return st != KVX_OK ? st : joined;
 }
@@ -691,10 +703,12 @@ kvx_status state_copy(kvx_ctx* ctx, int32_t L, void* const* layer_base, int64_t 
   if (mode == KVX_MODE_ZEROCOPY && !mapped) return KVX_ENOTPINNED;
 
   std::lock_guard<std::mutex> lock(ctx->mu);
+  // Ordered copies run on the caller's stream itself (stream order is the
+  // dependency); the negative control (KVX_FLAG_UNORDERED) runs them on a side
+  // stream that does not wait for the caller's work.
   const bool ordered = (ctx->opts.flags & KVX_FLAG_UNORDERED) == 0;
-  KVX_CUDA(cudaEventRecord(ctx->ev_in, stream));
   if (mode == KVX_MODE_ZEROCOPY) {
-    if (ordered) KVX_CUDA(cudaStreamWaitEvent(ctx->s_kern, ctx->ev_in, 0));
+    cudaStream_t ks = ordered ? stream : ctx->s_kern;
     SegmentParams p;
     memset(&p, 0, sizeof(p));
     int64_t bytes = 0;
@@ -704,47 +718,59 @@ kvx_status state_copy(kvx_ctx* ctx, int32_t L, void* const* layer_base, int64_t 
       Segment& s = p.seg[p.n_seg++];
       s.src = to_host ? dev : host;
       s.dst = to_host ? host : dev;
-      s.bytes = slot_bytes;
-      p.total_units += (slot_bytes + 32767) / 32768;
-      s.unit_end = p.total_units;
+      p.total_bytes += slot_bytes;
+      s.byte_end = p.total_bytes;
       bytes += slot_bytes;
       if (p.n_seg == kMaxSegments || l == L - 1) {
-        int64_t grid = (p.total_units + 7) / 8;
+        // Warps of at most 32 KiB units, then the unit size that splits the
+        // bytes evenly over those warps in whole rounds: with 32 KiB units a
+        // 48-layer state snapshot took 3 rounds of 608 warps where 2.7 suffice.
+        constexpr int64_t kMaxUnit = 32 << 10, kWarps = kThreads / 32;
+        int64_t grid = (p.total_bytes + kMaxUnit * kWarps - 1) / (kMaxUnit * kWarps);
         int64_t cap = (int64_t)ctx->num_sms * ctx->seg_occ;
         cap = std::min<int64_t>(cap, ctx->opts.max_ctas > 0 ? ctx->opts.max_ctas : ctx->link_ctas);
         grid = std::max<int64_t>(1, std::min(grid, cap));
+        const int64_t warps = grid * kWarps;
+        const int64_t rounds = (p.total_bytes + warps * kMaxUnit - 1) / (warps * kMaxUnit);
+        const int64_t share = (p.total_bytes + warps * rounds - 1) / (warps * rounds);
+        p.unit_bytes = std::max<int64_t>(512, (share + 511) / 512 * 512);
+        p.total_units = (p.total_bytes + p.unit_bytes - 1) / p.unit_bytes;
         const bool timing = (ctx->opts.flags & KVX_FLAG_TIME_KERNELS) != 0;
         cudaEvent_t a = timing ? take_timing_event(ctx) : nullptr;
         cudaEvent_t b = timing ? take_timing_event(ctx) : nullptr;
-        if (a && b) KVX_CUDA(cudaEventRecord(a, ctx->s_kern));
-        KVX_CUDA(launch_segments(p, (int)grid, ctx->s_kern));
+        if (a && b) KVX_CUDA(cudaEventRecord(a, ks));
+        KVX_CUDA(launch_segments(p, (int)grid, ks));
         ctx->launches++;
         if (a && b) {
-          KVX_CUDA(cudaEventRecord(b, ctx->s_kern));
+          KVX_CUDA(cudaEventRecord(b, ks));
           ctx->pending.push_back({a, b, 2 * bytes, to_host ? 0 : 1});
         }
         memset(&p, 0, sizeof(p));
         bytes = 0;
       }
     }
-    KVX_CUDA(cudaEventRecord(ctx->ev_kern_done, ctx->s_kern));
-    KVX_CUDA(cudaStreamWaitEvent(stream, ctx->ev_kern_done, 0));
+    if (!ordered) {
+      KVX_CUDA(cudaEventRecord(ctx->ev_kern_done, ctx->s_kern));
+      KVX_CUDA(cudaStreamWaitEvent(stream, ctx->ev_kern_done, 0));
+    }
     return KVX_OK;
   }
   // Staged mode: the slot of each layer is already contiguous, so the copy
   // engines move it directly; no staging buffer is needed.
-  if (ordered) KVX_CUDA(cudaStreamWaitEvent(ctx->s_copy, ctx->ev_in, 0));
+  cudaStream_t cs = ordered ? stream : ctx->s_copy;
   for (int32_t l = 0; l < L; ++l) {
     uint8_t* dev = (uint8_t*)layer_base[l] + slot * slot_bytes;
     uint8_t* host = (uint8_t*)host_obj + (int64_t)l * slot_bytes;
     if (to_host)
-      KVX_CUDA(cudaMemcpyAsync(host, dev, (size_t)slot_bytes, cudaMemcpyDeviceToHost, ctx->s_copy));
+      KVX_CUDA(cudaMemcpyAsync(host, dev, (size_t)slot_bytes, cudaMemcpyDeviceToHost, cs));
     else
-      KVX_CUDA(cudaMemcpyAsync(dev, host, (size_t)slot_bytes, cudaMemcpyHostToDevice, ctx->s_copy));
+      KVX_CUDA(cudaMemcpyAsync(dev, host, (size_t)slot_bytes, cudaMemcpyHostToDevice, cs));
     ctx->memcpys++;
   }
-  KVX_CUDA(cudaEventRecord(ctx->ev_copy_done, ctx->s_copy));
-  KVX_CUDA(cudaStreamWaitEvent(stream, ctx->ev_copy_done, 0));
+  if (!ordered) {
+    KVX_CUDA(cudaEventRecord(ctx->ev_copy_done, ctx->s_copy));
+    KVX_CUDA(cudaStreamWaitEvent(stream, ctx->ev_copy_done, 0));
+  }
   return KVX_OK;
 }
 

@@ -181,9 +181,9 @@ __global__ void __launch_bounds__(kThreads, 4) move_kernel(const __grid_constant
   }
 }
 
-// Opaque byte segments (recurrent-state slots), 32 KiB per warp unit.
-constexpr int64_t kSegUnit = 32 * 1024;
-
+// Opaque byte segments (recurrent-state slots): warp units of p.unit_bytes
+// over the concatenated segments; a unit that crosses a segment end continues
+// in the next segment.  Every piece is a multiple of 16 bytes.
 __global__ void __launch_bounds__(kThreads) segment_kernel(const __grid_constant__ SegmentParams p) {
   const int lane = threadIdx.x & 31;
   const int64_t nwarps = ((int64_t)gridDim.x * kThreads) >> 5;
@@ -191,14 +191,22 @@ __global__ void __launch_bounds__(kThreads) segment_kernel(const __grid_constant
   int j = 0;
   int64_t seg_begin = 0;
   for (; u < p.total_units; u += nwarps) {
-    while (u >= p.seg[j].unit_end) {
-      seg_begin = p.seg[j].unit_end;
+    int64_t b = u * p.unit_bytes;
+    const int64_t b_end = min(b + p.unit_bytes, p.total_bytes);
+    while (b >= p.seg[j].byte_end) {  // warp-uniform; units ascend per warp
+      seg_begin = p.seg[j].byte_end;
       ++j;
     }
-    const Segment& S = p.seg[j];
-    const int64_t off = (u - seg_begin) * kSegUnit;
-    const int64_t n = min(kSegUnit, S.bytes - off);
-    move_flat<kPack>(const_cast<uint8_t*>(S.src) + off, S.dst + off, n, lane);
+    while (b < b_end) {
+      const Segment& S = p.seg[j];
+      const int64_t n = min(b_end, S.byte_end) - b;
+      move_flat<kPack>(const_cast<uint8_t*>(S.src) + (b - seg_begin), S.dst + (b - seg_begin), n, lane);
+      b += n;
+      if (b >= S.byte_end && b < b_end) {
+        seg_begin = S.byte_end;
+        ++j;
+      }
+    }
   }
 }
 

@@ -23,9 +23,10 @@ def disarm():
     kvx().kv_fault_inject(None)
 
 
-# (mode, point, after): a launch failing after the first launch of a 3-launch zero-copy store;
-# a staged copy failing after a few copies; the ordering event failing at once
-CASES = [(2, "launch", 1), (1, "memcpy", 3), (1, "launch", 2), (2, "event", 0), (1, "event", 0)]
+# (mode, point, after): the first, or the second, launch of a 3-launch zero-copy store
+# failing (zero-copy moves run on the caller's stream: no event); a staged copy failing
+# after a few copies; a staged launch failing; the staged pipeline's ordering event failing
+CASES = [(2, "launch", 1), (2, "launch", 0), (1, "memcpy", 3), (1, "launch", 2), (1, "event", 0)]
 
 
 @pytest.mark.parametrize("mode,point,after", CASES)

@@ -282,10 +282,13 @@ def test_special_streams(orc, ctxs, which):
 
 
 @pytest.mark.parametrize("mode", list(MODES))
-def test_state_snapshot_parity(orc, ctxs, mode):
-    """Recurrent-state snapshots: slot 3 of 5 layers out to host, then into slot 1."""
+@pytest.mark.parametrize("L,slots,sb", [(5, 4, 16 * 128 * 128 * 4 // 64), (3, 4, 81968), (120, 4, 16016),
+                                         (1, 4, 16), (48, 4, 1097728)])
+def test_state_snapshot_parity(orc, ctxs, mode, L, slots, sb):
+    """Recurrent-state snapshots: slot 3 of L layers out to host, then into slot 1.
+    Slot sizes that are not multiples of the copy unit make units cross layer
+    ends; 120 layers take two launches; 48 x 1,097,728 B is the hybrid model's."""
     k = kvx()
-    L, slots, sb = 5, 4, 16 * 128 * 128 * 4 // 64
     layers_np = [synth.splitmix64_bytes(slots * sb, 900 + l) for l in range(L)]
     layers = [torch.from_numpy(a).cuda() for a in layers_np]
     obj = torch.full((L * sb,), POISON, dtype=torch.uint8).pin_memory()
