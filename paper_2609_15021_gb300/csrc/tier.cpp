@@ -50,7 +50,7 @@ using namespace kvx;
 
 namespace {
 
-constexpr uint64_t kMagic = 0x3252454954584B56ull;  // "VKXTIER2"
+constexpr uint64_t kMagic = 0x3352454954584B56ull;  // "VKXTIER3"
 constexpr int64_t kDataAlign = 2ll << 20;
 constexpr int kHolders = 8;  // processes that may pin one entry at the same time
 
@@ -59,6 +59,7 @@ enum SlotState : int32_t { kFree = 0, kWriting = 1, kCommitting = 2, kReady = 3 
 struct Header {
   uint64_t magic;
   int64_t slot_bytes, n_slots, data_offset, total_bytes;
+  int64_t index_size;  // entries of the key index: a power of two >= 2 * n_slots
   pthread_mutex_t mu;
   uint64_t clock;
   int64_t hits, misses, evictions;
@@ -133,9 +134,10 @@ struct PendingEvent {
 }  // namespace
 
 struct kvx_tier {
-  // the slot table and counters: in shared memory for a shared tier
+  // the slot table, key index and counters: in shared memory for a shared tier
   Header* hdr = nullptr;
   SlotMeta* meta = nullptr;
+  int64_t* index = nullptr;  // open addressing, linear probing: slot or -1 (empty)
   uint8_t* data = nullptr;
   // ownership
   void* mapping = nullptr;   // shared: the whole mmap; private: the metadata allocation
@@ -152,7 +154,6 @@ struct kvx_tier {
   std::unordered_map<int64_t, cudaEvent_t> commit_event;  // slot -> event readers here may wait on
   std::vector<cudaEvent_t> spare;
   std::mutex local;          // guards the members above
-  std::unordered_map<uint64_t, int64_t> index;  // private tier: key -> slot
 };
 
 namespace {
@@ -220,16 +221,70 @@ void poll_locked(kvx_tier* t, bool wait) {
   }
 }
 
-int64_t find_slot(kvx_tier* t, uint64_t key) {
-  if (!t->shared) {
-    auto it = t->index.find(key);
-    if (it == t->index.end()) return -1;
-    const SlotMeta& m = t->meta[it->second];
-    return m.state != kFree && m.key == key ? it->second : -1;
+// Key index: every slot that is not FREE has exactly one entry, at or after
+// (cyclically) the home position of its key; lookups cost O(1) on average
+// instead of a scan of every slot.
+int64_t index_size_for(int64_t n_slots) {
+  int64_t h = 2;
+  while (h < 2 * n_slots) h <<= 1;
+  return h;
+}
+
+int64_t index_home(const kvx_tier* t, uint64_t key) {
+  return (int64_t)(mix64(key) & (uint64_t)(t->hdr->index_size - 1));
+}
+
+// Position of key in the index, or -1.
+int64_t index_pos(const kvx_tier* t, uint64_t key) {
+  const int64_t mask = t->hdr->index_size - 1;
+  int64_t i = index_home(t, key);
+  for (int64_t n = 0; n <= mask; ++n, i = (i + 1) & mask) {
+    const int64_t s = t->index[i];
+    if (s < 0) return -1;
+    if (t->meta[s].key == key) return i;
   }
-  for (int64_t i = 0; i < t->hdr->n_slots; ++i)
-    if (t->meta[i].state != kFree && t->meta[i].key == key) return i;
   return -1;
+}
+
+// The index has twice as many entries as slots, so a free entry always exists.
+void index_insert(kvx_tier* t, uint64_t key, int64_t slot) {
+  const int64_t mask = t->hdr->index_size - 1;
+  int64_t i = index_home(t, key);
+  while (t->index[i] >= 0) i = (i + 1) & mask;
+  t->index[i] = slot;
+}
+
+// Removes the entry at position i, moving later entries of the same probe run
+// back so that no lookup meets a hole before its key (deletion without
+// tombstones for linear probing, Knuth TAOCP vol. 3, 6.4 Algorithm R).
+void index_erase_at(kvx_tier* t, int64_t i) {
+  const int64_t mask = t->hdr->index_size - 1;
+  int64_t j = i;
+  for (;;) {
+    j = (j + 1) & mask;
+    const int64_t s = t->index[j];
+    if (s < 0) break;
+    const int64_t k = index_home(t, t->meta[s].key);
+    const bool stays = i <= j ? (i < k && k <= j) : (i < k || k <= j);
+    if (stays) continue;
+    t->index[i] = s;
+    i = j;
+  }
+  t->index[i] = -1;
+}
+
+// Drops the index entry of a slot that becomes FREE or takes another key
+// (called while the slot still holds its old key).
+void index_erase(kvx_tier* t, uint64_t key) {
+  const int64_t i = index_pos(t, key);
+  if (i >= 0) index_erase_at(t, i);
+}
+
+int64_t find_slot(kvx_tier* t, uint64_t key) {
+  const int64_t i = index_pos(t, key);
+  if (i < 0) return -1;
+  const int64_t s = t->index[i];
+  return t->meta[s].state != kFree ? s : -1;
 }
 
 // Free slot, else the least recently used slot that is READY and unpinned; -1 if none.
@@ -276,6 +331,7 @@ int64_t reclaim_locked(kvx_tier* t) {
     if (m.state == kFree) continue;
     bool c = false;
     if ((m.state == kWriting || m.state == kCommitting) && is_gone(m.writer_pid)) {
+      index_erase(t, m.key);
       m.state = kFree;
       clear_pins(m);
       c = true;
@@ -319,24 +375,36 @@ void destroy_tier(kvx_tier* t) {
   delete t;
 }
 
+// Bytes of the header, the slot table and the key index of an n-slot tier.
+int64_t metadata_bytes(int64_t n_slots) {
+  return (int64_t)sizeof(Header) + n_slots * (int64_t)sizeof(SlotMeta) + index_size_for(n_slots) * 8;
+}
+
+// Points t's table and index into the metadata at m (the header already filled).
+void attach_metadata(kvx_tier* t, void* m) {
+  t->hdr = (Header*)m;
+  t->meta = (SlotMeta*)((uint8_t*)m + sizeof(Header));
+  t->index = (int64_t*)((uint8_t*)t->meta + t->hdr->n_slots * (int64_t)sizeof(SlotMeta));
+}
+
 kvx_status init_private(void* base, int64_t slot_bytes, int64_t n_slots, kvx_tier** out) {
   kvx_tier* t = new (std::nothrow) kvx_tier;
   if (!t) return KVX_ENOMEM;
-  const int64_t meta_bytes = (int64_t)sizeof(Header) + n_slots * (int64_t)sizeof(SlotMeta);
-  void* m = calloc(1, (size_t)meta_bytes);
+  void* m = calloc(1, (size_t)metadata_bytes(n_slots));
   if (!m) {
     delete t;
     return KVX_ENOMEM;
   }
   t->mapping = m;
-  t->hdr = (Header*)m;
-  t->meta = (SlotMeta*)((uint8_t*)m + sizeof(Header));
-  t->data = (uint8_t*)base;
-  t->pid = (int32_t)getpid();
-  Header* h = t->hdr;
+  Header* h = (Header*)m;
   h->magic = kMagic;
   h->slot_bytes = slot_bytes;
   h->n_slots = n_slots;
+  h->index_size = index_size_for(n_slots);
+  attach_metadata(t, m);
+  memset(t->index, 0xFF, (size_t)h->index_size * 8);  // every entry -1: empty
+  t->data = (uint8_t*)base;
+  t->pid = (int32_t)getpid();
   pthread_mutex_init(&h->mu, nullptr);
   h->initialised = 1;
   *out = t;
@@ -401,7 +469,7 @@ kvx_status kv_tier_open_shared(const char* name, int64_t slot_bytes, int64_t n_s
   }
   int64_t total = 0, data_offset = 0;
   if (create) {
-    const int64_t meta_bytes = (int64_t)sizeof(Header) + n_slots * (int64_t)sizeof(SlotMeta);
+    const int64_t meta_bytes = metadata_bytes(n_slots);
     data_offset = (meta_bytes + kDataAlign - 1) / kDataAlign * kDataAlign;
     if (n_slots > (INT64_MAX - data_offset) / slot_bytes) {
       close(fd);
@@ -446,15 +514,17 @@ kvx_status kv_tier_open_shared(const char* name, int64_t slot_bytes, int64_t n_s
   t->mapping_bytes = total;
   t->pid = (int32_t)getpid();
   snprintf(t->name, sizeof(t->name), "%s", name);
-  t->hdr = (Header*)map;
-  t->meta = (SlotMeta*)((uint8_t*)map + sizeof(Header));
-  Header* h = t->hdr;
+  Header* h = (Header*)map;
+  t->hdr = h;
   if (create) {
     h->magic = kMagic;
     h->slot_bytes = slot_bytes;
     h->n_slots = n_slots;
     h->data_offset = data_offset;
     h->total_bytes = total;
+    h->index_size = index_size_for(n_slots);
+    attach_metadata(t, map);
+    memset(t->index, 0xFF, (size_t)h->index_size * 8);  // every entry -1: empty
     pthread_mutexattr_t a;
     pthread_mutexattr_init(&a);
     pthread_mutexattr_setpshared(&a, PTHREAD_PROCESS_SHARED);
@@ -465,12 +535,14 @@ kvx_status kv_tier_open_shared(const char* name, int64_t slot_bytes, int64_t n_s
   } else {
     int i = 0;
     while (__atomic_load_n(&h->initialised, __ATOMIC_ACQUIRE) != 1 && i++ < 5000) usleep(1000);
-    if (h->initialised != 1 || h->magic != kMagic || h->total_bytes != total) {
+    if (h->initialised != 1 || h->magic != kMagic || h->total_bytes != total ||
+        h->index_size != index_size_for(h->n_slots) || metadata_bytes(h->n_slots) > h->data_offset) {
       munmap(map, (size_t)total);
       delete t;
       set_error_text("the shared tier is not initialised or does not match");
       return KVX_EINVAL;
     }
+    attach_metadata(t, map);
   }
   t->data = (uint8_t*)map + h->data_offset;
   if (!(flags & KVX_TIER_NO_PIN)) {
@@ -516,10 +588,11 @@ kvx_status kv_tier_reserve(kvx_tier* t, uint64_t key, void** slot) {
     if (i >= 0) {
       SlotMeta& m = t->meta[i];
       if (m.state != kFree) {
-        if (!t->shared) t->index.erase(m.key);
+        index_erase(t, m.key);
         t->hdr->evictions++;
       }
-      if (!t->shared) t->index[key] = i;
+      m.key = key;
+      index_insert(t, key, i);
       break;
     }
   }
@@ -621,8 +694,8 @@ kvx_status kv_tier_release(kvx_tier* t, uint64_t key, kvx_stream_t stream) {
   if (no_stream(stream)) {
     add_pins(m, t->pid, -1);
     if (m.state == kWriting && m.pins == 0) {  // a writer giving up its reservation
+      index_erase(t, m.key);
       m.state = kFree;
-      if (!t->shared) t->index.erase(m.key);
     }
     return KVX_OK;
   }

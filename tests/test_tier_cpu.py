@@ -122,3 +122,131 @@ def test_abandoned_reservation_frees_its_key(k):
     assert e.value.status == k.KVX_ENOENT
     assert int(tier.acquire(22, NO)[0]) == 22
     tier.release(22, NO)
+
+
+class _Model:
+    """The tier's documented rules for one process with KVX_NO_STREAM: a reserve takes
+    the key's own READY unpinned slot, else the first FREE slot, else the least
+    recently used READY unpinned slot; commit makes READY; acquire pins a READY
+    entry; release unpins, and frees a reservation given up."""
+
+    def __init__(self, n):
+        self.slots = [{"key": None, "state": "FREE", "pins": 0, "tick": 0} for _ in range(n)]
+        self.clock = 0
+        self.hits = self.misses = self.evictions = 0
+
+    def find(self, key):
+        for i, s in enumerate(self.slots):
+            if s["state"] != "FREE" and s["key"] == key:
+                return i
+        return None
+
+    def reserve(self, key):
+        i = self.find(key)
+        if i is not None:
+            s = self.slots[i]
+            if s["pins"] > 0 or s["state"] != "READY":
+                return "EBUSY", None
+        else:
+            free = [j for j, s in enumerate(self.slots) if s["state"] == "FREE"]
+            if free:
+                i = free[0]
+            else:
+                cand = [j for j, s in enumerate(self.slots) if s["state"] == "READY" and s["pins"] == 0]
+                if not cand:
+                    return "ENOMEM", None
+                i = min(cand, key=lambda j: self.slots[j]["tick"])
+                self.evictions += 1
+        self.clock += 1
+        self.slots[i] = {"key": key, "state": "WRITING", "pins": 1, "tick": self.clock}
+        return "OK", i
+
+    def commit(self, key):
+        i = self.find(key)
+        if i is None:
+            return "ENOENT"
+        s = self.slots[i]
+        if s["state"] != "WRITING":
+            return "EINVAL"
+        s["state"], s["pins"] = "READY", s["pins"] - 1
+        self.clock += 1
+        s["tick"] = self.clock
+        return "OK"
+
+    def acquire(self, key):
+        i = self.find(key)
+        if i is None or self.slots[i]["state"] != "READY":
+            self.misses += 1
+            return "ENOENT"
+        s = self.slots[i]
+        s["pins"] += 1
+        self.clock += 1
+        s["tick"] = self.clock
+        self.hits += 1
+        return "OK"
+
+    def release(self, key):
+        i = self.find(key)
+        if i is None:
+            return "ENOENT"
+        s = self.slots[i]
+        if s["pins"] < 1:
+            return "EINVAL"
+        s["pins"] -= 1
+        if s["state"] == "WRITING" and s["pins"] == 0:
+            s["state"] = "FREE"
+        return "OK"
+
+    def prefix_hits(self, keys):
+        h = 0
+        for key in keys:
+            i = self.find(key)
+            if i is None or self.slots[i]["state"] != "READY":
+                break
+            h += 1
+        return h
+
+
+@pytest.mark.parametrize("seed,n_slots,n_keys", [(1, 5, 12), (2, 1, 3), (3, 16, 40), (4, 64, 70)])
+def test_tier_follows_its_rules_under_random_operations(k, seed, n_slots, n_keys):
+    """Thousands of random operations against a model of the documented rules:
+    statuses, hits / misses / evictions, prefix hits, and the bytes in every slot
+    handed out (each key's slot holds that key's pattern)."""
+    tier, buf = _tier(k, n_slots)
+    model = _Model(n_slots)
+    rng = np.random.default_rng(seed)
+    status = {k.KVX_EBUSY: "EBUSY", k.KVX_ENOMEM: "ENOMEM", k.KVX_ENOENT: "ENOENT", k.KVX_EINVAL: "EINVAL"}
+
+    def call(fn, *a):
+        try:
+            return "OK", fn(*a)
+        except k.KvxError as e:
+            return status[e.status], None
+
+    for step in range(4000):
+        key = int(rng.integers(1, n_keys + 1)) * 1000003
+        op = rng.choice(["reserve", "commit", "acquire", "release", "prefix"], p=[0.3, 0.25, 0.2, 0.2, 0.05])
+        if op == "reserve":
+            got, view = call(tier.reserve, key)
+            want, _ = model.reserve(key)
+            if got == "OK":
+                view.fill_(key % 251)
+        elif op == "commit":
+            got, _ = call(tier.commit, key, NO)
+            want = model.commit(key)
+        elif op == "acquire":
+            got, view = call(tier.acquire, key, NO)
+            want = model.acquire(key)
+            if got == "OK":
+                assert int(view[0]) == key % 251 and int(view[-1]) == key % 251, step
+        elif op == "release":
+            got, _ = call(tier.release, key, NO)
+            want = model.release(key)
+        else:
+            keys = [int(x) * 1000003 for x in rng.integers(1, n_keys + 1, size=4)]
+            got, want = tier.prefix_hits(keys), model.prefix_hits(keys)
+        assert got == want, (step, op, key, got, want)
+    st = tier.stats()
+    assert (st["hits"], st["misses"], st["evictions"]) == (model.hits, model.misses, model.evictions)
+    assert st["entries"] == sum(s["state"] != "FREE" for s in model.slots)
+    assert st["pinned"] == sum(s["pins"] > 0 for s in model.slots)
