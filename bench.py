@@ -185,9 +185,9 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-hbm-roofline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--host-alloc", choices=["cuda", "numa"], default="cuda",
-                    help="pinned pool from kv_host_alloc (cudaHostAlloc) or kv_host_alloc_numa on the "
-                         "host node nearest the GPU")
+    ap.add_argument("--host-alloc", choices=["plain", "numa"], default="plain",
+                    help="pinned pool from kv_host_alloc, or from kv_host_alloc_numa on the host NUMA "
+                         "node nearest the GPU")
     ap.add_argument("--no-concurrent", action="store_true",
                     help="skip the two-replica leg (one stores while the other restores)")
     ap.add_argument("--device-engine", choices=["lsu", "tma"], default="tma",
@@ -356,6 +356,24 @@ def host_mem_available() -> int:
     except OSError:
         pass
     return 0
+
+
+def huge_page_bytes(ptr: int, nbytes: int) -> int | None:
+    """Bytes of [ptr, ptr + nbytes) that transparent huge pages back (AnonHugePages of
+    the overlapping mappings in /proc/self/smaps), or None where that is unknown."""
+    try:
+        total, overlap = 0, False
+        with open("/proc/self/smaps") as f:
+            for line in f:
+                head = line.split()[0]
+                if "-" in head and ":" not in head:
+                    lo, hi = (int(x, 16) for x in head.split("-"))
+                    overlap = lo < ptr + nbytes and hi > ptr
+                elif overlap and line.startswith("AnonHugePages:"):
+                    total += int(line.split()[1]) * 1024
+        return total
+    except (OSError, ValueError):
+        return None
 
 
 def cpu_model() -> str:
@@ -623,6 +641,7 @@ def run_ours(args):
                    "parallelism": f"replicas x{world}", "pinned_host_bytes": n_chunks * cb,
                    "host_alloc": args.host_alloc if host_pool.numa_node is None
                    else f"numa node {host_pool.numa_node}",
+                   "host_pool_huge_page_bytes": huge_page_bytes(host_pool.ptr, n_chunks * cb),
                    "pin_seconds": pin_seconds},
         "restore_ms": {"median": statistics.median(restore_ms), "min": min(restore_ms), "max": max(restore_ms),
                        "n": len(restore_ms)},

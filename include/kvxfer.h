@@ -315,11 +315,13 @@ kvx_status kv_store_noalloc(const kvx_pool* pool, const int32_t* block_table, in
  * Page-locked host memory for a shared chunk pool (Sec. 3.3: the shared tier
  * is one full-size pinned allocation; the paper's 256 GiB + 4096 B request
  * was rounded up to a power of two by the framework's pinned allocator and
- * silently fell back to pageable memory).  kv_host_alloc allocates exactly
- * `bytes` (no rounding), portable to every device and mapped for zero-copy,
- * checks that the result is page-locked, and otherwise fails: KVX_ENOMEM when
- * the memory is not available, never a pageable fallback.  Free with
- * kv_host_free (NULL is ignored).
+ * silently fell back to pageable memory).  kv_host_alloc maps `bytes` (the
+ * mapping is rounded up to whole huge pages, never to a power of two), backs
+ * pools of at least one huge page with transparent huge pages, and registers
+ * it page-locked, portable to every device and mapped for zero-copy.  Huge
+ * pages are what let the copy engines (KVX_MODE_STAGED) reach the link peak
+ * on a host with small base pages.  Failure is KVX_ENOMEM or KVX_ECUDA, never
+ * a pageable fallback.  Free with kv_host_free (NULL is ignored).
  */
 kvx_status kv_host_alloc(int64_t bytes, void** out);
 /*
@@ -327,9 +329,8 @@ kvx_status kv_host_alloc(int64_t bytes, void** out);
  * nodes the pool belongs on the node next to the GPU that uses it, or every
  * zero-copy access also crosses the link between sockets.  numa_node >= 0
  * names the node; KVX_NUMA_NEAREST asks for the node CUDA reports as closest
- * to the current device (no placement if it reports none).  The memory is
- * anonymous memory with a preferred-node policy (mbind), registered
- * page-locked, portable and mapped, exactly `bytes` long as seen by callers.
+ * to the current device (no placement if it reports none).  The memory gets
+ * a preferred-node policy (mbind) before it is faulted in.
  * KVX_EINVAL for a node that does not exist, KVX_ENOMEM if the node has less
  * free memory than `bytes` or the memory cannot be pinned (never a pageable
  * fallback).  *numa_out (may be NULL) receives the node of the first page,
@@ -337,7 +338,8 @@ kvx_status kv_host_alloc(int64_t bytes, void** out);
  */
 #define KVX_NUMA_NEAREST (-1)
 kvx_status kv_host_alloc_numa(int32_t numa_node, int64_t bytes, void** out, int32_t* numa_out);
-/* Frees kv_host_alloc and kv_host_alloc_numa memory; NULL is ignored. */
+/* Frees kv_host_alloc and kv_host_alloc_numa memory; NULL and pointers the
+   library did not allocate are ignored. */
 void kv_host_free(void* host);
 
 /* ------------------------------------------------------------------------

@@ -107,8 +107,7 @@ int segment_ctas_per_sm();
 // Records the last CUDA error seen by this thread (kv_last_cuda_error).
 void set_last_cuda_error(int e);
 
-// True if p was allocated by kv_host_alloc_numa; it is then unregistered and
-// unmapped (numa_alloc.cpp).
-bool free_numa_allocation(void* p);
+// Host-side fault injection (kv_fault_inject): true if the armed point fails now.
+bool fault_point(const char* point);
 
 }  // namespace kvx

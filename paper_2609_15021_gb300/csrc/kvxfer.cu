@@ -67,6 +67,10 @@ bool fault_now(const char* point) {
 }
 }  // namespace
 
+namespace kvx {
+bool fault_point(const char* point) { return fault_now(point); }
+}  // namespace kvx
+
 #define KVX_CUDA_AT(point, call)                                                   \
   do {                                                                             \
     cudaError_t e_ = fault_now(point) ? cudaErrorUnknown : (call);                 \
@@ -1046,39 +1050,6 @@ kvx_status kv_pool_view_check(const kvx_pool* pool, int32_t ndim, const int64_t*
     stride *= shape[d];
   }
   return KVX_OK;
-}
-
-kvx_status kv_host_alloc(int64_t bytes, void** out) {
-  if (!out) return KVX_EINVAL;
-  *out = nullptr;
-  if (bytes <= 0) return KVX_EINVAL;
-  void* p = nullptr;
-  // Exactly `bytes`, no rounding; portable and mapped so every context and
-  // the zero-copy kernels can use it.  No pageable fallback: a failure is an
-  // error (Sec. 3.3: a full-pool request that silently fell back to pageable
-  // memory).
-  cudaError_t e = fault_now("host_alloc")
-                      ? cudaErrorMemoryAllocation
-                      : cudaHostAlloc(&p, (size_t)bytes, cudaHostAllocPortable | cudaHostAllocMapped);
-  if (e != cudaSuccess) {
-    record_cuda_error((int)e, "cudaHostAlloc", __LINE__);
-    cudaGetLastError();
-    return e == cudaErrorMemoryAllocation ? KVX_ENOMEM : KVX_ECUDA;
-  }
-  uint8_t* mapped = nullptr;
-  if (check_pinned_range(p, bytes, &mapped) != KVX_OK) {
-    cudaFreeHost(p);
-    return KVX_ENOTPINNED;
-  }
-  *out = p;
-  return KVX_OK;
-}
-
-void kv_host_free(void* p) {
-  if (p && !free_numa_allocation(p)) {
-    cudaFreeHost(p);
-    cudaGetLastError();
-  }
 }
 
 kvx_status kv_get_device_error(kvx_ctx* ctx, int64_t* first_bad_block) {
