@@ -75,9 +75,15 @@ def load_peaks():
 
 
 def kernel_source_hash(source="pack_kernels.cu"):
-    p = os.path.join(ROOT, "paper_2609_15021_gb300", "csrc", source)
-    with open(p, "rb") as f:
-        return hashlib.sha256(f.read()).hexdigest()[:16]
+    """sha256 prefix of a kernel source file and the device headers (.cuh) it includes."""
+    csrc = os.path.join(ROOT, "paper_2609_15021_gb300", "csrc")
+    with open(os.path.join(csrc, source), "rb") as f:
+        text = f.read()
+    h = hashlib.sha256(text)
+    for inc in re.findall(rb'#include "([^"]+\.cuh)"', text):
+        with open(os.path.join(csrc, inc.decode()), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
 
 
 def shape_key(s):
@@ -185,9 +191,9 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-hbm-roofline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--host-alloc", choices=["plain", "numa"], default="plain",
-                    help="pinned pool from kv_host_alloc, or from kv_host_alloc_numa on the host NUMA "
-                         "node nearest the GPU")
+    ap.add_argument("--host-alloc", choices=["plain", "numa", "driver"], default="plain",
+                    help="pinned pool from kv_host_alloc, from kv_host_alloc_numa on the host NUMA "
+                         "node nearest the GPU, or from the driver's allocator (KVX_HOST_DRIVER)")
     ap.add_argument("--no-concurrent", action="store_true",
                     help="skip the two-replica leg (one stores while the other restores)")
     ap.add_argument("--device-engine", choices=["lsu", "tma"], default="tma",
@@ -423,7 +429,8 @@ def run_ours(args):
     tb = torch.from_numpy(tb_np).to(dev)
     t_pin = time.perf_counter()
     # exact-size pinned, mapped pool (no power-of-two rounding)
-    host_pool = k.HostBuffer(n_chunks * cb, numa_node=k.KVX_NUMA_NEAREST if args.host_alloc == "numa" else None)
+    host_pool = k.HostBuffer(n_chunks * cb, numa_node=k.KVX_NUMA_NEAREST if args.host_alloc == "numa" else None,
+                             driver=args.host_alloc == "driver")
     pin_seconds = time.perf_counter() - t_pin
     chunks = [host_pool.tensor[i * cb:(i + 1) * cb] for i in range(n_chunks)]
 

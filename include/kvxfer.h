@@ -338,6 +338,21 @@ kvx_status kv_host_alloc(int64_t bytes, void** out);
  */
 #define KVX_NUMA_NEAREST (-1)
 kvx_status kv_host_alloc_numa(int32_t numa_node, int64_t bytes, void** out, int32_t* numa_out);
+/*
+ * Both of the above, with the choices spelled out.  numa_node: KVX_NUMA_ANY
+ * (no placement), KVX_NUMA_NEAREST, or a node.  flags: KVX_HOST_DRIVER takes
+ * the memory from the driver's pinned allocator (cudaHostAlloc, portable and
+ * mapped) instead of the library's huge-page mapping; numa_node must then be
+ * KVX_NUMA_ANY.  Without a placement, a pool smaller than one huge page, or
+ * any pool on a host without transparent huge pages, also comes from the
+ * driver's allocator.  kv_host_alloc(b, o) is kv_host_alloc_ex(b,
+ * KVX_NUMA_ANY, 0, o, NULL).  Memory from either source zero-copies at the
+ * link peak; only huge pages let the copy engines (KVX_MODE_STAGED) reach it
+ * steadily on a host with small base pages.
+ */
+#define KVX_NUMA_ANY (-2)
+#define KVX_HOST_DRIVER 0x1u
+kvx_status kv_host_alloc_ex(int64_t bytes, int32_t numa_node, uint32_t flags, void** out, int32_t* numa_out);
 /* Frees kv_host_alloc and kv_host_alloc_numa memory; NULL and pointers the
    library did not allocate are ignored. */
 void kv_host_free(void* host);

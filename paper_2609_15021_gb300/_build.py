@@ -13,7 +13,7 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "_lib", "libkvxfer.so")
 
-SOURCES = ["pack_kernels.cu", "tma_kernels.cu", "kvxfer.cu", "probe.cu", "no_alloc.cu", "tier.cpp",
+SOURCES = ["pack_kernels.cu", "segment_kernels.cu", "tma_kernels.cu", "kvxfer.cu", "probe.cu", "no_alloc.cu", "tier.cpp",
            "host_alloc.cpp"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC,-O2", f"-I{INCLUDE}"]
@@ -28,7 +28,7 @@ def _nvcc() -> str:
 
 def _inputs() -> list[str]:
     deps = [os.path.join(CSRC, s) for s in SOURCES]
-    deps += [os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith(".h")]
+    deps += [os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith((".h", ".cuh"))]
     deps += [os.path.join(INCLUDE, f) for f in os.listdir(INCLUDE) if f.endswith(".h")]
     return deps
 

@@ -1,5 +1,5 @@
 // host_alloc.cpp -- page-locked host pools for the shared tier (kv_host_alloc,
-// kv_host_alloc_numa, kv_host_free).
+// kv_host_alloc_numa, kv_host_alloc_ex, kv_host_free).
 //
 // Sec. 3.3: the shared tier is one exact-size pinned pool, and a request that
 // silently fell back to pageable memory was one of the paper's failures.  A
@@ -17,7 +17,10 @@
 // aligned, asked for huge pages, faulted in at once (MADV_POPULATE_WRITE),
 // and any range still on base pages is collapsed into huge pages
 // (MADV_COLLAPSE) before the pages are pinned; both are advice, so the pool
-// is still created if the kernel cannot comply.
+// is still created if the kernel cannot comply.  Where no huge page can back
+// the pool (smaller than one, or a host without transparent huge pages) and
+// no placement is asked, the driver's allocator serves instead, as it does on
+// request (KVX_HOST_DRIVER).
 //
 // NUMA: on a host with several memory nodes the pool belongs on the node next
 // to the GPU that uses it; mbind with a preferred-node policy places it there
@@ -90,12 +93,40 @@ int page_node(void* addr) {
   return status[0] >= 0 ? status[0] : -1;
 }
 
+// Transparent huge pages can be had for a mapping that asks (not "never").
+bool thp_available() {
+  FILE* f = fopen("/sys/kernel/mm/transparent_hugepage/enabled", "r");
+  if (!f) return false;
+  char line[128] = "";
+  const bool ok = fgets(line, sizeof(line), f) != nullptr && strstr(line, "[never]") == nullptr;
+  fclose(f);
+  return ok;
+}
+
+// The driver's pinned allocator (cudaHostAlloc, portable and mapped).
+kvx_status driver_pool(int64_t bytes, void** out) {
+  void* p = nullptr;
+  const cudaError_t e = cudaHostAlloc(&p, (size_t)bytes, cudaHostAllocPortable | cudaHostAllocMapped);
+  if (e != cudaSuccess) {
+    set_last_cuda_error((int)e);
+    set_error_text("cudaHostAlloc of the host pool");
+    cudaGetLastError();
+    return e == cudaErrorMemoryAllocation ? KVX_ENOMEM : KVX_ECUDA;
+  }
+  {
+    std::lock_guard<std::mutex> g(g_mu);
+    g_mappings[p] = 0;  // length 0: freed with cudaFreeHost
+  }
+  *out = p;
+  return KVX_OK;
+}
+
 // Maps, places (node >= 0), backs with huge pages where possible and pins a
 // pool of at least `bytes`.  On success *out is the pool and *len_out the
 // mapped length.
 kvx_status map_pool(int node, int64_t bytes, void** out, size_t* len_out) {
   const size_t page = (size_t)sysconf(_SC_PAGESIZE);
-  const size_t huge = huge_page_bytes();
+  const size_t huge = thp_available() ? huge_page_bytes() : 0;
   const bool use_huge = huge >= page && (size_t)bytes >= huge;
   const size_t unit = use_huge ? huge : page;
   const size_t len = ((size_t)bytes + unit - 1) / unit * unit;
@@ -148,26 +179,29 @@ kvx_status map_pool(int node, int64_t bytes, void** out, size_t* len_out) {
 
 extern "C" {
 
-kvx_status kv_host_alloc(int64_t bytes, void** out) {
-  if (!out) return KVX_EINVAL;
-  *out = nullptr;
-  if (bytes <= 0) return KVX_EINVAL;
-  if (fault_point("host_alloc")) {
-    set_last_cuda_error((int)cudaErrorMemoryAllocation);
-    set_error_text("cudaHostRegister of the host pool (injected fault)");
-    return KVX_ENOMEM;
-  }
-  size_t len = 0;
-  return map_pool(-1, bytes, out, &len);
-}
-
-kvx_status kv_host_alloc_numa(int32_t numa_node, int64_t bytes, void** out, int32_t* numa_out) {
+kvx_status kv_host_alloc_ex(int64_t bytes, int32_t numa_node, uint32_t flags, void** out, int32_t* numa_out) {
   if (!out) return KVX_EINVAL;
   *out = nullptr;
   if (numa_out) *numa_out = -1;
-  if (bytes <= 0 || numa_node < KVX_NUMA_NEAREST || numa_node >= kMaxNodes) return KVX_EINVAL;
+  if (bytes <= 0 || numa_node < KVX_NUMA_ANY || numa_node >= kMaxNodes || (flags & ~KVX_HOST_DRIVER))
+    return KVX_EINVAL;
+  if ((flags & KVX_HOST_DRIVER) && numa_node != KVX_NUMA_ANY) return KVX_EINVAL;
+  if (fault_point("host_alloc")) {
+    set_last_cuda_error((int)cudaErrorMemoryAllocation);
+    set_error_text("pinning of the host pool (injected fault)");
+    return KVX_ENOMEM;
+  }
+  // The driver's allocator where asked, and where the library's mapping would
+  // get no huge pages and no placement anyway (a small pool, or no
+  // transparent huge pages): its memory serves the copy engines better than
+  // base pages do.
+  const size_t huge = thp_available() ? huge_page_bytes() : 0;
+  if ((flags & KVX_HOST_DRIVER) || (numa_node == KVX_NUMA_ANY && (huge == 0 || (size_t)bytes < huge)))
+    return driver_pool(bytes, out);
   int node = numa_node;
-  if (node == KVX_NUMA_NEAREST) {
+  if (node == KVX_NUMA_ANY) {
+    node = -1;
+  } else if (node == KVX_NUMA_NEAREST) {
     int dev = 0, id = -1;
     if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&id, cudaDevAttrHostNumaId, dev) != cudaSuccess)
       id = -1;
@@ -190,6 +224,18 @@ kvx_status kv_host_alloc_numa(int32_t numa_node, int64_t bytes, void** out, int3
   return st;
 }
 
+kvx_status kv_host_alloc(int64_t bytes, void** out) {
+  return kv_host_alloc_ex(bytes, KVX_NUMA_ANY, 0, out, nullptr);
+}
+
+kvx_status kv_host_alloc_numa(int32_t numa_node, int64_t bytes, void** out, int32_t* numa_out) {
+  if (numa_node < KVX_NUMA_NEAREST) {
+    if (out) *out = nullptr;
+    return KVX_EINVAL;
+  }
+  return kv_host_alloc_ex(bytes, numa_node, 0, out, numa_out);
+}
+
 void kv_host_free(void* p) {
   if (!p) return;
   size_t len = 0;
@@ -200,9 +246,14 @@ void kv_host_free(void* p) {
     len = it->second;
     g_mappings.erase(it);
   }
-  cudaHostUnregister(p);
+  if (len == 0) {
+    cudaFreeHost(p);
+  } else {
+    cudaHostUnregister(p);
+    cudaGetLastError();
+    munmap(p, len);
+  }
   cudaGetLastError();
-  munmap(p, len);
 }
 
 }  // extern "C"

@@ -19,61 +19,11 @@
 // Out-of-range block-table entries skip their unit and lower a device error
 // word (atomicMin of the logical block index); nothing traps.
 
+#include "copy16.cuh"
 #include "kvx_internal.h"
 
 namespace kvx {
 namespace {
-
-constexpr int kInflight = 8;  // 16-byte vectors per lane between loads and stores
-
-// Streaming (evict-first) accesses: every byte is touched exactly once.
-__device__ __forceinline__ uint4 ld16(const uint8_t* p) {
-  return __ldcs(reinterpret_cast<const uint4*>(p));
-}
-__device__ __forceinline__ void st16(uint8_t* p, const uint4& v) {
-  __stcs(reinterpret_cast<uint4*>(p), v);
-}
-
-// Move kInflight vectors: pack reads the page side, unpack reads the chunk side.
-template <int DIR>
-__device__ __forceinline__ void move_batch(uint8_t* pg, uint8_t* ck, const int64_t (&po)[kInflight],
-                                           const int64_t (&co)[kInflight]) {
-  uint4 v[kInflight];
-  if (DIR == kPack) {
-#pragma unroll
-    for (int i = 0; i < kInflight; ++i) v[i] = ld16(pg + po[i]);
-#pragma unroll
-    for (int i = 0; i < kInflight; ++i) st16(ck + co[i], v[i]);
-  } else {
-#pragma unroll
-    for (int i = 0; i < kInflight; ++i) v[i] = ld16(ck + co[i]);
-#pragma unroll
-    for (int i = 0; i < kInflight; ++i) st16(pg + po[i], v[i]);
-  }
-}
-
-template <int DIR>
-__device__ __forceinline__ void move_one(uint8_t* pg, uint8_t* ck, int64_t po, int64_t co) {
-  if (DIR == kPack)
-    st16(ck + co, ld16(pg + po));
-  else
-    st16(pg + po, ld16(ck + co));
-}
-
-// Same byte order on both sides (NHD pages, opaque segments): a flat copy of
-// nbytes (a multiple of 16).
-template <int DIR>
-__device__ __forceinline__ void move_flat(uint8_t* pg, uint8_t* ck, int64_t nbytes, int lane) {
-  int64_t off = (int64_t)lane * 16;
-  constexpr int64_t kStep = 32 * 16;
-  for (; off + (kInflight - 1) * kStep < nbytes; off += kInflight * kStep) {
-    int64_t o[kInflight];
-#pragma unroll
-    for (int i = 0; i < kInflight; ++i) o[i] = off + i * kStep;
-    move_batch<DIR>(pg, ck, o, o);
-  }
-  for (; off < nbytes; off += kStep) move_one<DIR>(pg, ck, off, off);
-}
 
 // HND page side [H][B][R] <-> chunk side [nb][H][R], nr = nb * H rows, when
 // R / 16 is a power of two no larger than 32: a warp covers 32 / (R/16) whole
@@ -181,35 +131,6 @@ __global__ void __launch_bounds__(kThreads, 4) move_kernel(const __grid_constant
   }
 }
 
-// Opaque byte segments (recurrent-state slots): warp units of p.unit_bytes
-// over the concatenated segments; a unit that crosses a segment end continues
-// in the next segment.  Every piece is a multiple of 16 bytes.
-__global__ void __launch_bounds__(kThreads) segment_kernel(const __grid_constant__ SegmentParams p) {
-  const int lane = threadIdx.x & 31;
-  const int64_t nwarps = ((int64_t)gridDim.x * kThreads) >> 5;
-  int64_t u = ((int64_t)blockIdx.x * kThreads + threadIdx.x) >> 5;
-  int j = 0;
-  int64_t seg_begin = 0;
-  for (; u < p.total_units; u += nwarps) {
-    int64_t b = u * p.unit_bytes;
-    const int64_t b_end = min(b + p.unit_bytes, p.total_bytes);
-    while (b >= p.seg[j].byte_end) {  // warp-uniform; units ascend per warp
-      seg_begin = p.seg[j].byte_end;
-      ++j;
-    }
-    while (b < b_end) {
-      const Segment& S = p.seg[j];
-      const int64_t n = min(b_end, S.byte_end) - b;
-      move_flat<kPack>(const_cast<uint8_t*>(S.src) + (b - seg_begin), S.dst + (b - seg_begin), n, lane);
-      b += n;
-      if (b >= S.byte_end && b < b_end) {
-        seg_begin = S.byte_end;
-        ++j;
-      }
-    }
-  }
-}
-
 template <int DIR, int LAYOUT>
 int occupancy_of() {
   int n = 0;
@@ -235,25 +156,11 @@ cudaError_t launch_move(int dir, int layout, const MoveParams& p, int grid, cuda
   return cudaGetLastError();
 }
 
-cudaError_t launch_segments(const SegmentParams& p, int grid, cudaStream_t s) {
-  segment_kernel<<<grid, kThreads, 0, s>>>(p);
-  return cudaGetLastError();
-}
-
 int move_ctas_per_sm(int dir, int layout) {
   if (dir == kPack) return layout == KVX_LAYOUT_HND ? occupancy_of<kPack, KVX_LAYOUT_HND>()
                                                     : occupancy_of<kPack, KVX_LAYOUT_NHD>();
   return layout == KVX_LAYOUT_HND ? occupancy_of<kUnpack, KVX_LAYOUT_HND>()
                                   : occupancy_of<kUnpack, KVX_LAYOUT_NHD>();
-}
-
-int segment_ctas_per_sm() {
-  int n = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, segment_kernel, kThreads, 0) != cudaSuccess) {
-    cudaGetLastError();
-    return 1;
-  }
-  return n > 0 ? n : 1;
 }
 
 }  // namespace kvx

@@ -39,7 +39,7 @@ EXPORTED = (
     "kv_host_alloc", "kv_host_free", "kv_pool_view_check",
     "kv_chunk_keys", "kv_tier_create", "kv_tier_create_on", "kv_tier_destroy", "kv_tier_reserve", "kv_tier_commit",
     "kv_tier_acquire", "kv_tier_release", "kv_tier_prefix_hits", "kv_tier_stats", "kv_fault_inject",
-    "kv_tier_open_shared", "kv_tier_poll", "kv_tier_reclaim", "kv_host_alloc_numa",
+    "kv_tier_open_shared", "kv_tier_poll", "kv_tier_reclaim", "kv_host_alloc_numa", "kv_host_alloc_ex",
 )
 KVX_ENOENT, KVX_EBUSY = -8, -9
 KVX_TIER_CREATE, KVX_TIER_NO_PIN = 0x1, 0x2
@@ -112,6 +112,7 @@ def _declare(lib):
         "kv_host_alloc": (st, [i64, P(vp)]),
         "kv_host_free": (None, [vp]),
         "kv_host_alloc_numa": (st, [i32, i64, P(vp), P(i32)]),
+        "kv_host_alloc_ex": (st, [i64, i32, ctypes.c_uint32, P(vp), P(i32)]),
         "kv_pool_view_check": (st, [P(kvx_pool), i32, P(i64), P(i64)]),
         "kv_chunk_keys": (st, [P(i32), i64, i32, ctypes.c_uint64, P(ctypes.c_uint64), i64]),
         "kv_tier_create": (st, [i64, i64, P(vp)]),
@@ -354,7 +355,8 @@ def kv_host_alloc(nbytes: int) -> int:
     return out.value
 
 
-KVX_NUMA_NEAREST = -1
+KVX_NUMA_NEAREST, KVX_NUMA_ANY = -1, -2
+KVX_HOST_DRIVER = 0x1
 
 
 def kv_host_alloc_numa(nbytes: int, numa_node: int = KVX_NUMA_NEAREST) -> tuple[int, int]:
@@ -363,6 +365,15 @@ def kv_host_alloc_numa(nbytes: int, numa_node: int = KVX_NUMA_NEAREST) -> tuple[
     out = ctypes.c_void_p()
     node = ctypes.c_int32(-1)
     _check(_lib.kv_host_alloc_numa(numa_node, nbytes, ctypes.byref(out), ctypes.byref(node)), "kv_host_alloc_numa")
+    return out.value, node.value
+
+
+def kv_host_alloc_ex(nbytes: int, numa_node: int = KVX_NUMA_ANY, flags: int = 0) -> tuple[int, int]:
+    """kv_host_alloc with the placement and the allocator chosen (see kvxfer.h).
+    Returns (pointer, node of the first page or -1)."""
+    out = ctypes.c_void_p()
+    node = ctypes.c_int32(-1)
+    _check(_lib.kv_host_alloc_ex(nbytes, numa_node, flags, ctypes.byref(out), ctypes.byref(node)), "kv_host_alloc_ex")
     return out.value, node.value
 
 
@@ -376,13 +387,18 @@ class HostBuffer:
     Views of ``.tensor`` keep the allocation alive; ``close()`` frees it at once
     and must only be called when no view is used any more."""
 
-    def __init__(self, nbytes: int, numa_node: int | None = None):
+    def __init__(self, nbytes: int, numa_node: int | None = None, driver: bool = False):
         """numa_node: None for kv_host_alloc, else kv_host_alloc_numa on that node
-        (KVX_NUMA_NEAREST: the node nearest the current GPU); see .numa_node."""
+        (KVX_NUMA_NEAREST: the node nearest the current GPU); see .numa_node.
+        driver: the driver's pinned allocator instead (KVX_HOST_DRIVER)."""
         import torch
         self.nbytes = nbytes
         self.numa_node = None
-        if numa_node is None:
+        if driver:
+            if numa_node is not None:
+                raise ValueError("the driver's allocator takes no NUMA placement")
+            self.ptr, _ = kv_host_alloc_ex(nbytes, KVX_NUMA_ANY, KVX_HOST_DRIVER)
+        elif numa_node is None:
             self.ptr = kv_host_alloc(nbytes)
         else:
             self.ptr, self.numa_node = kv_host_alloc_numa(nbytes, numa_node)

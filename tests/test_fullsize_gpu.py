@@ -167,19 +167,21 @@ def test_host_alloc_exact_and_pinned():
         buf.close()
 
 
-@pytest.mark.parametrize("node", ["nearest", 0])
+@pytest.mark.parametrize("node", ["nearest", 0, "driver", "plain"])
 def test_host_alloc_numa_round_trip(orc, node):
-    """kv_host_alloc_numa: a pinned, mapped pool on a host NUMA node (the node
-    nearest the GPU, or node 0), used as the chunks of a zero-copy store and
-    restore that must match the oracle."""
+    """Each kind of pinned pool (kv_host_alloc_numa on the node nearest the GPU or
+    on node 0, the driver's allocator, plain kv_host_alloc) used as the chunks of
+    a zero-copy store and restore that must match the oracle."""
     k = kvx()
     spec = oracle.PoolSpec(4, 64, 16, 8, 128, 2, oracle.HND)
     Cs, n_used = 256, 40
     T = n_used * 16 - 5
     cb = orc.chunk_bytes(spec, Cs)
     n_chunks = -(-T // Cs)
-    want_node = k.KVX_NUMA_NEAREST if node == "nearest" else node
-    buf = k.HostBuffer(n_chunks * cb, numa_node=want_node)
+    if node in ("driver", "plain"):
+        buf = k.HostBuffer(n_chunks * cb, driver=node == "driver")
+    else:
+        buf = k.HostBuffer(n_chunks * cb, numa_node=k.KVX_NUMA_NEAREST if node == "nearest" else node)
     try:
         if node == 0:
             assert buf.numa_node == 0
