@@ -7,6 +7,8 @@
 
 #include <cuda_runtime.h>
 
+#include <mutex>
+
 #include "kvx_internal.h"
 #include "kvxfer_probe.h"
 
@@ -35,6 +37,21 @@ __global__ void delayed_copy_kernel(uint4* dst, const uint4* src, long long n16,
   const long long stride = (long long)gridDim.x * blockDim.x;
   for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < n16; i += stride)
     dst[i] = src[i];
+}
+
+// The probe kernels use no shared memory, but an SM's shared-memory carveout
+// is set for the kernels resident on it: asking for the largest carveout lets
+// kernels that need shared memory (the TMA engine) start beside a spinning
+// probe, so an unordered transfer really runs before the probe finishes.
+void prefer_max_shared_carveout() {
+  static std::once_flag once;
+  std::call_once(once, [] {
+    cudaFuncSetAttribute(delayed_fill_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                         cudaSharedmemCarveoutMaxShared);
+    cudaFuncSetAttribute(delayed_copy_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                         cudaSharedmemCarveoutMaxShared);
+    cudaGetLastError();
+  });
 }
 
 // One CTA per SM keeps every CTA resident, so the whole grid waits about
@@ -70,6 +87,7 @@ extern "C" kvx_status kvx_probe_delayed_fill(void* dev, int64_t bytes, int32_t v
   if (!dev || bytes <= 0 || value < 0 || value > 255) return KVX_EINVAL;
   kvx_status st = device_ptr_ok(dev);
   if (st != KVX_OK) return st;
+  prefer_max_shared_carveout();
   delayed_fill_kernel<<<resident_grid(), kProbeThreads, 0, (cudaStream_t)stream>>>(
       (uint8_t*)dev, bytes, (uint8_t)value, clamp_cycles(cycles));
   cudaError_t e = cudaGetLastError();
@@ -87,6 +105,7 @@ extern "C" kvx_status kvx_probe_delayed_copy(void* dst, const void* src, int64_t
   kvx_status st = device_ptr_ok(dst);
   if (st == KVX_OK) st = device_ptr_ok(src);
   if (st != KVX_OK) return st;
+  prefer_max_shared_carveout();
   delayed_copy_kernel<<<resident_grid(), kProbeThreads, 0, (cudaStream_t)stream>>>(
       (uint4*)dst, (const uint4*)src, bytes / 16, clamp_cycles(cycles));
   cudaError_t e = cudaGetLastError();

@@ -150,13 +150,13 @@ def ctxs():
 
 
 # (name, mode, unordered, force the load/store device engine).  The staged
-# negative control packs with the load/store engine.  With the TMA engine the
-# unordered pack did not see stale bytes: its CTAs ask for 32-96 KiB of shared
-# memory, and (the likely cause) an SM whose carveout is set for the spinning
-# producer, which uses none, takes them only after the producer leaves, so the
-# pack runs after it and the missing dependency stays hidden.
+# negative control runs with both device engines.  The TMA engine's CTAs need
+# 32-96 KiB of shared memory; an SM whose carveout was set for a probe that
+# uses none took them only after the probe left, which hid the missing
+# dependency until the probe kernels asked for the largest carveout.
 VARIANTS = [("staged", 1, False, False), ("staged_lsu", 1, False, True), ("zerocopy", 2, False, False),
-            ("staged_unordered", 1, True, True), ("zerocopy_unordered", 2, True, False)]
+            ("staged_unordered", 1, True, True), ("staged_unordered_tma", 1, True, False),
+            ("zerocopy_unordered", 2, True, False)]
 
 
 @pytest.mark.parametrize("n_bytes", SIZES)
