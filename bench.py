@@ -364,24 +364,6 @@ def host_mem_available() -> int:
     return 0
 
 
-def huge_page_bytes(ptr: int, nbytes: int) -> int | None:
-    """Bytes of [ptr, ptr + nbytes) that transparent huge pages back (AnonHugePages of
-    the overlapping mappings in /proc/self/smaps), or None where that is unknown."""
-    try:
-        total, overlap = 0, False
-        with open("/proc/self/smaps") as f:
-            for line in f:
-                head = line.split()[0]
-                if "-" in head and ":" not in head:
-                    lo, hi = (int(x, 16) for x in head.split("-"))
-                    overlap = lo < ptr + nbytes and hi > ptr
-                elif overlap and line.startswith("AnonHugePages:"):
-                    total += int(line.split()[1]) * 1024
-        return total
-    except (OSError, ValueError):
-        return None
-
-
 def cpu_model() -> str:
     try:
         out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
@@ -578,6 +560,7 @@ def run_ours(args):
     concurrent = None
     if not args.no_concurrent and world == 1 and host_mem_available() > n_chunks * cb + (32 << 30):
         host_pool2 = k.HostBuffer(n_chunks * cb)
+        pool2 = host_pool2.info()
         chunks2 = [host_pool2.tensor[i * cb:(i + 1) * cb] for i in range(n_chunks)]
         ctx_b = k.kv_ctx_create(local, store_mode=mode, load_mode=mode, staging_slot_bytes=args.slot_mib << 20)
         s_b = torch.cuda.Stream(device=dev)
@@ -608,6 +591,7 @@ def run_ours(args):
                       "span_ms": span, "aggregate_gbs": agg, "peak_bidir_gbs": link["bidir"],
                       "frac": agg / link["bidir"], "reps": len(span_ms),
                       "second_store_equals_first_on_sampled_chunks": same,
+                      "second_pool": pool2,
                       "what": "replica A kv_store of the context into a second pinned chunk set while replica B "
                               "kv_load of the timed steps' chunks into its pool, own context and stream each; "
                               "peak = pinned cudaMemcpyAsync of 1 GiB each way at once"}
@@ -648,7 +632,7 @@ def run_ours(args):
                    "parallelism": f"replicas x{world}", "pinned_host_bytes": n_chunks * cb,
                    "host_alloc": args.host_alloc if host_pool.numa_node is None
                    else f"numa node {host_pool.numa_node}",
-                   "host_pool_huge_page_bytes": huge_page_bytes(host_pool.ptr, n_chunks * cb),
+                   "host_pool": host_pool.info(),
                    "pin_seconds": pin_seconds},
         "restore_ms": {"median": statistics.median(restore_ms), "min": min(restore_ms), "max": max(restore_ms),
                        "n": len(restore_ms)},

@@ -343,9 +343,10 @@ kvx_status kv_host_alloc_numa(int32_t numa_node, int64_t bytes, void** out, int3
  * (no placement), KVX_NUMA_NEAREST, or a node.  flags: KVX_HOST_DRIVER takes
  * the memory from the driver's pinned allocator (cudaHostAlloc, portable and
  * mapped) instead of the library's huge-page mapping; numa_node must then be
- * KVX_NUMA_ANY.  Without a placement, a pool smaller than one huge page, or
- * any pool on a host without transparent huge pages, also comes from the
- * driver's allocator.  kv_host_alloc(b, o) is kv_host_alloc_ex(b,
+ * KVX_NUMA_ANY.  Without a placement, a pool that whole huge pages would
+ * overshoot by more than an eighth (for 512 MiB pages: anything below 4 GiB
+ * that is not a near multiple), or any pool on a host without transparent
+ * huge pages, also comes from the driver's allocator.  kv_host_alloc(b, o) is kv_host_alloc_ex(b,
  * KVX_NUMA_ANY, 0, o, NULL).  Memory from either source zero-copies at the
  * link peak; only huge pages let the copy engines (KVX_MODE_STAGED) reach it
  * steadily on a host with small base pages.
@@ -353,6 +354,26 @@ kvx_status kv_host_alloc_numa(int32_t numa_node, int64_t bytes, void** out, int3
 #define KVX_NUMA_ANY (-2)
 #define KVX_HOST_DRIVER 0x1u
 kvx_status kv_host_alloc_ex(int64_t bytes, int32_t numa_node, uint32_t flags, void** out, int32_t* numa_out);
+
+/*
+ * What backs a pool from the calls above.  A pool of the library's own
+ * mapping is either wholly on huge pages or wholly on base pages, never a
+ * mixture: on GB300 a pool partly on huge pages zero-copied at 76 GB/s where
+ * either kind alone reached 202 GB/s.  When huge pages cannot back the whole
+ * pool, the call falls back to the driver's allocator (no placement asked) or
+ * to base pages (placement asked).
+ */
+#define KVX_HOST_SOURCE_DRIVER 0 /* cudaHostAlloc                               */
+#define KVX_HOST_SOURCE_MAPPED 1 /* the library's mapping, then cudaHostRegister */
+typedef struct {
+  int64_t bytes;            /* requested                                        */
+  int64_t mapped_bytes;     /* mapped (rounded up to whole pages)               */
+  int64_t huge_page_bytes;  /* backed by transparent huge pages when pinned     */
+  int32_t numa_node;        /* node of the first page, or -1 if unknown          */
+  int32_t source;           /* KVX_HOST_SOURCE_*                                 */
+} kvx_host_pool_info;
+/* KVX_ENOENT if `host` is not the start of a pool these calls returned. */
+kvx_status kv_host_pool_info(const void* host, kvx_host_pool_info* info);
 /* Frees kv_host_alloc and kv_host_alloc_numa memory; NULL and pointers the
    library did not allocate are ignored. */
 void kv_host_free(void* host);

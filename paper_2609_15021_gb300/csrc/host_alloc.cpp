@@ -50,8 +50,18 @@ constexpr int kMaxNodes = 1024;      // nodes a node mask below can name
 constexpr int kMadvPopulateWrite = 23;
 constexpr int kMadvCollapse = 25;
 
+// A pool made here.  Mapped pools sit between two inaccessible guard pages,
+// so the kernel never merges their mapping with a neighbour's and
+// /proc/self/smaps describes exactly the pool.
+struct Pool {
+  size_t len = 0;           // mapped length; 0 for the driver's allocator
+  int64_t bytes = 0;        // requested
+  int64_t huge_bytes = 0;   // backed by huge pages when pinned
+  int32_t node = -1;        // NUMA node of the first page, or -1
+  int32_t source = KVX_HOST_SOURCE_DRIVER;
+};
 std::mutex g_mu;
-std::unordered_map<void*, size_t> g_mappings;  // pools made here: base -> mapped length
+std::unordered_map<void*, Pool> g_pools;
 
 bool node_exists(int node) {
   char path[64];
@@ -113,65 +123,115 @@ kvx_status driver_pool(int64_t bytes, void** out) {
     cudaGetLastError();
     return e == cudaErrorMemoryAllocation ? KVX_ENOMEM : KVX_ECUDA;
   }
+  Pool rec;
+  rec.bytes = bytes;
   {
     std::lock_guard<std::mutex> g(g_mu);
-    g_mappings[p] = 0;  // length 0: freed with cudaFreeHost
+    g_pools[p] = rec;
   }
   *out = p;
   return KVX_OK;
 }
 
-// Maps, places (node >= 0), backs with huge pages where possible and pins a
-// pool of at least `bytes`.  On success *out is the pool and *len_out the
-// mapped length.
-kvx_status map_pool(int node, int64_t bytes, void** out, size_t* len_out) {
+// Bytes of [p, p + len) backed by transparent huge pages (AnonHugePages of the
+// mappings inside that range in /proc/self/smaps), or -1 if unreadable.
+int64_t huge_backed_bytes(const void* p, size_t len) {
+  FILE* f = fopen("/proc/self/smaps", "r");
+  if (!f) return -1;
+  const uintptr_t a = (uintptr_t)p, b = a + len;
+  char line[512];
+  bool inside = false;
+  long long total_kb = 0;
+  while (fgets(line, sizeof(line), f)) {
+    unsigned long lo = 0, hi = 0;
+    long long kb = 0;
+    if (sscanf(line, "%lx-%lx ", &lo, &hi) == 2 && strchr(line, ':') != nullptr && line[0] != ' ' &&
+        strncmp(line, "AnonHugePages", 13) != 0) {
+      inside = lo >= a && hi <= b;
+    } else if (inside && sscanf(line, "AnonHugePages: %lld kB", &kb) == 1) {
+      total_kb += kb;
+    }
+  }
+  fclose(f);
+  return (int64_t)total_kb * 1024;
+}
+
+// Maps a pool of at least `bytes` between two guard pages, places it on
+// `node` (>= 0), backs it with huge pages (huge) or explicitly with base
+// pages, faults it in and pins it.  KVX_EAGAIN-like outcome: returns
+// KVX_ENOMEM with *partial set when huge pages were asked but did not back
+// the whole pool; the mapping is then already released.
+kvx_status map_pool(int node, int64_t bytes, bool huge_pages, void** out, bool* partial) {
+  *partial = false;
   const size_t page = (size_t)sysconf(_SC_PAGESIZE);
-  const size_t huge = thp_available() ? huge_page_bytes() : 0;
-  const bool use_huge = huge >= page && (size_t)bytes >= huge;
-  const size_t unit = use_huge ? huge : page;
+  const size_t huge = huge_page_bytes();
+  const size_t unit = huge_pages ? huge : page;
   const size_t len = ((size_t)bytes + unit - 1) / unit * unit;
-  const size_t span = use_huge ? len + huge : len;  // room to align the start
+  const size_t span = len + 2 * unit;  // room to align the start and keep a guard page on each side
   uint8_t* raw = (uint8_t*)mmap(nullptr, span, PROT_READ | PROT_WRITE, MAP_PRIVATE | MAP_ANONYMOUS, -1, 0);
   if (raw == (uint8_t*)MAP_FAILED) {
     set_error_text("mmap of the host pool failed");
     return KVX_ENOMEM;
   }
-  uint8_t* p = raw;
-  if (use_huge) {
-    p = (uint8_t*)(((uintptr_t)raw + huge - 1) / huge * huge);
-    if (p > raw) munmap(raw, (size_t)(p - raw));
-    const size_t tail = (size_t)(raw + span - (p + len));
-    if (tail) munmap(p + len, tail);
-  }
+  uint8_t* p = (uint8_t*)(((uintptr_t)raw + page + unit - 1) / unit * unit);  // >= one page in
+  uint8_t* lo = p - page;
+  uint8_t* hi = p + len + page;
+  if (lo > raw) munmap(raw, (size_t)(lo - raw));
+  if (raw + span > hi) munmap(hi, (size_t)(raw + span - hi));
+  mprotect(lo, page, PROT_NONE);
+  mprotect(p + len, page, PROT_NONE);
+  auto release = [&] { munmap(lo, (size_t)(hi - lo)); };
   if (node >= 0) {
     unsigned long mask[kMaxNodes / (8 * sizeof(unsigned long))] = {};
     mask[node / (8 * sizeof(unsigned long))] |= 1ul << (node % (8 * sizeof(unsigned long)));
     // maxnode counts one more than the bits the kernel reads from the mask
     if (syscall(SYS_mbind, p, len, kMpolPreferred, mask, (unsigned long)kMaxNodes + 1, 0u) != 0) {
-      munmap(p, len);
+      release();
       set_error_text("mbind of the host pool failed");
       return KVX_EINVAL;
     }
   }
-  if (use_huge) {
+  int64_t huge_bytes = 0;
+  if (huge_pages) {
     madvise(p, len, MADV_HUGEPAGE);
     madvise(p, len, kMadvPopulateWrite);  // fault in now, as huge pages where the kernel can
-    madvise(p, len, kMadvCollapse);       // and collapse what it could not
+    for (int attempt = 0; attempt < 3; ++attempt) {
+      huge_bytes = huge_backed_bytes(p, len);
+      if (huge_bytes >= (int64_t)len) break;
+      madvise(p, len, kMadvCollapse);     // collapse what is still on base pages
+    }
+    huge_bytes = huge_backed_bytes(p, len);
+    if (huge_bytes < (int64_t)len) {
+      // Measured on GB300: a pool partly on huge pages zero-copied at 76 GB/s
+      // where one wholly on either kind ran at 202 GB/s.  Never hand one out.
+      release();
+      *partial = true;
+      set_error_text("huge pages could not back the whole host pool");
+      return KVX_ENOMEM;
+    }
+  } else {
+    madvise(p, len, MADV_NOHUGEPAGE);    // all base pages: no mixture either
+    madvise(p, len, kMadvPopulateWrite);
   }
   const cudaError_t e = cudaHostRegister(p, len, cudaHostRegisterPortable | cudaHostRegisterMapped);
   if (e != cudaSuccess) {
     set_last_cuda_error((int)e);
     set_error_text("cudaHostRegister of the host pool");
     cudaGetLastError();
-    munmap(p, len);
+    release();
     return e == cudaErrorMemoryAllocation ? KVX_ENOMEM : KVX_ECUDA;
   }
+  Pool rec;
+  rec.len = len;
+  rec.bytes = bytes;
+  rec.huge_bytes = huge_bytes;
+  rec.node = page_node(p);
+  rec.source = KVX_HOST_SOURCE_MAPPED;
   {
     std::lock_guard<std::mutex> g(g_mu);
-    g_mappings[p] = len;
+    g_pools[p] = rec;
   }
   *out = p;
-  *len_out = len;
   return KVX_OK;
 }
 
@@ -192,12 +252,15 @@ kvx_status kv_host_alloc_ex(int64_t bytes, int32_t numa_node, uint32_t flags, vo
     return KVX_ENOMEM;
   }
   // The driver's allocator where asked, and where the library's mapping would
-  // get no huge pages and no placement anyway (a small pool, or no
-  // transparent huge pages): its memory serves the copy engines better than
-  // base pages do.
+  // get no huge pages and no placement anyway (a pool small next to a huge
+  // page, or no transparent huge pages): its memory serves the copy engines
+  // better than base pages do.
+  // Huge pages where rounding the pool up to whole huge pages wastes at most
+  // an eighth of it.
   const size_t huge = thp_available() ? huge_page_bytes() : 0;
-  if ((flags & KVX_HOST_DRIVER) || (numa_node == KVX_NUMA_ANY && (huge == 0 || (size_t)bytes < huge)))
-    return driver_pool(bytes, out);
+  const size_t rounded = huge ? ((size_t)bytes + huge - 1) / huge * huge : 0;
+  const bool huge_fits = huge != 0 && (rounded - (size_t)bytes) * 8 <= (size_t)bytes;
+  if ((flags & KVX_HOST_DRIVER) || (numa_node == KVX_NUMA_ANY && !huge_fits)) return driver_pool(bytes, out);
   int node = numa_node;
   if (node == KVX_NUMA_ANY) {
     node = -1;
@@ -218,10 +281,34 @@ kvx_status kv_host_alloc_ex(int64_t bytes, int32_t numa_node, uint32_t flags, vo
       return KVX_ENOMEM;
     }
   }
-  size_t len = 0;
-  const kvx_status st = map_pool(node, bytes, out, &len);
+  // If huge pages cannot back all of it: the driver's allocator (no placement
+  // asked) or base pages (placement asked).
+  bool partial = false;
+  kvx_status st = KVX_ENOMEM;
+  if (huge_fits) {
+    st = map_pool(node, bytes, true, out, &partial);
+    if (st != KVX_OK && !partial) return st;
+  }
+  if (st != KVX_OK) {
+    if (numa_node == KVX_NUMA_ANY) return driver_pool(bytes, out);
+    st = map_pool(node, bytes, false, out, &partial);
+  }
   if (st == KVX_OK && numa_out) *numa_out = page_node(*out);
   return st;
+}
+
+kvx_status kv_host_pool_info(const void* host, kvx_host_pool_info* info) {
+  if (!host || !info) return KVX_EINVAL;
+  std::lock_guard<std::mutex> g(g_mu);
+  auto it = g_pools.find(const_cast<void*>(host));
+  if (it == g_pools.end()) return KVX_ENOENT;
+  const Pool& r = it->second;
+  info->bytes = r.bytes;
+  info->mapped_bytes = r.len ? (int64_t)r.len : r.bytes;
+  info->huge_page_bytes = r.huge_bytes;
+  info->numa_node = r.node;
+  info->source = r.source;
+  return KVX_OK;
 }
 
 kvx_status kv_host_alloc(int64_t bytes, void** out) {
@@ -238,20 +325,21 @@ kvx_status kv_host_alloc_numa(int32_t numa_node, int64_t bytes, void** out, int3
 
 void kv_host_free(void* p) {
   if (!p) return;
-  size_t len = 0;
+  Pool rec;
   {
     std::lock_guard<std::mutex> g(g_mu);
-    auto it = g_mappings.find(p);
-    if (it == g_mappings.end()) return;  // not a pool of this library
-    len = it->second;
-    g_mappings.erase(it);
+    auto it = g_pools.find(p);
+    if (it == g_pools.end()) return;  // not a pool of this library
+    rec = it->second;
+    g_pools.erase(it);
   }
-  if (len == 0) {
+  if (rec.source == KVX_HOST_SOURCE_DRIVER) {
     cudaFreeHost(p);
   } else {
     cudaHostUnregister(p);
     cudaGetLastError();
-    munmap(p, len);
+    const size_t page = (size_t)sysconf(_SC_PAGESIZE);
+    munmap((uint8_t*)p - page, rec.len + 2 * page);  // the pool and its two guard pages
   }
   cudaGetLastError();
 }

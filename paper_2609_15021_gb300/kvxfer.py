@@ -40,6 +40,7 @@ EXPORTED = (
     "kv_chunk_keys", "kv_tier_create", "kv_tier_create_on", "kv_tier_destroy", "kv_tier_reserve", "kv_tier_commit",
     "kv_tier_acquire", "kv_tier_release", "kv_tier_prefix_hits", "kv_tier_stats", "kv_fault_inject",
     "kv_tier_open_shared", "kv_tier_poll", "kv_tier_reclaim", "kv_host_alloc_numa", "kv_host_alloc_ex",
+    "kv_host_pool_info",
 )
 KVX_ENOENT, KVX_EBUSY = -8, -9
 KVX_TIER_CREATE, KVX_TIER_NO_PIN = 0x1, 0x2
@@ -64,6 +65,11 @@ class kvx_pool(ctypes.Structure):
                 ("num_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
                 ("elem_bytes", ctypes.c_int32), ("layout", ctypes.c_int32),
                 ("pages_per_block", ctypes.c_int32)]
+
+
+class kvx_host_pool_info(ctypes.Structure):
+    _fields_ = [("bytes", ctypes.c_int64), ("mapped_bytes", ctypes.c_int64), ("huge_page_bytes", ctypes.c_int64),
+                ("numa_node", ctypes.c_int32), ("source", ctypes.c_int32)]
 
 
 class kvx_chunk_layout(ctypes.Structure):
@@ -113,6 +119,7 @@ def _declare(lib):
         "kv_host_free": (None, [vp]),
         "kv_host_alloc_numa": (st, [i32, i64, P(vp), P(i32)]),
         "kv_host_alloc_ex": (st, [i64, i32, ctypes.c_uint32, P(vp), P(i32)]),
+        "kv_host_pool_info": (st, [vp, P(kvx_host_pool_info)]),
         "kv_pool_view_check": (st, [P(kvx_pool), i32, P(i64), P(i64)]),
         "kv_chunk_keys": (st, [P(i32), i64, i32, ctypes.c_uint64, P(ctypes.c_uint64), i64]),
         "kv_tier_create": (st, [i64, i64, P(vp)]),
@@ -357,6 +364,16 @@ def kv_host_alloc(nbytes: int) -> int:
 
 KVX_NUMA_NEAREST, KVX_NUMA_ANY = -1, -2
 KVX_HOST_DRIVER = 0x1
+KVX_HOST_SOURCE_DRIVER, KVX_HOST_SOURCE_MAPPED = 0, 1
+
+
+def kv_host_pool_info(ptr: int) -> dict:
+    """What backs a pool from kv_host_alloc / _numa / _ex (see kvxfer.h)."""
+    out = kvx_host_pool_info()
+    _check(_lib.kv_host_pool_info(ptr, ctypes.byref(out)), "kv_host_pool_info")
+    return {"bytes": out.bytes, "mapped_bytes": out.mapped_bytes, "huge_page_bytes": out.huge_page_bytes,
+            "numa_node": out.numa_node,
+            "source": "driver" if out.source == KVX_HOST_SOURCE_DRIVER else "mapped"}
 
 
 def kv_host_alloc_numa(nbytes: int, numa_node: int = KVX_NUMA_NEAREST) -> tuple[int, int]:
@@ -405,6 +422,9 @@ class HostBuffer:
         raw = (ctypes.c_uint8 * nbytes).from_address(self.ptr)
         raw._owner = self  # the tensor holds `raw`, `raw` holds this buffer
         self.tensor = torch.frombuffer(raw, dtype=torch.uint8, count=nbytes)
+
+    def info(self) -> dict:
+        return kv_host_pool_info(self.ptr)
 
     def close(self):
         if self.ptr:

@@ -151,11 +151,26 @@ def test_fullsize_device_pack_unpack_sampled(orc, engine):
 
 
 def test_host_alloc_exact_and_pinned():
-    """kv_host_alloc returns exactly the requested, page-locked, mapped size (no rounding)."""
+    """kv_host_alloc returns exactly the requested, page-locked, mapped size (no
+    power-of-two rounding), backed wholly by huge pages or wholly by the driver's
+    allocator, never by a mixture."""
     k = kvx()
     n = (1 << 30) + 4096  # a size a power-of-two rounding allocator would double
     buf = k.HostBuffer(n)
     try:
+        info = buf.info()
+        print(f"\n{n} B pool: {info}")
+        assert info["bytes"] == n and info["mapped_bytes"] <= n + n // 8 + (64 << 10)
+        if info["source"] == "mapped":
+            assert info["huge_page_bytes"] in (0, info["mapped_bytes"])
+        big = k.HostBuffer(33 << 30)                        # a tier-sized pool: huge pages, or the driver's
+        bi = big.info()
+        assert bi["huge_page_bytes"] in (0, bi["mapped_bytes"]) and bi["mapped_bytes"] <= (33 << 30) + (512 << 20)
+        print(f"33 GiB pool: {bi}")
+        big.close()
+        small = k.HostBuffer(1 << 20)                      # below one huge page: the driver's allocator
+        assert small.info()["source"] == "driver"
+        small.close()
         assert buf.tensor.numel() == n
         buf.tensor[-1] = 7
         assert int(buf.tensor[-1]) == 7
@@ -185,6 +200,8 @@ def test_host_alloc_numa_round_trip(orc, node):
     try:
         if node == 0:
             assert buf.numa_node == 0
+        info = buf.info()
+        assert info["huge_page_bytes"] in (0, info["mapped_bytes"]) or info["source"] == "driver"
         print(f"\nhost pool on NUMA node {buf.numa_node} (asked: {node})")
         chunks = [buf.tensor[i * cb:(i + 1) * cb] for i in range(n_chunks)]
         src_np = host_layers(spec, 61)
