@@ -429,7 +429,9 @@ kvx_status kv_tier_create_on(void* base, int64_t slot_bytes, int64_t n_slots, kv
  * has seen that work complete (any tier call or kv_tier_poll in that process);
  * in the writer's own process it is readable at once, the reader's stream
  * waiting on the writer's event.  The creator's kv_tier_destroy removes the
- * name; mappings in other processes stay valid.
+ * name; mappings in other processes stay valid.  The shared data is kept on
+ * base pages.  Zero-copy runs at the link peak on it; the copy engines
+ * (KVX_MODE_STAGED) do not, so use zero-copy with a shared tier.
  */
 #define KVX_TIER_CREATE 0x1u
 #define KVX_TIER_NO_PIN 0x2u

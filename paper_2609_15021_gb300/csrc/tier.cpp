@@ -545,6 +545,11 @@ kvx_status kv_tier_open_shared(const char* name, int64_t slot_bytes, int64_t n_s
     attach_metadata(t, map);
   }
   t->data = (uint8_t*)map + h->data_offset;
+  // Shared memory is kept on base pages: the SMs' zero-copy accesses run at the
+  // link peak on them, and a mixture of page sizes slowed zero-copy on GB300
+  // to a third.  (The copy engines are slow on base pages: with a shared tier,
+  // zero-copy, the default mode, is the one to use.)
+  madvise(t->data, (size_t)(h->slot_bytes * h->n_slots), MADV_NOHUGEPAGE);
   if (!(flags & KVX_TIER_NO_PIN)) {
     const cudaError_t e = cudaHostRegister(t->data, (size_t)(h->slot_bytes * h->n_slots),
                                            cudaHostRegisterPortable | cudaHostRegisterMapped);
