@@ -121,7 +121,7 @@ typedef struct {
   int32_t store_mode;         /* kvx_mode                                       */
   int32_t load_mode;          /* kvx_mode                                       */
   int32_t staging_slots;      /* staged ring depth (>= 2); 0 = 4                */
-  int64_t staging_slot_bytes; /* bytes per slot; 0 = 32 MiB; a slot must hold
+  int64_t staging_slot_bytes; /* bytes per slot; 0 = 128 MiB; a slot must hold
                                  one layer of one chunk                         */
   int32_t max_ctas;           /* cap on CTAs per kernel launch; 0 = default:
                                  launches that read or write host memory

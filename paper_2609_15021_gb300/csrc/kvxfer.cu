@@ -85,7 +85,11 @@ bool fault_point(const char* point) { return fault_now(point); }
 namespace {
 
 constexpr int32_t kDefaultSlots = 4;
-constexpr int64_t kDefaultSlotBytes = 32ll << 20;
+// 4 x 128 MiB: measured on GB300 at 128k tokens, staged stores and restores
+// run at 200.0 GB/s against 198.3 with 32 MiB slots, and the host enqueues a
+// 32k-token store in 0.6 ms instead of 10.4 (a quarter of the launches, each
+// carrying its layers' tensor maps).
+constexpr int64_t kDefaultSlotBytes = 128ll << 20;
 constexpr long long kNoError = LLONG_MAX;
 
 struct TimedLaunch {
