@@ -14,6 +14,16 @@ value  = bytes moved over the host link (both directions) / device time of
 e2e    = the same metric timed on the host clock around the public API calls,
          including per-step block-table uploads from pinned memory and the
          host synchronisation that must precede host use of the chunks.
+After the timed region (none of it is in `value`):
+roofline             the dominant kernel against the host link's pinned-copy
+                     peak measured in the same run (zero-copy) or HBM (staged),
+                     with DRAM traffic from the committed ncu record;
+hbm_roofline         kv_pack / kv_unpack of the same context into device chunks
+                     against the measured HBM copy peak;
+concurrent_replicas  one context stored while another context's chunks are
+                     restored, each through its own context and stream;
+cpu_baseline         the oracle on the host cores over a sample of the chunks,
+                     which also checks those GPU chunks byte for byte.
 Prints one JSON line.  --impl reference times the CPU oracle instead.
 """
 from __future__ import annotations
