@@ -527,34 +527,45 @@ def run_ours(args):
     if not args.no_hbm_roofline:
         dev_slab = torch.empty(n_chunks * cb, dtype=torch.uint8, device=dev)
         dchunks = [dev_slab[i * cb:(i + 1) * cb] for i in range(n_chunks)]
+
+        def device_leg(tma):
+            """Per direction: (launches, bytes per launch, ms per launch) of kv_pack / kv_unpack."""
+            hctx = k.kv_ctx_create(local, flags=k.KVX_FLAG_TIME_KERNELS | (0 if tma else k.KVX_FLAG_DEVICE_LSU))
+            for _ in range(2):
+                k.kv_pack(hctx, src, ta, 0, T, C, dchunks, stream=stream)
+                k.kv_unpack(hctx, dst, tb, 0, T, C, dchunks, stream=stream)
+            stream.synchronize()
+            k.kv_ctx_reset_stats(hctx)
+            for _ in range(3):
+                k.kv_pack(hctx, src, ta, 0, T, C, dchunks, stream=stream)
+                k.kv_unpack(hctx, dst, tb, 0, T, C, dchunks, stream=stream)
+            stream.synchronize()
+            hs = k.kv_ctx_stats(hctx)
+            assert k.kv_get_device_error(hctx) == -1
+            k.kv_ctx_destroy(hctx)
+            return [(hs["timed_launches"][d], hs["kernel_bytes"][d] / hs["timed_launches"][d],
+                     hs["kernel_ms"][d] / hs["timed_launches"][d]) for d in (0, 1)]
+
         tma = args.device_engine == "tma"
-        hctx = k.kv_ctx_create(local, flags=k.KVX_FLAG_TIME_KERNELS | (0 if tma else k.KVX_FLAG_DEVICE_LSU))
-        for _ in range(2):
-            k.kv_pack(hctx, src, ta, 0, T, C, dchunks, stream=stream)
-            k.kv_unpack(hctx, dst, tb, 0, T, C, dchunks, stream=stream)
-        stream.synchronize()
-        k.kv_ctx_reset_stats(hctx)
-        for _ in range(3):
-            k.kv_pack(hctx, src, ta, 0, T, C, dchunks, stream=stream)
-            k.kv_unpack(hctx, dst, tb, 0, T, C, dchunks, stream=stream)
-        stream.synchronize()
-        hs = k.kv_ctx_stats(hctx)
-        assert k.kv_get_device_error(hctx) == -1
-        k.kv_ctx_destroy(hctx)
+        legs = {tma: device_leg(tma), not tma: device_leg(not tma)}  # the chosen engine and the other one
         dev_traffic = recorded_traffic(s, "tma_kernels.cu") if tma else traffic
         hbm_roofline = {"bound": "hbm", "peak": hbm_peak, "unit": "GB/s", "peak_source": peak_src,
                         "engine": "TMA tensor-map boxes (tmap_move_kernel)" if tma else
                                   "16-byte loads/stores (move_kernel)"}
         for d, name in ((0, "pack"), (1, "unpack")):
-            nl = hs["timed_launches"][d]
-            per_launch = hs["kernel_bytes"][d] / nl
-            achieved = per_launch / (hs["kernel_ms"][d] / nl * 1e-3) / GB
+            nl, per_launch, ms = legs[tma][d]
+            achieved = per_launch / (ms * 1e-3) / GB
             kname = f"tmap_move_kernel<{name}>" if tma else f"move_kernel<{name},HND>"
             hbm_roofline[name] = {"kernel": f"{kname} (device chunks)", "achieved": achieved,
                                   "frac": achieved / hbm_peak, "launches": nl,
-                                  "algorithmic_bytes_per_launch": per_launch,
-                                  "avg_launch_ms": hs["kernel_ms"][d] / nl,
+                                  "algorithmic_bytes_per_launch": per_launch, "avg_launch_ms": ms,
                                   "traffic": dev_traffic.get(f"device_{name}", per_launch)}
+        other = legs[not tma]
+        hbm_roofline["other_engine"] = {
+            "engine": "16-byte loads/stores (move_kernel)" if tma else "TMA tensor-map boxes (tmap_move_kernel)",
+            **{name: {"achieved": other[d][1] / (other[d][2] * 1e-3) / GB,
+                      "frac": other[d][1] / (other[d][2] * 1e-3) / GB / hbm_peak, "avg_launch_ms": other[d][2]}
+               for d, name in ((0, "pack"), (1, "unpack"))}}
         del dev_slab, dchunks
 
     store_gbs = X / (statistics.median(store_ms) * 1e-3) / GB
