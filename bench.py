@@ -560,6 +560,21 @@ def run_ours(args):
                                   "frac": achieved / hbm_peak, "launches": nl,
                                   "algorithmic_bytes_per_launch": per_launch, "avg_launch_ms": ms,
                                   "traffic": dev_traffic.get(f"device_{name}", per_launch)}
+        # this GPU's device-to-device copy rate right now (context for the peak above)
+        a = dev_slab[: len(dev_slab) // 2]
+        b = dev_slab[len(dev_slab) // 2: 2 * (len(dev_slab) // 2)]
+        best = None
+        for i in range(6):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            with torch.cuda.stream(stream):
+                b.copy_(a)
+            e1.record(stream)
+            e1.synchronize()
+            if i >= 1:
+                best = e0.elapsed_time(e1) if best is None else min(best, e0.elapsed_time(e1))
+        hbm_roofline["copy_this_run_gbs"] = 2 * a.numel() / (best * 1e-3) / GB
+        del a, b
         other = legs[not tma]
         hbm_roofline["other_engine"] = {
             "engine": "16-byte loads/stores (move_kernel)" if tma else "TMA tensor-map boxes (tmap_move_kernel)",
