@@ -315,13 +315,16 @@ kvx_status kv_store_noalloc(const kvx_pool* pool, const int32_t* block_table, in
  * Page-locked host memory for a shared chunk pool (Sec. 3.3: the shared tier
  * is one full-size pinned allocation; the paper's 256 GiB + 4096 B request
  * was rounded up to a power of two by the framework's pinned allocator and
- * silently fell back to pageable memory).  kv_host_alloc maps `bytes` (the
- * mapping is rounded up to whole huge pages, never to a power of two), backs
- * pools of at least one huge page with transparent huge pages, and registers
- * it page-locked, portable to every device and mapped for zero-copy.  Huge
- * pages are what let the copy engines (KVX_MODE_STAGED) reach the link peak
- * on a host with small base pages.  Failure is KVX_ENOMEM or KVX_ECUDA, never
- * a pageable fallback.  Free with kv_host_free (NULL is ignored).
+ * silently fell back to pageable memory).  kv_host_alloc returns `bytes` of
+ * page-locked memory, portable to every device and mapped for zero-copy.  A
+ * pool that whole huge pages fit within an eighth is mapped by the library
+ * on transparent huge pages (rounded up to whole huge pages, never to a power
+ * of two), which is what lets the copy engines (KVX_MODE_STAGED) reach the
+ * link peak on a host with small base pages; other pools, and pools huge
+ * pages cannot wholly back, come from the driver's allocator (see
+ * kv_host_alloc_ex and kv_host_pool_info).  Failure is KVX_ENOMEM or
+ * KVX_ECUDA, never a pageable fallback.  Free with kv_host_free (NULL is
+ * ignored).
  */
 kvx_status kv_host_alloc(int64_t bytes, void** out);
 /*
@@ -346,10 +349,10 @@ kvx_status kv_host_alloc_numa(int32_t numa_node, int64_t bytes, void** out, int3
  * KVX_NUMA_ANY.  Without a placement, a pool that whole huge pages would
  * overshoot by more than an eighth (for 512 MiB pages: anything below 4 GiB
  * that is not a near multiple), or any pool on a host without transparent
- * huge pages, also comes from the driver's allocator.  kv_host_alloc(b, o) is kv_host_alloc_ex(b,
- * KVX_NUMA_ANY, 0, o, NULL).  Memory from either source zero-copies at the
- * link peak; only huge pages let the copy engines (KVX_MODE_STAGED) reach it
- * steadily on a host with small base pages.
+ * huge pages, also comes from the driver's allocator.  kv_host_alloc(b, o)
+ * is kv_host_alloc_ex(b, KVX_NUMA_ANY, 0, o, NULL).  Memory from either
+ * source zero-copies at the link peak; only huge pages let the copy engines
+ * (KVX_MODE_STAGED) reach it steadily on a host with small base pages.
  */
 #define KVX_NUMA_ANY (-2)
 #define KVX_HOST_DRIVER 0x1u
