@@ -27,6 +27,10 @@ CASES = {
     "ragged_tail_nhd": (3, 40, 16, 4, 64, 2, NHD, 37, 64, 2, 9),
     "rows_48B_generic": (2, 20, 4, 3, 24, 2, HND, 17, 8, 0, 3),
     "rows_1KiB_generic": (2, 12, 8, 2, 256, 4, HND, 10, 16, 0, 1),
+    # rows of 2 KiB (the widest a tensor map describes: 256 eight-byte elements) and of
+    # 4 KiB (beyond it: the TMA engine falls back to row copies, the default to loads/stores)
+    "rows_2KiB_esz8": (2, 16, 4, 1, 512, 4, HND, 12, 8, 0, 1),
+    "rows_4KiB_no_tensor_map": (1, 10, 2, 1, 1024, 4, HND, 8, 4, 0, 1),
     "rows_16B_16_heads": (1, 30, 2, 16, 16, 1, HND, 25, 4, 2, 1),
     "fp8_1568_token_chunks": (4, 120, 32, 4, 256, 1, HND, 103, 1568, 0, 7),
     "many_chunks_three_launches": (1, 300, 1, 1, 8, 2, HND, 300, 2, 0, 1),
@@ -137,7 +141,8 @@ ENGINES = {"lsu": ("KVX_FLAG_DEVICE_LSU", 0), "default": (None, 0), "tma": ("KVX
 @pytest.mark.parametrize("engine", list(ENGINES))
 @pytest.mark.parametrize("name", ["tiny_cfg_hnd", "ragged_tail_nhd", "rows_48B_generic", "many_chunks_three_launches",
                                   "27b_shape_two_chunks", "paper_logical_blocks_49", "logical_blocks_4_nhd_ragged",
-                                  "rows_16B_16_heads", "one_token"])
+                                  "rows_16B_16_heads", "one_token", "rows_1KiB_generic", "rows_2KiB_esz8",
+                                  "rows_4KiB_no_tensor_map", "fp8_1568_token_chunks"])
 def test_device_pack_unpack_parity(orc, ctxs, name, engine):
     k = kvx()
     case = CASES[name]
