@@ -310,3 +310,72 @@ def test_state_snapshot_parity(orc, ctxs, mode, L, slots, sb):
     assert orc.state_copy(dst_np, sb, 1, want, False) == 0
     for a, b in zip(dst, dst_np):
         assert first_mismatch(np_of(a), b) is None
+
+
+def test_two_contexts_at_once_and_one_context_from_two_threads(orc):
+    """Replica A stores while replica B restores other chunks (two contexts, two
+    streams, overlapping on the GPU); then one context serves two host threads at
+    once.  Every result must match the oracle."""
+    import threading
+    k = kvx()
+    L, N, B, H, D, e, C = 3, 64, 16, 4, 64, 2, 128
+    spec = oracle.PoolSpec(L, N, B, H, D, e, HND)
+    T = 40 * B - 3
+    src_np, other_np = host_layers(spec, 501), host_layers(spec, 502)
+    ta, tb = synth.permuted_table(N, 40, 31), synth.permuted_table(N, 40, 32)
+    want_a, _ = oracle_store(orc, spec, src_np, ta, 0, T, C)
+    want_b, _ = oracle_store(orc, spec, other_np, ta, 0, T, C)
+    restored_b, _ = oracle_load(orc, spec, [np.full(spec.layer_bytes, POISON, np.uint8)] * L, tb, 0, T, C, want_b)
+    ta_d, tb_d = torch.from_numpy(ta).cuda(), torch.from_numpy(tb).cuda()
+
+    # two contexts at once
+    src = device_pool(spec, src_np)
+    dst_b = device_pool(spec)
+    out_a = pinned_chunks(orc, spec, 0, T, C)
+    in_b = [torch.from_numpy(w).pin_memory() for w in want_b]
+    ca, cb_ = k.kv_ctx_create(0), k.kv_ctx_create(0)
+    try:
+        sa, sb = torch.cuda.Stream(), torch.cuda.Stream()
+        torch.cuda.synchronize()
+        k.kv_store(ca, src, ta_d, 0, T, C, out_a, stream=sa)
+        k.kv_load(cb_, dst_b, tb_d, 0, T, C, in_b, stream=sb)
+        torch.cuda.synchronize()
+        assert k.kv_get_device_error(ca) == -1 and k.kv_get_device_error(cb_) == -1
+    finally:
+        k.kv_ctx_destroy(ca)
+        k.kv_ctx_destroy(cb_)
+    for got, w in zip(out_a, want_a):
+        assert first_mismatch(np_of(got)[:w.size], w) is None
+    for l in range(L):
+        assert first_mismatch(np_of(dst_b.layers[l]), restored_b[l]) is None
+
+    # one context, two host threads, each with its own stream and buffers
+    ctx = k.kv_ctx_create(0)
+    pools = [device_pool(spec, src_np), device_pool(spec, other_np)]
+    outs = [pinned_chunks(orc, spec, 0, T, C) for _ in range(2)]
+    errors = []
+
+    def worker(i):
+        try:
+            s = torch.cuda.Stream()
+            for _ in range(5):
+                k.kv_store(ctx, pools[i], ta_d, 0, T, C, outs[i], stream=s)
+            s.synchronize()
+        except Exception as ex:  # reported below
+            errors.append(ex)
+
+    try:
+        torch.cuda.synchronize()
+        threads = [threading.Thread(target=worker, args=(i,)) for i in range(2)]
+        for t in threads:
+            t.start()
+        for t in threads:
+            t.join(timeout=120)
+        assert not errors, errors
+        assert k.kv_get_device_error(ctx) == -1
+    finally:
+        k.kv_ctx_destroy(ctx)
+    for got, w in zip(outs[0], want_a):
+        assert first_mismatch(np_of(got)[:w.size], w) is None
+    for got, w in zip(outs[1], want_b):
+        assert first_mismatch(np_of(got)[:w.size], w) is None
