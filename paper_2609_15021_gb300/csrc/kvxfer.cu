@@ -452,6 +452,7 @@ kvx_status enqueue_direct(kvx_ctx* ctx, const Plan& pl, cudaStream_t s) {
     add_job(&p, pl.side[i], (pl.first_chunk + i) * pl.bpc, pl.tokens[i], 0, pl.P->num_layers);
     bytes += chunk_bytes_of(pl.P, pl.g, pl.tokens[i]);
     if (p.n_jobs == kMaxJobs || i == pl.n - 1) {
+      TraceRange trace("kvx launch: chunks");
       kvx_status st = launch_move_timed(ctx, pl.P, pl.dir, pl.P->layout, p, bytes, s, pl.over_link);
       if (st != KVX_OK) return st;
       p.n_jobs = 0;
@@ -474,6 +475,7 @@ kvx_status enqueue_staged(kvx_ctx* ctx, const Plan& pl) {
   auto layer_bytes = [&](int64_t i) { return 2ll * pl.tokens[i] * P->num_heads * pl.g.row; };
   auto flush = [&]() -> kvx_status {
     if (batch.empty()) return KVX_OK;
+    TraceRange trace(pl.dir == kPack ? "kvx staged batch: pack, copy out" : "kvx staged batch: copy in, unpack");
     const int k = ctx->next_slot;
     ctx->next_slot = (ctx->next_slot + 1) % ctx->nslots;
     uint8_t* slot = ctx->slots[k];
