@@ -204,6 +204,8 @@ def parse():
     ap.add_argument("--host-alloc", choices=["plain", "numa", "driver"], default="plain",
                     help="pinned pool from kv_host_alloc, from kv_host_alloc_numa on the host NUMA "
                          "node nearest the GPU, or from the driver's allocator (KVX_HOST_DRIVER)")
+    ap.add_argument("--no-tier", action="store_true",
+                    help="skip the leg that stores and restores chunk by chunk through the host tier")
     ap.add_argument("--no-concurrent", action="store_true",
                     help="skip the two-replica leg (one stores while the other restores)")
     ap.add_argument("--device-engine", choices=["lsu", "tma"], default="tma",
@@ -457,6 +459,9 @@ def run_ours(args):
         barrier(world)
         torch.cuda.synchronize()
     clock_info = clocks.summary()
+    # the link peak again right after the timed steps: a drop shows traffic from
+    # outside this process (the host memory is shared) during the measurement
+    link_after = host_link_peak(torch, dev)
     total_ms = ev[0][0].elapsed_time(ev[-1][2])
     store_ms = [e_[0].elapsed_time(e_[1]) for e_ in ev]
     restore_ms = [e_[1].elapsed_time(e_[2]) for e_ in ev]
@@ -588,7 +593,9 @@ def run_ours(args):
     host_link = {"store_gbs": store_gbs, "restore_gbs": restore_gbs, "peak_d2h_gbs": link["d2h"],
                  "peak_h2d_gbs": link["h2d"], "peak_bidir_gbs": link["bidir"], "store_frac": store_gbs / link["d2h"],
                  "restore_frac": restore_gbs / link["h2d"],
-                 "peak_source": "pinned cudaMemcpyAsync of 1 GiB, best of 5, measured in this run"}
+                 "peak_after_d2h_gbs": link_after["d2h"], "peak_after_h2d_gbs": link_after["h2d"],
+                 "peak_source": "pinned cudaMemcpyAsync of 1 GiB, best of 5, measured in this run before "
+                                "(peak_*) and right after (peak_after_*) the timed steps"}
 
     # Two replicas at once, each with its own context and stream: replica A stores
     # the context into a second chunk set while replica B restores the chunks the
@@ -631,6 +638,56 @@ def run_ours(args):
                       "what": "replica A kv_store of the context into a second pinned chunk set while replica B "
                               "kv_load of the timed steps' chunks into its pool, own context and stream each; "
                               "peak = pinned cudaMemcpyAsync of 1 GiB each way at once"}
+
+    # The tier path: the same store and restore through a private host tier, as a
+    # replica uses it: reserve a slot per chunk key, one kv_store into those slots,
+    # commit each key on the stream; prefix lookup; acquire each key on the stream,
+    # one kv_load from those slots, release each key on the stream.  Commit and
+    # release are ordered by events on the stream, so the host never waits.
+    tier_leg = None
+    if not args.no_tier and world == 1 and host_mem_available() > n_chunks * cb + (32 << 30):
+        tier = k.KvTier(cb, n_chunks)
+        token_ids = synth.rng(synth.SEED).integers(0, 150000, size=T).astype(np.int32)
+        keys = k.kv_chunk_keys(token_ids, C, salt=synth.SEED)
+        st_ms, ld_ms, host_ms, hits = [], [], [], 0
+        for rep in range(2 + 3):
+            a, b, c = (torch.cuda.Event(enable_timing=True) for _ in range(3))
+            torch.cuda.synchronize()
+            t0 = time.perf_counter()
+            a.record(stream)
+            slots = [tier.reserve(key) for key in keys]
+            k.kv_store(ctx, src, ta, 0, T, C, slots, stream=stream)
+            for key in keys:
+                tier.commit(key, stream=stream)
+            b.record(stream)
+            hits = tier.prefix_hits(keys)
+            slots = [tier.acquire(key, stream=stream) for key in keys[:hits]]
+            k.kv_load(ctx, dst, tb, 0, T, C, slots, stream=stream)
+            for key in keys[:hits]:
+                tier.release(key, stream=stream)
+            c.record(stream)
+            del slots
+            t1 = time.perf_counter()
+            torch.cuda.synchronize()
+            tier.poll()
+            if rep >= 2:
+                st_ms.append(a.elapsed_time(b))
+                ld_ms.append(b.elapsed_time(c))
+                host_ms.append((t1 - t0) * 1e3)
+        assert k.kv_get_device_error(ctx) == -1
+        same = all(torch.equal(tier.acquire(keys[ci], k.KVX_NO_STREAM), chunks[ci])
+                   for ci in sorted({0, n_chunks // 2, n_chunks - 1}))
+        for ci in sorted({0, n_chunks // 2, n_chunks - 1}):
+            tier.release(keys[ci], k.KVX_NO_STREAM)
+        tstats = tier.stats()
+        tier.close()
+        tier_leg = {"store_ms": statistics.median(st_ms), "restore_ms": statistics.median(ld_ms),
+                    "store_gbs": X / (statistics.median(st_ms) * 1e-3) / GB,
+                    "restore_gbs": X / (statistics.median(ld_ms) * 1e-3) / GB,
+                    "host_ms_per_store_and_restore": statistics.median(host_ms),
+                    "prefix_hits": hits, "chunks": n_chunks, "tier_calls_per_chunk": 4,
+                    "transfer_calls_per_direction": 1,
+                    "slots_equal_timed_chunks_on_sample": same, "evictions": tstats["evictions"]}
 
     cpu = None
     verified = None
@@ -680,6 +737,7 @@ def run_ours(args):
         "cpu_baseline": cpu,
         "verified_sample_vs_oracle": verified,
         "concurrent_replicas": concurrent,
+        "tier_path": tier_leg,
         "e2e": e2e,
         "gpu_launches": stats["kernel_launches"],
         "memcpy_calls": stats["memcpy_calls"],

@@ -39,6 +39,7 @@
 #include <time.h>
 #include <unistd.h>
 
+#include <deque>
 #include <mutex>
 #include <new>
 #include <unordered_map>
@@ -149,8 +150,9 @@ struct kvx_tier {
   char name[128] = "";
   int32_t pid = 0;
   // this process's pending GPU work on slots
-  std::vector<PendingEvent> commits;   // COMMITTING entries written by this process
-  std::vector<PendingEvent> releases;  // pins held until queued work completes
+  std::deque<PendingEvent> commits;    // COMMITTING entries written by this process, oldest first
+  std::deque<PendingEvent> releases;   // pins held until queued work completes, oldest first
+  std::unordered_map<int64_t, int32_t> queued;  // slot -> its releases in `releases`
   std::unordered_map<int64_t, cudaEvent_t> commit_event;  // slot -> event readers here may wait on
   std::vector<cudaEvent_t> spare;
   std::mutex local;          // guards the members above
@@ -187,38 +189,52 @@ cudaEvent_t take_event(kvx_tier* t) {
 }
 
 // Settle this process's completed GPU work: COMMITTING -> READY, pins dropped.
-void poll_locked(kvx_tier* t, bool wait) {
+// kFront settles completed work from the front of each queue up to the first
+// that is still pending (O(1) amortised: every tier call does it, and work on
+// one stream completes in order); kAll checks every entry; kWait waits for all.
+enum PollMode { kFront, kAll, kWait };
+
+void settle_commit(kvx_tier* t, const PendingEvent& p) {
+  SlotMeta& m = t->meta[p.slot];
+  if (m.state == kCommitting && m.writer_pid == t->pid) m.state = kReady;
+  auto it = t->commit_event.find(p.slot);
+  if (it != t->commit_event.end() && it->second == p.ev) t->commit_event.erase(it);
+  t->spare.push_back(p.ev);
+}
+
+void settle_release(kvx_tier* t, const PendingEvent& p) {
+  add_pins(t->meta[p.slot], t->pid, -1);
+  auto it = t->queued.find(p.slot);
+  if (it != t->queued.end() && --it->second <= 0) t->queued.erase(it);
+  t->spare.push_back(p.ev);
+}
+
+void poll_locked(kvx_tier* t, PollMode mode) {
   auto done = [&](cudaEvent_t e) {
-    cudaError_t q = wait ? cudaEventSynchronize(e) : cudaEventQuery(e);
+    const cudaError_t q = mode == kWait ? cudaEventSynchronize(e) : cudaEventQuery(e);
     if (q == cudaErrorNotReady) return false;
     cudaGetLastError();
     return true;
   };
-  for (size_t i = 0; i < t->commits.size();) {
-    PendingEvent& p = t->commits[i];
-    if (!done(p.ev)) {
-      ++i;
-      continue;
+  auto settle = [&](std::deque<PendingEvent>& q, void (*fn)(kvx_tier*, const PendingEvent&)) {
+    if (mode == kFront) {
+      while (!q.empty() && done(q.front().ev)) {
+        fn(t, q.front());
+        q.pop_front();
+      }
+      return;
     }
-    SlotMeta& m = t->meta[p.slot];
-    if (m.state == kCommitting && m.writer_pid == t->pid) m.state = kReady;
-    auto it = t->commit_event.find(p.slot);
-    if (it != t->commit_event.end() && it->second == p.ev) t->commit_event.erase(it);
-    t->spare.push_back(p.ev);
-    t->commits[i] = t->commits.back();
-    t->commits.pop_back();
-  }
-  for (size_t i = 0; i < t->releases.size();) {
-    PendingEvent& p = t->releases[i];
-    if (!done(p.ev)) {
-      ++i;
-      continue;
+    std::deque<PendingEvent> pending;
+    for (const PendingEvent& p : q) {
+      if (done(p.ev))
+        fn(t, p);
+      else
+        pending.push_back(p);
     }
-    add_pins(t->meta[p.slot], t->pid, -1);
-    t->spare.push_back(p.ev);
-    t->releases[i] = t->releases.back();
-    t->releases.pop_back();
-  }
+    q.swap(pending);
+  };
+  settle(t->commits, settle_commit);
+  settle(t->releases, settle_release);
 }
 
 // Key index: every slot that is not FREE has exactly one entry, at or after
@@ -301,9 +317,8 @@ int64_t pick_slot(kvx_tier* t) {
 
 // Pins of this process on `slot` whose release is queued behind GPU work.
 int64_t queued_releases(const kvx_tier* t, int64_t slot) {
-  int64_t n = 0;
-  for (const PendingEvent& p : t->releases) n += p.slot == slot;
-  return n;
+  auto it = t->queued.find(slot);
+  return it == t->queued.end() ? 0 : it->second;
 }
 
 int32_t pins_of(const SlotMeta& m, int32_t pid) {
@@ -355,7 +370,7 @@ void destroy_tier(kvx_tier* t) {
     if (t->hdr) {
       int r = pthread_mutex_lock(&t->hdr->mu);
       if (r == EOWNERDEAD) pthread_mutex_consistent(&t->hdr->mu);
-      poll_locked(t, true);  // settle this process's pending work
+      poll_locked(t, kWait);  // settle this process's pending work
       pthread_mutex_unlock(&t->hdr->mu);
     }
     for (cudaEvent_t e : t->spare) cudaEventDestroy(e);
@@ -570,18 +585,21 @@ void kv_tier_destroy(kvx_tier* t) { destroy_tier(t); }
 kvx_status kv_tier_poll(kvx_tier* t) {
   if (!t) return KVX_EINVAL;
   TierLock lock(t);
-  poll_locked(t, false);
+  poll_locked(t, kAll);
   return KVX_OK;
 }
 
 kvx_status kv_tier_reserve(kvx_tier* t, uint64_t key, void** slot) {
   if (!t || !slot) return KVX_EINVAL;
   TierLock lock(t);
-  poll_locked(t, false);
+  poll_locked(t, kFront);
   int64_t i = -1;
   // a second pass after reclaiming what processes that died left behind
   for (int pass = 0; pass < 2; ++pass) {
-    if (pass == 1 && reclaim_locked(t) == 0) break;
+    if (pass == 1) {
+      poll_locked(t, kAll);  // completed work behind a pending one frees slots too
+      if (reclaim_locked(t) == 0 && pick_slot(t) < 0 && find_slot(t, key) < 0) break;
+    }
     i = find_slot(t, key);
     if (i >= 0) {
       const SlotMeta& m = t->meta[i];
@@ -623,7 +641,7 @@ kvx_status kv_tier_reserve(kvx_tier* t, uint64_t key, void** slot) {
 kvx_status kv_tier_commit(kvx_tier* t, uint64_t key, kvx_stream_t stream) {
   if (!t) return KVX_EINVAL;
   TierLock lock(t);
-  poll_locked(t, false);
+  poll_locked(t, kFront);
   const int64_t i = find_slot(t, key);
   if (i < 0) return KVX_ENOENT;
   SlotMeta& m = t->meta[i];
@@ -650,7 +668,7 @@ kvx_status kv_tier_commit(kvx_tier* t, uint64_t key, kvx_stream_t stream) {
 kvx_status kv_tier_acquire(kvx_tier* t, uint64_t key, kvx_stream_t stream, void** slot) {
   if (!t || !slot) return KVX_EINVAL;
   TierLock lock(t);
-  poll_locked(t, false);
+  poll_locked(t, kFront);
   const int64_t i = find_slot(t, key);
   bool ok = i >= 0 && t->meta[i].state == kReady;
   cudaEvent_t wait_on = nullptr;
@@ -688,7 +706,7 @@ kvx_status kv_tier_acquire(kvx_tier* t, uint64_t key, kvx_stream_t stream, void*
 kvx_status kv_tier_release(kvx_tier* t, uint64_t key, kvx_stream_t stream) {
   if (!t) return KVX_EINVAL;
   TierLock lock(t);
-  poll_locked(t, false);
+  poll_locked(t, kFront);
   const int64_t i = find_slot(t, key);
   if (i < 0) return KVX_ENOENT;
   SlotMeta& m = t->meta[i];
@@ -712,13 +730,14 @@ kvx_status kv_tier_release(kvx_tier* t, uint64_t key, kvx_stream_t stream) {
     return cuda_fail(r, "cudaEventRecord (tier release)");
   }
   t->releases.push_back({i, e});  // the pin stays until the queued work completes
+  t->queued[i]++;
   return KVX_OK;
 }
 
 kvx_status kv_tier_reclaim(kvx_tier* t, int64_t* reclaimed) {
   if (!t) return KVX_EINVAL;
   TierLock lock(t);
-  poll_locked(t, false);
+  poll_locked(t, kFront);
   const int64_t n = reclaim_locked(t);
   if (reclaimed) *reclaimed = n;
   return KVX_OK;
@@ -727,7 +746,7 @@ kvx_status kv_tier_reclaim(kvx_tier* t, int64_t* reclaimed) {
 kvx_status kv_tier_prefix_hits(kvx_tier* t, const uint64_t* keys, int64_t n, int64_t* hits) {
   if (!t || !hits || n < 0 || (n > 0 && !keys)) return KVX_EINVAL;
   TierLock lock(t);
-  poll_locked(t, false);
+  poll_locked(t, kFront);
   int64_t h = 0;
   while (h < n) {
     const int64_t i = find_slot(t, keys[h]);
@@ -744,7 +763,7 @@ kvx_status kv_tier_prefix_hits(kvx_tier* t, const uint64_t* keys, int64_t n, int
 kvx_status kv_tier_stats(kvx_tier* t, kvx_tier_stats* out) {
   if (!t || !out) return KVX_EINVAL;
   TierLock lock(t);
-  poll_locked(t, false);
+  poll_locked(t, kFront);
   out->slots = t->hdr->n_slots;
   out->slot_bytes = t->hdr->slot_bytes;
   int64_t used = 0, pinned = 0;
