@@ -20,6 +20,7 @@
 #include <string.h>
 
 #include <algorithm>
+#include <atomic>
 #include <mutex>
 #include <new>
 #include <vector>
@@ -54,14 +55,17 @@ void record_cuda_error(int e, const char* call, int line) {
 // n-th next call with cudaErrorUnknown instead of calling CUDA.
 namespace {
 std::mutex g_fault_mu;
-char g_fault_point[32] = "";
-int g_fault_countdown = -1;
+char g_fault_point[32] = "";               // guarded by g_fault_mu
+std::atomic<int> g_fault_countdown{-1};    // -1: unarmed; written under g_fault_mu
 
 bool fault_now(const char* point) {
-  if (g_fault_countdown < 0) return false;  // unarmed (racy read is benign: re-checked under the lock)
+  // Unarmed is the common case and takes no lock; the armed state is re-read under it.
+  if (g_fault_countdown.load(std::memory_order_relaxed) < 0) return false;
   std::lock_guard<std::mutex> lock(g_fault_mu);
-  if (g_fault_countdown < 0 || strcmp(point, g_fault_point) != 0) return false;
-  if (g_fault_countdown-- > 0) return false;
+  const int n = g_fault_countdown.load(std::memory_order_relaxed);
+  if (n < 0 || strcmp(point, g_fault_point) != 0) return false;
+  g_fault_countdown.store(n - 1, std::memory_order_relaxed);  // 0 fires now and disarms
+  if (n > 0) return false;
   g_fault_point[0] = 0;
   return true;
 }
@@ -814,9 +818,11 @@ void destroy_ctx(kvx_ctx* ctx) {
 int32_t resolve_mode(int32_t m) {
   // Measured on GB300 (Grace host, NVLink-C2C) for a 128k-token 27B-class
   // context: zero-copy moves every step at the pinned-copy peak of both
-  // directions (193 / 211 GB/s) with 32 CTAs, while the staged pipeline
-  // alternates between that and about 25% slower steps.  Zero-copy also needs
-  // no staging memory and one launch per 64 chunks.
+  // directions (193 / 211 GB/s) from any pinned pool, including a tier in
+  // POSIX shared memory; the staged pipeline reaches 0.98-0.99 of that only
+  // from a pool wholly on huge pages.  Zero-copy also needs no staging memory,
+  // no second pass over HBM and one launch per 64 chunks, and two replicas
+  // moving at once get more of the bidirectional link with it.
   return m == KVX_MODE_AUTO ? (int32_t)KVX_MODE_ZEROCOPY : m;
 }
 
@@ -997,14 +1003,14 @@ kvx_status kv_fault_inject(const char* point, int32_t after_calls) {
   std::lock_guard<std::mutex> lock(g_fault_mu);
   if (!point || !point[0]) {
     g_fault_point[0] = 0;
-    g_fault_countdown = -1;
+    g_fault_countdown.store(-1, std::memory_order_relaxed);
     return KVX_OK;
   }
   bool known = false;
   for (const char* q : points) known |= strcmp(q, point) == 0;
   if (!known || after_calls < 0) return KVX_EINVAL;
   snprintf(g_fault_point, sizeof(g_fault_point), "%s", point);
-  g_fault_countdown = after_calls;
+  g_fault_countdown.store(after_calls, std::memory_order_relaxed);
   return KVX_OK;
 }
 
