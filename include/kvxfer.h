@@ -467,7 +467,10 @@ kvx_status kv_tier_release(kvx_tier* tier, uint64_t key, kvx_stream_t stream);
    kv_tier_reserve does the same by itself when it finds no usable slot.
    Liveness is judged by process id within this host's pid namespace; a
    private tier has nothing to reclaim.  An entry can be pinned by at most 8
-   processes at once (KVX_EBUSY beyond). */
+   processes at once (KVX_EBUSY beyond).  A process that dies inside a tier
+   call, holding the table lock, leaves no entry readable under a wrong key:
+   the next call in another process takes the lock over and rebuilds the key
+   index from the slot table, and the dead process's slot is reclaimed. */
 kvx_status kv_tier_reclaim(kvx_tier* tier, int64_t* reclaimed);
 /* Number of leading keys with committed entries (the cached prefix). */
 kvx_status kv_tier_prefix_hits(kvx_tier* tier, const uint64_t* keys, int64_t n, int64_t* hits);
@@ -501,8 +504,12 @@ const char* kv_last_error_message(void);
  * fails with cudaErrorUnknown (cudaErrorMemoryAllocation for "host_alloc")
  * instead of being made.  Points: "launch" (kernel launches), "memcpy"
  * (staged-mode copies), "event" (the staged pipeline's ordering event
- * recorded on the caller's stream), "host_alloc" (kv_host_alloc).  One point is armed at a time;
- * point NULL or "" disarms.  KVX_EINVAL for an unknown point.
+ * recorded on the caller's stream), "host_alloc" (kv_host_alloc).  One more
+ * point fails differently: "tier_exit" ends the process (_exit(3)) inside
+ * kv_tier_reserve, while it holds a shared tier's table lock, right after it
+ * has taken a slot for the new key; it tests how the processes left recover
+ * the tier from a replica that died mid-update.  One point is armed at a
+ * time; point NULL or "" disarms.  KVX_EINVAL for an unknown point.
  */
 kvx_status kv_fault_inject(const char* point, int32_t after_calls);
 

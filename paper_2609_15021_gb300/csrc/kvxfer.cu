@@ -999,7 +999,7 @@ kvx_status kv_state_load(kvx_ctx* ctx, int32_t num_layers, void* const* layer_ba
 }
 
 kvx_status kv_fault_inject(const char* point, int32_t after_calls) {
-  static const char* const points[] = {"launch", "memcpy", "event", "host_alloc"};
+  static const char* const points[] = {"launch", "memcpy", "event", "host_alloc", "tier_exit"};
   std::lock_guard<std::mutex> lock(g_fault_mu);
   if (!point || !point[0]) {
     g_fault_point[0] = 0;

@@ -160,13 +160,24 @@ struct kvx_tier {
 
 namespace {
 
-// Process-shared lock over the slot table (robust: a holder that died leaves it usable).
+void rebuild_index_locked(kvx_tier* t);
+
+// Takes the process-shared table lock.  It is robust: when its holder died,
+// the next taker gets it, marks it consistent and rebuilds the key index from
+// the slot table, since the holder may have died halfway through moving
+// index entries.
+void lock_table(kvx_tier* t) {
+  if (pthread_mutex_lock(&t->hdr->mu) == EOWNERDEAD) {
+    pthread_mutex_consistent(&t->hdr->mu);
+    rebuild_index_locked(t);
+  }
+}
+
 struct TierLock {
   kvx_tier* t;
   explicit TierLock(kvx_tier* tier) : t(tier) {
     t->local.lock();
-    int r = pthread_mutex_lock(&t->hdr->mu);
-    if (r == EOWNERDEAD) pthread_mutex_consistent(&t->hdr->mu);
+    lock_table(t);
   }
   ~TierLock() {
     pthread_mutex_unlock(&t->hdr->mu);
@@ -296,6 +307,25 @@ void index_erase(kvx_tier* t, uint64_t key) {
   if (i >= 0) index_erase_at(t, i);
 }
 
+// The slot table is the record and the index is derived from it.  The table
+// itself is kept valid after every single store: a slot changes its key only
+// while WRITING, so a process that dies mid-update leaves at worst a WRITING
+// slot of a dead writer (freed by reclaim), never a readable entry under the
+// wrong key.  Two live slots with one key cannot arise; should they, the newer
+// is indexed and the other is evicted or reclaimed like any unindexed slot.
+void rebuild_index_locked(kvx_tier* t) {
+  memset(t->index, 0xFF, (size_t)t->hdr->index_size * 8);  // every entry -1: empty
+  for (int64_t i = 0; i < t->hdr->n_slots; ++i) {
+    const SlotMeta& m = t->meta[i];
+    if (m.state == kFree) continue;
+    const int64_t pos = index_pos(t, m.key);
+    if (pos < 0)
+      index_insert(t, m.key, i);
+    else if (t->meta[t->index[pos]].tick < m.tick)
+      t->index[pos] = i;
+  }
+}
+
 int64_t find_slot(kvx_tier* t, uint64_t key) {
   const int64_t i = index_pos(t, key);
   if (i < 0) return -1;
@@ -368,8 +398,7 @@ void destroy_tier(kvx_tier* t) {
   {
     std::lock_guard<std::mutex> g(t->local);
     if (t->hdr) {
-      int r = pthread_mutex_lock(&t->hdr->mu);
-      if (r == EOWNERDEAD) pthread_mutex_consistent(&t->hdr->mu);
+      lock_table(t);
       poll_locked(t, kWait);  // settle this process's pending work
       pthread_mutex_unlock(&t->hdr->mu);
     }
@@ -614,8 +643,14 @@ kvx_status kv_tier_reserve(kvx_tier* t, uint64_t key, void** slot) {
         index_erase(t, m.key);
         t->hdr->evictions++;
       }
+      // WRITING before the key changes: were this process to die from here
+      // on, the slot is a dead writer's reservation, never old bytes
+      // readable under the new key.
+      m.writer_pid = t->pid;
+      m.state = kWriting;
       m.key = key;
       index_insert(t, key, i);
+      if (fault_point("tier_exit")) _exit(3);  // test hook: die holding the lock, mid-reserve
       break;
     }
   }
@@ -628,9 +663,8 @@ kvx_status kv_tier_reserve(kvx_tier* t, uint64_t key, void** slot) {
     return KVX_ENOMEM;
   }
   SlotMeta& m = t->meta[i];
-  m.key = key;
-  m.state = kWriting;
   m.writer_pid = t->pid;
+  m.state = kWriting;
   clear_pins(m);
   add_pins(m, t->pid, 1);
   m.tick = ++t->hdr->clock;

@@ -141,6 +141,62 @@ def test_dead_process_pins_and_writes_are_reclaimed():
         t.close()
 
 
+def _child_dies_mid_reserve(name, after_calls):
+    sys.path.insert(0, ROOT)
+    from paper_2609_15021_gb300 import kvxfer as k
+    t = k.KvTier(shared_name=name, pin=False)
+    k.kv_fault_inject("tier_exit", after_calls)
+    for key in (30, 31):
+        t.reserve(key)                 # the armed reservation ends the process inside the lock
+    os._exit(0)                        # not reached when the hook fires
+
+
+@pytest.mark.parametrize("after_calls", [0, 1])
+def test_process_dying_mid_reserve_leaves_no_wrong_entry(after_calls):
+    """Failure detection on the host: a replica that dies inside kv_tier_reserve,
+    holding the table lock, right after it has evicted an entry and indexed
+    its new key, leaves neither that key readable (the slot still holds the
+    evicted bytes) nor a lock that blocks the others.  The next call here takes
+    the lock over (the mutex is robust), rebuilds the key index, and the dead
+    process's slot is reclaimed."""
+    sys.path.insert(0, ROOT)
+    from paper_2609_15021_gb300 import _build
+    _build.build()
+    from paper_2609_15021_gb300 import kvxfer as k
+    NO = -1
+    name = _name(f"midres{after_calls}")
+    t = k.KvTier(64, 3, shared_name=name, create=True, pin=False)
+    try:
+        for key, fill in ((1, 11), (2, 22), (3, 33)):      # a full tier: the child must evict
+            t.reserve(key).fill_(fill)
+            t.commit(key, NO)
+        ctx = mp.get_context("spawn")
+        p = ctx.Process(target=_child_dies_mid_reserve, args=(name, after_calls))
+        p.start()
+        p.join(timeout=120)
+        assert p.exitcode == 3                              # the hook's exit, inside the lock
+        died_at = 30 + after_calls
+        assert t.prefix_hits([died_at]) == 0                # never readable under the new key
+        with pytest.raises(k.KvxError) as e:
+            t.acquire(died_at, NO)
+        assert e.value.status == k.KVX_ENOENT
+        survivors = [key for key in (1, 2, 3) if t.prefix_hits([key]) == 1]
+        assert len(survivors) == 2 - after_calls           # one eviction per reservation the child made
+        for key in survivors:                               # what survives reads its own bytes
+            assert int(t.acquire(key, NO)[0]) == key * 11
+            t.release(key, NO)
+        assert t.reclaim() == 1 + after_calls               # the dead writer's reservation(s)
+        s = t.reserve(died_at)                              # the key is usable again
+        s.fill_(44)
+        t.commit(died_at, NO)
+        assert int(t.acquire(died_at, NO)[0]) == 44
+        t.release(died_at, NO)
+        st = t.stats()
+        assert st["pinned"] == 0 and st["entries"] == len(survivors) + 1
+    finally:
+        t.close()
+
+
 def test_reclaim_leaves_live_processes_alone():
     sys.path.insert(0, ROOT)
     from paper_2609_15021_gb300 import _build
