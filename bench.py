@@ -742,6 +742,10 @@ def run_ours(args):
         "gpu_launches": stats["kernel_launches"],
         "memcpy_calls": stats["memcpy_calls"],
         "clocks": clock_info,
+        "device": {"gpu": torch.cuda.get_device_name(dev),
+                   "sms": torch.cuda.get_device_properties(dev).multi_processor_count,
+                   "host_cpu": cpu_model(), "host_threads": os.cpu_count(),
+                   "pinned_pool_numa_node": host_pool.info()["numa_node"]},
     }
     print(json.dumps(line), flush=True)
     return 0

@@ -510,6 +510,9 @@ const char* kv_last_error_message(void);
  * has taken a slot for the new key; it tests how the processes left recover
  * the tier from a replica that died mid-update.  One point is armed at a
  * time; point NULL or "" disarms.  KVX_EINVAL for an unknown point.
+ * The environment variable KVX_FAULT="<point>[:<after_calls>]" arms a point
+ * the same way when the library is loaded (a malformed value is reported on
+ * stderr and ignored), for programs that do not call this function.
  */
 kvx_status kv_fault_inject(const char* point, int32_t after_calls);
 

@@ -17,6 +17,7 @@
 #include <cuda_runtime.h>
 #include <limits.h>
 #include <stdio.h>
+#include <stdlib.h>
 #include <string.h>
 
 #include <algorithm>
@@ -1013,6 +1014,40 @@ kvx_status kv_fault_inject(const char* point, int32_t after_calls) {
   g_fault_countdown.store(after_calls, std::memory_order_relaxed);
   return KVX_OK;
 }
+
+}  // extern "C"
+
+namespace {
+// KVX_FAULT="<point>[:<after_calls>]" arms one fault point when the library is
+// loaded, so that a program which never calls kv_fault_inject (a serving
+// engine under test) can be made to fail the same way.  A value naming no
+// point, or a count that is not a non-negative integer, is reported on stderr
+// and ignored.
+struct FaultFromEnv {
+  FaultFromEnv() {
+    const char* v = getenv("KVX_FAULT");
+    if (!v || !v[0]) return;
+    char point[32];
+    const char* colon = strchr(v, ':');
+    const size_t len = colon ? (size_t)(colon - v) : strlen(v);
+    long n = 0;
+    bool ok = len > 0 && len < sizeof(point);
+    if (ok && colon) {
+      char* end = nullptr;
+      n = strtol(colon + 1, &end, 10);
+      ok = end != colon + 1 && *end == 0 && n >= 0 && n <= INT32_MAX;
+    }
+    if (ok) {
+      memcpy(point, v, len);
+      point[len] = 0;
+      ok = kv_fault_inject(point, (int32_t)n) == KVX_OK;
+    }
+    if (!ok) fprintf(stderr, "libkvxfer: ignoring KVX_FAULT=%s (expected <point>[:<after_calls>])\n", v);
+  }
+} g_fault_from_env;
+}  // namespace
+
+extern "C" {
 
 kvx_status kv_pool_view_check(const kvx_pool* pool, int32_t ndim, const int64_t* shape,
                               const int64_t* strides_bytes) {

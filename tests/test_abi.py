@@ -208,3 +208,44 @@ def test_host_alloc_numa_arguments(k):
     assert ex(4096, 0, k.KVX_HOST_DRIVER, ctypes.byref(out), None) == k.KVX_EINVAL         # driver + node
     assert ex(4096, -3, 0, ctypes.byref(out), None) == k.KVX_EINVAL
     assert k._lib.kv_host_alloc_numa(k.KVX_NUMA_ANY, 4096, ctypes.byref(out), None) == k.KVX_EINVAL
+
+
+_FAULT_PROBE = r"""
+import ctypes, json, sys
+sys.path.insert(0, sys.argv[1])
+from paper_2609_15021_gb300 import kvxfer as k
+out = ctypes.c_void_p()
+res = []
+for _ in range(3):
+    code = k._lib.kv_host_alloc(4096, ctypes.byref(out))
+    res.append([code, k._lib.kv_last_error_message().decode()])
+    k._lib.kv_host_free(out)
+print(json.dumps(res))
+"""
+
+
+def _run_with_fault_env(value):
+    import json
+    import subprocess
+    import sys
+    env = dict(os.environ, KVX_FAULT=value)
+    r = subprocess.run([sys.executable, "-c", _FAULT_PROBE, ROOT], env=env, capture_output=True, text=True,
+                       timeout=300)
+    assert r.returncode == 0, r.stderr
+    return json.loads(r.stdout.strip().splitlines()[-1]), r.stderr
+
+
+@pytest.mark.parametrize("value, injected_at", [("host_alloc", 0), ("host_alloc:1", 1), ("host_alloc:0", 0)])
+def test_fault_armed_from_environment(k, value, injected_at):
+    """KVX_FAULT arms a fault point when the library loads: exactly the
+    (n + 1)-th pinned allocation fails as injected, the others do not."""
+    res, _ = _run_with_fault_env(value)
+    injected = [code == k.KVX_ENOMEM and "injected" in msg for code, msg in res]
+    assert injected == [i == injected_at for i in range(3)]
+
+
+@pytest.mark.parametrize("value", ["no_such_point", "host_alloc:x", "host_alloc:-1", ":3", "host_alloc:"])
+def test_malformed_fault_environment_is_reported_and_ignored(k, value):
+    res, err = _run_with_fault_env(value)
+    assert "ignoring KVX_FAULT" in err
+    assert not any("injected" in msg for _, msg in res)
