@@ -3,7 +3,9 @@
 Replica A (this process) prefills nothing here: it fills its paged KV pool
 with data, stores the prefix chunk by chunk into a shared tier (POSIX shared
 memory, registered pinned and mapped in each process), and commits each chunk
-on its stream.  Replica B (a second process on the same GPU) asks the tier
+on its stream: the GPU publishes each commit into the shared slot table once
+the chunk's bytes are written, so other processes see it with no further call
+from A.  Replica B (a second process on the same GPU) asks the tier
 how much of the prefix it holds, acquires those chunks, restores them into
 its own pool through a different block table, and checks the bytes it got
 against A's pages, which A hands it through the tier as well.
@@ -74,9 +76,8 @@ def main():
         for c, key in enumerate(keys):
             slot = tier.reserve(key)
             k.kv_store(ctx, pool, table, c * C, (c + 1) * C, C, [slot], stream=stream)
-            tier.commit(key, stream=stream)      # readable once the store has completed
+            tier.commit(key, stream=stream)      # readable everywhere once the GPU has passed this point
         stream.synchronize()
-        tier.poll()                              # other processes see the entries from here on
         want = [t.view(N, PAGE)[table.long()].cpu().numpy() for t in layers]
         k.kv_ctx_destroy(ctx)
 

@@ -14,7 +14,7 @@ BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "_lib", "libkvxfer.so")
 
 SOURCES = ["pack_kernels.cu", "segment_kernels.cu", "tma_kernels.cu", "kvxfer.cu", "probe.cu", "no_alloc.cu", "tier.cpp",
-           "host_alloc.cpp"]
+           "tier_kernels.cu", "host_alloc.cpp"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC,-O2,-Wall,-Wextra", f"-I{INCLUDE}"]
 

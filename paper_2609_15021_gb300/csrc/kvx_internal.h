@@ -103,6 +103,11 @@ cudaError_t launch_move_tmap(int dir, const MoveParams& p, const void* maps, int
                              int stage_bytes, int stages, int* timeout, cudaStream_t s);
 int move_ctas_per_sm(int dir, int layout);
 int segment_ctas_per_sm();
+// Shared tier (tier_kernels.cu): enqueues on s a system-scope release store of
+// seq to dev_flag (a device address of mapped host memory).
+cudaError_t launch_tier_publish(uint64_t* dev_flag, uint64_t seq, cudaStream_t s);
+// Loads the publication kernel (at tier open, never inside a commit).
+cudaError_t prepare_tier_kernels();
 
 // Records the last CUDA error seen by this thread (kv_last_cuda_error).
 void set_last_cuda_error(int e);

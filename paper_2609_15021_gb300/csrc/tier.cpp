@@ -11,13 +11,18 @@
 // memory holding the slot table, a process-shared robust mutex and the data,
 // which every process registers as pinned, mapped memory).  Entry states:
 //   WRITING    reserved by a writer, not readable
-//   COMMITTING committed on the writer's stream, GPU work still pending:
+//   COMMITTING committed on the writer's stream, not yet published:
 //              readable in the writer's process (the reader's stream waits on
 //              the writer's event), invisible to other processes
 //   READY      the data is complete: readable everywhere
-// The writer's process turns COMMITTING into READY when its event completes
-// (checked at every tier call of that process and by kv_tier_poll), which is
-// the paper's completion-before-consumption rule applied across processes.
+// A commit on a stream enqueues, behind the writer's work, a publication of
+// the commit's sequence number into the shared slot table (a system-scope
+// release store by the GPU, tier_kernels.cu).  Any process that finds the
+// number there turns COMMITTING into READY, so the entry becomes readable
+// everywhere as soon as the GPU has passed the commit, with no further call
+// of the writer's process; the writer's own event does the same in its
+// process (and is the only path for a private tier).  This is the paper's
+// completion-before-consumption rule applied across processes.
 // Readers pin entries; a release on a stream keeps the pin until the work on
 // that stream completes, so a slot in use by queued GPU work is never evicted.
 // Pins are kept per process: when a process sharing the tier dies, its pins
@@ -30,6 +35,7 @@
 #include <fcntl.h>
 #include <pthread.h>
 #include <signal.h>
+#include <stddef.h>
 #include <stdint.h>
 #include <stdio.h>
 #include <stdlib.h>
@@ -51,7 +57,7 @@ using namespace kvx;
 
 namespace {
 
-constexpr uint64_t kMagic = 0x3352454954584B56ull;  // "VKXTIER3"
+constexpr uint64_t kMagic = 0x3452454954584B56ull;  // "VKXTIER4"
 constexpr int64_t kDataAlign = 2ll << 20;
 constexpr int kHolders = 8;  // processes that may pin one entry at the same time
 
@@ -63,6 +69,7 @@ struct Header {
   int64_t index_size;  // entries of the key index: a power of two >= 2 * n_slots
   pthread_mutex_t mu;
   uint64_t clock;
+  uint64_t seq;        // commits made on a stream, for their publication
   int64_t hits, misses, evictions;
   volatile int32_t initialised;
 };
@@ -76,6 +83,10 @@ struct SlotMeta {
   // the pins by process, so that a process that died can be dropped from them
   int32_t holder_pid[kHolders];
   int32_t holder_pins[kHolders];
+  // A commit on a stream takes the next sequence number; the GPU writes it to
+  // `published` once the stream has passed the commit (tier_kernels.cu).
+  uint64_t commit_seq;
+  uint64_t published;  // written by the GPU: read with acquire loads only
 };
 
 // Adds n (may be negative) to pid's pins of m; false if pid holds none and
@@ -130,6 +141,7 @@ kvx_status cuda_fail(cudaError_t e, const char* what) {
 struct PendingEvent {
   int64_t slot;
   cudaEvent_t ev;
+  uint64_t seq;  // commits: the commit's sequence number
 };
 
 }  // namespace
@@ -140,6 +152,7 @@ struct kvx_tier {
   SlotMeta* meta = nullptr;
   int64_t* index = nullptr;  // open addressing, linear probing: slot or -1 (empty)
   uint8_t* data = nullptr;
+  uint8_t* meta_dev = nullptr;  // device address of meta (shared, registered tiers): publication target
   // ownership
   void* mapping = nullptr;   // shared: the whole mmap; private: the metadata allocation
   int64_t mapping_bytes = 0;
@@ -199,6 +212,16 @@ cudaEvent_t take_event(kvx_tier* t) {
   return e;
 }
 
+// COMMITTING -> READY once the GPU has published the commit (any process may
+// do this: the acquire load pairs with the GPU's system-scope release, so the
+// chunk's bytes are complete when the number is seen).
+bool promote_published(SlotMeta& m) {
+  if (m.state != kCommitting || m.commit_seq == 0) return false;
+  if (__atomic_load_n(&m.published, __ATOMIC_ACQUIRE) != m.commit_seq) return false;
+  m.state = kReady;
+  return true;
+}
+
 // Settle this process's completed GPU work: COMMITTING -> READY, pins dropped.
 // kFront settles completed work from the front of each queue up to the first
 // that is still pending (O(1) amortised: every tier call does it, and work on
@@ -207,7 +230,7 @@ enum PollMode { kFront, kAll, kWait };
 
 void settle_commit(kvx_tier* t, const PendingEvent& p) {
   SlotMeta& m = t->meta[p.slot];
-  if (m.state == kCommitting && m.writer_pid == t->pid) m.state = kReady;
+  if (m.state == kCommitting && m.writer_pid == t->pid && m.commit_seq == p.seq) m.state = kReady;
   auto it = t->commit_event.find(p.slot);
   if (it != t->commit_event.end() && it->second == p.ev) t->commit_event.erase(it);
   t->spare.push_back(p.ev);
@@ -246,6 +269,8 @@ void poll_locked(kvx_tier* t, PollMode mode) {
   };
   settle(t->commits, settle_commit);
   settle(t->releases, settle_release);
+  if (mode != kFront && t->meta_dev)  // commits of every process that the GPU has published
+    for (int64_t i = 0; i < t->hdr->n_slots; ++i) promote_published(t->meta[i]);
 }
 
 // Key index: every slot that is not FREE has exactly one entry, at or after
@@ -330,6 +355,7 @@ int64_t find_slot(kvx_tier* t, uint64_t key) {
   const int64_t i = index_pos(t, key);
   if (i < 0) return -1;
   const int64_t s = t->index[i];
+  promote_published(t->meta[s]);
   return t->meta[s].state != kFree ? s : -1;
 }
 
@@ -337,8 +363,9 @@ int64_t find_slot(kvx_tier* t, uint64_t key) {
 int64_t pick_slot(kvx_tier* t) {
   int64_t best = -1;
   for (int64_t i = 0; i < t->hdr->n_slots; ++i) {
-    const SlotMeta& m = t->meta[i];
+    SlotMeta& m = t->meta[i];
     if (m.state == kFree) return i;
+    promote_published(m);
     if (m.state != kReady || m.pins > 0) continue;
     if (best < 0 || m.tick < t->meta[best].tick) best = i;
   }
@@ -375,6 +402,7 @@ int64_t reclaim_locked(kvx_tier* t) {
     SlotMeta& m = t->meta[i];
     if (m.state == kFree) continue;
     bool c = false;
+    promote_published(m);  // a published commit is complete, whoever made it
     if ((m.state == kWriting || m.state == kCommitting) && is_gone(m.writer_pid)) {
       index_erase(t, m.key);
       m.state = kFree;
@@ -406,7 +434,7 @@ void destroy_tier(kvx_tier* t) {
     cudaGetLastError();
   }
   if (t->registered) {
-    cudaHostUnregister(t->data);
+    cudaHostUnregister(t->mapping);
     cudaGetLastError();
   }
   if (t->shared) {
@@ -595,8 +623,8 @@ kvx_status kv_tier_open_shared(const char* name, int64_t slot_bytes, int64_t n_s
   // zero-copy, the default mode, is the one to use.)
   madvise(t->data, (size_t)(h->slot_bytes * h->n_slots), MADV_NOHUGEPAGE);
   if (!(flags & KVX_TIER_NO_PIN)) {
-    const cudaError_t e = cudaHostRegister(t->data, (size_t)(h->slot_bytes * h->n_slots),
-                                           cudaHostRegisterPortable | cudaHostRegisterMapped);
+    // The whole region, slot table included: the GPU publishes commits into it.
+    const cudaError_t e = cudaHostRegister(map, (size_t)total, cudaHostRegisterPortable | cudaHostRegisterMapped);
     if (e != cudaSuccess) {
       kvx_status st = cuda_fail(e, "cudaHostRegister of the shared tier");
       t->creator = create;
@@ -604,6 +632,10 @@ kvx_status kv_tier_open_shared(const char* name, int64_t slot_bytes, int64_t n_s
       return st;
     }
     t->registered = true;
+    void* dmap = nullptr;
+    if (cudaHostGetDevicePointer(&dmap, map, 0) == cudaSuccess && dmap && prepare_tier_kernels() == cudaSuccess)
+      t->meta_dev = (uint8_t*)dmap + ((uint8_t*)t->meta - (uint8_t*)map);
+    cudaGetLastError();  // without publication, commits turn READY through the writer's events only
   }
   *out = t;
   return KVX_OK;
@@ -683,6 +715,15 @@ kvx_status kv_tier_commit(kvx_tier* t, uint64_t key, kvx_stream_t stream) {
   if (no_stream(stream)) {
     m.state = kReady;
   } else {
+    // The sequence number is this commit's alone; a publication that lands
+    // after a failure below matches no commit.
+    const uint64_t seq = ++t->hdr->seq;
+    if (t->meta_dev) {
+      uint64_t* flag = (uint64_t*)(t->meta_dev + i * (int64_t)sizeof(SlotMeta) + offsetof(SlotMeta, published));
+      const cudaError_t r = fault_point("launch") ? cudaErrorUnknown
+                                                  : launch_tier_publish(flag, seq, (cudaStream_t)stream);
+      if (r != cudaSuccess) return cuda_fail(r, "publication kernel launch (tier commit)");
+    }
     cudaEvent_t e = take_event(t);
     if (!e) return cuda_fail(cudaErrorMemoryAllocation, "cudaEventCreate (tier commit)");
     const cudaError_t r = cudaEventRecord(e, (cudaStream_t)stream);
@@ -690,8 +731,9 @@ kvx_status kv_tier_commit(kvx_tier* t, uint64_t key, kvx_stream_t stream) {
       t->spare.push_back(e);
       return cuda_fail(r, "cudaEventRecord (tier commit)");
     }
+    m.commit_seq = seq;
     m.state = kCommitting;
-    t->commits.push_back({i, e});
+    t->commits.push_back({i, e, seq});
     t->commit_event[i] = e;
   }
   add_pins(m, t->pid, -1);
@@ -763,7 +805,7 @@ kvx_status kv_tier_release(kvx_tier* t, uint64_t key, kvx_stream_t stream) {
     t->spare.push_back(e);
     return cuda_fail(r, "cudaEventRecord (tier release)");
   }
-  t->releases.push_back({i, e});  // the pin stays until the queued work completes
+  t->releases.push_back({i, e, 0});  // the pin stays until the queued work completes
   t->queued[i]++;
   return KVX_OK;
 }

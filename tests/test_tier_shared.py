@@ -6,10 +6,13 @@ committed by one process are found, read and pinned by the other; LRU and
 pinning hold across processes.
 
 GPU test: process A stores chunks of a pool into the shared pool on its
-stream, behind a ~10^8-cycle delayed producer; process B must not see them
-before A has observed its GPU work complete, then restores them into its own
-pool on the same GPU and checks every byte against the oracle.  The
-processes synchronise on the host only (no kernel waits on another process).
+stream, behind a producer delayed by ~2*10^9 GPU cycles, and commits them on
+that stream.  Process B must not see them while A's GPU work is pending,
+must see them once the GPU has published the commits although A makes no
+further call, and then restores them into its own pool on the same GPU and
+checks every byte against the oracle (so the publication came after the
+bytes).  The processes synchronise on the host only (no kernel waits on
+another process).
 """
 import multiprocessing as mp
 import os
@@ -236,11 +239,8 @@ def _child_gpu(name, q_in, q_out):
     from paper_2609_15021_gb300 import synth
     spec = oracle.PoolSpec(4, 64, 16, 8, 128, 2, oracle.HND)
     C, n_used = 256, 32
+    import time
     t = k.KvTier(shared_name=name)
-    keys = q_in.get()
-    q_out.put(t.prefix_hits(keys))                 # A's GPU work is still delayed: nothing visible
-    assert q_in.get() == "committed"
-    q_out.put(t.prefix_hits(keys))
     final_np = host_layers(spec, 2)
     ta = synth.permuted_table(64, n_used, 3)
     tb = synth.permuted_table(64, n_used, 4)
@@ -248,6 +248,15 @@ def _child_gpu(name, q_in, q_out):
     ctx = k.kv_ctx_create(0)
     s = torch.cuda.Stream()
     tb_d = torch.from_numpy(tb).cuda()
+    torch.cuda.synchronize()
+    q_out.put("ready")                             # every slow set-up step is done
+    keys = q_in.get()
+    q_out.put(t.prefix_hits(keys))                 # A's GPU work is still delayed: nothing visible
+    t0, hits = time.monotonic(), 0
+    while hits < len(keys) and time.monotonic() - t0 < 120:
+        hits = t.prefix_hits(keys)                 # A makes no call meanwhile: the GPU publishes
+        time.sleep(0.001)
+    q_out.put(hits)
     for c, key in enumerate(keys):
         slot = t.acquire(key, stream=s)
         k.kv_load(ctx, dst, tb_d, c * C, (c + 1) * C, C, [slot], stream=s)
@@ -291,19 +300,20 @@ def test_shared_tier_store_in_one_process_restore_in_another():
         keys = k.kv_chunk_keys(synth.rng(11).integers(0, 150000, size=T).astype(np.int32), C, salt=1)
         s = torch.cuda.Stream()
         torch.cuda.synchronize()
-        for l in range(4):   # the producer finishes writing the KV ~10^8 cycles later
-            k.kvx_probe_delayed_copy(pool.layers[l], final_dev[l], spec.layer_bytes, 10 ** 8 if l == 0 else 0, s)
+        assert q_out.get(timeout=300) == "ready"  # the other process waits for the keys from here on
+        for l in range(4):   # the producer finishes writing the KV ~2*10^9 cycles (~1 s) later
+            k.kvx_probe_delayed_copy(pool.layers[l], final_dev[l], spec.layer_bytes, 2 * 10 ** 9 if l == 0 else 0, s)
         for c, key in enumerate(keys):
             slot = tier.reserve(key)
             k.kv_store(ctx, pool, ta_d, c * C, (c + 1) * C, C, [slot], stream=s)
             tier.commit(key, stream=s)
         q_in.put(keys)
         assert q_out.get(timeout=120) == 0      # still in flight on our stream: invisible elsewhere
-        s.synchronize()
-        tier.poll()                             # we observed completion: entries become READY
-        q_in.put("committed")
-        assert q_out.get(timeout=120) == len(keys)
+        # no tier call and no synchronisation here until the other process has seen every entry
+        assert q_out.get(timeout=180) == len(keys)
         assert q_out.get(timeout=300) is True   # the other process restored every byte
+        s.synchronize()
+        tier.poll()
         p.join(timeout=120)
         assert p.exitcode == 0
     finally:
