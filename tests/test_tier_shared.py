@@ -321,3 +321,89 @@ def test_shared_tier_store_in_one_process_restore_in_another():
             p.kill()
         k.kv_ctx_destroy(ctx)
         tier.close()
+
+
+def _child_commits_then_dies(name, q_out):
+    sys.path.insert(0, ROOT)
+    sys.path.insert(0, os.path.join(ROOT, "tests"))
+    import torch
+
+    import oracle
+    from gpu_util import device_pool, host_layers
+    from paper_2609_15021_gb300 import kvxfer as k
+    from paper_2609_15021_gb300 import synth
+    spec = oracle.PoolSpec(4, 64, 16, 8, 128, 2, oracle.HND)
+    C, n_used = 256, 32
+    t = k.KvTier(shared_name=name)
+    pool = device_pool(spec, host_layers(spec, 21))
+    ta_d = torch.from_numpy(synth.permuted_table(64, n_used, 22)).cuda()
+    ctx = k.kv_ctx_create(0)
+    s = torch.cuda.Stream()
+    t.reserve(503)                   # a reservation left unfinished
+    scratch = torch.empty(4096, dtype=torch.uint8, device="cuda")
+    torch.cuda.synchronize()
+    k.kvx_probe_delayed_fill(scratch, 4096, 0, 4 * 10 ** 8, s)   # the stores start ~0.2 s from now
+    for c, key in enumerate([501, 502]):
+        slot = t.reserve(key)
+        k.kv_store(ctx, pool, ta_d, c * C, (c + 1) * C, C, [slot], stream=s)
+        t.commit(key, stream=s)      # every tier call of this process comes before the GPU work ends
+    s.synchronize()                  # the GPU has published both commits; no tier call after this
+    q_out.put("done")
+    q_out.close()
+    q_out.join_thread()
+    os._exit(0)
+
+
+@pytest.mark.gpu
+def test_published_entries_of_a_dead_writer_stay_readable():
+    """Failure detection: a replica that committed chunks on its stream and died
+    after its GPU work finished, with no tier call in between, leaves those
+    entries complete and readable (the GPU published them); reclaim frees only
+    the reservation it never finished.  The bytes restored in this process
+    match the oracle."""
+    sys.path.insert(0, ROOT)
+    sys.path.insert(0, os.path.join(ROOT, "tests"))
+    import torch
+
+    import oracle
+    from gpu_util import POISON, device_pool, first_mismatch, host_layers, np_of, oracle_load, oracle_store
+    from paper_2609_15021_gb300 import kvxfer as k
+    from paper_2609_15021_gb300 import synth
+    spec = oracle.PoolSpec(4, 64, 16, 8, 128, 2, oracle.HND)
+    C, n_used = 256, 32
+    orc = oracle.c_oracle()
+    name = _name("pubdead")
+    tier = k.KvTier(orc.chunk_bytes(spec, C), 4, shared_name=name, create=True)
+    try:
+        ctx_mp = mp.get_context("spawn")
+        q_out = ctx_mp.Queue()
+        p = ctx_mp.Process(target=_child_commits_then_dies, args=(name, q_out))
+        p.start()
+        assert q_out.get(timeout=300) == "done"
+        p.join(timeout=120)
+        assert p.exitcode == 0
+        assert tier.prefix_hits([501, 502]) == 2
+        assert tier.reclaim() == 1                           # the unfinished reservation only
+        assert tier.prefix_hits([501, 502, 503]) == 2
+        dst = device_pool(spec)
+        tb = synth.permuted_table(64, n_used, 23)
+        tb_d = torch.from_numpy(tb).cuda()
+        ctx = k.kv_ctx_create(0)
+        s = torch.cuda.Stream()
+        try:
+            for c, key in enumerate([501, 502]):
+                slot = tier.acquire(key, stream=s)
+                k.kv_load(ctx, dst, tb_d, c * C, (c + 1) * C, C, [slot], stream=s)
+                tier.release(key, stream=s)
+            s.synchronize()
+            assert k.kv_get_device_error(ctx) == -1
+        finally:
+            k.kv_ctx_destroy(ctx)
+        ta = synth.permuted_table(64, n_used, 22)
+        want, _ = oracle_store(orc, spec, host_layers(spec, 21), ta, 0, n_used * 16, C)
+        loaded, _ = oracle_load(orc, spec, [np.full(spec.layer_bytes, POISON, np.uint8)] * 4, tb, 0,
+                                n_used * 16, C, want)
+        for l in range(4):
+            assert first_mismatch(np_of(dst.layers[l]), loaded[l]) is None, f"layer {l}"
+    finally:
+        tier.close()
