@@ -457,8 +457,15 @@ void kv_tier_destroy(kvx_tier* tier);
    slot is pinned or busy; KVX_EBUSY if `key` itself is. */
 kvx_status kv_tier_reserve(kvx_tier* tier, uint64_t key, void** slot);
 /* Marks a reserved entry readable once the work already enqueued on
-   `stream` (the store into it) completes; unpins it. */
+   `stream` (the store into it) completes; unpins it.  On a shared tier the
+   commit enqueues its publication (see kv_tier_open_shared): a one-thread
+   kernel launch per call. */
 kvx_status kv_tier_commit(kvx_tier* tier, uint64_t key, kvx_stream_t stream);
+/* kv_tier_commit of n keys on one stream at once: one publication launch per
+   512 keys and one event for all of them (a 128k-token context is 512 chunks).
+   Every key must be reserved by this process and listed once; otherwise
+   KVX_ENOENT / KVX_EINVAL and nothing is committed. */
+kvx_status kv_tier_commit_many(kvx_tier* tier, const uint64_t* keys, int64_t n, kvx_stream_t stream);
 /* Slot of a committed entry; `stream` is made to wait for its commit event.
    Pins it until kv_tier_release.  KVX_ENOENT if absent or not committed. */
 kvx_status kv_tier_acquire(kvx_tier* tier, uint64_t key, kvx_stream_t stream, void** slot);

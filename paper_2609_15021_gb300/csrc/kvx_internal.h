@@ -103,9 +103,19 @@ cudaError_t launch_move_tmap(int dir, const MoveParams& p, const void* maps, int
                              int stage_bytes, int stages, int* timeout, cudaStream_t s);
 int move_ctas_per_sm(int dir, int layout);
 int segment_ctas_per_sm();
-// Shared tier (tier_kernels.cu): enqueues on s a system-scope release store of
-// seq to dev_flag (a device address of mapped host memory).
-cudaError_t launch_tier_publish(uint64_t* dev_flag, uint64_t seq, cudaStream_t s);
+// Shared tier (tier_kernels.cu): publication of up to kMaxPublish commits in
+// one launch.  Thread j makes a system-scope release store of seq0 + j to the
+// 8-byte flag at meta + slot[j] * stride + offset (meta: the device address of
+// the mapped slot table).
+constexpr int kMaxPublish = 512;
+struct TierPublish {
+  uint8_t* meta;
+  int64_t stride, offset;
+  uint64_t seq0;
+  int32_t n;
+  int32_t slot[kMaxPublish];
+};
+cudaError_t launch_tier_publish(const TierPublish& b, cudaStream_t s);
 // Loads the publication kernel (at tier open, never inside a commit).
 cudaError_t prepare_tier_kernels();
 

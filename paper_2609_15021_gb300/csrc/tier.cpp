@@ -45,6 +45,7 @@
 #include <time.h>
 #include <unistd.h>
 
+#include <algorithm>
 #include <deque>
 #include <mutex>
 #include <new>
@@ -141,7 +142,8 @@ kvx_status cuda_fail(cudaError_t e, const char* what) {
 struct PendingEvent {
   int64_t slot;
   cudaEvent_t ev;
-  uint64_t seq;  // commits: the commit's sequence number
+  uint64_t seq;   // commits: the commit's sequence number
+  bool owns_ev;   // the event goes back to the spares with this entry (the last of its batch)
 };
 
 }  // namespace
@@ -233,7 +235,7 @@ void settle_commit(kvx_tier* t, const PendingEvent& p) {
   if (m.state == kCommitting && m.writer_pid == t->pid && m.commit_seq == p.seq) m.state = kReady;
   auto it = t->commit_event.find(p.slot);
   if (it != t->commit_event.end() && it->second == p.ev) t->commit_event.erase(it);
-  t->spare.push_back(p.ev);
+  if (p.owns_ev) t->spare.push_back(p.ev);
 }
 
 void settle_release(kvx_tier* t, const PendingEvent& p) {
@@ -244,11 +246,18 @@ void settle_release(kvx_tier* t, const PendingEvent& p) {
 }
 
 void poll_locked(kvx_tier* t, PollMode mode) {
+  // The entries of one batch share an event and sit next to each other: the
+  // event is asked once for all of them, so they settle together and the
+  // last one returns the event only when the others are done with it.
+  cudaEvent_t last = nullptr;
+  bool last_done = false;
   auto done = [&](cudaEvent_t e) {
+    if (e == last) return last_done;
     const cudaError_t q = mode == kWait ? cudaEventSynchronize(e) : cudaEventQuery(e);
-    if (q == cudaErrorNotReady) return false;
-    cudaGetLastError();
-    return true;
+    last = e;
+    last_done = q != cudaErrorNotReady;
+    if (last_done) cudaGetLastError();
+    return last_done;
   };
   auto settle = [&](std::deque<PendingEvent>& q, void (*fn)(kvx_tier*, const PendingEvent&)) {
     if (mode == kFront) {
@@ -705,39 +714,71 @@ kvx_status kv_tier_reserve(kvx_tier* t, uint64_t key, void** slot) {
 }
 
 kvx_status kv_tier_commit(kvx_tier* t, uint64_t key, kvx_stream_t stream) {
-  if (!t) return KVX_EINVAL;
+  return kv_tier_commit_many(t, &key, 1, stream);
+}
+
+kvx_status kv_tier_commit_many(kvx_tier* t, const uint64_t* keys, int64_t n, kvx_stream_t stream) {
+  if (!t || n < 0 || (n > 0 && !keys)) return KVX_EINVAL;
+  if (n == 0) return KVX_OK;
   TierLock lock(t);
   poll_locked(t, kFront);
-  const int64_t i = find_slot(t, key);
-  if (i < 0) return KVX_ENOENT;
-  SlotMeta& m = t->meta[i];
-  if (m.state != kWriting || m.writer_pid != t->pid) return KVX_EINVAL;
+  std::vector<int64_t> slots((size_t)n);
+  std::unordered_map<int64_t, bool> seen;
+  for (int64_t j = 0; j < n; ++j) {  // every key first: on an error nothing is committed
+    const int64_t i = find_slot(t, keys[j]);
+    if (i < 0) return KVX_ENOENT;
+    const SlotMeta& m = t->meta[i];
+    if (m.state != kWriting || m.writer_pid != t->pid) return KVX_EINVAL;
+    if (!seen.emplace(i, true).second) {
+      set_error_text("a key is listed twice");
+      return KVX_EINVAL;
+    }
+    slots[(size_t)j] = i;
+  }
   if (no_stream(stream)) {
-    m.state = kReady;
-  } else {
-    // The sequence number is this commit's alone; a publication that lands
-    // after a failure below matches no commit.
-    const uint64_t seq = ++t->hdr->seq;
-    if (t->meta_dev) {
-      uint64_t* flag = (uint64_t*)(t->meta_dev + i * (int64_t)sizeof(SlotMeta) + offsetof(SlotMeta, published));
-      const cudaError_t r = fault_point("launch") ? cudaErrorUnknown
-                                                  : launch_tier_publish(flag, seq, (cudaStream_t)stream);
+    for (int64_t i : slots) {
+      SlotMeta& m = t->meta[i];
+      m.state = kReady;
+      add_pins(m, t->pid, -1);
+      m.tick = ++t->hdr->clock;
+    }
+    return KVX_OK;
+  }
+  // The sequence numbers are these commits' alone; a publication that lands
+  // after a failure below matches no commit.
+  const uint64_t seq0 = t->hdr->seq + 1;
+  t->hdr->seq += (uint64_t)n;
+  if (t->meta_dev) {
+    TierPublish b;
+    b.meta = t->meta_dev;
+    b.stride = (int64_t)sizeof(SlotMeta);
+    b.offset = (int64_t)offsetof(SlotMeta, published);
+    for (int64_t j0 = 0; j0 < n; j0 += kMaxPublish) {
+      b.n = (int32_t)std::min<int64_t>(kMaxPublish, n - j0);
+      b.seq0 = seq0 + (uint64_t)j0;
+      for (int32_t j = 0; j < b.n; ++j) b.slot[j] = (int32_t)slots[(size_t)(j0 + j)];
+      const cudaError_t r = fault_point("launch") ? cudaErrorUnknown : launch_tier_publish(b, (cudaStream_t)stream);
       if (r != cudaSuccess) return cuda_fail(r, "publication kernel launch (tier commit)");
     }
-    cudaEvent_t e = take_event(t);
-    if (!e) return cuda_fail(cudaErrorMemoryAllocation, "cudaEventCreate (tier commit)");
-    const cudaError_t r = cudaEventRecord(e, (cudaStream_t)stream);
-    if (r != cudaSuccess) {
-      t->spare.push_back(e);
-      return cuda_fail(r, "cudaEventRecord (tier commit)");
-    }
-    m.commit_seq = seq;
-    m.state = kCommitting;
-    t->commits.push_back({i, e, seq});
-    t->commit_event[i] = e;
   }
-  add_pins(m, t->pid, -1);
-  m.tick = ++t->hdr->clock;
+  cudaEvent_t e = take_event(t);
+  if (!e) return cuda_fail(cudaErrorMemoryAllocation, "cudaEventCreate (tier commit)");
+  const cudaError_t r = cudaEventRecord(e, (cudaStream_t)stream);
+  if (r != cudaSuccess) {
+    t->spare.push_back(e);
+    return cuda_fail(r, "cudaEventRecord (tier commit)");
+  }
+  for (int64_t j = 0; j < n; ++j) {
+    const int64_t i = slots[(size_t)j];
+    SlotMeta& m = t->meta[i];
+    m.commit_seq = seq0 + (uint64_t)j;
+    m.state = kCommitting;
+    // one event for the batch: the last entry gives it back
+    t->commits.push_back({i, e, m.commit_seq, j == n - 1});
+    t->commit_event[i] = e;
+    add_pins(m, t->pid, -1);
+    m.tick = ++t->hdr->clock;
+  }
   return KVX_OK;
 }
 
@@ -805,7 +846,7 @@ kvx_status kv_tier_release(kvx_tier* t, uint64_t key, kvx_stream_t stream) {
     t->spare.push_back(e);
     return cuda_fail(r, "cudaEventRecord (tier release)");
   }
-  t->releases.push_back({i, e, 0});  // the pin stays until the queued work completes
+  t->releases.push_back({i, e, 0, true});  // the pin stays until the queued work completes
   t->queued[i]++;
   return KVX_OK;
 }

@@ -16,7 +16,13 @@
 namespace kvx {
 namespace {
 
-__global__ void tier_publish_kernel(unsigned long long* flag, unsigned long long seq) {
+// Thread j publishes commit seq0 + j of slot slot[j]: its flag lies at
+// meta + slot[j] * stride + offset.
+__global__ void tier_publish_kernel(TierPublish b) {
+  const int j = threadIdx.x;
+  if (j >= b.n) return;
+  unsigned long long* flag = reinterpret_cast<unsigned long long*>(b.meta + (int64_t)b.slot[j] * b.stride + b.offset);
+  const unsigned long long seq = b.seq0 + (unsigned long long)j;
   asm volatile("st.release.sys.global.u64 [%0], %1;" ::"l"(flag), "l"(seq) : "memory");
 }
 
@@ -29,9 +35,9 @@ cudaError_t prepare_tier_kernels() {
   return cudaFuncGetAttributes(&a, tier_publish_kernel);
 }
 
-cudaError_t launch_tier_publish(uint64_t* dev_flag, uint64_t seq, cudaStream_t s) {
-  tier_publish_kernel<<<1, 1, 0, s>>>(reinterpret_cast<unsigned long long*>(dev_flag),
-                                      static_cast<unsigned long long>(seq));
+cudaError_t launch_tier_publish(const TierPublish& b, cudaStream_t s) {
+  if (b.n < 1 || b.n > kMaxPublish) return cudaErrorInvalidValue;
+  tier_publish_kernel<<<1, b.n, 0, s>>>(b);
   return cudaGetLastError();
 }
 

@@ -37,7 +37,7 @@ EXPORTED = (
     "kv_ctx_modes", "kv_last_cuda_error", "kv_last_error_message", "kv_status_string", "kv_abi_version",
     "kvx_probe_delayed_fill", "kvx_probe_delayed_copy", "kvx_probe_copy", "kv_store_noalloc",
     "kv_host_alloc", "kv_host_free", "kv_pool_view_check",
-    "kv_chunk_keys", "kv_tier_create", "kv_tier_create_on", "kv_tier_destroy", "kv_tier_reserve", "kv_tier_commit",
+    "kv_chunk_keys", "kv_tier_create", "kv_tier_create_on", "kv_tier_destroy", "kv_tier_reserve", "kv_tier_commit", "kv_tier_commit_many",
     "kv_tier_acquire", "kv_tier_release", "kv_tier_prefix_hits", "kv_tier_stats", "kv_fault_inject",
     "kv_tier_open_shared", "kv_tier_poll", "kv_tier_reclaim", "kv_host_alloc_numa", "kv_host_alloc_ex",
     "kv_host_pool_info",
@@ -130,6 +130,7 @@ def _declare(lib):
         "kv_tier_destroy": (None, [vp]),
         "kv_tier_reserve": (st, [vp, ctypes.c_uint64, P(vp)]),
         "kv_tier_commit": (st, [vp, ctypes.c_uint64, vp]),
+        "kv_tier_commit_many": (st, [vp, P(ctypes.c_uint64), i64, vp]),
         "kv_tier_acquire": (st, [vp, ctypes.c_uint64, vp, P(vp)]),
         "kv_tier_release": (st, [vp, ctypes.c_uint64, vp]),
         "kv_tier_prefix_hits": (st, [vp, P(ctypes.c_uint64), i64, P(i64)]),
@@ -576,6 +577,10 @@ class KvTier:
 
     def commit(self, key: int, stream=None):
         _check(_lib.kv_tier_commit(self.handle, key, self._stream(stream)), "kv_tier_commit")
+
+    def commit_many(self, keys, stream=None):
+        arr = (ctypes.c_uint64 * max(1, len(keys)))(*keys)
+        _check(_lib.kv_tier_commit_many(self.handle, arr, len(keys), self._stream(stream)), "kv_tier_commit_many")
 
     def acquire(self, key: int, stream=None):
         out = ctypes.c_void_p()

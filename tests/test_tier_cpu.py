@@ -173,6 +173,22 @@ class _Model:
         s["tick"] = self.clock
         return "OK"
 
+    def commit_many(self, keys):
+        idx = []
+        for key in keys:                      # every key is checked before any is committed
+            i = self.find(key)
+            if i is None:
+                return "ENOENT"
+            if self.slots[i]["state"] != "WRITING" or i in idx:
+                return "EINVAL"
+            idx.append(i)
+        for i in idx:
+            s = self.slots[i]
+            s["state"], s["pins"] = "READY", s["pins"] - 1
+            self.clock += 1
+            s["tick"] = self.clock
+        return "OK"
+
     def acquire(self, key):
         i = self.find(key)
         if i is None or self.slots[i]["state"] != "READY":
@@ -225,7 +241,8 @@ def test_tier_follows_its_rules_under_random_operations(k, seed, n_slots, n_keys
 
     for step in range(4000):
         key = int(rng.integers(1, n_keys + 1)) * 1000003
-        op = rng.choice(["reserve", "commit", "acquire", "release", "prefix"], p=[0.3, 0.25, 0.2, 0.2, 0.05])
+        op = rng.choice(["reserve", "commit", "commit_many", "acquire", "release", "prefix"],
+                        p=[0.3, 0.17, 0.08, 0.2, 0.2, 0.05])
         if op == "reserve":
             got, view = call(tier.reserve, key)
             want, _ = model.reserve(key)
@@ -234,6 +251,10 @@ def test_tier_follows_its_rules_under_random_operations(k, seed, n_slots, n_keys
         elif op == "commit":
             got, _ = call(tier.commit, key, NO)
             want = model.commit(key)
+        elif op == "commit_many":
+            keys = [int(x) * 1000003 for x in rng.integers(1, n_keys + 1, size=int(rng.integers(0, 4)))]
+            got, _ = call(tier.commit_many, keys, NO)
+            want = model.commit_many(keys)
         elif op == "acquire":
             got, view = call(tier.acquire, key, NO)
             want = model.acquire(key)

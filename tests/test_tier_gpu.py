@@ -18,7 +18,10 @@ pytestmark = pytest.mark.gpu
 DELAY = 10 ** 8
 
 
-def test_store_then_restore_across_streams_through_the_tier(orc):
+@pytest.mark.parametrize("commit", ["per_key", "many"])
+def test_store_then_restore_across_streams_through_the_tier(orc, commit):
+    """commit="many": one kv_store of every chunk into its slot and one
+    kv_tier_commit_many, whose entries share one event."""
     k = kvx()
     spec = oracle.PoolSpec(4, 64, 16, 8, 128, 2, oracle.HND)
     C, n_used = 256, 48
@@ -42,10 +45,15 @@ def test_store_then_restore_across_streams_through_the_tier(orc):
         for l in range(spec.num_layers):
             k.kvx_probe_delayed_copy(pool_a.layers[l], final_dev[l], spec.layer_bytes, DELAY if l == 0 else 0, s_a)
         ta_d = torch.from_numpy(ta).cuda()
-        for c, key in enumerate(keys):
-            slot = tier.reserve(key)
-            k.kv_store(ctx, pool_a, ta_d, c * C, (c + 1) * C, C, [slot], stream=s_a)
-            tier.commit(key, stream=s_a)
+        if commit == "many":
+            slots = [tier.reserve(key) for key in keys]
+            k.kv_store(ctx, pool_a, ta_d, 0, T, C, slots, stream=s_a)
+            tier.commit_many(keys, stream=s_a)
+        else:
+            for c, key in enumerate(keys):
+                slot = tier.reserve(key)
+                k.kv_store(ctx, pool_a, ta_d, c * C, (c + 1) * C, C, [slot], stream=s_a)
+                tier.commit(key, stream=s_a)
         # replica B, its own stream, no host synchronisation: ordered by the commit events
         assert tier.prefix_hits(keys) == len(keys)
         tb_d = torch.from_numpy(tb).cuda()
@@ -64,6 +72,9 @@ def test_store_then_restore_across_streams_through_the_tier(orc):
             slot = tier.acquire(key, stream=k.KVX_NO_STREAM)
             assert first_mismatch(np_of(slot), want[c]) is None, c
             tier.release(key, stream=k.KVX_NO_STREAM)
+        tier.poll()
+        st = tier.stats()
+        assert st["pinned"] == 0 and st["entries"] == len(keys)
     finally:
         k.kv_ctx_destroy(ctx)
         tier.close()

@@ -272,7 +272,8 @@ def _child_gpu(name, q_in, q_out):
 
 
 @pytest.mark.gpu
-def test_shared_tier_store_in_one_process_restore_in_another():
+@pytest.mark.parametrize("commit", ["per_key", "many"])
+def test_shared_tier_store_in_one_process_restore_in_another(commit):
     sys.path.insert(0, ROOT)
     sys.path.insert(0, os.path.join(ROOT, "tests"))
     import torch
@@ -285,7 +286,7 @@ def test_shared_tier_store_in_one_process_restore_in_another():
     C, n_used = 256, 32
     T = n_used * 16
     orc = oracle.c_oracle()
-    name = _name("gpu")
+    name = _name(f"gpu{commit}")
     tier = k.KvTier(orc.chunk_bytes(spec, C), 4, shared_name=name, create=True)
     ctx_mp = mp.get_context("spawn")
     q_in, q_out = ctx_mp.Queue(), ctx_mp.Queue()
@@ -303,10 +304,15 @@ def test_shared_tier_store_in_one_process_restore_in_another():
         assert q_out.get(timeout=300) == "ready"  # the other process waits for the keys from here on
         for l in range(4):   # the producer finishes writing the KV ~2*10^9 cycles (~1 s) later
             k.kvx_probe_delayed_copy(pool.layers[l], final_dev[l], spec.layer_bytes, 2 * 10 ** 9 if l == 0 else 0, s)
-        for c, key in enumerate(keys):
-            slot = tier.reserve(key)
-            k.kv_store(ctx, pool, ta_d, c * C, (c + 1) * C, C, [slot], stream=s)
-            tier.commit(key, stream=s)
+        if commit == "many":                    # one store, one publication launch for both chunks
+            slots = [tier.reserve(key) for key in keys]
+            k.kv_store(ctx, pool, ta_d, 0, T, C, slots, stream=s)
+            tier.commit_many(keys, stream=s)
+        else:
+            for c, key in enumerate(keys):
+                slot = tier.reserve(key)
+                k.kv_store(ctx, pool, ta_d, c * C, (c + 1) * C, C, [slot], stream=s)
+                tier.commit(key, stream=s)
         q_in.put(keys)
         assert q_out.get(timeout=120) == 0      # still in flight on our stream: invisible elsewhere
         # no tier call and no synchronisation here until the other process has seen every entry
