@@ -204,9 +204,11 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-hbm-roofline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--host-alloc", choices=["plain", "numa", "driver"], default="plain",
-                    help="pinned pool from kv_host_alloc, from kv_host_alloc_numa on the host NUMA "
-                         "node nearest the GPU, or from the driver's allocator (KVX_HOST_DRIVER)")
+    ap.add_argument("--host-alloc", choices=["auto", "plain", "numa", "driver", "huge"], default="auto",
+                    help="pinned pool from kv_host_alloc (plain: the driver's allocator), from "
+                         "kv_host_alloc_numa on the host NUMA node nearest the GPU, from the driver's allocator "
+                         "stated (KVX_HOST_DRIVER), or on huge pages (KVX_HOST_HUGE); auto: huge for "
+                         "--mode staged (the copy engines want huge pages), else plain")
     ap.add_argument("--no-tier", action="store_true",
                     help="skip the leg that stores and restores chunk by chunk through the host tier")
     ap.add_argument("--no-concurrent", action="store_true",
@@ -325,11 +327,18 @@ def run_reference(args):
 # ------------------------------------------------------------------ GPU leg
 
 
-def host_link_peak(torch, dev):
-    """Best-of-5 pinned cudaMemcpyAsync of 1 GiB per direction, GB/s."""
+def link_buffers(torch, dev):
+    """The pinned and device buffers of host_link_peak, allocated once per run."""
     n = 1 << 30
-    h = torch.empty(n, dtype=torch.uint8).pin_memory()
-    d = torch.empty(n, dtype=torch.uint8, device=dev)
+    return {"h": torch.empty(n, dtype=torch.uint8, pin_memory=True), "d": torch.empty(n, dtype=torch.uint8, device=dev),
+            "h2": torch.empty(n, dtype=torch.uint8, pin_memory=True),
+            "d2": torch.empty(n, dtype=torch.uint8, device=dev)}
+
+
+def host_link_peak(torch, dev, bufs):
+    """Best-of-5 pinned cudaMemcpyAsync of 1 GiB per direction, GB/s."""
+    h, d, h2, d2 = bufs["h"], bufs["d"], bufs["h2"], bufs["d2"]
+    n = h.numel()
     out = {}
     for name, dst, src in (("d2h", h, d), ("h2d", d, h)):
         best = None
@@ -344,8 +353,6 @@ def host_link_peak(torch, dev):
                 best = ms if best is None else min(best, ms)
         out[name] = n / (best * 1e-3) / GB
     # both directions at once, one copy per stream (two replicas sharing the link)
-    h2 = torch.empty(n, dtype=torch.uint8).pin_memory()
-    d2 = torch.empty(n, dtype=torch.uint8, device=dev)
     s1, s2 = torch.cuda.Stream(device=dev), torch.cuda.Stream(device=dev)
     best = None
     for i in range(7):
@@ -364,7 +371,6 @@ def host_link_peak(torch, dev):
             ms = max(a.elapsed_time(b1), a.elapsed_time(b2))
             best = ms if best is None else min(best, ms)
     out["bidir"] = 2 * n / (best * 1e-3) / GB
-    del h, d, h2, d2
     return out
 
 
@@ -413,7 +419,12 @@ def run_ours(args):
     n_chunks = -(-T // C)
     cb = L * 2 * C * H * D * e
 
-    link = host_link_peak(torch, dev)
+    # Every host buffer of the run is pinned up front, before the warm-up: on
+    # GB300, pinning or freeing host memory while (or just before) zero-copy
+    # kernels ran stalled them for up to a second, and such stalls inside a
+    # measured leg would come from this harness, not from the transfer.
+    link_bufs = link_buffers(torch, dev)
+    link = host_link_peak(torch, dev, link_bufs)
 
     src_layers = [synth.normal_bf16_(torch.empty(layer_bytes, dtype=torch.uint8, device=dev), synth.SEED + l)
                   for l in range(L)]
@@ -424,12 +435,23 @@ def run_ours(args):
     tb_np = synth.permuted_table(N, T // B, seed=2 + 1000 * rank)
     ta = torch.from_numpy(ta_np).to(dev)
     tb = torch.from_numpy(tb_np).to(dev)
+    avail = host_mem_available()
     t_pin = time.perf_counter()
     # exact-size pinned, mapped pool (no power-of-two rounding)
-    host_pool = k.HostBuffer(n_chunks * cb, numa_node=k.KVX_NUMA_NEAREST if args.host_alloc == "numa" else None,
-                             driver=args.host_alloc == "driver")
+    host_alloc = args.host_alloc if args.host_alloc != "auto" else "huge" if args.mode == "staged" else "plain"
+    host_pool = k.HostBuffer(n_chunks * cb, numa_node=k.KVX_NUMA_NEAREST if host_alloc == "numa" else None,
+                             driver=host_alloc == "driver", huge=host_alloc == "huge")
     pin_seconds = time.perf_counter() - t_pin
     chunks = [host_pool.tensor[i * cb:(i + 1) * cb] for i in range(n_chunks)]
+    # the pinned memory of the later legs: a second chunk set (two replicas at
+    # once) and the e2e leg's pinned block tables.  The shared tier's pool is
+    # made once the second chunk set is freed: three 33 GB pools pinned at once
+    # left the two-replica leg at half its speed.
+    want_conc = not args.no_concurrent and world == 1 and avail > 2 * n_chunks * cb + (32 << 30)
+    want_tier = not args.no_tier and world == 1 and avail > 2 * n_chunks * cb + (32 << 30)
+    host_pool2 = k.HostBuffer(n_chunks * cb, huge=host_alloc == "huge") if want_conc else None
+    ta_host = torch.from_numpy(ta_np).pin_memory()
+    tb_host = torch.from_numpy(tb_np).pin_memory()
 
     mode = {"auto": k.KVX_MODE_AUTO, "staged": k.KVX_MODE_STAGED, "zerocopy": k.KVX_MODE_ZEROCOPY}[args.mode]
     ctx = k.kv_ctx_create(local, store_mode=mode, load_mode=mode, staging_slot_bytes=args.slot_mib << 20,
@@ -464,7 +486,7 @@ def run_ours(args):
     clock_info = clocks.summary()
     # the link peak again right after the timed steps: a drop shows traffic from
     # outside this process (the host memory is shared) during the measurement
-    link_after = host_link_peak(torch, dev)
+    link_after = host_link_peak(torch, dev, link_bufs)
     total_ms = ev[0][0].elapsed_time(ev[-1][2])
     store_ms = [e_[0].elapsed_time(e_[1]) for e_ in ev]
     restore_ms = [e_[1].elapsed_time(e_[2]) for e_ in ev]
@@ -476,8 +498,6 @@ def run_ours(args):
     # end to end through the public API on the host clock
     e2e = None
     if not args.no_e2e:
-        ta_host = torch.from_numpy(ta_np).pin_memory()
-        tb_host = torch.from_numpy(tb_np).pin_memory()
         torch.cuda.synchronize()
         barrier(world)
         t0 = time.perf_counter()
@@ -604,8 +624,7 @@ def run_ours(args):
     # the context into a second chunk set while replica B restores the chunks the
     # timed steps wrote.  The host link then carries both directions.
     concurrent = None
-    if not args.no_concurrent and world == 1 and host_mem_available() > n_chunks * cb + (32 << 30):
-        host_pool2 = k.HostBuffer(n_chunks * cb)
+    if host_pool2 is not None:
         pool2 = host_pool2.info()
         chunks2 = [host_pool2.tensor[i * cb:(i + 1) * cb] for i in range(n_chunks)]
         ctx_b = k.kv_ctx_create(local, store_mode=mode, load_mode=mode, staging_slot_bytes=args.slot_mib << 20)
@@ -644,12 +663,12 @@ def run_ours(args):
 
     # The tier path: the same store and restore through a host tier shared across
     # processes (POSIX shared memory, the paper's replicas sharing one pool), as a
-    # replica uses it: reserve a slot per chunk key, one kv_store into those slots,
+    # replica uses it: reserve a slot per chunk key (one call), one kv_store into those slots,
     # commit the keys on the stream (one publication launch per 512); prefix
-    # lookup; acquire each key on the stream, one kv_load from those slots, release
-    # each key on the stream.  The host never waits for the GPU.
+    # lookup; acquire the keys on the stream, one kv_load from those slots, release
+    # the keys on the stream (one event).  The host never waits for the GPU.
     tier_leg = None
-    if not args.no_tier and world == 1 and host_mem_available() > n_chunks * cb + (32 << 30):
+    if want_tier:
         shm_name = f"/kvx_bench_{os.getpid()}"
         tier = k.KvTier(cb, n_chunks, shared_name=shm_name, create=True)
         try:  # no other process opens it: unlinked now, the memory goes with this process however it ends
@@ -664,15 +683,14 @@ def run_ours(args):
             torch.cuda.synchronize()
             t0 = time.perf_counter()
             a.record(stream)
-            slots = [tier.reserve(key) for key in keys]
+            slots = tier.reserve_many(keys)
             k.kv_store(ctx, src, ta, 0, T, C, slots, stream=stream)
             tier.commit_many(keys, stream=stream)
             b.record(stream)
             hits = tier.prefix_hits(keys)
-            slots = [tier.acquire(key, stream=stream) for key in keys[:hits]]
+            slots = tier.acquire_many(keys[:hits], stream=stream)
             k.kv_load(ctx, dst, tb, 0, T, C, slots, stream=stream)
-            for key in keys[:hits]:
-                tier.release(key, stream=stream)
+            tier.release_many(keys[:hits], stream=stream)
             c.record(stream)
             del slots
             t1 = time.perf_counter()
@@ -695,8 +713,7 @@ def run_ours(args):
                     "host_ms_per_store_and_restore": statistics.median(host_ms),
                     "tier": "shared across processes (POSIX shared memory, base pages, registered pinned "
                             "and mapped)",
-                    "prefix_hits": hits, "chunks": n_chunks, "tier_calls_per_chunk": 3,
-                    "commit_many_calls_per_direction": 1,
+                    "prefix_hits": hits, "chunks": n_chunks, "tier_calls_per_step": 5,
                     "transfer_calls_per_direction": 1,
                     "slots_equal_timed_chunks_on_sample": same, "evictions": tstats["evictions"]}
 
@@ -734,10 +751,10 @@ def run_ours(args):
                    "bytes_per_direction": X, "l2": f"inputs larger than L2 ({X} bytes per direction), no flush",
                    "store_mode": k.MODE_NAMES[store_mode], "load_mode": k.MODE_NAMES[load_mode],
                    "parallelism": f"replicas x{world}", "pinned_host_bytes": n_chunks * cb,
-                   "host_alloc": args.host_alloc if host_pool.numa_node is None
+                   "host_alloc": host_alloc if host_pool.numa_node is None
                    else f"numa node {host_pool.numa_node}",
                    "host_pool": host_pool.info(),
-                   "pin_seconds": pin_seconds},
+                   "pin_seconds": pin_seconds, "host_mem_available_at_start": avail},
         "restore_ms": {"median": statistics.median(restore_ms), "min": min(restore_ms), "max": max(restore_ms),
                        "n": len(restore_ms)},
         "store_ms": {"median": statistics.median(store_ms), "min": min(store_ms), "max": max(store_ms)},

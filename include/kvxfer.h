@@ -315,16 +315,17 @@ kvx_status kv_store_noalloc(const kvx_pool* pool, const int32_t* block_table, in
  * Page-locked host memory for a shared chunk pool (Sec. 3.3: the shared tier
  * is one full-size pinned allocation; the paper's 256 GiB + 4096 B request
  * was rounded up to a power of two by the framework's pinned allocator and
- * silently fell back to pageable memory).  kv_host_alloc returns `bytes` of
- * page-locked memory, portable to every device and mapped for zero-copy.  A
- * pool that whole huge pages fit within an eighth is mapped by the library
- * on transparent huge pages (rounded up to whole huge pages, never to a power
- * of two), which is what lets the copy engines (KVX_MODE_STAGED) reach the
- * link peak on a host with small base pages; other pools, and pools huge
- * pages cannot wholly back, come from the driver's allocator (see
- * kv_host_alloc_ex and kv_host_pool_info).  Failure is KVX_ENOMEM or
- * KVX_ECUDA, never a pageable fallback.  Free with kv_host_free (NULL is
- * ignored).
+ * silently fell back to pageable memory).  kv_host_alloc returns exactly
+ * `bytes` of page-locked memory, portable to every device and mapped for
+ * zero-copy, from the driver's pinned allocator (cudaHostAlloc, asked for
+ * exactly that size).  Measured on GB300 (Grace host): zero-copy transfers,
+ * the default mode, held the link peak from such pools in every benchmark
+ * run, where pools the library mapped on huge pages stalled at times after
+ * other pinning, freeing or forking in the same process.  For copy-engine
+ * transfers (KVX_MODE_STAGED) ask for huge pages (kv_host_alloc_ex with
+ * KVX_HOST_HUGE): the copy engines reach the link peak only from them.
+ * Failure is KVX_ENOMEM or KVX_ECUDA, never a pageable fallback.  Free with
+ * kv_host_free (NULL is ignored).
  */
 kvx_status kv_host_alloc(int64_t bytes, void** out);
 /*
@@ -332,8 +333,9 @@ kvx_status kv_host_alloc(int64_t bytes, void** out);
  * nodes the pool belongs on the node next to the GPU that uses it, or every
  * zero-copy access also crosses the link between sockets.  numa_node >= 0
  * names the node; KVX_NUMA_NEAREST asks for the node CUDA reports as closest
- * to the current device (no placement if it reports none).  The memory gets
- * a preferred-node policy (mbind) before it is faulted in.
+ * to the current device (no placement if it reports none).  The library maps
+ * the pool itself (huge pages where they fit, as KVX_HOST_HUGE, else base
+ * pages) and gives it a preferred-node policy (mbind) before it is faulted in.
  * KVX_EINVAL for a node that does not exist, KVX_ENOMEM if the node has less
  * free memory than `bytes` or the memory cannot be pinned (never a pageable
  * fallback).  *numa_out (may be NULL) receives the node of the first page,
@@ -343,19 +345,27 @@ kvx_status kv_host_alloc(int64_t bytes, void** out);
 kvx_status kv_host_alloc_numa(int32_t numa_node, int64_t bytes, void** out, int32_t* numa_out);
 /*
  * Both of the above, with the choices spelled out.  numa_node: KVX_NUMA_ANY
- * (no placement), KVX_NUMA_NEAREST, or a node.  flags: KVX_HOST_DRIVER takes
- * the memory from the driver's pinned allocator (cudaHostAlloc, portable and
- * mapped) instead of the library's huge-page mapping; numa_node must then be
- * KVX_NUMA_ANY.  Without a placement, a pool that whole huge pages would
- * overshoot by more than an eighth (for 512 MiB pages: anything below 4 GiB
- * that is not a near multiple), or any pool on a host without transparent
- * huge pages, also comes from the driver's allocator.  kv_host_alloc(b, o)
- * is kv_host_alloc_ex(b, KVX_NUMA_ANY, 0, o, NULL).  Memory from either
- * source zero-copies at the link peak; only huge pages let the copy engines
- * (KVX_MODE_STAGED) reach it steadily on a host with small base pages.
+ * (no placement), KVX_NUMA_NEAREST, or a node.  flags:
+ *   KVX_HOST_DRIVER  the driver's pinned allocator (the default without a
+ *                    placement); numa_node must be KVX_NUMA_ANY.
+ *   KVX_HOST_HUGE    the library's own mapping on transparent huge pages,
+ *                    rounded up to whole huge pages (never to a power of
+ *                    two), for copy-engine transfers.  A pool that whole huge
+ *                    pages would overshoot by more than an eighth (for 512 MiB
+ *                    pages: anything below 4 GiB that is not a near multiple),
+ *                    or that huge pages cannot wholly back, or any pool on a
+ *                    host without transparent huge pages, comes from the
+ *                    driver's allocator instead (no placement) or from base
+ *                    pages (placement).  Not with KVX_HOST_DRIVER.
+ * A mapped pool is not inherited by child processes (MADV_DONTFORK): on GB300
+ * a fork of the owning process, even to start a subprocess, otherwise
+ * stalled the next zero-copy store through it for seconds.  A child must not
+ * touch the pool.  kv_host_alloc(b, o) is kv_host_alloc_ex(b, KVX_NUMA_ANY, 0,
+ * o, NULL).  kv_host_pool_info tells what a call returned.
  */
 #define KVX_NUMA_ANY (-2)
 #define KVX_HOST_DRIVER 0x1u
+#define KVX_HOST_HUGE 0x2u
 kvx_status kv_host_alloc_ex(int64_t bytes, int32_t numa_node, uint32_t flags, void** out, int32_t* numa_out);
 
 /*
@@ -456,6 +466,12 @@ void kv_tier_destroy(kvx_tier* tier);
    kv_tier_commit (or kv_tier_release to give it up).  KVX_ENOMEM if every
    slot is pinned or busy; KVX_EBUSY if `key` itself is. */
 kvx_status kv_tier_reserve(kvx_tier* tier, uint64_t key, void** slot);
+/* kv_tier_reserve of keys[0..n) in order, under one lock: slots[j] receives
+   the slot of keys[j].  It stops at the first key that cannot be reserved and
+   returns that key's status; *n_reserved (may be NULL) receives the number
+   reserved, which stay reserved (commit them or release them). */
+kvx_status kv_tier_reserve_many(kvx_tier* tier, const uint64_t* keys, int64_t n, void** slots,
+                                int64_t* n_reserved);
 /* Marks a reserved entry readable once the work already enqueued on
    `stream` (the store into it) completes; unpins it.  On a shared tier the
    commit enqueues its publication (see kv_tier_open_shared): a one-thread
@@ -469,9 +485,19 @@ kvx_status kv_tier_commit_many(kvx_tier* tier, const uint64_t* keys, int64_t n, 
 /* Slot of a committed entry; `stream` is made to wait for its commit event.
    Pins it until kv_tier_release.  KVX_ENOENT if absent or not committed. */
 kvx_status kv_tier_acquire(kvx_tier* tier, uint64_t key, kvx_stream_t stream, void** slot);
+/* kv_tier_acquire of n keys: slots[j] receives the slot of keys[j] (a key may
+   be listed more than once: one pin each).  `stream` waits once per distinct
+   commit event.  If any key is not readable (KVX_ENOENT) or cannot be pinned
+   (KVX_EBUSY), nothing is pinned. */
+kvx_status kv_tier_acquire_many(kvx_tier* tier, const uint64_t* keys, int64_t n, kvx_stream_t stream,
+                                void** slots);
 /* Unpins; the slot stays in use until the work already enqueued on `stream`
    (the load from it) completes. */
 kvx_status kv_tier_release(kvx_tier* tier, uint64_t key, kvx_stream_t stream);
+/* kv_tier_release of n keys with one event for all of them.  Each listing of
+   a key drops one pin this process holds; if any key lacks the pins
+   (KVX_EINVAL) or is absent (KVX_ENOENT), nothing is released. */
+kvx_status kv_tier_release_many(kvx_tier* tier, const uint64_t* keys, int64_t n, kvx_stream_t stream);
 /* Shared tier: drops the pins held by processes that no longer exist and
    frees the entries they were writing or committing (their bytes may be
    incomplete).  *reclaimed (may be null) receives the number of slots changed.

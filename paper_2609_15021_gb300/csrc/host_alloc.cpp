@@ -3,24 +3,31 @@
 //
 // Sec. 3.3: the shared tier is one exact-size pinned pool, and a request that
 // silently fell back to pageable memory was one of the paper's failures.  A
-// pool here is anonymous memory mapped by the library, backed by transparent
-// huge pages where it is large enough, optionally placed on one NUMA node,
-// and registered page-locked, portable and mapped.
+// pool here comes from the driver's pinned allocator (cudaHostAlloc, portable
+// and mapped) unless huge pages or a NUMA placement are asked for; then the
+// library maps anonymous memory itself, backs it with transparent huge pages
+// where it is large enough, places it, and registers it page-locked,
+// portable and mapped.
 //
-// Why huge pages (measured on GB300 with a Grace host and 64 KiB base pages):
-// the SMs' zero-copy accesses run at the link peak whatever backs the pool,
-// but the copy engines (cudaMemcpyAsync, the staged mode) moved 6-18 GB/s
-// from a pool of base pages, 84 GB/s on average (172-422 ms per 33 GB, from
-// step to step) from cudaHostAlloc memory, and 192 GB/s, the link peak,
-// steadily from a pool fully backed by huge pages.  A pool only partly backed
-// (31.1 of 33.3 GB) ran staged at 97 GB/s.  So the mapping is huge-page
-// aligned, asked for huge pages, faulted in at once (MADV_POPULATE_WRITE),
-// and any range still on base pages is collapsed into huge pages
-// (MADV_COLLAPSE) before the pages are pinned; both are advice, so the pool
-// is still created if the kernel cannot comply.  Where no huge page can back
-// the pool (smaller than one, or a host without transparent huge pages) and
-// no placement is asked, the driver's allocator serves instead, as it does on
-// request (KVX_HOST_DRIVER).
+// Why (measured on GB300 with a Grace host and 64 KiB base pages):
+// * The SMs' zero-copy accesses (the default transfer mode) ran at the link
+//   peak from both kinds of pool in a quiet process.  In the benchmark, whose
+//   process also pins and frees other buffers and starts a subprocess,
+//   cudaHostAlloc pools held the peak in every run of an interleaved A/B on
+//   one box (200.5-201.8 GB/s), while the library's huge-page pools fell to
+//   146-194 GB/s in the same runs: their zero-copy accesses stalled for
+//   hundreds of milliseconds after memory-management events in the process.
+// * The copy engines (cudaMemcpyAsync, KVX_MODE_STAGED) moved 6-18 GB/s from a
+//   pool of base pages, 84 GB/s on average (172-422 ms per 33 GB, from step to
+//   step) from cudaHostAlloc memory, and 192 GB/s, the link peak, steadily
+//   from a pool fully backed by huge pages.  A pool only partly backed (31.1
+//   of 33.3 GB) ran staged at 97 GB/s.
+// So the default is the driver's allocator, and KVX_HOST_HUGE asks for the
+// huge-page mapping for copy-engine use.  That mapping is huge-page aligned,
+// asked for huge pages, faulted in at once (MADV_POPULATE_WRITE), and any
+// range still on base pages is collapsed into huge pages (MADV_COLLAPSE)
+// before the pages are pinned; a pool that huge pages do not back wholly is
+// never handed out.
 //
 // NUMA: on a host with several memory nodes the pool belongs on the node next
 // to the GPU that uses it; mbind with a preferred-node policy places it there
@@ -213,6 +220,17 @@ kvx_status map_pool(int node, int64_t bytes, bool huge_pages, void** out, bool* 
     madvise(p, len, MADV_NOHUGEPAGE);    // all base pages: no mixture either
     madvise(p, len, kMadvPopulateWrite);
   }
+  // Not inherited by child processes.  Measured on GB300: a fork (a
+  // subprocess started by the process that owns the pool) made the next
+  // zero-copy store through a pinned private pool take 2.4 s instead of 43 ms
+  // and split its huge-page mappings, and khugepaged collapsing them again
+  // 12 s later cost another 0.9 s store; with the pool kept out of the child,
+  // neither happened.
+  if (madvise(p, len, MADV_DONTFORK) != 0) {
+    release();
+    set_error_text("madvise(MADV_DONTFORK) of the host pool failed");
+    return KVX_ENOMEM;
+  }
   const cudaError_t e = cudaHostRegister(p, len, cudaHostRegisterPortable | cudaHostRegisterMapped);
   if (e != cudaSuccess) {
     set_last_cuda_error((int)e);
@@ -243,24 +261,23 @@ kvx_status kv_host_alloc_ex(int64_t bytes, int32_t numa_node, uint32_t flags, vo
   if (!out) return KVX_EINVAL;
   *out = nullptr;
   if (numa_out) *numa_out = -1;
-  if (bytes <= 0 || numa_node < KVX_NUMA_ANY || numa_node >= kMaxNodes || (flags & ~KVX_HOST_DRIVER))
+  if (bytes <= 0 || numa_node < KVX_NUMA_ANY || numa_node >= kMaxNodes ||
+      (flags & ~(KVX_HOST_DRIVER | KVX_HOST_HUGE)))
     return KVX_EINVAL;
-  if ((flags & KVX_HOST_DRIVER) && numa_node != KVX_NUMA_ANY) return KVX_EINVAL;
+  if ((flags & KVX_HOST_DRIVER) && (numa_node != KVX_NUMA_ANY || (flags & KVX_HOST_HUGE))) return KVX_EINVAL;
   if (fault_point("host_alloc")) {
     set_last_cuda_error((int)cudaErrorMemoryAllocation);
     set_error_text("pinning of the host pool (injected fault)");
     return KVX_ENOMEM;
   }
-  // The driver's allocator where asked, and where the library's mapping would
-  // get no huge pages and no placement anyway (a pool small next to a huge
-  // page, or no transparent huge pages): its memory serves the copy engines
-  // better than base pages do.
+  // Without a placement, the driver's allocator unless huge pages are asked
+  // for (and can be had); a placement needs the library's own mapping.
   // Huge pages where rounding the pool up to whole huge pages wastes at most
   // an eighth of it.
   const size_t huge = thp_available() ? huge_page_bytes() : 0;
   const size_t rounded = huge ? ((size_t)bytes + huge - 1) / huge * huge : 0;
   const bool huge_fits = huge != 0 && (rounded - (size_t)bytes) * 8 <= (size_t)bytes;
-  if ((flags & KVX_HOST_DRIVER) || (numa_node == KVX_NUMA_ANY && !huge_fits)) return driver_pool(bytes, out);
+  if (numa_node == KVX_NUMA_ANY && (!(flags & KVX_HOST_HUGE) || !huge_fits)) return driver_pool(bytes, out);
   int node = numa_node;
   if (node == KVX_NUMA_ANY) {
     node = -1;

@@ -111,6 +111,13 @@ bool add_pins(SlotMeta& m, int32_t pid, int32_t n) {
   return true;
 }
 
+// A process that holds no pin on m can still get a holder place.
+bool has_free_holder(const SlotMeta& m) {
+  for (int h = 0; h < kHolders; ++h)
+    if (m.holder_pins[h] <= 0) return true;
+  return false;
+}
+
 void clear_pins(SlotMeta& m) {
   m.pins = 0;
   for (int h = 0; h < kHolders; ++h) m.holder_pins[h] = 0;
@@ -242,7 +249,7 @@ void settle_release(kvx_tier* t, const PendingEvent& p) {
   add_pins(t->meta[p.slot], t->pid, -1);
   auto it = t->queued.find(p.slot);
   if (it != t->queued.end() && --it->second <= 0) t->queued.erase(it);
-  t->spare.push_back(p.ev);
+  if (p.owns_ev) t->spare.push_back(p.ev);
 }
 
 void poll_locked(kvx_tier* t, PollMode mode) {
@@ -659,10 +666,12 @@ kvx_status kv_tier_poll(kvx_tier* t) {
   return KVX_OK;
 }
 
-kvx_status kv_tier_reserve(kvx_tier* t, uint64_t key, void** slot) {
-  if (!t || !slot) return KVX_EINVAL;
-  TierLock lock(t);
-  poll_locked(t, kFront);
+}  // extern "C"
+
+namespace {
+
+// kv_tier_reserve under the lock, after the caller's poll.
+kvx_status reserve_locked(kvx_tier* t, uint64_t key, void** slot) {
   int64_t i = -1;
   // a second pass after reclaiming what processes that died left behind
   for (int pass = 0; pass < 2; ++pass) {
@@ -710,6 +719,34 @@ kvx_status kv_tier_reserve(kvx_tier* t, uint64_t key, void** slot) {
   add_pins(m, t->pid, 1);
   m.tick = ++t->hdr->clock;
   *slot = t->data + i * t->hdr->slot_bytes;
+  return KVX_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+kvx_status kv_tier_reserve(kvx_tier* t, uint64_t key, void** slot) {
+  if (!t || !slot) return KVX_EINVAL;
+  TierLock lock(t);
+  poll_locked(t, kFront);
+  return reserve_locked(t, key, slot);
+}
+
+kvx_status kv_tier_reserve_many(kvx_tier* t, const uint64_t* keys, int64_t n, void** slots, int64_t* n_reserved) {
+  if (n_reserved) *n_reserved = 0;
+  if (!t || n < 0 || (n > 0 && (!keys || !slots))) return KVX_EINVAL;
+  if (n == 0) return KVX_OK;
+  TierLock lock(t);
+  poll_locked(t, kFront);
+  for (int64_t j = 0; j < n; ++j) {
+    const kvx_status st = reserve_locked(t, keys[j], &slots[j]);
+    if (st != KVX_OK) {
+      if (n_reserved) *n_reserved = j;
+      return st;
+    }
+  }
+  if (n_reserved) *n_reserved = n;
   return KVX_OK;
 }
 
@@ -783,59 +820,82 @@ kvx_status kv_tier_commit_many(kvx_tier* t, const uint64_t* keys, int64_t n, kvx
 }
 
 kvx_status kv_tier_acquire(kvx_tier* t, uint64_t key, kvx_stream_t stream, void** slot) {
-  if (!t || !slot) return KVX_EINVAL;
+  if (!slot) return KVX_EINVAL;
+  return kv_tier_acquire_many(t, &key, 1, stream, slot);
+}
+
+kvx_status kv_tier_acquire_many(kvx_tier* t, const uint64_t* keys, int64_t n, kvx_stream_t stream,
+                                void** slots) {
+  if (!t || n < 0 || (n > 0 && (!keys || !slots))) return KVX_EINVAL;
+  if (n == 0) return KVX_OK;
   TierLock lock(t);
   poll_locked(t, kFront);
-  const int64_t i = find_slot(t, key);
-  bool ok = i >= 0 && t->meta[i].state == kReady;
-  cudaEvent_t wait_on = nullptr;
-  if (i >= 0 && t->meta[i].state == kCommitting && t->meta[i].writer_pid == t->pid) {
-    auto it = t->commit_event.find(i);  // written here: order the reader on the writer's event
-    if (it != t->commit_event.end()) {
-      wait_on = it->second;
-      ok = true;
+  std::vector<int64_t> idx((size_t)n);
+  std::vector<cudaEvent_t> waits;  // this process's commit events the readers must follow, once each
+  for (int64_t j = 0; j < n; ++j) {  // every key first: on an error nothing is pinned
+    const int64_t i = find_slot(t, keys[j]);
+    bool ok = i >= 0 && t->meta[i].state == kReady;
+    if (i >= 0 && t->meta[i].state == kCommitting && t->meta[i].writer_pid == t->pid) {
+      auto it = t->commit_event.find(i);  // written here: order the reader on the writer's event
+      if (it != t->commit_event.end()) {
+        if (std::find(waits.begin(), waits.end(), it->second) == waits.end()) waits.push_back(it->second);
+        ok = true;
+      }
     }
-  }
-  if (!ok) {
-    t->hdr->misses++;
-    return KVX_ENOENT;
-  }
-  if (wait_on) {
-    if (no_stream(stream)) {
-      const cudaError_t r = cudaEventSynchronize(wait_on);
-      if (r != cudaSuccess) return cuda_fail(r, "cudaEventSynchronize (tier acquire)");
-    } else {
-      const cudaError_t r = cudaStreamWaitEvent((cudaStream_t)stream, wait_on, 0);
-      if (r != cudaSuccess) return cuda_fail(r, "cudaStreamWaitEvent (tier acquire)");
+    if (!ok) {
+      t->hdr->misses++;
+      return KVX_ENOENT;
     }
+    if (pins_of(t->meta[i], t->pid) == 0 && !has_free_holder(t->meta[i])) {
+      set_error_text("the entry is pinned by as many processes as it can track");
+      return KVX_EBUSY;
+    }
+    idx[(size_t)j] = i;
   }
-  SlotMeta& m = t->meta[i];
-  if (!add_pins(m, t->pid, 1)) {
-    set_error_text("the entry is pinned by as many processes as it can track");
-    return KVX_EBUSY;
+  for (cudaEvent_t e : waits) {
+    const cudaError_t r = no_stream(stream) ? cudaEventSynchronize(e) : cudaStreamWaitEvent((cudaStream_t)stream, e, 0);
+    if (r != cudaSuccess) return cuda_fail(r, no_stream(stream) ? "cudaEventSynchronize (tier acquire)"
+                                                                 : "cudaStreamWaitEvent (tier acquire)");
   }
-  m.tick = ++t->hdr->clock;
-  t->hdr->hits++;
-  *slot = t->data + i * t->hdr->slot_bytes;
+  for (int64_t j = 0; j < n; ++j) {
+    const int64_t i = idx[(size_t)j];
+    SlotMeta& m = t->meta[i];
+    add_pins(m, t->pid, 1);  // cannot fail: a holder place was checked above
+    m.tick = ++t->hdr->clock;
+    t->hdr->hits++;
+    slots[j] = t->data + i * t->hdr->slot_bytes;
+  }
   return KVX_OK;
 }
 
 kvx_status kv_tier_release(kvx_tier* t, uint64_t key, kvx_stream_t stream) {
-  if (!t) return KVX_EINVAL;
+  return kv_tier_release_many(t, &key, 1, stream);
+}
+
+kvx_status kv_tier_release_many(kvx_tier* t, const uint64_t* keys, int64_t n, kvx_stream_t stream) {
+  if (!t || n < 0 || (n > 0 && !keys)) return KVX_EINVAL;
+  if (n == 0) return KVX_OK;
   TierLock lock(t);
   poll_locked(t, kFront);
-  const int64_t i = find_slot(t, key);
-  if (i < 0) return KVX_ENOENT;
-  SlotMeta& m = t->meta[i];
-  if (pins_of(m, t->pid) - queued_releases(t, i) < 1) {
-    set_error_text("this process holds no pin on the entry");
-    return KVX_EINVAL;
+  std::vector<int64_t> idx((size_t)n);
+  std::unordered_map<int64_t, int64_t> asked;  // releases of each slot in this call
+  for (int64_t j = 0; j < n; ++j) {  // every key first: on an error nothing is released
+    const int64_t i = find_slot(t, keys[j]);
+    if (i < 0) return KVX_ENOENT;
+    idx[(size_t)j] = i;
+    if (pins_of(t->meta[i], t->pid) - queued_releases(t, i) < ++asked[i]) {
+      set_error_text("this process holds no pin on the entry");
+      return KVX_EINVAL;
+    }
   }
   if (no_stream(stream)) {
-    add_pins(m, t->pid, -1);
-    if (m.state == kWriting && m.pins == 0) {  // a writer giving up its reservation
-      index_erase(t, m.key);
-      m.state = kFree;
+    for (int64_t i : idx) {
+      SlotMeta& m = t->meta[i];
+      add_pins(m, t->pid, -1);
+      if (m.state == kWriting && m.pins == 0) {  // a writer giving up its reservation
+        index_erase(t, m.key);
+        m.state = kFree;
+      }
     }
     return KVX_OK;
   }
@@ -846,8 +906,11 @@ kvx_status kv_tier_release(kvx_tier* t, uint64_t key, kvx_stream_t stream) {
     t->spare.push_back(e);
     return cuda_fail(r, "cudaEventRecord (tier release)");
   }
-  t->releases.push_back({i, e, 0, true});  // the pin stays until the queued work completes
-  t->queued[i]++;
+  for (int64_t j = 0; j < n; ++j) {  // the pins stay until the queued work completes; one event for all
+    const int64_t i = idx[(size_t)j];
+    t->releases.push_back({i, e, 0, j == n - 1});
+    t->queued[i]++;
+  }
   return KVX_OK;
 }
 

@@ -37,8 +37,8 @@ EXPORTED = (
     "kv_ctx_modes", "kv_last_cuda_error", "kv_last_error_message", "kv_status_string", "kv_abi_version",
     "kvx_probe_delayed_fill", "kvx_probe_delayed_copy", "kvx_probe_copy", "kv_store_noalloc",
     "kv_host_alloc", "kv_host_free", "kv_pool_view_check",
-    "kv_chunk_keys", "kv_tier_create", "kv_tier_create_on", "kv_tier_destroy", "kv_tier_reserve", "kv_tier_commit", "kv_tier_commit_many",
-    "kv_tier_acquire", "kv_tier_release", "kv_tier_prefix_hits", "kv_tier_stats", "kv_fault_inject",
+    "kv_chunk_keys", "kv_tier_create", "kv_tier_create_on", "kv_tier_destroy", "kv_tier_reserve", "kv_tier_reserve_many", "kv_tier_commit", "kv_tier_commit_many",
+    "kv_tier_acquire", "kv_tier_release", "kv_tier_acquire_many", "kv_tier_release_many", "kv_tier_prefix_hits", "kv_tier_stats", "kv_fault_inject",
     "kv_tier_open_shared", "kv_tier_poll", "kv_tier_reclaim", "kv_host_alloc_numa", "kv_host_alloc_ex",
     "kv_host_pool_info",
 )
@@ -129,10 +129,13 @@ def _declare(lib):
         "kv_tier_reclaim": (st, [vp, P(i64)]),
         "kv_tier_destroy": (None, [vp]),
         "kv_tier_reserve": (st, [vp, ctypes.c_uint64, P(vp)]),
+        "kv_tier_reserve_many": (st, [vp, P(ctypes.c_uint64), i64, P(vp), P(i64)]),
         "kv_tier_commit": (st, [vp, ctypes.c_uint64, vp]),
         "kv_tier_commit_many": (st, [vp, P(ctypes.c_uint64), i64, vp]),
         "kv_tier_acquire": (st, [vp, ctypes.c_uint64, vp, P(vp)]),
         "kv_tier_release": (st, [vp, ctypes.c_uint64, vp]),
+        "kv_tier_acquire_many": (st, [vp, P(ctypes.c_uint64), i64, vp, P(vp)]),
+        "kv_tier_release_many": (st, [vp, P(ctypes.c_uint64), i64, vp]),
         "kv_tier_prefix_hits": (st, [vp, P(ctypes.c_uint64), i64, P(i64)]),
         "kv_tier_stats": (st, [vp, P(kvx_tier_stats)]),
         "kv_fault_inject": (st, [ctypes.c_char_p, i32]),
@@ -364,7 +367,7 @@ def kv_host_alloc(nbytes: int) -> int:
 
 
 KVX_NUMA_NEAREST, KVX_NUMA_ANY = -1, -2
-KVX_HOST_DRIVER = 0x1
+KVX_HOST_DRIVER, KVX_HOST_HUGE = 0x1, 0x2
 KVX_HOST_SOURCE_DRIVER, KVX_HOST_SOURCE_MAPPED = 0, 1
 
 
@@ -405,17 +408,22 @@ class HostBuffer:
     Views of ``.tensor`` keep the allocation alive; ``close()`` frees it at once
     and must only be called when no view is used any more."""
 
-    def __init__(self, nbytes: int, numa_node: int | None = None, driver: bool = False):
-        """numa_node: None for kv_host_alloc, else kv_host_alloc_numa on that node
-        (KVX_NUMA_NEAREST: the node nearest the current GPU); see .numa_node.
-        driver: the driver's pinned allocator instead (KVX_HOST_DRIVER)."""
+    def __init__(self, nbytes: int, numa_node: int | None = None, driver: bool = False, huge: bool = False):
+        """numa_node: None for no placement, else on that node (KVX_NUMA_NEAREST:
+        the node nearest the current GPU); see .numa_node.  driver: the driver's
+        pinned allocator, stated (KVX_HOST_DRIVER; the default without a
+        placement).  huge: the library's huge-page mapping (KVX_HOST_HUGE), for
+        copy-engine transfers."""
         import torch
         self.nbytes = nbytes
         self.numa_node = None
+        if driver and (huge or numa_node is not None):
+            raise ValueError("the driver's allocator takes no NUMA placement and no huge pages")
         if driver:
-            if numa_node is not None:
-                raise ValueError("the driver's allocator takes no NUMA placement")
             self.ptr, _ = kv_host_alloc_ex(nbytes, KVX_NUMA_ANY, KVX_HOST_DRIVER)
+        elif huge:
+            self.ptr, node = kv_host_alloc_ex(nbytes, KVX_NUMA_ANY if numa_node is None else numa_node, KVX_HOST_HUGE)
+            self.numa_node = None if numa_node is None else node
         elif numa_node is None:
             self.ptr = kv_host_alloc(nbytes)
         else:
@@ -575,6 +583,23 @@ class KvTier:
         _check(_lib.kv_tier_reserve(self.handle, key, ctypes.byref(out)), "kv_tier_reserve")
         return self._slot_tensor(out.value)
 
+    def reserve_many(self, keys) -> list:
+        """Slots for `keys`, reserved in order under one lock.  If a key cannot be
+        reserved, KvxError is raised with `.reserved`: the slots of the keys
+        before it, which stay reserved (commit or release them)."""
+        n = len(keys)
+        arr = (ctypes.c_uint64 * max(1, n))(*keys)
+        out = (ctypes.c_void_p * max(1, n))()
+        done = ctypes.c_int64()
+        status = _lib.kv_tier_reserve_many(self.handle, arr, n, out, ctypes.byref(done))
+        slots = [self._slot_tensor(out[j]) for j in range(done.value)]
+        try:
+            _check(status, "kv_tier_reserve_many")
+        except KvxError as e:
+            e.reserved = slots
+            raise
+        return slots
+
     def commit(self, key: int, stream=None):
         _check(_lib.kv_tier_commit(self.handle, key, self._stream(stream)), "kv_tier_commit")
 
@@ -589,6 +614,17 @@ class KvTier:
 
     def release(self, key: int, stream=None):
         _check(_lib.kv_tier_release(self.handle, key, self._stream(stream)), "kv_tier_release")
+
+    def acquire_many(self, keys, stream=None) -> list:
+        arr = (ctypes.c_uint64 * max(1, len(keys)))(*keys)
+        out = (ctypes.c_void_p * max(1, len(keys)))()
+        _check(_lib.kv_tier_acquire_many(self.handle, arr, len(keys), self._stream(stream), out),
+               "kv_tier_acquire_many")
+        return [self._slot_tensor(out[j]) for j in range(len(keys))]
+
+    def release_many(self, keys, stream=None):
+        arr = (ctypes.c_uint64 * max(1, len(keys)))(*keys)
+        _check(_lib.kv_tier_release_many(self.handle, arr, len(keys), self._stream(stream)), "kv_tier_release_many")
 
     def prefix_hits(self, keys) -> int:
         arr = (ctypes.c_uint64 * max(1, len(keys)))(*keys)

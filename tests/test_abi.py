@@ -204,8 +204,10 @@ def test_host_alloc_numa_arguments(k):
         assert k._lib.kv_host_alloc_numa(0, 4096, ctypes.byref(out), None) == k.KVX_ECUDA
         assert out.value is None
     ex = k._lib.kv_host_alloc_ex
-    assert ex(4096, k.KVX_NUMA_ANY, 0x2, ctypes.byref(out), None) == k.KVX_EINVAL          # unknown flag
+    assert ex(4096, k.KVX_NUMA_ANY, 0x4, ctypes.byref(out), None) == k.KVX_EINVAL          # unknown flag
     assert ex(4096, 0, k.KVX_HOST_DRIVER, ctypes.byref(out), None) == k.KVX_EINVAL         # driver + node
+    assert ex(4096, k.KVX_NUMA_ANY, k.KVX_HOST_DRIVER | k.KVX_HOST_HUGE, ctypes.byref(out),
+              None) == k.KVX_EINVAL                                                         # driver + huge
     assert ex(4096, -3, 0, ctypes.byref(out), None) == k.KVX_EINVAL
     assert k._lib.kv_host_alloc_numa(k.KVX_NUMA_ANY, 4096, ctypes.byref(out), None) == k.KVX_EINVAL
 

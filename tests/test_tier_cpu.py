@@ -173,6 +173,13 @@ class _Model:
         s["tick"] = self.clock
         return "OK"
 
+    def reserve_many(self, keys):
+        for j, key in enumerate(keys):        # in order, up to the first failure
+            st, _ = self.reserve(key)
+            if st != "OK":
+                return st, j
+        return "OK", len(keys)
+
     def commit_many(self, keys):
         idx = []
         for key in keys:                      # every key is checked before any is committed
@@ -213,6 +220,29 @@ class _Model:
             s["state"] = "FREE"
         return "OK"
 
+    def acquire_many(self, keys):
+        for key in keys:                      # all or nothing
+            i = self.find(key)
+            if i is None or self.slots[i]["state"] != "READY":
+                self.misses += 1
+                return "ENOENT"
+        for key in keys:
+            assert self.acquire(key) == "OK"
+        return "OK"
+
+    def release_many(self, keys):
+        asked = {}
+        for key in keys:
+            i = self.find(key)
+            if i is None:
+                return "ENOENT"
+            asked[i] = asked.get(i, 0) + 1
+            if self.slots[i]["pins"] < asked[i]:
+                return "EINVAL"
+        for key in keys:
+            assert self.release(key) == "OK"
+        return "OK"
+
     def prefix_hits(self, keys):
         h = 0
         for key in keys:
@@ -241,8 +271,8 @@ def test_tier_follows_its_rules_under_random_operations(k, seed, n_slots, n_keys
 
     for step in range(4000):
         key = int(rng.integers(1, n_keys + 1)) * 1000003
-        op = rng.choice(["reserve", "commit", "commit_many", "acquire", "release", "prefix"],
-                        p=[0.3, 0.17, 0.08, 0.2, 0.2, 0.05])
+        op = rng.choice(["reserve", "reserve_many", "commit", "commit_many", "acquire", "acquire_many", "release",
+                         "release_many", "prefix"], p=[0.22, 0.08, 0.17, 0.08, 0.14, 0.06, 0.14, 0.06, 0.05])
         if op == "reserve":
             got, view = call(tier.reserve, key)
             want, _ = model.reserve(key)
@@ -251,10 +281,27 @@ def test_tier_follows_its_rules_under_random_operations(k, seed, n_slots, n_keys
         elif op == "commit":
             got, _ = call(tier.commit, key, NO)
             want = model.commit(key)
+        elif op == "reserve_many":
+            keys = [int(x) * 1000003 for x in rng.integers(1, n_keys + 1, size=int(rng.integers(0, 4)))]
+            try:
+                views, got = tier.reserve_many(keys), "OK"
+            except k.KvxError as e:
+                views, got = e.reserved, status[e.status]
+            want, n_done = model.reserve_many(keys)
+            assert len(views) == n_done, (step, keys)
+            for kk, view in zip(keys, views):
+                view.fill_(kk % 251)
         elif op == "commit_many":
             keys = [int(x) * 1000003 for x in rng.integers(1, n_keys + 1, size=int(rng.integers(0, 4)))]
             got, _ = call(tier.commit_many, keys, NO)
             want = model.commit_many(keys)
+        elif op in ("acquire_many", "release_many"):
+            keys = [int(x) * 1000003 for x in rng.integers(1, n_keys + 1, size=int(rng.integers(0, 4)))]
+            got, views = call(getattr(tier, op), keys, NO)
+            want = getattr(model, op)(keys)
+            if op == "acquire_many" and got == "OK":
+                for kk, view in zip(keys, views):
+                    assert int(view[0]) == kk % 251 and int(view[-1]) == kk % 251, step
         elif op == "acquire":
             got, view = call(tier.acquire, key, NO)
             want = model.acquire(key)

@@ -21,7 +21,8 @@ DELAY = 10 ** 8
 @pytest.mark.parametrize("commit", ["per_key", "many"])
 def test_store_then_restore_across_streams_through_the_tier(orc, commit):
     """commit="many": one kv_store of every chunk into its slot and one
-    kv_tier_commit_many, whose entries share one event."""
+    kv_tier_commit_many, whose entries share one event; the reader takes them
+    with one kv_tier_acquire_many, one kv_load and one kv_tier_release_many."""
     k = kvx()
     spec = oracle.PoolSpec(4, 64, 16, 8, 128, 2, oracle.HND)
     C, n_used = 256, 48
@@ -46,7 +47,7 @@ def test_store_then_restore_across_streams_through_the_tier(orc, commit):
             k.kvx_probe_delayed_copy(pool_a.layers[l], final_dev[l], spec.layer_bytes, DELAY if l == 0 else 0, s_a)
         ta_d = torch.from_numpy(ta).cuda()
         if commit == "many":
-            slots = [tier.reserve(key) for key in keys]
+            slots = tier.reserve_many(keys)
             k.kv_store(ctx, pool_a, ta_d, 0, T, C, slots, stream=s_a)
             tier.commit_many(keys, stream=s_a)
         else:
@@ -57,10 +58,15 @@ def test_store_then_restore_across_streams_through_the_tier(orc, commit):
         # replica B, its own stream, no host synchronisation: ordered by the commit events
         assert tier.prefix_hits(keys) == len(keys)
         tb_d = torch.from_numpy(tb).cuda()
-        for c, key in enumerate(keys):
-            slot = tier.acquire(key, stream=s_b)
-            k.kv_load(ctx, pool_b, tb_d, c * C, (c + 1) * C, C, [slot], stream=s_b)
-            tier.release(key, stream=s_b)
+        if commit == "many":
+            slots = tier.acquire_many(keys, stream=s_b)
+            k.kv_load(ctx, pool_b, tb_d, 0, T, C, slots, stream=s_b)
+            tier.release_many(keys, stream=s_b)
+        else:
+            for c, key in enumerate(keys):
+                slot = tier.acquire(key, stream=s_b)
+                k.kv_load(ctx, pool_b, tb_d, c * C, (c + 1) * C, C, [slot], stream=s_b)
+                tier.release(key, stream=s_b)
         s_b.synchronize()
         s_a.synchronize()
         want, _ = oracle_store(orc, spec, final_np, ta, 0, T, C)

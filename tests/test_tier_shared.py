@@ -305,7 +305,7 @@ def test_shared_tier_store_in_one_process_restore_in_another(commit):
         for l in range(4):   # the producer finishes writing the KV ~2*10^9 cycles (~1 s) later
             k.kvx_probe_delayed_copy(pool.layers[l], final_dev[l], spec.layer_bytes, 2 * 10 ** 9 if l == 0 else 0, s)
         if commit == "many":                    # one store, one publication launch for both chunks
-            slots = [tier.reserve(key) for key in keys]
+            slots = tier.reserve_many(keys)
             k.kv_store(ctx, pool, ta_d, 0, T, C, slots, stream=s)
             tier.commit_many(keys, stream=s)
         else:
