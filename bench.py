@@ -327,6 +327,15 @@ def run_reference(args):
 # ------------------------------------------------------------------ GPU leg
 
 
+def shm_free_bytes() -> int:
+    """Room left in the POSIX shared-memory file system (0 if unknown)."""
+    try:
+        st = os.statvfs("/dev/shm")
+        return st.f_bavail * st.f_frsize
+    except OSError:
+        return 0
+
+
 def link_buffers(torch, dev):
     """The pinned and device buffers of host_link_peak, allocated once per run."""
     n = 1 << 30
@@ -448,7 +457,8 @@ def run_ours(args):
     # made once the second chunk set is freed: three 33 GB pools pinned at once
     # left the two-replica leg at half its speed.
     want_conc = not args.no_concurrent and world == 1 and avail > 2 * n_chunks * cb + (32 << 30)
-    want_tier = not args.no_tier and world == 1 and avail > 2 * n_chunks * cb + (32 << 30)
+    want_tier = (not args.no_tier and world == 1 and avail > 2 * n_chunks * cb + (32 << 30)
+                 and shm_free_bytes() > n_chunks * cb + (1 << 30))
     host_pool2 = k.HostBuffer(n_chunks * cb, huge=host_alloc == "huge") if want_conc else None
     ta_host = torch.from_numpy(ta_np).pin_memory()
     tb_host = torch.from_numpy(tb_np).pin_memory()

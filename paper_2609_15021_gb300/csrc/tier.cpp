@@ -571,6 +571,15 @@ kvx_status kv_tier_open_shared(const char* name, int64_t slot_bytes, int64_t n_s
       set_error_text("ftruncate of the shared tier failed");
       return KVX_ENOMEM;
     }
+    // Reserve the pages now: a shared-memory file system without room for
+    // them would otherwise end the process with SIGBUS at first touch.
+    const int fr = posix_fallocate(fd, 0, (off_t)total);
+    if (fr != 0 && fr != EOPNOTSUPP && fr != EINVAL) {
+      close(fd);
+      shm_unlink(name);
+      set_error_text("the shared-memory file system has no room for the tier");
+      return KVX_ENOMEM;
+    }
   } else {
     struct stat sb;
     // wait (bounded) for the creator to size and initialise the region
