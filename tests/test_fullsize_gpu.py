@@ -201,8 +201,8 @@ def _pool_smaps(ptr: int, nbytes: int):
 def test_pool_is_not_disturbed_by_a_subprocess():
     """A pool the library maps (here on huge pages) is kept out of child processes (MADV_DONTFORK, VmFlags "dc"):
     starting a subprocess leaves its huge-page mappings whole, and the zero-copy
-    store and restore right after run as fast as before.  Without it, a fork
-    stalled the next store through such a pool for seconds on GB300."""
+    store and restore right after do not stall.  Without it, a fork stalled the
+    next store through such a pool for seconds on GB300."""
     import subprocess
     k = kvx()
     spec = oracle.PoolSpec(L, 4096, B, H, D, E, oracle.HND)
@@ -241,7 +241,10 @@ def test_pool_is_not_disturbed_by_a_subprocess():
             print(f"\nstore + restore of {T} tokens: {before:.1f} ms before a subprocess, {after:.1f} ms after; "
                   f"huge-page bytes {huge0} -> {huge1}")
             assert huge1 == huge0
-            assert after < 1.5 * before
+            # A fork stalled the next step 28-fold without MADV_DONTFORK; other
+            # host memory activity on a shared machine has stalled steps up to
+            # about 5-fold, so the bound only catches the fork stall.
+            assert after < 10 * before
             assert k.kv_get_device_error(ctx) == -1
         finally:
             k.kv_ctx_destroy(ctx)
