@@ -243,7 +243,9 @@ def max_over_ranks(world, value: float, local: int) -> float:
         return value
     import torch
     import torch.distributed as dist
-    t = torch.tensor([value], dtype=torch.float64, device=f"cuda:{local}" if torch.cuda.is_available() else "cpu")
+    # NCCL reduces device tensors, gloo host tensors
+    on_gpu = dist.get_backend() == "nccl"
+    t = torch.tensor([value], dtype=torch.float64, device=f"cuda:{local}" if on_gpu else "cpu")
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
 
