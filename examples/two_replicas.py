@@ -45,10 +45,9 @@ def replica_b(name, q):
     ctx = k.kv_ctx_create(0)
     stream = torch.cuda.Stream()
     torch.cuda.synchronize()
-    for c in range(hits):                                  # acquire, restore, release: all on `stream`
-        slot = tier.acquire(keys[c], stream=stream)
-        k.kv_load(ctx, pool, table, c * C, (c + 1) * C, C, [slot], stream=stream)
-        tier.release(keys[c], stream=stream)
+    slots = tier.acquire_many(keys[:hits], stream=stream)  # acquire, restore, release: all on `stream`
+    k.kv_load(ctx, pool, table, 0, hits * C, C, slots, stream=stream)
+    tier.release_many(keys[:hits], stream=stream)
     stream.synchronize()
     assert k.kv_get_device_error(ctx) == -1
     got = [t.view(N, PAGE)[table.long()].cpu() for t in layers]
@@ -73,10 +72,9 @@ def main():
         stream = torch.cuda.Stream()
         torch.cuda.synchronize()
         keys = chunk_keys(k)
-        for c, key in enumerate(keys):
-            slot = tier.reserve(key)
-            k.kv_store(ctx, pool, table, c * C, (c + 1) * C, C, [slot], stream=stream)
-            tier.commit(key, stream=stream)      # readable everywhere once the GPU has passed this point
+        slots = tier.reserve_many(keys)              # one slot per chunk key
+        k.kv_store(ctx, pool, table, 0, TOKENS, C, slots, stream=stream)
+        tier.commit_many(keys, stream=stream)        # readable everywhere once the GPU has passed this point
         stream.synchronize()
         want = [t.view(N, PAGE)[table.long()].cpu().numpy() for t in layers]
         k.kv_ctx_destroy(ctx)
