@@ -132,6 +132,7 @@ kvx_status driver_pool(int64_t bytes, void** out) {
   }
   Pool rec;
   rec.bytes = bytes;
+  rec.node = page_node(p);  // -1 where the kernel does not say for the driver's mapping
   {
     std::lock_guard<std::mutex> g(g_mu);
     g_pools[p] = rec;
