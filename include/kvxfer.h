@@ -403,6 +403,10 @@ void kv_host_free(void* host);
  * release events not yet complete): the premature reuse of asynchronous-copy
  * buffers the paper cites is ruled out.  All tier calls are host-thread safe.
  * Pass KVX_NO_STREAM when the caller has already synchronised (no event).
+ * Tier calls keep their bookkeeping on the host at call time, so a call given
+ * a stream that is being captured into a CUDA graph returns KVX_EINVAL and
+ * leaves the capture as it was: a replay would repeat its events and
+ * publications without the bookkeeping.
  * ------------------------------------------------------------------------ */
 #define KVX_NO_STREAM ((kvx_stream_t)(intptr_t)-1)
 

@@ -139,6 +139,20 @@ uint64_t mix64(uint64_t z) {
 
 bool no_stream(kvx_stream_t s) { return s == KVX_NO_STREAM; }
 
+// Tier calls keep their bookkeeping on the host at call time; on a stream
+// being captured into a graph, a replay would repeat their GPU work without it.
+bool capturing(kvx_stream_t s) {
+  if (no_stream(s)) return false;
+  cudaStreamCaptureStatus st = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing((cudaStream_t)s, &st) != cudaSuccess) {
+    cudaGetLastError();
+    return false;  // an unusable stream fails at its first use below
+  }
+  if (st == cudaStreamCaptureStatusNone) return false;
+  set_error_text("tier calls cannot be captured into a CUDA graph");
+  return true;
+}
+
 kvx_status cuda_fail(cudaError_t e, const char* what) {
   set_last_cuda_error((int)e);
   set_error_text(what);
@@ -195,15 +209,23 @@ void lock_table(kvx_tier* t) {
   }
 }
 
+// The tier's own event queries and creations run in relaxed capture mode:
+// a tier call made while the calling thread is capturing a graph on another
+// stream (reserve, a lookup) then leaves that capture alone.
 struct TierLock {
   kvx_tier* t;
+  cudaStreamCaptureMode mode = cudaStreamCaptureModeRelaxed;
+  bool swapped = false;
   explicit TierLock(kvx_tier* tier) : t(tier) {
+    swapped = cudaThreadExchangeStreamCaptureMode(&mode) == cudaSuccess;
+    if (!swapped) cudaGetLastError();
     t->local.lock();
     lock_table(t);
   }
   ~TierLock() {
     pthread_mutex_unlock(&t->hdr->mu);
     t->local.unlock();
+    if (swapped && cudaThreadExchangeStreamCaptureMode(&mode) != cudaSuccess) cudaGetLastError();
   }
 };
 
@@ -764,7 +786,7 @@ kvx_status kv_tier_commit(kvx_tier* t, uint64_t key, kvx_stream_t stream) {
 }
 
 kvx_status kv_tier_commit_many(kvx_tier* t, const uint64_t* keys, int64_t n, kvx_stream_t stream) {
-  if (!t || n < 0 || (n > 0 && !keys)) return KVX_EINVAL;
+  if (!t || n < 0 || (n > 0 && !keys) || capturing(stream)) return KVX_EINVAL;
   if (n == 0) return KVX_OK;
   TierLock lock(t);
   poll_locked(t, kFront);
@@ -835,7 +857,7 @@ kvx_status kv_tier_acquire(kvx_tier* t, uint64_t key, kvx_stream_t stream, void*
 
 kvx_status kv_tier_acquire_many(kvx_tier* t, const uint64_t* keys, int64_t n, kvx_stream_t stream,
                                 void** slots) {
-  if (!t || n < 0 || (n > 0 && (!keys || !slots))) return KVX_EINVAL;
+  if (!t || n < 0 || (n > 0 && (!keys || !slots)) || capturing(stream)) return KVX_EINVAL;
   if (n == 0) return KVX_OK;
   TierLock lock(t);
   poll_locked(t, kFront);
@@ -882,7 +904,7 @@ kvx_status kv_tier_release(kvx_tier* t, uint64_t key, kvx_stream_t stream) {
 }
 
 kvx_status kv_tier_release_many(kvx_tier* t, const uint64_t* keys, int64_t n, kvx_stream_t stream) {
-  if (!t || n < 0 || (n > 0 && !keys)) return KVX_EINVAL;
+  if (!t || n < 0 || (n > 0 && !keys) || capturing(stream)) return KVX_EINVAL;
   if (n == 0) return KVX_OK;
   TierLock lock(t);
   poll_locked(t, kFront);

@@ -57,3 +57,53 @@ def test_store_restore_replayed_from_a_cuda_graph(orc):
         assert k.kv_get_device_error(ctx) == -1
     finally:
         k.kv_ctx_destroy(ctx)
+
+
+def test_tier_calls_during_a_capture(orc):
+    """Tier calls keep host bookkeeping, so one given a capturing stream is
+    refused (KVX_EINVAL) and the capture goes on; calls without a stream
+    (reserve, lookups) made while the thread captures leave the capture alone.
+    The captured store is replayed, then committed outside the capture, and
+    its bytes match the oracle."""
+    k = kvx()
+    spec = oracle.PoolSpec(4, 64, 16, 8, 128, 2, oracle.HND)
+    C, n_used = 256, 32
+    T = n_used * 16
+    layers_np = host_layers(spec, 5)
+    src = device_pool(spec, layers_np)
+    ta = synth.permuted_table(64, n_used, 6)
+    ta_d = torch.from_numpy(ta).cuda()
+    keys = [901, 902]
+    tier = k.KvTier(orc.chunk_bytes(spec, C), 4, shared_name=f"/kvx_graph_{__import__('os').getpid()}", create=True)
+    ctx = k.kv_ctx_create(0)
+    try:
+        s = torch.cuda.Stream()
+        slots = tier.reserve_many(keys)
+        with torch.cuda.stream(s):  # warm up outside the capture
+            k.kv_store(ctx, src, ta_d, 0, T, C, slots)
+        s.synchronize()
+        tier.reserve(903)                       # an entry with GPU work pending when the capture starts
+        tier.commit(903, stream=s)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=s):     # the strictest capture mode: global
+            k.kv_store(ctx, src, ta_d, 0, T, C, slots)
+            for call in (lambda: tier.commit_many(keys, stream=s), lambda: tier.acquire(903, stream=s),
+                         lambda: tier.release(903, stream=s)):
+                with pytest.raises(k.KvxError) as e:
+                    call()
+                assert e.value.status == k.KVX_EINVAL
+            assert tier.prefix_hits(keys) == 0  # host-side calls go on (with event queries) inside the capture
+            tier.reserve(904)
+        g.replay()
+        tier.commit_many(keys, stream=s)
+        s.synchronize()
+        assert tier.prefix_hits(keys) == 2
+        want, _ = oracle_store(orc, spec, layers_np, ta, 0, T, C)
+        for c, key in enumerate(keys):
+            got = tier.acquire(key, k.KVX_NO_STREAM)
+            assert first_mismatch(np_of(got), want[c]) is None, c
+            tier.release(key, k.KVX_NO_STREAM)
+        assert k.kv_get_device_error(ctx) == -1
+    finally:
+        k.kv_ctx_destroy(ctx)
+        tier.close()
