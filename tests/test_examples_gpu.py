@@ -1,4 +1,4 @@
-"""The Python example runs as a user would run it, and succeeds."""
+"""The Python examples run as a user would run them, and succeed."""
 import os
 import subprocess
 import sys
@@ -14,4 +14,21 @@ def test_two_replicas_example():
     r = subprocess.run([sys.executable, os.path.join(ROOT, "examples", "two_replicas.py")], cwd=ROOT,
                        capture_output=True, text=True, timeout=600)
     assert r.returncode == 0, r.stdout + r.stderr
+    assert "bit-exact" in r.stdout
+
+
+def test_cross_replica_128k_example():
+    """The full-size cross-process restore: A stores and commits 128k tokens, B
+    sees the published entries, restores them and checks sampled pages."""
+    import torch
+    free, _ = torch.cuda.mem_get_info()
+    st = os.statvfs("/dev/shm")
+    with open("/proc/meminfo") as f:
+        avail = next(int(l.split()[1]) * 1024 for l in f if l.startswith("MemAvailable:"))
+    if free < (130 << 30) or st.f_bavail * st.f_frsize < (34 << 30) or avail < (80 << 30):
+        pytest.skip("needs ~130 GB of device memory, 34 GB of /dev/shm and 80 GB of host memory")
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "examples", "cross_replica_128k.py")], cwd=ROOT,
+                       capture_output=True, text=True, timeout=900)
+    assert r.returncode == 0, r.stdout + r.stderr
+    print("\n" + r.stdout.strip())
     assert "bit-exact" in r.stdout
