@@ -22,6 +22,8 @@ hbm_roofline         kv_pack / kv_unpack of the same context into device chunks
                      against the measured HBM copy peak;
 concurrent_replicas  one context stored while another context's chunks are
                      restored, each through its own context and stream;
+restore_after_idle   a restore after the pool sat untouched for a few seconds,
+                     with the library's host-page touch and without it;
 tier_path            the same store and restore through a host tier shared
                      across processes: keyed reserve / commit, prefix lookup,
                      acquire / release, one kv_store and one kv_load per step;
@@ -209,6 +211,9 @@ def parse():
                          "kv_host_alloc_numa on the host NUMA node nearest the GPU, from the driver's allocator "
                          "stated (KVX_HOST_DRIVER), or on huge pages (KVX_HOST_HUGE); auto: huge for "
                          "--mode staged (the copy engines want huge pages), else plain")
+    ap.add_argument("--no-cold", action="store_true",
+                    help="skip the leg that restores after the pool sat untouched (--cold-idle-s seconds)")
+    ap.add_argument("--cold-idle-s", type=float, default=10.0)
     ap.add_argument("--no-tier", action="store_true",
                     help="skip the leg that stores and restores chunk by chunk through the host tier")
     ap.add_argument("--no-concurrent", action="store_true",
@@ -758,6 +763,29 @@ def run_ours(args):
                     "transfer_calls_per_direction": 1,
                     "slots_equal_timed_chunks_on_sample": same, "evictions": tstats["evictions"]}
 
+    # A restore after idle time: the pool untouched for a few seconds, as before
+    # the first cross-replica hit after a quiet period.  Once as the library
+    # does it by default (it reads one byte per host page first when the
+    # context was idle), once with that off (KVX_FLAG_NO_HOST_TOUCH).  The
+    # events bracket the call, so the host's reads are inside the time.
+    cold = None
+    if not args.no_cold and world == 1:
+        ctx_nt = k.kv_ctx_create(local, store_mode=mode, load_mode=mode, staging_slot_bytes=args.slot_mib << 20,
+                                 flags=k.KVX_FLAG_NO_HOST_TOUCH)
+        cold = {"idle_s": args.cold_idle_s}
+        for name, c in (("restore_ms_without_host_touch", ctx_nt), ("restore_ms", ctx)):
+            torch.cuda.synchronize()
+            time.sleep(args.cold_idle_s)
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            k.kv_load(c, dst, tb, 0, T, C, chunks, stream=stream)
+            b.record(stream)
+            b.synchronize()
+            cold[name] = a.elapsed_time(b)
+        assert k.kv_get_device_error(ctx) == -1 and k.kv_get_device_error(ctx_nt) == -1
+        k.kv_ctx_destroy(ctx_nt)
+        cold["warm_restore_ms"] = statistics.median(restore_ms)
+
     cpu = None
     verified = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -807,6 +835,7 @@ def run_ours(args):
         "verified_sample_vs_oracle": verified,
         "concurrent_replicas": concurrent,
         "tier_path": tier_leg,
+        "restore_after_idle": cold,
         "e2e": e2e,
         "gpu_launches": stats["kernel_launches"],
         "memcpy_calls": stats["memcpy_calls"],

@@ -113,9 +113,19 @@ typedef enum {
 #define KVX_FLAG_DEVICE_TMA 0x4u   /* TMA everywhere it fits, with one bulk
                                       copy per row where no tensor map does  */
 #define KVX_FLAG_DEVICE_LSU 0x8u   /* the 16-byte load/store kernel always   */
+/* Host memory after idle time.  Measured on GB300 (Grace host): after the
+   pinned pool had sat untouched for 10 s, a 128k-token restore through it took
+   337 ms instead of 159 ms (219 ms after 3 s, 165-168 after 1 s), the next one
+   159 ms again; the slowdown followed parts of the pool's host memory, not the
+   GPU or the link.  A CPU read of one byte per host page of the chunks just
+   before the transfer (13.8 ms on one thread for 33 GB) brought it back to
+   159 ms.  So when a context has begun no transfer for more than 1 s,
+   kv_store and kv_load first read one byte of every host page of the chunks
+   they are given, on up to 16 host threads.  This flag turns that off.      */
+#define KVX_FLAG_NO_HOST_TOUCH 0x10u
 /* Every defined flag.  kv_ctx_create rejects (KVX_EINVAL) other bits, and
    KVX_FLAG_DEVICE_TMA together with KVX_FLAG_DEVICE_LSU.                     */
-#define KVX_FLAGS_ALL 0xFu
+#define KVX_FLAGS_ALL 0x1Fu
 
 typedef struct {
   int32_t store_mode;         /* kvx_mode                                       */

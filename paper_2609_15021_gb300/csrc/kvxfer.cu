@@ -20,9 +20,13 @@
 #include <stdlib.h>
 #include <string.h>
 
+#include <unistd.h>
+
 #include <algorithm>
 #include <atomic>
+#include <chrono>
 #include <mutex>
+#include <thread>
 #include <new>
 #include <vector>
 
@@ -129,6 +133,8 @@ struct kvx_ctx {
   long long* d_err = nullptr;  // 16-byte allocation: error word, then the timeout flag
   int* d_timeout = nullptr;
   std::mutex mu;
+  // end of this context's last transfer call (host clock, ns), for the host touch
+  int64_t last_call_ns = 0;
   int64_t launches = 0, memcpys = 0;
   int64_t timed[2] = {0, 0}, timed_bytes[2] = {0, 0};
   double timed_ms[2] = {0.0, 0.0};
@@ -638,6 +644,54 @@ int64_t chunk_bytes(const kvx_pool* P, const Geometry& g, int64_t tokens) { retu
 
 namespace {
 
+int64_t now_ns() {
+  return std::chrono::duration_cast<std::chrono::nanoseconds>(std::chrono::steady_clock::now().time_since_epoch())
+      .count();
+}
+
+// A context that began no transfer for this long reads its host chunks' pages
+// before it moves them.  Measured from the previous call's start, since the
+// library does not see when the GPU finishes; 1 s keeps a caller that waits
+// for each 128k-256k transfer before the next (160-350 ms) from touching at
+// every call, and the slowdown after 1 s of idle time was still small (+4 %).
+constexpr int64_t kIdleTouchNs = 1000ll * 1000 * 1000;
+
+// Reads one byte of every host page of the chunks, on up to 16 threads.  On
+// GB300 a transfer through pinned host memory that had sat untouched for
+// seconds ran at half speed or less until the CPU had read the pages (one
+// byte per page, 13.8 ms on one thread for 33 GB, then the restore ran at the
+// link peak).  The reads are volatile and their values unused; the pages
+// are pinned, so no read faults.
+void touch_host_pages(void* const* chunks, const std::vector<int32_t>& tokens, const kvx_pool* P,
+                      const Geometry& g) {
+  const int64_t page = std::max<int64_t>(4096, (int64_t)sysconf(_SC_PAGESIZE));
+  struct Range {
+    const volatile uint8_t* p;
+    int64_t bytes;
+  };
+  std::vector<Range> ranges;
+  int64_t pages = 0;
+  for (size_t i = 0; i < tokens.size(); ++i) {
+    const int64_t bytes = chunk_bytes_of(P, g, tokens[i]);
+    ranges.push_back({(const volatile uint8_t*)chunks[i], bytes});
+    pages += (bytes + page - 1) / page;
+  }
+  const int threads = (int)std::min<int64_t>(16, std::max<int64_t>(1, pages / 4096));
+  auto work = [&](int w) {
+    // pages are dealt out round-robin over the threads, chunk by chunk
+    uint8_t sink = 0;
+    int64_t k = 0;
+    for (const Range& r : ranges)
+      for (int64_t off = 0; off < r.bytes; off += page, ++k)
+        if (k % threads == w) sink ^= r.p[off];
+    (void)sink;
+  };
+  std::vector<std::thread> pool;
+  for (int w = 1; w < threads; ++w) pool.emplace_back(work, w);
+  work(0);
+  for (std::thread& t : pool) t.join();
+}
+
 // The shared body of kv_store / kv_load / kv_pack / kv_unpack.
 kvx_status transfer(kvx_ctx* ctx, const kvx_pool* P, const int32_t* table, int64_t table_len, int64_t t0,
                     int64_t t1, int32_t C, void* const* chunks, int64_t n_chunks, cudaStream_t stream,
@@ -671,6 +725,12 @@ kvx_status transfer(kvx_ctx* ctx, const kvx_pool* P, const int32_t* table, int64
   if (staged && max_layer_bytes > ctx->slot_bytes) return KVX_EINVAL;
 
   std::lock_guard<std::mutex> lock(ctx->mu);
+  const int64_t now = now_ns();
+  if (where == kHostChunks && !(ctx->opts.flags & KVX_FLAG_NO_HOST_TOUCH) && now - ctx->last_call_ns > kIdleTouchNs) {
+    TraceRange trace("kvx host touch after idle time");
+    touch_host_pages(chunks, pl.tokens, P, pl.g);
+  }
+  ctx->last_call_ns = now;
   const bool ordered = (ctx->opts.flags & KVX_FLAG_UNORDERED) == 0;
   // Kernel-only moves (zero-copy or device chunks) run on the caller's stream
   // itself: stream order is the dependency, with no event hop in between.

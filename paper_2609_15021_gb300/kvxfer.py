@@ -22,7 +22,8 @@ KVX_ENOTPINNED, KVX_ECUDA, KVX_ENOMEM, KVX_EDEVICE = -4, -5, -6, -7
 KVX_LAYOUT_HND, KVX_LAYOUT_NHD = 0, 1
 KVX_MODE_AUTO, KVX_MODE_STAGED, KVX_MODE_ZEROCOPY = 0, 1, 2
 KVX_FLAG_TIME_KERNELS, KVX_FLAG_UNORDERED, KVX_FLAG_DEVICE_TMA, KVX_FLAG_DEVICE_LSU = 0x1, 0x2, 0x4, 0x8
-KVX_FLAGS_ALL = 0xF
+KVX_FLAG_NO_HOST_TOUCH = 0x10
+KVX_FLAGS_ALL = 0x1F
 KVX_ETIMEOUT = -10
 KVX_MAX_LAYERS = 128
 KVX_PROBE_RAW, KVX_PROBE_WAIT_THEN_COPY, KVX_PROBE_ASYNC_ON_STREAM = 0, 1, 2

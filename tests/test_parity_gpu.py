@@ -379,3 +379,39 @@ def test_two_contexts_at_once_and_one_context_from_two_threads(orc):
         assert first_mismatch(np_of(got)[:w.size], w) is None
     for got, w in zip(outs[1], want_b):
         assert first_mismatch(np_of(got)[:w.size], w) is None
+
+
+@pytest.mark.parametrize("touch", [True, False])
+def test_calls_after_idle_time(orc, touch):
+    """A context idle for more than 1 s reads one byte per host page of its
+    chunks before a transfer (unless KVX_FLAG_NO_HOST_TOUCH): the store and the
+    restore that follow idle gaps, across several host buffers and a short last
+    chunk, still match the oracle byte for byte."""
+    import time
+    k = kvx()
+    spec = oracle.PoolSpec(4, 96, 16, 8, 128, 2, oracle.HND)
+    C, n_used = 256, 72
+    T = n_used * 16 - 9
+    src_np = host_layers(spec, 31)
+    src, dst = device_pool(spec, src_np), device_pool(spec)
+    ta, tb = synth.permuted_table(96, n_used, 32), synth.permuted_table(96, n_used, 33)
+    ta_d, tb_d = torch.from_numpy(ta).cuda(), torch.from_numpy(tb).cuda()
+    host = pinned_chunks(orc, spec, 0, T, C)
+    ctx = k.kv_ctx_create(0, flags=0 if touch else k.KVX_FLAG_NO_HOST_TOUCH)
+    try:
+        s = torch.cuda.Stream()
+        time.sleep(1.1)
+        k.kv_store(ctx, src, ta_d, 0, T, C, host, stream=s)
+        s.synchronize()
+        time.sleep(1.1)
+        k.kv_load(ctx, dst, tb_d, 0, T, C, host, stream=s)
+        s.synchronize()
+        assert k.kv_get_device_error(ctx) == -1
+    finally:
+        k.kv_ctx_destroy(ctx)
+    want, _ = oracle_store(orc, spec, src_np, ta, 0, T, C)
+    for c, w in enumerate(want):
+        assert first_mismatch(np_of(host[c]), w) is None, c
+    loaded, _ = oracle_load(orc, spec, [np.full(spec.layer_bytes, POISON, np.uint8)] * 4, tb, 0, T, C, want)
+    for l in range(4):
+        assert first_mismatch(np_of(dst.layers[l]), loaded[l]) is None, l
