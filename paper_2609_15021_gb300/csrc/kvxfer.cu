@@ -687,7 +687,14 @@ void touch_host_pages(void* const* chunks, const std::vector<int32_t>& tokens, c
     (void)sink;
   };
   std::vector<std::thread> pool;
-  for (int w = 1; w < threads; ++w) pool.emplace_back(work, w);
+  int w = 1;
+  try {
+    pool.reserve((size_t)threads);
+    for (; w < threads; ++w) pool.emplace_back(work, w);
+  } catch (...) {
+    // no more threads to be had: the calling thread takes the rest
+  }
+  for (int r = w; r < threads; ++r) work(r);
   work(0);
   for (std::thread& t : pool) t.join();
 }
@@ -728,7 +735,11 @@ kvx_status transfer(kvx_ctx* ctx, const kvx_pool* P, const int32_t* table, int64
   const int64_t now = now_ns();
   if (where == kHostChunks && !(ctx->opts.flags & KVX_FLAG_NO_HOST_TOUCH) && now - ctx->last_call_ns > kIdleTouchNs) {
     TraceRange trace("kvx host touch after idle time");
-    touch_host_pages(chunks, pl.tokens, P, pl.g);
+    try {
+      touch_host_pages(chunks, pl.tokens, P, pl.g);
+    } catch (...) {
+      // only a speed-up: the transfer goes ahead without it
+    }
   }
   ctx->last_call_ns = now;
   const bool ordered = (ctx->opts.flags & KVX_FLAG_UNORDERED) == 0;
