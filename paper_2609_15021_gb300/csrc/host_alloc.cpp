@@ -259,60 +259,62 @@ kvx_status map_pool(int node, int64_t bytes, bool huge_pages, void** out, bool* 
 extern "C" {
 
 kvx_status kv_host_alloc_ex(int64_t bytes, int32_t numa_node, uint32_t flags, void** out, int32_t* numa_out) {
-  if (!out) return KVX_EINVAL;
-  *out = nullptr;
-  if (numa_out) *numa_out = -1;
-  if (bytes <= 0 || numa_node < KVX_NUMA_ANY || numa_node >= kMaxNodes ||
-      (flags & ~(KVX_HOST_DRIVER | KVX_HOST_HUGE)))
-    return KVX_EINVAL;
-  if ((flags & KVX_HOST_DRIVER) && (numa_node != KVX_NUMA_ANY || (flags & KVX_HOST_HUGE))) return KVX_EINVAL;
-  if (fault_point("host_alloc")) {
-    set_last_cuda_error((int)cudaErrorMemoryAllocation);
-    set_error_text("pinning of the host pool (injected fault)");
-    return KVX_ENOMEM;
-  }
-  // Without a placement, the driver's allocator unless huge pages are asked
-  // for (and can be had); a placement needs the library's own mapping.
-  // Huge pages where rounding the pool up to whole huge pages wastes at most
-  // an eighth of it.
-  const size_t huge = thp_available() ? huge_page_bytes() : 0;
-  const size_t rounded = huge ? ((size_t)bytes + huge - 1) / huge * huge : 0;
-  const bool huge_fits = huge != 0 && (rounded - (size_t)bytes) * 8 <= (size_t)bytes;
-  if (numa_node == KVX_NUMA_ANY && (!(flags & KVX_HOST_HUGE) || !huge_fits)) return driver_pool(bytes, out);
-  int node = numa_node;
-  if (node == KVX_NUMA_ANY) {
-    node = -1;
-  } else if (node == KVX_NUMA_NEAREST) {
-    int dev = 0, id = -1;
-    if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&id, cudaDevAttrHostNumaId, dev) != cudaSuccess)
-      id = -1;
-    cudaGetLastError();
-    node = id >= 0 && id < kMaxNodes && node_exists(id) ? id : -1;  // -1: no placement asked
-  } else if (!node_exists(node)) {
-    set_error_text("no such host NUMA node");
-    return KVX_EINVAL;
-  }
-  if (node >= 0) {
-    const int64_t avail = node_free_bytes(node);
-    if (avail >= 0 && avail < bytes) {
-      set_error_text("the NUMA node has less free memory than requested");
+  return guarded([&]() -> kvx_status {
+    if (!out) return KVX_EINVAL;
+    *out = nullptr;
+    if (numa_out) *numa_out = -1;
+    if (bytes <= 0 || numa_node < KVX_NUMA_ANY || numa_node >= kMaxNodes ||
+        (flags & ~(KVX_HOST_DRIVER | KVX_HOST_HUGE)))
+      return KVX_EINVAL;
+    if ((flags & KVX_HOST_DRIVER) && (numa_node != KVX_NUMA_ANY || (flags & KVX_HOST_HUGE))) return KVX_EINVAL;
+    if (fault_point("host_alloc")) {
+      set_last_cuda_error((int)cudaErrorMemoryAllocation);
+      set_error_text("pinning of the host pool (injected fault)");
       return KVX_ENOMEM;
     }
-  }
-  // If huge pages cannot back all of it: the driver's allocator (no placement
-  // asked) or base pages (placement asked).
-  bool partial = false;
-  kvx_status st = KVX_ENOMEM;
-  if (huge_fits) {
-    st = map_pool(node, bytes, true, out, &partial);
-    if (st != KVX_OK && !partial) return st;
-  }
-  if (st != KVX_OK) {
-    if (numa_node == KVX_NUMA_ANY) return driver_pool(bytes, out);
-    st = map_pool(node, bytes, false, out, &partial);
-  }
-  if (st == KVX_OK && numa_out) *numa_out = page_node(*out);
-  return st;
+    // Without a placement, the driver's allocator unless huge pages are asked
+    // for (and can be had); a placement needs the library's own mapping.
+    // Huge pages where rounding the pool up to whole huge pages wastes at most
+    // an eighth of it.
+    const size_t huge = thp_available() ? huge_page_bytes() : 0;
+    const size_t rounded = huge ? ((size_t)bytes + huge - 1) / huge * huge : 0;
+    const bool huge_fits = huge != 0 && (rounded - (size_t)bytes) * 8 <= (size_t)bytes;
+    if (numa_node == KVX_NUMA_ANY && (!(flags & KVX_HOST_HUGE) || !huge_fits)) return driver_pool(bytes, out);
+    int node = numa_node;
+    if (node == KVX_NUMA_ANY) {
+      node = -1;
+    } else if (node == KVX_NUMA_NEAREST) {
+      int dev = 0, id = -1;
+      if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&id, cudaDevAttrHostNumaId, dev) != cudaSuccess)
+        id = -1;
+      cudaGetLastError();
+      node = id >= 0 && id < kMaxNodes && node_exists(id) ? id : -1;  // -1: no placement asked
+    } else if (!node_exists(node)) {
+      set_error_text("no such host NUMA node");
+      return KVX_EINVAL;
+    }
+    if (node >= 0) {
+      const int64_t avail = node_free_bytes(node);
+      if (avail >= 0 && avail < bytes) {
+        set_error_text("the NUMA node has less free memory than requested");
+        return KVX_ENOMEM;
+      }
+    }
+    // If huge pages cannot back all of it: the driver's allocator (no placement
+    // asked) or base pages (placement asked).
+    bool partial = false;
+    kvx_status st = KVX_ENOMEM;
+    if (huge_fits) {
+      st = map_pool(node, bytes, true, out, &partial);
+      if (st != KVX_OK && !partial) return st;
+    }
+    if (st != KVX_OK) {
+      if (numa_node == KVX_NUMA_ANY) return driver_pool(bytes, out);
+      st = map_pool(node, bytes, false, out, &partial);
+    }
+    if (st == KVX_OK && numa_out) *numa_out = page_node(*out);
+    return st;
+  });
 }
 
 kvx_status kv_host_pool_info(const void* host, kvx_host_pool_info* info) {

@@ -4,6 +4,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <new>
+
 #include "kvxfer.h"
 
 namespace kvx {
@@ -124,5 +126,20 @@ void set_last_cuda_error(int e);
 
 // Host-side fault injection (kv_fault_inject): true if the armed point fails now.
 bool fault_point(const char* point);
+
+// Runs an entry point's body so that no C++ exception leaves the C ABI: a
+// failed host allocation (a caller's absurd count, say) returns KVX_ENOMEM.
+template <class F>
+kvx_status guarded(F&& body) {
+  try {
+    return body();
+  } catch (const std::bad_alloc&) {
+    set_error_text("out of host memory");
+    return KVX_ENOMEM;
+  } catch (...) {
+    set_error_text("unexpected failure inside the library");
+    return KVX_EINVAL;
+  }
+}
 
 }  // namespace kvx

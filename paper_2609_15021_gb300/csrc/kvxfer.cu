@@ -926,76 +926,78 @@ const char* kv_status_string(kvx_status s) {
 }
 
 kvx_status kv_ctx_create(int device, const kvx_opts* opts, kvx_ctx** out) {
-  if (!out) return KVX_EINVAL;
-  *out = nullptr;
-  kvx_opts o{};
-  if (opts) o = *opts;
-  for (int32_t m : {o.store_mode, o.load_mode})
-    if (m != KVX_MODE_AUTO && m != KVX_MODE_STAGED && m != KVX_MODE_ZEROCOPY) return KVX_EINVAL;
-  if (o.staging_slots != 0 && o.staging_slots < 2) return KVX_EINVAL;
-  if (o.staging_slots > 64) return KVX_EINVAL;
-  if (o.staging_slot_bytes < 0 || o.staging_slot_bytes % 16 != 0) return KVX_EINVAL;
-  if (o.max_ctas < 0) return KVX_EINVAL;
-  if (o.flags & ~KVX_FLAGS_ALL) return KVX_EINVAL;
-  if ((o.flags & KVX_FLAG_DEVICE_TMA) && (o.flags & KVX_FLAG_DEVICE_LSU)) return KVX_EINVAL;
-  int count = 0;
-  if (cudaGetDeviceCount(&count) != cudaSuccess) {
-    g_last_cuda_error = (int)cudaGetLastError();
-    return KVX_ECUDA;
-  }
-  if (device < 0 || device >= count) return KVX_EINVAL;
-  DeviceGuard guard(device);
-  if (!guard.ok) return KVX_ECUDA;
-  kvx_ctx* ctx = new (std::nothrow) kvx_ctx;
-  if (!ctx) return KVX_ENOMEM;
-  ctx->device = device;
-  ctx->opts = o;
-  ctx->store_mode = resolve_mode(o.store_mode);
-  ctx->load_mode = resolve_mode(o.load_mode);
-  ctx->nslots = o.staging_slots ? o.staging_slots : kDefaultSlots;
-  ctx->slot_bytes = o.staging_slot_bytes ? o.staging_slot_bytes : kDefaultSlotBytes;
-  auto fail = [&](cudaError_t e) {
-    g_last_cuda_error = (int)e;
-    cudaGetLastError();
-    destroy_ctx(ctx);
-    return e == cudaErrorMemoryAllocation ? KVX_ENOMEM : KVX_ECUDA;
-  };
-  cudaError_t e;
-  if ((e = cudaDeviceGetAttribute(&ctx->num_sms, cudaDevAttrMultiProcessorCount, device)) != cudaSuccess)
-    return fail(e);
-  // Host-link launches: half the SMs.  A quarter already saturates the link on
-  // an idle GPU; half keeps it within 2-4 % of that while a full-GPU GEMM runs
-  // beside the transfer (a quarter then loses 16-21 %), for 1-2 % more GEMM time.
-  ctx->link_ctas = std::max(1, (ctx->num_sms + 1) / 2);
-  if ((e = cudaStreamCreateWithFlags(&ctx->s_kern, cudaStreamNonBlocking)) != cudaSuccess) return fail(e);
-  if ((e = cudaStreamCreateWithFlags(&ctx->s_copy, cudaStreamNonBlocking)) != cudaSuccess) return fail(e);
-  if ((e = cudaStreamCreateWithFlags(&ctx->s_aux, cudaStreamNonBlocking)) != cudaSuccess) return fail(e);
-  for (cudaEvent_t* ev : {&ctx->ev_in, &ctx->ev_kern_done, &ctx->ev_copy_done})
-    if ((e = cudaEventCreateWithFlags(ev, cudaEventDisableTiming)) != cudaSuccess) return fail(e);
-  for (int32_t k = 0; k < ctx->nslots; ++k) {
-    cudaEvent_t a = nullptr, b = nullptr;
-    if ((e = cudaEventCreateWithFlags(&a, cudaEventDisableTiming)) != cudaSuccess) return fail(e);
-    ctx->ev_ready.push_back(a);
-    if ((e = cudaEventCreateWithFlags(&b, cudaEventDisableTiming)) != cudaSuccess) return fail(e);
-    ctx->ev_free.push_back(b);
-  }
-  if ((e = cudaMalloc(&ctx->d_err, 16)) != cudaSuccess) return fail(e);
-  ctx->d_timeout = reinterpret_cast<int*>(ctx->d_err + 1);
-  const long long init[2] = {kNoError, 0};
-  if ((e = cudaMemcpy(ctx->d_err, init, sizeof(init), cudaMemcpyHostToDevice)) != cudaSuccess) return fail(e);
-  for (int d = 0; d < 2; ++d)
-    for (int l = 0; l < 2; ++l) ctx->move_occ[d][l] = move_ctas_per_sm(d, l);
-  ctx->seg_occ = segment_ctas_per_sm();
-  if ((e = prepare_tma_kernels()) != cudaSuccess) return fail(e);
-  if (ctx->store_mode == KVX_MODE_STAGED || ctx->load_mode == KVX_MODE_STAGED) {
-    kvx_status st = ensure_staging(ctx);
-    if (st != KVX_OK) {
-      destroy_ctx(ctx);
-      return st;
+  return guarded([&]() -> kvx_status {
+    if (!out) return KVX_EINVAL;
+    *out = nullptr;
+    kvx_opts o{};
+    if (opts) o = *opts;
+    for (int32_t m : {o.store_mode, o.load_mode})
+      if (m != KVX_MODE_AUTO && m != KVX_MODE_STAGED && m != KVX_MODE_ZEROCOPY) return KVX_EINVAL;
+    if (o.staging_slots != 0 && o.staging_slots < 2) return KVX_EINVAL;
+    if (o.staging_slots > 64) return KVX_EINVAL;
+    if (o.staging_slot_bytes < 0 || o.staging_slot_bytes % 16 != 0) return KVX_EINVAL;
+    if (o.max_ctas < 0) return KVX_EINVAL;
+    if (o.flags & ~KVX_FLAGS_ALL) return KVX_EINVAL;
+    if ((o.flags & KVX_FLAG_DEVICE_TMA) && (o.flags & KVX_FLAG_DEVICE_LSU)) return KVX_EINVAL;
+    int count = 0;
+    if (cudaGetDeviceCount(&count) != cudaSuccess) {
+      g_last_cuda_error = (int)cudaGetLastError();
+      return KVX_ECUDA;
     }
-  }
-  *out = ctx;
-  return KVX_OK;
+    if (device < 0 || device >= count) return KVX_EINVAL;
+    DeviceGuard guard(device);
+    if (!guard.ok) return KVX_ECUDA;
+    kvx_ctx* ctx = new (std::nothrow) kvx_ctx;
+    if (!ctx) return KVX_ENOMEM;
+    ctx->device = device;
+    ctx->opts = o;
+    ctx->store_mode = resolve_mode(o.store_mode);
+    ctx->load_mode = resolve_mode(o.load_mode);
+    ctx->nslots = o.staging_slots ? o.staging_slots : kDefaultSlots;
+    ctx->slot_bytes = o.staging_slot_bytes ? o.staging_slot_bytes : kDefaultSlotBytes;
+    auto fail = [&](cudaError_t e) {
+      g_last_cuda_error = (int)e;
+      cudaGetLastError();
+      destroy_ctx(ctx);
+      return e == cudaErrorMemoryAllocation ? KVX_ENOMEM : KVX_ECUDA;
+    };
+    cudaError_t e;
+    if ((e = cudaDeviceGetAttribute(&ctx->num_sms, cudaDevAttrMultiProcessorCount, device)) != cudaSuccess)
+      return fail(e);
+    // Host-link launches: half the SMs.  A quarter already saturates the link on
+    // an idle GPU; half keeps it within 2-4 % of that while a full-GPU GEMM runs
+    // beside the transfer (a quarter then loses 16-21 %), for 1-2 % more GEMM time.
+    ctx->link_ctas = std::max(1, (ctx->num_sms + 1) / 2);
+    if ((e = cudaStreamCreateWithFlags(&ctx->s_kern, cudaStreamNonBlocking)) != cudaSuccess) return fail(e);
+    if ((e = cudaStreamCreateWithFlags(&ctx->s_copy, cudaStreamNonBlocking)) != cudaSuccess) return fail(e);
+    if ((e = cudaStreamCreateWithFlags(&ctx->s_aux, cudaStreamNonBlocking)) != cudaSuccess) return fail(e);
+    for (cudaEvent_t* ev : {&ctx->ev_in, &ctx->ev_kern_done, &ctx->ev_copy_done})
+      if ((e = cudaEventCreateWithFlags(ev, cudaEventDisableTiming)) != cudaSuccess) return fail(e);
+    for (int32_t k = 0; k < ctx->nslots; ++k) {
+      cudaEvent_t a = nullptr, b = nullptr;
+      if ((e = cudaEventCreateWithFlags(&a, cudaEventDisableTiming)) != cudaSuccess) return fail(e);
+      ctx->ev_ready.push_back(a);
+      if ((e = cudaEventCreateWithFlags(&b, cudaEventDisableTiming)) != cudaSuccess) return fail(e);
+      ctx->ev_free.push_back(b);
+    }
+    if ((e = cudaMalloc(&ctx->d_err, 16)) != cudaSuccess) return fail(e);
+    ctx->d_timeout = reinterpret_cast<int*>(ctx->d_err + 1);
+    const long long init[2] = {kNoError, 0};
+    if ((e = cudaMemcpy(ctx->d_err, init, sizeof(init), cudaMemcpyHostToDevice)) != cudaSuccess) return fail(e);
+    for (int d = 0; d < 2; ++d)
+      for (int l = 0; l < 2; ++l) ctx->move_occ[d][l] = move_ctas_per_sm(d, l);
+    ctx->seg_occ = segment_ctas_per_sm();
+    if ((e = prepare_tma_kernels()) != cudaSuccess) return fail(e);
+    if (ctx->store_mode == KVX_MODE_STAGED || ctx->load_mode == KVX_MODE_STAGED) {
+      kvx_status st = ensure_staging(ctx);
+      if (st != KVX_OK) {
+        destroy_ctx(ctx);
+        return st;
+      }
+    }
+    *out = ctx;
+    return KVX_OK;
+  });
 }
 
 void kv_ctx_destroy(kvx_ctx* ctx) { destroy_ctx(ctx); }
@@ -1027,47 +1029,59 @@ kvx_status kv_chunk_layout(const kvx_pool* pool, int32_t chunk_tokens, int32_t t
 kvx_status kv_store(kvx_ctx* ctx, const kvx_pool* pool, const int32_t* block_table, int64_t table_len,
                     int64_t tok_begin, int64_t tok_end, int32_t chunk_tokens, void* const* host_chunks,
                     int64_t n_chunks, kvx_stream_t stream) {
-  TraceRange trace("kv_store");
-  return transfer(ctx, pool, block_table, table_len, tok_begin, tok_end, chunk_tokens, host_chunks, n_chunks,
-                  (cudaStream_t)stream, kPack, kHostChunks);
+  return guarded([&]() -> kvx_status {
+    TraceRange trace("kv_store");
+    return transfer(ctx, pool, block_table, table_len, tok_begin, tok_end, chunk_tokens, host_chunks, n_chunks,
+                    (cudaStream_t)stream, kPack, kHostChunks);
+  });
 }
 
 kvx_status kv_load(kvx_ctx* ctx, const kvx_pool* pool, const int32_t* block_table, int64_t table_len,
                    int64_t tok_begin, int64_t tok_end, int32_t chunk_tokens, const void* const* host_chunks,
                    int64_t n_chunks, kvx_stream_t stream) {
-  TraceRange trace("kv_load");
-  return transfer(ctx, pool, block_table, table_len, tok_begin, tok_end, chunk_tokens,
-                  const_cast<void* const*>(host_chunks), n_chunks, (cudaStream_t)stream, kUnpack, kHostChunks);
+  return guarded([&]() -> kvx_status {
+    TraceRange trace("kv_load");
+    return transfer(ctx, pool, block_table, table_len, tok_begin, tok_end, chunk_tokens,
+                    const_cast<void* const*>(host_chunks), n_chunks, (cudaStream_t)stream, kUnpack, kHostChunks);
+  });
 }
 
 kvx_status kv_pack(kvx_ctx* ctx, const kvx_pool* pool, const int32_t* block_table, int64_t table_len,
                    int64_t tok_begin, int64_t tok_end, int32_t chunk_tokens, void* const* dev_chunks,
                    int64_t n_chunks, kvx_stream_t stream) {
-  TraceRange trace("kv_pack");
-  return transfer(ctx, pool, block_table, table_len, tok_begin, tok_end, chunk_tokens, dev_chunks, n_chunks,
-                  (cudaStream_t)stream, kPack, kDeviceChunks);
+  return guarded([&]() -> kvx_status {
+    TraceRange trace("kv_pack");
+    return transfer(ctx, pool, block_table, table_len, tok_begin, tok_end, chunk_tokens, dev_chunks, n_chunks,
+                    (cudaStream_t)stream, kPack, kDeviceChunks);
+  });
 }
 
 kvx_status kv_unpack(kvx_ctx* ctx, const kvx_pool* pool, const int32_t* block_table, int64_t table_len,
                      int64_t tok_begin, int64_t tok_end, int32_t chunk_tokens, const void* const* dev_chunks,
                      int64_t n_chunks, kvx_stream_t stream) {
-  TraceRange trace("kv_unpack");
-  return transfer(ctx, pool, block_table, table_len, tok_begin, tok_end, chunk_tokens,
-                  const_cast<void* const*>(dev_chunks), n_chunks, (cudaStream_t)stream, kUnpack, kDeviceChunks);
+  return guarded([&]() -> kvx_status {
+    TraceRange trace("kv_unpack");
+    return transfer(ctx, pool, block_table, table_len, tok_begin, tok_end, chunk_tokens,
+                    const_cast<void* const*>(dev_chunks), n_chunks, (cudaStream_t)stream, kUnpack, kDeviceChunks);
+  });
 }
 
 kvx_status kv_state_store(kvx_ctx* ctx, int32_t num_layers, void* const* layer_base, int64_t num_slots,
                           int64_t slot_bytes, int64_t slot, void* host_obj, kvx_stream_t stream) {
-  TraceRange trace("kv_state_store");
-  return state_copy(ctx, num_layers, layer_base, num_slots, slot_bytes, slot, host_obj, (cudaStream_t)stream,
-                    true);
+  return guarded([&]() -> kvx_status {
+    TraceRange trace("kv_state_store");
+    return state_copy(ctx, num_layers, layer_base, num_slots, slot_bytes, slot, host_obj, (cudaStream_t)stream,
+                      true);
+  });
 }
 
 kvx_status kv_state_load(kvx_ctx* ctx, int32_t num_layers, void* const* layer_base, int64_t num_slots,
                          int64_t slot_bytes, int64_t slot, const void* host_obj, kvx_stream_t stream) {
-  TraceRange trace("kv_state_load");
-  return state_copy(ctx, num_layers, layer_base, num_slots, slot_bytes, slot, const_cast<void*>(host_obj),
-                    (cudaStream_t)stream, false);
+  return guarded([&]() -> kvx_status {
+    TraceRange trace("kv_state_load");
+    return state_copy(ctx, num_layers, layer_base, num_slots, slot_bytes, slot, const_cast<void*>(host_obj),
+                      (cudaStream_t)stream, false);
+  });
 }
 
 kvx_status kv_fault_inject(const char* point, int32_t after_calls) {
@@ -1186,29 +1200,31 @@ kvx_status kv_get_device_error(kvx_ctx* ctx, int64_t* first_bad_block) {
 }
 
 kvx_status kv_ctx_stats(kvx_ctx* ctx, kvx_stats* out) {
-  if (!ctx || !out) return KVX_EINVAL;
-  DeviceGuard guard(ctx->device);
-  if (!guard.ok) return KVX_ECUDA;
-  std::lock_guard<std::mutex> lock(ctx->mu);
-  for (const TimedLaunch& t : ctx->pending) {
-    KVX_CUDA(cudaEventSynchronize(t.b));
-    float ms = 0.f;
-    KVX_CUDA(cudaEventElapsedTime(&ms, t.a, t.b));
-    ctx->timed_ms[t.dir] += ms;
-    ctx->timed[t.dir]++;
-    ctx->timed_bytes[t.dir] += t.bytes;
-    ctx->spare_events.push_back(t.a);
-    ctx->spare_events.push_back(t.b);
-  }
-  ctx->pending.clear();
-  out->kernel_launches = ctx->launches;
-  out->memcpy_calls = ctx->memcpys;
-  for (int d = 0; d < 2; ++d) {
-    out->timed_launches[d] = ctx->timed[d];
-    out->kernel_ms[d] = ctx->timed_ms[d];
-    out->kernel_bytes[d] = ctx->timed_bytes[d];
-  }
-  return KVX_OK;
+  return guarded([&]() -> kvx_status {
+    if (!ctx || !out) return KVX_EINVAL;
+    DeviceGuard guard(ctx->device);
+    if (!guard.ok) return KVX_ECUDA;
+    std::lock_guard<std::mutex> lock(ctx->mu);
+    for (const TimedLaunch& t : ctx->pending) {
+      KVX_CUDA(cudaEventSynchronize(t.b));
+      float ms = 0.f;
+      KVX_CUDA(cudaEventElapsedTime(&ms, t.a, t.b));
+      ctx->timed_ms[t.dir] += ms;
+      ctx->timed[t.dir]++;
+      ctx->timed_bytes[t.dir] += t.bytes;
+      ctx->spare_events.push_back(t.a);
+      ctx->spare_events.push_back(t.b);
+    }
+    ctx->pending.clear();
+    out->kernel_launches = ctx->launches;
+    out->memcpy_calls = ctx->memcpys;
+    for (int d = 0; d < 2; ++d) {
+      out->timed_launches[d] = ctx->timed[d];
+      out->kernel_ms[d] = ctx->timed_ms[d];
+      out->kernel_bytes[d] = ctx->timed_bytes[d];
+    }
+    return KVX_OK;
+  });
 }
 
 kvx_status kv_ctx_reset_stats(kvx_ctx* ctx) {

@@ -542,159 +542,167 @@ kvx_status kv_chunk_keys(const int32_t* tokens, int64_t n_tokens, int32_t chunk_
 }
 
 kvx_status kv_tier_create_on(void* base, int64_t slot_bytes, int64_t n_slots, kvx_tier** out) {
-  if (!out) return KVX_EINVAL;
-  *out = nullptr;
-  if (!base || slot_bytes < 16 || slot_bytes % 16 != 0 || n_slots < 1) return KVX_EINVAL;
-  if ((uintptr_t)base & 15) return KVX_EALIGN;
-  return init_private(base, slot_bytes, n_slots, out);
+  return guarded([&]() -> kvx_status {
+    if (!out) return KVX_EINVAL;
+    *out = nullptr;
+    if (!base || slot_bytes < 16 || slot_bytes % 16 != 0 || n_slots < 1) return KVX_EINVAL;
+    if ((uintptr_t)base & 15) return KVX_EALIGN;
+    return init_private(base, slot_bytes, n_slots, out);
+  });
 }
 
 kvx_status kv_tier_create(int64_t slot_bytes, int64_t n_slots, kvx_tier** out) {
-  if (!out) return KVX_EINVAL;
-  *out = nullptr;
-  if (slot_bytes < 16 || slot_bytes % 16 != 0 || n_slots < 1) return KVX_EINVAL;
-  if (n_slots > INT64_MAX / slot_bytes) return KVX_EINVAL;
-  void* p = nullptr;
-  kvx_status st = kv_host_alloc(slot_bytes * n_slots, &p);
-  if (st != KVX_OK) return st;
-  st = init_private(p, slot_bytes, n_slots, out);
-  if (st != KVX_OK) {
-    kv_host_free(p);
-    return st;
-  }
-  (*out)->owns_data = true;
-  return KVX_OK;
+  return guarded([&]() -> kvx_status {
+    if (!out) return KVX_EINVAL;
+    *out = nullptr;
+    if (slot_bytes < 16 || slot_bytes % 16 != 0 || n_slots < 1) return KVX_EINVAL;
+    if (n_slots > INT64_MAX / slot_bytes) return KVX_EINVAL;
+    void* p = nullptr;
+    kvx_status st = kv_host_alloc(slot_bytes * n_slots, &p);
+    if (st != KVX_OK) return st;
+    st = init_private(p, slot_bytes, n_slots, out);
+    if (st != KVX_OK) {
+      kv_host_free(p);
+      return st;
+    }
+    (*out)->owns_data = true;
+    return KVX_OK;
+  });
 }
 
 kvx_status kv_tier_open_shared(const char* name, int64_t slot_bytes, int64_t n_slots, uint32_t flags,
                                kvx_tier** out) {
-  if (!out || !name || name[0] != '/' || strlen(name) >= 120) return KVX_EINVAL;
-  *out = nullptr;
-  const bool create = (flags & KVX_TIER_CREATE) != 0;
-  if (create && (slot_bytes < 16 || slot_bytes % 16 != 0 || n_slots < 1)) return KVX_EINVAL;
-  const int fd = shm_open(name, create ? (O_CREAT | O_EXCL | O_RDWR) : O_RDWR, 0600);
-  if (fd < 0) {
-    set_error_text(create ? "shm_open: the name exists or cannot be created" : "shm_open: no such tier");
-    return create ? KVX_EINVAL : KVX_ENOENT;
-  }
-  int64_t total = 0, data_offset = 0;
-  if (create) {
-    const int64_t meta_bytes = metadata_bytes(n_slots);
-    data_offset = (meta_bytes + kDataAlign - 1) / kDataAlign * kDataAlign;
-    if (n_slots > (INT64_MAX - data_offset) / slot_bytes) {
-      close(fd);
-      shm_unlink(name);
-      return KVX_EINVAL;
+  return guarded([&]() -> kvx_status {
+    if (!out || !name || name[0] != '/' || strlen(name) >= 120) return KVX_EINVAL;
+    *out = nullptr;
+    const bool create = (flags & KVX_TIER_CREATE) != 0;
+    if (create && (slot_bytes < 16 || slot_bytes % 16 != 0 || n_slots < 1)) return KVX_EINVAL;
+    const int fd = shm_open(name, create ? (O_CREAT | O_EXCL | O_RDWR) : O_RDWR, 0600);
+    if (fd < 0) {
+      set_error_text(create ? "shm_open: the name exists or cannot be created" : "shm_open: no such tier");
+      return create ? KVX_EINVAL : KVX_ENOENT;
     }
-    total = data_offset + slot_bytes * n_slots;
-    if (ftruncate(fd, (off_t)total) != 0) {
-      close(fd);
-      shm_unlink(name);
-      set_error_text("ftruncate of the shared tier failed");
+    int64_t total = 0, data_offset = 0;
+    if (create) {
+      const int64_t meta_bytes = metadata_bytes(n_slots);
+      data_offset = (meta_bytes + kDataAlign - 1) / kDataAlign * kDataAlign;
+      if (n_slots > (INT64_MAX - data_offset) / slot_bytes) {
+        close(fd);
+        shm_unlink(name);
+        return KVX_EINVAL;
+      }
+      total = data_offset + slot_bytes * n_slots;
+      if (ftruncate(fd, (off_t)total) != 0) {
+        close(fd);
+        shm_unlink(name);
+        set_error_text("ftruncate of the shared tier failed");
+        return KVX_ENOMEM;
+      }
+      // Reserve the pages now: a shared-memory file system without room for
+      // them would otherwise end the process with SIGBUS at first touch.
+      const int fr = posix_fallocate(fd, 0, (off_t)total);
+      if (fr != 0 && fr != EOPNOTSUPP && fr != EINVAL) {
+        close(fd);
+        shm_unlink(name);
+        set_error_text("the shared-memory file system has no room for the tier");
+        return KVX_ENOMEM;
+      }
+    } else {
+      struct stat sb;
+      // wait (bounded) for the creator to size and initialise the region
+      for (int i = 0; i < 5000; ++i) {
+        if (fstat(fd, &sb) == 0 && sb.st_size >= (off_t)sizeof(Header)) break;
+        usleep(1000);
+      }
+      if (fstat(fd, &sb) != 0 || sb.st_size < (off_t)sizeof(Header)) {
+        close(fd);
+        return KVX_ENOENT;
+      }
+      total = (int64_t)sb.st_size;
+    }
+    void* map = mmap(nullptr, (size_t)total, PROT_READ | PROT_WRITE, MAP_SHARED, fd, 0);
+    close(fd);
+    if (map == MAP_FAILED) {
+      if (create) shm_unlink(name);
       return KVX_ENOMEM;
     }
-    // Reserve the pages now: a shared-memory file system without room for
-    // them would otherwise end the process with SIGBUS at first touch.
-    const int fr = posix_fallocate(fd, 0, (off_t)total);
-    if (fr != 0 && fr != EOPNOTSUPP && fr != EINVAL) {
-      close(fd);
-      shm_unlink(name);
-      set_error_text("the shared-memory file system has no room for the tier");
-      return KVX_ENOMEM;
-    }
-  } else {
-    struct stat sb;
-    // wait (bounded) for the creator to size and initialise the region
-    for (int i = 0; i < 5000; ++i) {
-      if (fstat(fd, &sb) == 0 && sb.st_size >= (off_t)sizeof(Header)) break;
-      usleep(1000);
-    }
-    if (fstat(fd, &sb) != 0 || sb.st_size < (off_t)sizeof(Header)) {
-      close(fd);
-      return KVX_ENOENT;
-    }
-    total = (int64_t)sb.st_size;
-  }
-  void* map = mmap(nullptr, (size_t)total, PROT_READ | PROT_WRITE, MAP_SHARED, fd, 0);
-  close(fd);
-  if (map == MAP_FAILED) {
-    if (create) shm_unlink(name);
-    return KVX_ENOMEM;
-  }
-  kvx_tier* t = new (std::nothrow) kvx_tier;
-  if (!t) {
-    munmap(map, (size_t)total);
-    if (create) shm_unlink(name);
-    return KVX_ENOMEM;
-  }
-  t->shared = true;
-  t->creator = create;
-  t->mapping = map;
-  t->mapping_bytes = total;
-  t->pid = (int32_t)getpid();
-  snprintf(t->name, sizeof(t->name), "%s", name);
-  Header* h = (Header*)map;
-  t->hdr = h;
-  if (create) {
-    h->magic = kMagic;
-    h->slot_bytes = slot_bytes;
-    h->n_slots = n_slots;
-    h->data_offset = data_offset;
-    h->total_bytes = total;
-    h->index_size = index_size_for(n_slots);
-    attach_metadata(t, map);
-    memset(t->index, 0xFF, (size_t)h->index_size * 8);  // every entry -1: empty
-    pthread_mutexattr_t a;
-    pthread_mutexattr_init(&a);
-    pthread_mutexattr_setpshared(&a, PTHREAD_PROCESS_SHARED);
-    pthread_mutexattr_setrobust(&a, PTHREAD_MUTEX_ROBUST);
-    pthread_mutex_init(&h->mu, &a);
-    pthread_mutexattr_destroy(&a);
-    __atomic_store_n(&h->initialised, 1, __ATOMIC_RELEASE);
-  } else {
-    int i = 0;
-    while (__atomic_load_n(&h->initialised, __ATOMIC_ACQUIRE) != 1 && i++ < 5000) usleep(1000);
-    if (h->initialised != 1 || h->magic != kMagic || h->total_bytes != total ||
-        h->index_size != index_size_for(h->n_slots) || metadata_bytes(h->n_slots) > h->data_offset) {
+    kvx_tier* t = new (std::nothrow) kvx_tier;
+    if (!t) {
       munmap(map, (size_t)total);
-      delete t;
-      set_error_text("the shared tier is not initialised or does not match");
-      return KVX_EINVAL;
+      if (create) shm_unlink(name);
+      return KVX_ENOMEM;
     }
-    attach_metadata(t, map);
-  }
-  t->data = (uint8_t*)map + h->data_offset;
-  // Shared memory is kept on base pages: the SMs' zero-copy accesses run at the
-  // link peak on them, and a mixture of page sizes slowed zero-copy on GB300
-  // to a third.  (The copy engines are slow on base pages: with a shared tier,
-  // zero-copy, the default mode, is the one to use.)
-  madvise(t->data, (size_t)(h->slot_bytes * h->n_slots), MADV_NOHUGEPAGE);
-  if (!(flags & KVX_TIER_NO_PIN)) {
-    // The whole region, slot table included: the GPU publishes commits into it.
-    const cudaError_t e = cudaHostRegister(map, (size_t)total, cudaHostRegisterPortable | cudaHostRegisterMapped);
-    if (e != cudaSuccess) {
-      kvx_status st = cuda_fail(e, "cudaHostRegister of the shared tier");
-      t->creator = create;
-      destroy_tier(t);
-      return st;
+    t->shared = true;
+    t->creator = create;
+    t->mapping = map;
+    t->mapping_bytes = total;
+    t->pid = (int32_t)getpid();
+    snprintf(t->name, sizeof(t->name), "%s", name);
+    Header* h = (Header*)map;
+    t->hdr = h;
+    if (create) {
+      h->magic = kMagic;
+      h->slot_bytes = slot_bytes;
+      h->n_slots = n_slots;
+      h->data_offset = data_offset;
+      h->total_bytes = total;
+      h->index_size = index_size_for(n_slots);
+      attach_metadata(t, map);
+      memset(t->index, 0xFF, (size_t)h->index_size * 8);  // every entry -1: empty
+      pthread_mutexattr_t a;
+      pthread_mutexattr_init(&a);
+      pthread_mutexattr_setpshared(&a, PTHREAD_PROCESS_SHARED);
+      pthread_mutexattr_setrobust(&a, PTHREAD_MUTEX_ROBUST);
+      pthread_mutex_init(&h->mu, &a);
+      pthread_mutexattr_destroy(&a);
+      __atomic_store_n(&h->initialised, 1, __ATOMIC_RELEASE);
+    } else {
+      int i = 0;
+      while (__atomic_load_n(&h->initialised, __ATOMIC_ACQUIRE) != 1 && i++ < 5000) usleep(1000);
+      if (h->initialised != 1 || h->magic != kMagic || h->total_bytes != total ||
+          h->index_size != index_size_for(h->n_slots) || metadata_bytes(h->n_slots) > h->data_offset) {
+        munmap(map, (size_t)total);
+        delete t;
+        set_error_text("the shared tier is not initialised or does not match");
+        return KVX_EINVAL;
+      }
+      attach_metadata(t, map);
     }
-    t->registered = true;
-    void* dmap = nullptr;
-    if (cudaHostGetDevicePointer(&dmap, map, 0) == cudaSuccess && dmap && prepare_tier_kernels() == cudaSuccess)
-      t->meta_dev = (uint8_t*)dmap + ((uint8_t*)t->meta - (uint8_t*)map);
-    cudaGetLastError();  // without publication, commits turn READY through the writer's events only
-  }
-  *out = t;
-  return KVX_OK;
+    t->data = (uint8_t*)map + h->data_offset;
+    // Shared memory is kept on base pages: the SMs' zero-copy accesses run at the
+    // link peak on them, and a mixture of page sizes slowed zero-copy on GB300
+    // to a third.  (The copy engines are slow on base pages: with a shared tier,
+    // zero-copy, the default mode, is the one to use.)
+    madvise(t->data, (size_t)(h->slot_bytes * h->n_slots), MADV_NOHUGEPAGE);
+    if (!(flags & KVX_TIER_NO_PIN)) {
+      // The whole region, slot table included: the GPU publishes commits into it.
+      const cudaError_t e = cudaHostRegister(map, (size_t)total, cudaHostRegisterPortable | cudaHostRegisterMapped);
+      if (e != cudaSuccess) {
+        kvx_status st = cuda_fail(e, "cudaHostRegister of the shared tier");
+        t->creator = create;
+        destroy_tier(t);
+        return st;
+      }
+      t->registered = true;
+      void* dmap = nullptr;
+      if (cudaHostGetDevicePointer(&dmap, map, 0) == cudaSuccess && dmap && prepare_tier_kernels() == cudaSuccess)
+        t->meta_dev = (uint8_t*)dmap + ((uint8_t*)t->meta - (uint8_t*)map);
+      cudaGetLastError();  // without publication, commits turn READY through the writer's events only
+    }
+    *out = t;
+    return KVX_OK;
+  });
 }
 
 void kv_tier_destroy(kvx_tier* t) { destroy_tier(t); }
 
 kvx_status kv_tier_poll(kvx_tier* t) {
-  if (!t) return KVX_EINVAL;
-  TierLock lock(t);
-  poll_locked(t, kAll);
-  return KVX_OK;
+  return guarded([&]() -> kvx_status {
+    if (!t) return KVX_EINVAL;
+    TierLock lock(t);
+    poll_locked(t, kAll);
+    return KVX_OK;
+  });
 }
 
 }  // extern "C"
@@ -758,27 +766,31 @@ kvx_status reserve_locked(kvx_tier* t, uint64_t key, void** slot) {
 extern "C" {
 
 kvx_status kv_tier_reserve(kvx_tier* t, uint64_t key, void** slot) {
-  if (!t || !slot) return KVX_EINVAL;
-  TierLock lock(t);
-  poll_locked(t, kFront);
-  return reserve_locked(t, key, slot);
+  return guarded([&]() -> kvx_status {
+    if (!t || !slot) return KVX_EINVAL;
+    TierLock lock(t);
+    poll_locked(t, kFront);
+    return reserve_locked(t, key, slot);
+  });
 }
 
 kvx_status kv_tier_reserve_many(kvx_tier* t, const uint64_t* keys, int64_t n, void** slots, int64_t* n_reserved) {
-  if (n_reserved) *n_reserved = 0;
-  if (!t || n < 0 || (n > 0 && (!keys || !slots))) return KVX_EINVAL;
-  if (n == 0) return KVX_OK;
-  TierLock lock(t);
-  poll_locked(t, kFront);
-  for (int64_t j = 0; j < n; ++j) {
-    const kvx_status st = reserve_locked(t, keys[j], &slots[j]);
-    if (st != KVX_OK) {
-      if (n_reserved) *n_reserved = j;
-      return st;
+  return guarded([&]() -> kvx_status {
+    if (n_reserved) *n_reserved = 0;
+    if (!t || n < 0 || (n > 0 && (!keys || !slots))) return KVX_EINVAL;
+    if (n == 0) return KVX_OK;
+    TierLock lock(t);
+    poll_locked(t, kFront);
+    for (int64_t j = 0; j < n; ++j) {
+      const kvx_status st = reserve_locked(t, keys[j], &slots[j]);
+      if (st != KVX_OK) {
+        if (n_reserved) *n_reserved = j;
+        return st;
+      }
     }
-  }
-  if (n_reserved) *n_reserved = n;
-  return KVX_OK;
+    if (n_reserved) *n_reserved = n;
+    return KVX_OK;
+  });
 }
 
 kvx_status kv_tier_commit(kvx_tier* t, uint64_t key, kvx_stream_t stream) {
@@ -786,68 +798,70 @@ kvx_status kv_tier_commit(kvx_tier* t, uint64_t key, kvx_stream_t stream) {
 }
 
 kvx_status kv_tier_commit_many(kvx_tier* t, const uint64_t* keys, int64_t n, kvx_stream_t stream) {
-  if (!t || n < 0 || (n > 0 && !keys) || capturing(stream)) return KVX_EINVAL;
-  if (n == 0) return KVX_OK;
-  TierLock lock(t);
-  poll_locked(t, kFront);
-  std::vector<int64_t> slots((size_t)n);
-  std::unordered_map<int64_t, bool> seen;
-  for (int64_t j = 0; j < n; ++j) {  // every key first: on an error nothing is committed
-    const int64_t i = find_slot(t, keys[j]);
-    if (i < 0) return KVX_ENOENT;
-    const SlotMeta& m = t->meta[i];
-    if (m.state != kWriting || m.writer_pid != t->pid) return KVX_EINVAL;
-    if (!seen.emplace(i, true).second) {
-      set_error_text("a key is listed twice");
-      return KVX_EINVAL;
+  return guarded([&]() -> kvx_status {
+    if (!t || n < 0 || (n > 0 && !keys) || capturing(stream)) return KVX_EINVAL;
+    if (n == 0) return KVX_OK;
+    TierLock lock(t);
+    poll_locked(t, kFront);
+    std::vector<int64_t> slots((size_t)n);
+    std::unordered_map<int64_t, bool> seen;
+    for (int64_t j = 0; j < n; ++j) {  // every key first: on an error nothing is committed
+      const int64_t i = find_slot(t, keys[j]);
+      if (i < 0) return KVX_ENOENT;
+      const SlotMeta& m = t->meta[i];
+      if (m.state != kWriting || m.writer_pid != t->pid) return KVX_EINVAL;
+      if (!seen.emplace(i, true).second) {
+        set_error_text("a key is listed twice");
+        return KVX_EINVAL;
+      }
+      slots[(size_t)j] = i;
     }
-    slots[(size_t)j] = i;
-  }
-  if (no_stream(stream)) {
-    for (int64_t i : slots) {
+    if (no_stream(stream)) {
+      for (int64_t i : slots) {
+        SlotMeta& m = t->meta[i];
+        m.state = kReady;
+        add_pins(m, t->pid, -1);
+        m.tick = ++t->hdr->clock;
+      }
+      return KVX_OK;
+    }
+    // The sequence numbers are these commits' alone; a publication that lands
+    // after a failure below matches no commit.
+    const uint64_t seq0 = t->hdr->seq + 1;
+    t->hdr->seq += (uint64_t)n;
+    if (t->meta_dev) {
+      TierPublish b;
+      b.meta = t->meta_dev;
+      b.stride = (int64_t)sizeof(SlotMeta);
+      b.offset = (int64_t)offsetof(SlotMeta, published);
+      for (int64_t j0 = 0; j0 < n; j0 += kMaxPublish) {
+        b.n = (int32_t)std::min<int64_t>(kMaxPublish, n - j0);
+        b.seq0 = seq0 + (uint64_t)j0;
+        for (int32_t j = 0; j < b.n; ++j) b.slot[j] = (int32_t)slots[(size_t)(j0 + j)];
+        const cudaError_t r = fault_point("launch") ? cudaErrorUnknown : launch_tier_publish(b, (cudaStream_t)stream);
+        if (r != cudaSuccess) return cuda_fail(r, "publication kernel launch (tier commit)");
+      }
+    }
+    cudaEvent_t e = take_event(t);
+    if (!e) return cuda_fail(cudaErrorMemoryAllocation, "cudaEventCreate (tier commit)");
+    const cudaError_t r = cudaEventRecord(e, (cudaStream_t)stream);
+    if (r != cudaSuccess) {
+      t->spare.push_back(e);
+      return cuda_fail(r, "cudaEventRecord (tier commit)");
+    }
+    for (int64_t j = 0; j < n; ++j) {
+      const int64_t i = slots[(size_t)j];
       SlotMeta& m = t->meta[i];
-      m.state = kReady;
+      m.commit_seq = seq0 + (uint64_t)j;
+      m.state = kCommitting;
+      // one event for the batch: the last entry gives it back
+      t->commits.push_back({i, e, m.commit_seq, j == n - 1});
+      t->commit_event[i] = e;
       add_pins(m, t->pid, -1);
       m.tick = ++t->hdr->clock;
     }
     return KVX_OK;
-  }
-  // The sequence numbers are these commits' alone; a publication that lands
-  // after a failure below matches no commit.
-  const uint64_t seq0 = t->hdr->seq + 1;
-  t->hdr->seq += (uint64_t)n;
-  if (t->meta_dev) {
-    TierPublish b;
-    b.meta = t->meta_dev;
-    b.stride = (int64_t)sizeof(SlotMeta);
-    b.offset = (int64_t)offsetof(SlotMeta, published);
-    for (int64_t j0 = 0; j0 < n; j0 += kMaxPublish) {
-      b.n = (int32_t)std::min<int64_t>(kMaxPublish, n - j0);
-      b.seq0 = seq0 + (uint64_t)j0;
-      for (int32_t j = 0; j < b.n; ++j) b.slot[j] = (int32_t)slots[(size_t)(j0 + j)];
-      const cudaError_t r = fault_point("launch") ? cudaErrorUnknown : launch_tier_publish(b, (cudaStream_t)stream);
-      if (r != cudaSuccess) return cuda_fail(r, "publication kernel launch (tier commit)");
-    }
-  }
-  cudaEvent_t e = take_event(t);
-  if (!e) return cuda_fail(cudaErrorMemoryAllocation, "cudaEventCreate (tier commit)");
-  const cudaError_t r = cudaEventRecord(e, (cudaStream_t)stream);
-  if (r != cudaSuccess) {
-    t->spare.push_back(e);
-    return cuda_fail(r, "cudaEventRecord (tier commit)");
-  }
-  for (int64_t j = 0; j < n; ++j) {
-    const int64_t i = slots[(size_t)j];
-    SlotMeta& m = t->meta[i];
-    m.commit_seq = seq0 + (uint64_t)j;
-    m.state = kCommitting;
-    // one event for the batch: the last entry gives it back
-    t->commits.push_back({i, e, m.commit_seq, j == n - 1});
-    t->commit_event[i] = e;
-    add_pins(m, t->pid, -1);
-    m.tick = ++t->hdr->clock;
-  }
-  return KVX_OK;
+  });
 }
 
 kvx_status kv_tier_acquire(kvx_tier* t, uint64_t key, kvx_stream_t stream, void** slot) {
@@ -857,46 +871,48 @@ kvx_status kv_tier_acquire(kvx_tier* t, uint64_t key, kvx_stream_t stream, void*
 
 kvx_status kv_tier_acquire_many(kvx_tier* t, const uint64_t* keys, int64_t n, kvx_stream_t stream,
                                 void** slots) {
-  if (!t || n < 0 || (n > 0 && (!keys || !slots)) || capturing(stream)) return KVX_EINVAL;
-  if (n == 0) return KVX_OK;
-  TierLock lock(t);
-  poll_locked(t, kFront);
-  std::vector<int64_t> idx((size_t)n);
-  std::vector<cudaEvent_t> waits;  // this process's commit events the readers must follow, once each
-  for (int64_t j = 0; j < n; ++j) {  // every key first: on an error nothing is pinned
-    const int64_t i = find_slot(t, keys[j]);
-    bool ok = i >= 0 && t->meta[i].state == kReady;
-    if (i >= 0 && t->meta[i].state == kCommitting && t->meta[i].writer_pid == t->pid) {
-      auto it = t->commit_event.find(i);  // written here: order the reader on the writer's event
-      if (it != t->commit_event.end()) {
-        if (std::find(waits.begin(), waits.end(), it->second) == waits.end()) waits.push_back(it->second);
-        ok = true;
+  return guarded([&]() -> kvx_status {
+    if (!t || n < 0 || (n > 0 && (!keys || !slots)) || capturing(stream)) return KVX_EINVAL;
+    if (n == 0) return KVX_OK;
+    TierLock lock(t);
+    poll_locked(t, kFront);
+    std::vector<int64_t> idx((size_t)n);
+    std::vector<cudaEvent_t> waits;  // this process's commit events the readers must follow, once each
+    for (int64_t j = 0; j < n; ++j) {  // every key first: on an error nothing is pinned
+      const int64_t i = find_slot(t, keys[j]);
+      bool ok = i >= 0 && t->meta[i].state == kReady;
+      if (i >= 0 && t->meta[i].state == kCommitting && t->meta[i].writer_pid == t->pid) {
+        auto it = t->commit_event.find(i);  // written here: order the reader on the writer's event
+        if (it != t->commit_event.end()) {
+          if (std::find(waits.begin(), waits.end(), it->second) == waits.end()) waits.push_back(it->second);
+          ok = true;
+        }
       }
+      if (!ok) {
+        t->hdr->misses++;
+        return KVX_ENOENT;
+      }
+      if (pins_of(t->meta[i], t->pid) == 0 && !has_free_holder(t->meta[i])) {
+        set_error_text("the entry is pinned by as many processes as it can track");
+        return KVX_EBUSY;
+      }
+      idx[(size_t)j] = i;
     }
-    if (!ok) {
-      t->hdr->misses++;
-      return KVX_ENOENT;
+    for (cudaEvent_t e : waits) {
+      const cudaError_t r = no_stream(stream) ? cudaEventSynchronize(e) : cudaStreamWaitEvent((cudaStream_t)stream, e, 0);
+      if (r != cudaSuccess) return cuda_fail(r, no_stream(stream) ? "cudaEventSynchronize (tier acquire)"
+                                                                   : "cudaStreamWaitEvent (tier acquire)");
     }
-    if (pins_of(t->meta[i], t->pid) == 0 && !has_free_holder(t->meta[i])) {
-      set_error_text("the entry is pinned by as many processes as it can track");
-      return KVX_EBUSY;
+    for (int64_t j = 0; j < n; ++j) {
+      const int64_t i = idx[(size_t)j];
+      SlotMeta& m = t->meta[i];
+      add_pins(m, t->pid, 1);  // cannot fail: a holder place was checked above
+      m.tick = ++t->hdr->clock;
+      t->hdr->hits++;
+      slots[j] = t->data + i * t->hdr->slot_bytes;
     }
-    idx[(size_t)j] = i;
-  }
-  for (cudaEvent_t e : waits) {
-    const cudaError_t r = no_stream(stream) ? cudaEventSynchronize(e) : cudaStreamWaitEvent((cudaStream_t)stream, e, 0);
-    if (r != cudaSuccess) return cuda_fail(r, no_stream(stream) ? "cudaEventSynchronize (tier acquire)"
-                                                                 : "cudaStreamWaitEvent (tier acquire)");
-  }
-  for (int64_t j = 0; j < n; ++j) {
-    const int64_t i = idx[(size_t)j];
-    SlotMeta& m = t->meta[i];
-    add_pins(m, t->pid, 1);  // cannot fail: a holder place was checked above
-    m.tick = ++t->hdr->clock;
-    t->hdr->hits++;
-    slots[j] = t->data + i * t->hdr->slot_bytes;
-  }
-  return KVX_OK;
+    return KVX_OK;
+  });
 }
 
 kvx_status kv_tier_release(kvx_tier* t, uint64_t key, kvx_stream_t stream) {
@@ -904,90 +920,98 @@ kvx_status kv_tier_release(kvx_tier* t, uint64_t key, kvx_stream_t stream) {
 }
 
 kvx_status kv_tier_release_many(kvx_tier* t, const uint64_t* keys, int64_t n, kvx_stream_t stream) {
-  if (!t || n < 0 || (n > 0 && !keys) || capturing(stream)) return KVX_EINVAL;
-  if (n == 0) return KVX_OK;
-  TierLock lock(t);
-  poll_locked(t, kFront);
-  std::vector<int64_t> idx((size_t)n);
-  std::unordered_map<int64_t, int64_t> asked;  // releases of each slot in this call
-  for (int64_t j = 0; j < n; ++j) {  // every key first: on an error nothing is released
-    const int64_t i = find_slot(t, keys[j]);
-    if (i < 0) return KVX_ENOENT;
-    idx[(size_t)j] = i;
-    if (pins_of(t->meta[i], t->pid) - queued_releases(t, i) < ++asked[i]) {
-      set_error_text("this process holds no pin on the entry");
-      return KVX_EINVAL;
-    }
-  }
-  if (no_stream(stream)) {
-    for (int64_t i : idx) {
-      SlotMeta& m = t->meta[i];
-      add_pins(m, t->pid, -1);
-      if (m.state == kWriting && m.pins == 0) {  // a writer giving up its reservation
-        index_erase(t, m.key);
-        m.state = kFree;
+  return guarded([&]() -> kvx_status {
+    if (!t || n < 0 || (n > 0 && !keys) || capturing(stream)) return KVX_EINVAL;
+    if (n == 0) return KVX_OK;
+    TierLock lock(t);
+    poll_locked(t, kFront);
+    std::vector<int64_t> idx((size_t)n);
+    std::unordered_map<int64_t, int64_t> asked;  // releases of each slot in this call
+    for (int64_t j = 0; j < n; ++j) {  // every key first: on an error nothing is released
+      const int64_t i = find_slot(t, keys[j]);
+      if (i < 0) return KVX_ENOENT;
+      idx[(size_t)j] = i;
+      if (pins_of(t->meta[i], t->pid) - queued_releases(t, i) < ++asked[i]) {
+        set_error_text("this process holds no pin on the entry");
+        return KVX_EINVAL;
       }
     }
+    if (no_stream(stream)) {
+      for (int64_t i : idx) {
+        SlotMeta& m = t->meta[i];
+        add_pins(m, t->pid, -1);
+        if (m.state == kWriting && m.pins == 0) {  // a writer giving up its reservation
+          index_erase(t, m.key);
+          m.state = kFree;
+        }
+      }
+      return KVX_OK;
+    }
+    cudaEvent_t e = take_event(t);
+    if (!e) return cuda_fail(cudaErrorMemoryAllocation, "cudaEventCreate (tier release)");
+    const cudaError_t r = cudaEventRecord(e, (cudaStream_t)stream);
+    if (r != cudaSuccess) {
+      t->spare.push_back(e);
+      return cuda_fail(r, "cudaEventRecord (tier release)");
+    }
+    for (int64_t j = 0; j < n; ++j) {  // the pins stay until the queued work completes; one event for all
+      const int64_t i = idx[(size_t)j];
+      t->releases.push_back({i, e, 0, j == n - 1});
+      t->queued[i]++;
+    }
     return KVX_OK;
-  }
-  cudaEvent_t e = take_event(t);
-  if (!e) return cuda_fail(cudaErrorMemoryAllocation, "cudaEventCreate (tier release)");
-  const cudaError_t r = cudaEventRecord(e, (cudaStream_t)stream);
-  if (r != cudaSuccess) {
-    t->spare.push_back(e);
-    return cuda_fail(r, "cudaEventRecord (tier release)");
-  }
-  for (int64_t j = 0; j < n; ++j) {  // the pins stay until the queued work completes; one event for all
-    const int64_t i = idx[(size_t)j];
-    t->releases.push_back({i, e, 0, j == n - 1});
-    t->queued[i]++;
-  }
-  return KVX_OK;
+  });
 }
 
 kvx_status kv_tier_reclaim(kvx_tier* t, int64_t* reclaimed) {
-  if (!t) return KVX_EINVAL;
-  TierLock lock(t);
-  poll_locked(t, kFront);
-  const int64_t n = reclaim_locked(t);
-  if (reclaimed) *reclaimed = n;
-  return KVX_OK;
+  return guarded([&]() -> kvx_status {
+    if (!t) return KVX_EINVAL;
+    TierLock lock(t);
+    poll_locked(t, kFront);
+    const int64_t n = reclaim_locked(t);
+    if (reclaimed) *reclaimed = n;
+    return KVX_OK;
+  });
 }
 
 kvx_status kv_tier_prefix_hits(kvx_tier* t, const uint64_t* keys, int64_t n, int64_t* hits) {
-  if (!t || !hits || n < 0 || (n > 0 && !keys)) return KVX_EINVAL;
-  TierLock lock(t);
-  poll_locked(t, kFront);
-  int64_t h = 0;
-  while (h < n) {
-    const int64_t i = find_slot(t, keys[h]);
-    if (i < 0) break;
-    const SlotMeta& m = t->meta[i];
-    const bool visible = m.state == kReady || (m.state == kCommitting && m.writer_pid == t->pid);
-    if (!visible) break;
-    ++h;
-  }
-  *hits = h;
-  return KVX_OK;
+  return guarded([&]() -> kvx_status {
+    if (!t || !hits || n < 0 || (n > 0 && !keys)) return KVX_EINVAL;
+    TierLock lock(t);
+    poll_locked(t, kFront);
+    int64_t h = 0;
+    while (h < n) {
+      const int64_t i = find_slot(t, keys[h]);
+      if (i < 0) break;
+      const SlotMeta& m = t->meta[i];
+      const bool visible = m.state == kReady || (m.state == kCommitting && m.writer_pid == t->pid);
+      if (!visible) break;
+      ++h;
+    }
+    *hits = h;
+    return KVX_OK;
+  });
 }
 
 kvx_status kv_tier_stats(kvx_tier* t, kvx_tier_stats* out) {
-  if (!t || !out) return KVX_EINVAL;
-  TierLock lock(t);
-  poll_locked(t, kFront);
-  out->slots = t->hdr->n_slots;
-  out->slot_bytes = t->hdr->slot_bytes;
-  int64_t used = 0, pinned = 0;
-  for (int64_t i = 0; i < t->hdr->n_slots; ++i) {
-    used += t->meta[i].state != kFree;
-    pinned += t->meta[i].pins > 0;
-  }
-  out->entries = used;
-  out->pinned = pinned;
-  out->hits = t->hdr->hits;
-  out->misses = t->hdr->misses;
-  out->evictions = t->hdr->evictions;
-  return KVX_OK;
+  return guarded([&]() -> kvx_status {
+    if (!t || !out) return KVX_EINVAL;
+    TierLock lock(t);
+    poll_locked(t, kFront);
+    out->slots = t->hdr->n_slots;
+    out->slot_bytes = t->hdr->slot_bytes;
+    int64_t used = 0, pinned = 0;
+    for (int64_t i = 0; i < t->hdr->n_slots; ++i) {
+      used += t->meta[i].state != kFree;
+      pinned += t->meta[i].pins > 0;
+    }
+    out->entries = used;
+    out->pinned = pinned;
+    out->hits = t->hdr->hits;
+    out->misses = t->hdr->misses;
+    out->evictions = t->hdr->evictions;
+    return KVX_OK;
+  });
 }
 
 }  // extern "C"

@@ -318,3 +318,21 @@ def test_tier_follows_its_rules_under_random_operations(k, seed, n_slots, n_keys
     assert (st["hits"], st["misses"], st["evictions"]) == (model.hits, model.misses, model.evictions)
     assert st["entries"] == sum(s["state"] != "FREE" for s in model.slots)
     assert st["pinned"] == sum(s["pins"] > 0 for s in model.slots)
+
+
+def test_absurd_counts_return_enomem_not_a_crash(k):
+    """A batch call given a count no host could hold fails with KVX_ENOMEM (the
+    library's allocation fails inside the call); no C++ exception ends the
+    process, and the tier stays usable."""
+    import ctypes
+    tier, _ = _tier(k, 2)
+    key = (ctypes.c_uint64 * 1)(7)
+    slots = (ctypes.c_void_p * 1)()
+    n = ctypes.c_int64()
+    huge = 1 << 50
+    assert k._lib.kv_tier_commit_many(tier.handle, key, huge, NO) == k.KVX_ENOMEM
+    assert k._lib.kv_tier_acquire_many(tier.handle, key, huge, NO, slots) == k.KVX_ENOMEM
+    assert k._lib.kv_tier_release_many(tier.handle, key, huge, NO) == k.KVX_ENOMEM
+    tier.reserve(7).fill_(7)
+    tier.commit(7, NO)
+    assert tier.prefix_hits([7]) == 1
