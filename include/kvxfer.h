@@ -62,7 +62,7 @@
 extern "C" {
 #endif
 
-#define KVX_ABI_VERSION 2
+#define KVX_ABI_VERSION 3
 #define KVX_MAX_LAYERS 128 /* layers per pool description */
 
 /* Same handle as cudaStream_t; NULL is the legacy default stream. */
@@ -120,8 +120,17 @@ typedef enum {
    GPU or the link.  A CPU read of one byte per host page of the chunks just
    before the transfer (13.8 ms on one thread for 33 GB) brought it back to
    159 ms.  So when a context has begun no transfer for more than 1 s,
-   kv_store and kv_load first read one byte of every host page of the chunks
-   they are given, on up to 16 host threads.  This flag turns that off.      */
+   kv_store and kv_load read one byte of every host page of the chunks they
+   are given before moving them.  The reads run on a pool of up to 16
+   persistent library threads (started once per process), not on the calling
+   thread: the call enqueues on `stream`, ahead of its transfer, a host
+   function (cudaLaunchHostFunc) that waits until the pages have been read
+   (2-4 ms for 33 GB on GB300), so the transfer follows the reads, the call
+   itself returns without waiting, and `stream` completes only after the last
+   read.  It is skipped while `stream` is being captured.  If the library
+   cannot start threads (or in a forked child, which inherits none) the
+   calling thread reads the pages itself before it enqueues.  kv_host_touch
+   does the same reads on request.  This flag turns the idle-time touch off. */
 #define KVX_FLAG_NO_HOST_TOUCH 0x10u
 /* Every defined flag.  kv_ctx_create rejects (KVX_EINVAL) other bits, and
    KVX_FLAG_DEVICE_TMA together with KVX_FLAG_DEVICE_LSU.                     */
@@ -142,6 +151,15 @@ typedef struct {
                                  32 KiB unit its own warp or CTA.  With a cap,
                                  each warp or CTA strides over many units       */
   uint32_t flags;             /* KVX_FLAG_*                                     */
+  int64_t wait_cycles;        /* limit of every bounded wait inside a kernel, in
+                                 SM cycles (the TMA engine's waits for its
+                                 global -> shared copies); 0 = 4e9, about 2 s at
+                                 the maximum SM clock.  When a wait expires, the
+                                 CTA issues no further copy, waits once more
+                                 (same limit) for each copy it has started,
+                                 then returns; kv_get_device_error reports
+                                 KVX_ETIMEOUT and that call's output is
+                                 incomplete.  The context stays usable.         */
 } kvx_opts;
 
 /* Caller-owned description of one paged KV pool (device memory). */
@@ -233,7 +251,11 @@ kvx_status kv_pool_view_check(const kvx_pool* pool, int32_t ndim, const int64_t*
  * [tok_begin, tok_end) of the pages named by block_table into host_chunks.
  *   block_table : device int32 [table_len]; pages of logical blocks 0..
  *   tok_begin   : multiple of chunk_tokens (chunks start on aligned recovery
- *                 boundaries, Sec. 2.2);  tok_end <= table_len * B.
+ *                 boundaries, Sec. 2.2);
+ *   tok_end     : tok_begin <= tok_end <= table_len * P * B, where
+ *                 P = pool->pages_per_block (1 unless pages are packed into
+ *                 logical blocks) and B = pool->block_tokens; beyond that
+ *                 KVX_ERANGE.
  *   host_chunks : host array [n_chunks] of pinned host pointers; chunk i gets
  *                 chunk tok_begin/C + i; n_chunks >= ceil(tok_end/C) - tok_begin/C.
  *   stream      : the caller's current stream.  All reads of the pool happen
@@ -309,12 +331,21 @@ kvx_status kv_state_load(kvx_ctx* ctx, int32_t num_layers, void* const* layer_ba
  *                         atomicMin to the lowest logical block whose table
  *                         entry is out of range (initialise it, e.g. to
  *                         INT64_MAX); such tokens are stored as zeros.
- * Set-up: the first call on a device (with that device current) looks up the
- * array's device address with cudaGetSymbolAddress and caches it; make that
- * first call before any stream capture.  All calls share the one array and
- * nothing in it needs to start at zero (every staged byte is written before it
- * is copied).  Calls that overlap on the GPU -- on different streams without an
- * ordering between them -- race on the array: order them.
+ * Set-up: the first call in a CUDA context (on the thread's current device)
+ * looks up the array's device address with cudaGetSymbolAddress, loads the
+ * pack kernels, and keeps the address for that context.  A call in another
+ * context -- a driver-API context the caller made current, or the new primary
+ * context after cudaDeviceReset -- repeats this set-up there.  With CUDA's
+ * lazy module loading (the default) this set-up is also when the GPU takes the
+ * array's 64 MiB, so an engine that reserves all free GPU memory must make one
+ * call before it does.  A call with an empty range (tok_begin == tok_end,
+ * arguments otherwise valid) makes the set-up and moves nothing: make it at
+ * start-up, before the engine reserves GPU memory and before any stream
+ * capture.  Later calls in the same context allocate nothing on the device or
+ * the host.  All calls share the one array and nothing in it needs to start
+ * at zero (every staged byte is written before it is copied).  Calls that
+ * overlap on the GPU -- on different streams without an ordering between
+ * them -- race on the array: order them.
  */
 #define KVX_NOALLOC_SCRATCH_BYTES (64ll << 20)
 kvx_status kv_store_noalloc(const kvx_pool* pool, const int32_t* block_table, int64_t table_len,
@@ -400,6 +431,20 @@ kvx_status kv_host_pool_info(const void* host, kvx_host_pool_info* info);
 /* Frees kv_host_alloc and kv_host_alloc_numa memory; NULL and pointers the
    library did not allocate are ignored. */
 void kv_host_free(void* host);
+
+/*
+ * Read one byte of every host page of n ranges (ptrs[i], bytes[i] long) on the
+ * library's touch threads and the calling thread, returning when all have been
+ * read.  The idle-time touch of kv_store / kv_load (KVX_FLAG_NO_HOST_TOUCH)
+ * done ahead of time: a caller that knows a restore is coming (a request that
+ * hit the shared tier, say) can warm the chunks' pages before it calls
+ * kv_load.  Each range must be readable host memory (pinned or not) for the
+ * duration of the call.  KVX_EINVAL for n < 0, a negative size, or a null
+ * pointer with a positive size; zero-sized ranges are skipped.  Gives up after
+ * 5 s (pages left unread) and still returns KVX_OK: the touch is only a
+ * speed-up.
+ */
+kvx_status kv_host_touch(void* const* ptrs, const int64_t* bytes, int64_t n);
 
 /* ------------------------------------------------------------------------
  * Shared host tier (Table 1: one pinned RAM pool of fixed-token chunks with
@@ -530,7 +575,9 @@ kvx_status kv_tier_stats(kvx_tier* tier, kvx_tier_stats* out);
 /*
  * Lowest logical block index whose table entry was out of range in any call
  * completed since the last query, or -1.  Call after the caller's stream has
- * been synchronised.  Clears the record.
+ * been synchronised.  Clears the record.  Returns KVX_ETIMEOUT (and still fills
+ * *first_bad_block) if a bounded wait inside a kernel of this context expired
+ * since the last query (kvx_opts.wait_cycles); that clears too.
  */
 kvx_status kv_get_device_error(kvx_ctx* ctx, int64_t* first_bad_block);
 
@@ -555,8 +602,13 @@ const char* kv_last_error_message(void);
  * fails with cudaErrorUnknown (cudaErrorMemoryAllocation for "host_alloc")
  * instead of being made.  Points: "launch" (kernel launches), "memcpy"
  * (staged-mode copies), "event" (the staged pipeline's ordering event
- * recorded on the caller's stream), "host_alloc" (kv_host_alloc).  One more
- * point fails differently: "tier_exit" ends the process (_exit(3)) inside
+ * recorded on the caller's stream), "host_alloc" (kv_host_alloc).  Two more
+ * points fail differently.  "tma_wait": the (after_calls + 1)-th next launch
+ * of the TMA engine arms the shared-memory stage of its first unit for bytes
+ * that no copy brings, so that unit's bounded wait runs out (after
+ * kvx_opts.wait_cycles) with no copy in flight: the launch leaves that unit
+ * unmoved and kv_get_device_error returns KVX_ETIMEOUT; nothing faults or
+ * hangs.  "tier_exit" ends the process (_exit(3)) inside
  * kv_tier_reserve, while it holds a shared tier's table lock, right after it
  * has taken a slot for the new key; it tests how the processes left recover
  * the tier from a replica that died mid-update.  One point is armed at a

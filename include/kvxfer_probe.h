@@ -1,6 +1,9 @@
 /*
- * kvxfer_probe.h -- ordering probes shipped in libkvxfer.so.
+ * kvxfer_probe.h -- measuring instruments in libkvxfer_probe.so, a library of
+ * its own that the tests and the benchmark load beside libkvxfer.so.  It
+ * shares no code with the transfer library.
  *
+ * Ordering probes.
  * These reproduce the paper's controlled byte experiment (Sec. 3.2; Table 2,
  * "Copy-ordering controls"): a kernel on a non-default stream writes (or
  * reads) a buffer after an imposed delay of the order of 10^8 SM cycles, and
@@ -53,6 +56,22 @@ kvx_status kvx_probe_delayed_copy(void* dst, const void* src, int64_t bytes, int
  * fallback and is kept as a negative control only.
  */
 kvx_status kvx_probe_copy(void* dst, const void* src, int64_t bytes, int32_t how, kvx_stream_t stream);
+
+/*
+ * Host-link probe: on `stream`, copy `bytes` from src to dst with a plain
+ * contiguous streaming kernel on the SMs (16-byte loads and stores, whole
+ * 128-byte lines, `ctas` CTAs of 256 threads striding over the range).  Either
+ * side may be device memory or page-locked host memory mapped for the GPU, so
+ * device -> mapped host measures what SM stores can push over the host link
+ * and mapped host -> device what SM loads can pull: the ceiling of zero-copy
+ * transfers, beside the copy engines' cudaMemcpyAsync.  Both pointers and
+ * `bytes` must be multiples of 16 (KVX_EALIGN); a side that is neither device
+ * memory nor mapped over its whole length is KVX_ENOTPINNED.
+ */
+kvx_status kvx_probe_stream_copy(void* dst, const void* src, int64_t bytes, int32_t ctas, kvx_stream_t stream);
+
+/* The last CUDA error code a probe call of this thread saw (0 = none). */
+int kvx_probe_last_cuda_error(void);
 
 #ifdef __cplusplus
 }

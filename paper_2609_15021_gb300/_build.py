@@ -1,4 +1,6 @@
-"""Build libkvxfer.so in-tree with nvcc for sm_103a (no cmake, no torch)."""
+"""Build libkvxfer.so (the transfer library) and libkvxfer_probe.so (the
+measuring probes the tests and the benchmark use) in-tree with nvcc for
+sm_103a (no cmake, no torch)."""
 from __future__ import annotations
 
 import os
@@ -12,9 +14,11 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "_lib", "libkvxfer.so")
+PROBE_LIB = os.path.join(PKG, "_lib", "libkvxfer_probe.so")
 
-SOURCES = ["pack_kernels.cu", "segment_kernels.cu", "tma_kernels.cu", "kvxfer.cu", "probe.cu", "no_alloc.cu", "tier.cpp",
+SOURCES = ["pack_kernels.cu", "segment_kernels.cu", "tma_kernels.cu", "kvxfer.cu", "no_alloc.cu", "tier.cpp",
            "tier_kernels.cu", "host_alloc.cpp"]
+PROBE_SOURCES = ["probe.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC,-O2,-Wall,-Wextra", f"-I{INCLUDE}"]
 
@@ -26,23 +30,31 @@ def _nvcc() -> str:
     return "nvcc"
 
 
-def _inputs() -> list[str]:
-    deps = [os.path.join(CSRC, s) for s in SOURCES]
+def _inputs(sources) -> list[str]:
+    deps = [os.path.join(CSRC, s) for s in sources]
     deps += [os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith((".h", ".cuh"))]
     deps += [os.path.join(INCLUDE, f) for f in os.listdir(INCLUDE) if f.endswith(".h")]
+    deps.append(os.path.abspath(__file__))
     return deps
 
 
-def up_to_date() -> bool:
-    if not os.path.exists(LIB):
+def _fresh(lib, sources) -> bool:
+    if not os.path.exists(lib):
         return False
-    t = os.path.getmtime(LIB)
-    return all(os.path.getmtime(d) <= t for d in _inputs())
+    t = os.path.getmtime(lib)
+    return all(os.path.getmtime(d) <= t for d in _inputs(sources))
+
+
+def up_to_date() -> bool:
+    return _fresh(LIB, SOURCES) and _fresh(PROBE_LIB, PROBE_SOURCES)
 
 
 def build(force: bool = False, verbose: bool = False, ptxas_report: str | None = None) -> str:
-    """Compile every CUDA source in parallel and link the shared library."""
-    if not force and up_to_date():
+    """Compile every CUDA source in parallel and link both shared libraries;
+    returns the path of libkvxfer.so."""
+    todo = [(lib, srcs) for lib, srcs in ((LIB, SOURCES), (PROBE_LIB, PROBE_SOURCES))
+            if force or not _fresh(lib, srcs)]
+    if not todo:
         return LIB
     os.makedirs(BUILD, exist_ok=True)
     os.makedirs(os.path.dirname(LIB), exist_ok=True)
@@ -57,20 +69,22 @@ def build(force: bool = False, verbose: bool = False, ptxas_report: str | None =
             raise RuntimeError(f"nvcc failed for {src}:\n{r.stdout}\n{r.stderr}")
         return obj, r.stderr
 
-    with ThreadPoolExecutor(max_workers=len(SOURCES)) as ex:
-        results = list(ex.map(compile_one, SOURCES))
+    all_sources = [s for _, srcs in todo for s in srcs]
+    with ThreadPoolExecutor(max_workers=len(all_sources)) as ex:
+        results = dict(zip(all_sources, ex.map(compile_one, all_sources)))
     if ptxas_report:
         with open(ptxas_report, "w") as f:
-            for _, log in results:
+            for _, log in results.values():
                 f.write(log)
-    tmp = LIB + f".tmp{os.getpid()}"
-    cmd = [nvcc, *ARCH, "-shared", "-o", tmp, *[o for o, _ in results]]
-    r = subprocess.run(cmd, capture_output=True, text=True)
-    if r.returncode != 0:
-        raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")
-    os.replace(tmp, LIB)
-    if verbose:
-        print(f"built {LIB}", file=sys.stderr)
+    for lib, srcs in todo:
+        tmp = lib + f".tmp{os.getpid()}"
+        cmd = [nvcc, *ARCH, "-shared", "-o", tmp, *[results[s][0] for s in srcs]]
+        r = subprocess.run(cmd, capture_output=True, text=True)
+        if r.returncode != 0:
+            raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")
+        os.replace(tmp, lib)
+        if verbose:
+            print(f"built {lib}", file=sys.stderr)
     return LIB
 
 

@@ -88,11 +88,21 @@ void set_error_text(const char* text);
 // Launchers (pack_kernels.cu).  Return the cudaError_t of the launch.
 cudaError_t launch_move(int dir, int layout, const MoveParams& p, int grid, cudaStream_t s);
 cudaError_t launch_segments(const SegmentParams& p, int grid, cudaStream_t s);
+// Loads the pack kernels into the current context if lazy loading has not yet.
+cudaError_t load_pack_kernels();
+// Bounded waits of the TMA kernels: the limit of each mbarrier wait in SM
+// cycles, the device int set when one expires, and the unit (global index, -1
+// for none) whose load a kernel arms without issuing it (fault point "tma_wait").
+struct TmaWait {
+  long long cycles;
+  long long stall_unit;
+  int* timeout;
+};
+constexpr long long kDefaultWaitCycles = 4000000000ll;  // about 2 s at the maximum SM clock
 // Bulk-copy (TMA) variant for chunks in device memory (tma_kernels.cu): one
-// warp per CTA, `stages` shared-memory stages of stage_bytes each; sets
-// *timeout (device int) if a bounded wait expires.
+// warp per CTA, `stages` shared-memory stages of stage_bytes each.
 cudaError_t launch_move_tma(int dir, int layout, const MoveParams& p, int grid, int stage_bytes, int stages,
-                            int* timeout, cudaStream_t s);
+                            const TmaWait& wt, cudaStream_t s);
 // Sets the TMA kernels' shared-memory limit for the current device (once per
 // context creation; never on the launch path).
 cudaError_t prepare_tma_kernels();
@@ -102,7 +112,7 @@ constexpr int kTensorMapBytes = 128;
 // false if the pool's shape cannot be described (the row-copy variant is used).
 bool encode_tensor_maps(const kvx_pool* P, int64_t row_bytes, void* out);
 cudaError_t launch_move_tmap(int dir, const MoveParams& p, const void* maps, int num_layers, int grid,
-                             int stage_bytes, int stages, int* timeout, cudaStream_t s);
+                             int stage_bytes, int stages, const TmaWait& wt, cudaStream_t s);
 int move_ctas_per_sm(int dir, int layout);
 int segment_ctas_per_sm();
 // Shared tier (tier_kernels.cu): publication of up to kMaxPublish commits in

@@ -156,6 +156,14 @@ cudaError_t launch_move(int dir, int layout, const MoveParams& p, int grid, cuda
   return cudaGetLastError();
 }
 
+cudaError_t load_pack_kernels() {
+  // cudaFuncGetAttributes makes CUDA load a kernel that lazy loading has not loaded yet
+  cudaFuncAttributes a;
+  cudaError_t e = cudaFuncGetAttributes(&a, move_kernel<kPack, KVX_LAYOUT_HND>);
+  if (e == cudaSuccess) e = cudaFuncGetAttributes(&a, move_kernel<kPack, KVX_LAYOUT_NHD>);
+  return e;
+}
+
 int move_ctas_per_sm(int dir, int layout) {
   if (dir == kPack) return layout == KVX_LAYOUT_HND ? occupancy_of<kPack, KVX_LAYOUT_HND>()
                                                     : occupancy_of<kPack, KVX_LAYOUT_NHD>();

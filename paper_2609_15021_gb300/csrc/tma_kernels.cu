@@ -22,8 +22,13 @@
 // range is read into a chunk or written to a page.
 //
 // Only for chunks in device memory (kv_pack / kv_unpack / staged mode).  Every
-// mbarrier wait is bounded by a clock limit; on expiry the kernel sets a
-// timeout flag, drains its own bulk stores and returns.
+// mbarrier wait is bounded by a clock limit passed to the kernel.  When a wait
+// expires the CTA issues no further load; it waits again, under the same
+// limit, on every stage whose load it has issued and not yet consumed (so no
+// global -> shared copy it started can still be landing in its shared memory
+// when it leaves), waits for its bulk stores, sets the timeout flag and
+// returns.  A CTA therefore leaves a load behind only if that load has not
+// completed within twice the limit.
 
 #include <cuda.h>
 #include <string.h>
@@ -34,7 +39,6 @@ namespace kvx {
 namespace {
 
 constexpr int kStagesMax = 4;
-constexpr long long kWaitCycles = 4000000000ll;  // about 2 s at the maximum SM clock
 
 struct TensorMaps {
   CUtensorMap m[KVX_MAX_LAYERS];
@@ -60,12 +64,12 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
       : "memory");
   return done != 0;
 }
-// Bounded wait on an mbarrier phase; false when the limit expired.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+// Bounded wait on an mbarrier phase; false when `limit` SM cycles expired.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, long long limit) {
   if (mbar_try_wait(bar, parity)) return true;
   const long long t0 = clock64();
   while (!mbar_try_wait(bar, parity))
-    if (clock64() - t0 > kWaitCycles) return false;
+    if (clock64() - t0 > limit) return false;
   return true;
 }
 __device__ __forceinline__ void bulk_load(void* sdst, const void* gsrc, uint32_t bytes, uint64_t* bar) {
@@ -153,14 +157,16 @@ __device__ __forceinline__ Unit decode(const MoveParams& p, int64_t u, int& j, i
   return r;
 }
 
-// Issue the global -> shared copies of one unit into `stage`.
+// Issue the global -> shared copies of one unit into `stage`.  stall: arm the
+// stage's phase for bytes that no copy will bring (the host-side fault point
+// "tma_wait"), so that the wait on it runs out with nothing in flight.
 template <int DIR, int LAYOUT, bool TMAP>
 __device__ __forceinline__ void issue_loads(const MoveParams& p, const TensorMaps* maps, const Unit& w,
-                                            uint8_t* stage, uint64_t* bar, int lane) {
+                                            uint8_t* stage, uint64_t* bar, int lane, bool stall) {
   const uint32_t bytes = w.move ? (uint32_t)((TMAP && DIR == kPack && w.full ? p.B * p.H : w.nr) * p.R) : 0u;
-  if (lane == 0) mbar_expect_tx(bar, bytes);
+  if (lane == 0) mbar_expect_tx(bar, stall ? max(bytes, 16u) : bytes);
   __syncwarp();
-  if (!w.move) return;
+  if (!w.move || stall) return;
   if (DIR == kUnpack || LAYOUT == KVX_LAYOUT_NHD) {
     // chunk side (unpack) or an NHD page (pack): one contiguous run
     if (lane == 0) bulk_load(stage, DIR == kUnpack ? w.ck : w.pg, bytes, bar);
@@ -197,7 +203,7 @@ __device__ __forceinline__ void issue_stores(const MoveParams& p, const TensorMa
 
 template <int DIR, int LAYOUT, bool TMAP>
 __device__ __forceinline__ void tma_move_body(const MoveParams& p, const TensorMaps* maps, int stage_bytes,
-                                              int stages, int* timeout) {
+                                              int stages, const TmaWait& wt) {
   extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t bars[kStagesMax];
   // 128-byte aligned stages (tensor copies need it)
@@ -214,20 +220,26 @@ __device__ __forceinline__ void tma_move_body(const MoveParams& p, const TensorM
   int64_t bl = 0, bs = 0;
   // Loads run `ahead` units ahead of stores: stages - 1 with a ring, and one
   // with a single stage (the next unit's load then waits for the store to
-  // have read the stage).
+  // have read the stage).  Units [consumed, issued) have a load armed on
+  // stage (unit % stages); at most one per stage.
   const int ahead = stages > 1 ? stages - 1 : 1;
   const int64_t pro = n < ahead ? n : ahead;
   for (int64_t it = 0; it < pro; ++it) {
-    const Unit w = decode<DIR>(p, first + it * step, jl, bl, lane);
-    issue_loads<DIR, LAYOUT, TMAP>(p, maps, w, smem + it * stage_bytes, &bars[it], lane);
+    const int64_t u = first + it * step;
+    const Unit w = decode<DIR>(p, u, jl, bl, lane);
+    issue_loads<DIR, LAYOUT, TMAP>(p, maps, w, smem + it * stage_bytes, &bars[it], lane, u == wt.stall_unit);
   }
-  bool ok = true;
-  for (int64_t it = 0; it < n && ok; ++it) {
+  int64_t issued = pro, failed_at = -1;
+  for (int64_t it = 0; it < n; ++it) {
     const int k = (int)(it % stages);
     const Unit w = decode<DIR>(p, first + it * step, js, bs, -1);
-    if (lane == 0) ok = mbar_wait(&bars[k], (uint32_t)((it / stages) & 1));
+    bool ok = true;
+    if (lane == 0) ok = mbar_wait(&bars[k], (uint32_t)((it / stages) & 1), wt.cycles);
     ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
-    if (!ok) break;
+    if (!ok) {
+      failed_at = it;
+      break;
+    }
     issue_stores<DIR, LAYOUT, TMAP>(p, maps, w, smem + (int64_t)k * stage_bytes, lane);
     const int64_t nxt = it + ahead;
     if (nxt < n) {
@@ -239,25 +251,37 @@ __device__ __forceinline__ void tma_move_body(const MoveParams& p, const TensorM
         bulk_wait_read_0();
       __syncwarp();
       const int kn = (int)(nxt % stages);
-      const Unit wn = decode<DIR>(p, first + nxt * step, jl, bl, lane);
-      issue_loads<DIR, LAYOUT, TMAP>(p, maps, wn, smem + (int64_t)kn * stage_bytes, &bars[kn], lane);
+      const int64_t un = first + nxt * step;
+      const Unit wn = decode<DIR>(p, un, jl, bl, lane);
+      issue_loads<DIR, LAYOUT, TMAP>(p, maps, wn, smem + (int64_t)kn * stage_bytes, &bars[kn], lane,
+                                     un == wt.stall_unit);
+      issued = nxt + 1;
     }
   }
-  if (!ok && lane == 0) atomicExch(timeout, 1);
+  if (failed_at >= 0) {
+    // No new loads; every load still armed gets another bounded wait, so that
+    // none lands in this CTA's shared memory after it has left.
+    if (lane == 0) {
+      for (int64_t v = failed_at; v < issued; ++v)
+        mbar_wait(&bars[v % stages], (uint32_t)((v / stages) & 1), wt.cycles);
+      atomicExch(wt.timeout, 1);
+    }
+    __syncwarp();
+  }
   bulk_wait_all();
 }
 
 template <int DIR, int LAYOUT>
 __global__ void __launch_bounds__(32) tma_move_kernel(const __grid_constant__ MoveParams p, int stage_bytes,
-                                                      int stages, int* timeout) {
-  tma_move_body<DIR, LAYOUT, false>(p, nullptr, stage_bytes, stages, timeout);
+                                                      int stages, const TmaWait wt) {
+  tma_move_body<DIR, LAYOUT, false>(p, nullptr, stage_bytes, stages, wt);
 }
 
 template <int DIR>
 __global__ void __launch_bounds__(32) tmap_move_kernel(const __grid_constant__ MoveParams p,
                                                        const __grid_constant__ TensorMaps maps, int stage_bytes,
-                                                       int stages, int* timeout) {
-  tma_move_body<DIR, KVX_LAYOUT_HND, true>(p, &maps, stage_bytes, stages, timeout);
+                                                       int stages, const TmaWait wt) {
+  tma_move_body<DIR, KVX_LAYOUT_HND, true>(p, &maps, stage_bytes, stages, wt);
 }
 
 // Largest dynamic shared memory a TMA launch uses: 96 KiB of stages (three of
@@ -340,11 +364,11 @@ bool stages_ok(int stage_bytes, int stages) {
 }
 
 cudaError_t launch_move_tma(int dir, int layout, const MoveParams& p, int grid, int stage_bytes, int stages,
-                            int* timeout, cudaStream_t s) {
-  if (!stages_ok(stage_bytes, stages)) return cudaErrorInvalidValue;
+                            const TmaWait& wt, cudaStream_t s) {
+  if (!stages_ok(stage_bytes, stages) || wt.cycles < 1 || !wt.timeout) return cudaErrorInvalidValue;
   const size_t smem = (size_t)stage_bytes * stages + 128;
   auto go = [&](auto kernel) {
-    kernel<<<grid, 32, smem, s>>>(p, stage_bytes, stages, timeout);
+    kernel<<<grid, 32, smem, s>>>(p, stage_bytes, stages, wt);
     return cudaGetLastError();
   };
   if (dir == kPack)
@@ -355,13 +379,15 @@ cudaError_t launch_move_tma(int dir, int layout, const MoveParams& p, int grid, 
 }
 
 cudaError_t launch_move_tmap(int dir, const MoveParams& p, const void* maps, int num_layers, int grid,
-                             int stage_bytes, int stages, int* timeout, cudaStream_t s) {
-  if (!stages_ok(stage_bytes, stages) || num_layers < 1 || num_layers > KVX_MAX_LAYERS) return cudaErrorInvalidValue;
+                             int stage_bytes, int stages, const TmaWait& wt, cudaStream_t s) {
+  if (!stages_ok(stage_bytes, stages) || num_layers < 1 || num_layers > KVX_MAX_LAYERS || wt.cycles < 1 ||
+      !wt.timeout)
+    return cudaErrorInvalidValue;
   TensorMaps m;
   memcpy(m.m, maps, (size_t)num_layers * sizeof(CUtensorMap));
   const size_t smem = (size_t)stage_bytes * stages + 128;
   auto go = [&](auto kernel) {
-    kernel<<<grid, 32, smem, s>>>(p, m, stage_bytes, stages, timeout);
+    kernel<<<grid, 32, smem, s>>>(p, m, stage_bytes, stages, wt);
     return cudaGetLastError();
   };
   return dir == kPack ? go(tmap_move_kernel<kPack>) : go(tmap_move_kernel<kUnpack>);

@@ -1,7 +1,8 @@
 """Python binding of libkvxfer.so (ctypes): argument marshalling only.
 
-Every function has the name of the C entry point it calls (``include/kvxfer.h``,
-``include/kvxfer_probe.h``); all data movement happens in the library's CUDA
+Every function has the name of the C entry point it calls (``include/kvxfer.h``;
+the measuring probes of ``include/kvxfer_probe.h`` live in ``probe.py``, over a
+library of their own); all data movement happens in the library's CUDA
 kernels and copies.  Tensors are PyTorch tensors (device memory, pinned host
 buffers, streams); a C status other than ``KVX_OK`` raises ``KvxError``.
 
@@ -26,8 +27,6 @@ KVX_FLAG_NO_HOST_TOUCH = 0x10
 KVX_FLAGS_ALL = 0x1F
 KVX_ETIMEOUT = -10
 KVX_MAX_LAYERS = 128
-KVX_PROBE_RAW, KVX_PROBE_WAIT_THEN_COPY, KVX_PROBE_ASYNC_ON_STREAM = 0, 1, 2
-KVX_PROBE_MAX_CYCLES = 4_000_000_000
 
 MODE_NAMES = {KVX_MODE_AUTO: "auto", KVX_MODE_STAGED: "staged", KVX_MODE_ZEROCOPY: "zerocopy"}
 
@@ -36,12 +35,12 @@ EXPORTED = (
     "kv_ctx_create", "kv_ctx_destroy", "kv_chunk_layout", "kv_store", "kv_load", "kv_pack", "kv_unpack",
     "kv_state_store", "kv_state_load", "kv_get_device_error", "kv_ctx_stats", "kv_ctx_reset_stats",
     "kv_ctx_modes", "kv_last_cuda_error", "kv_last_error_message", "kv_status_string", "kv_abi_version",
-    "kvx_probe_delayed_fill", "kvx_probe_delayed_copy", "kvx_probe_copy", "kv_store_noalloc",
+    "kv_store_noalloc",
     "kv_host_alloc", "kv_host_free", "kv_pool_view_check",
     "kv_chunk_keys", "kv_tier_create", "kv_tier_create_on", "kv_tier_destroy", "kv_tier_reserve", "kv_tier_reserve_many", "kv_tier_commit", "kv_tier_commit_many",
     "kv_tier_acquire", "kv_tier_release", "kv_tier_acquire_many", "kv_tier_release_many", "kv_tier_prefix_hits", "kv_tier_stats", "kv_fault_inject",
     "kv_tier_open_shared", "kv_tier_poll", "kv_tier_reclaim", "kv_host_alloc_numa", "kv_host_alloc_ex",
-    "kv_host_pool_info",
+    "kv_host_pool_info", "kv_host_touch",
 )
 KVX_ENOENT, KVX_EBUSY = -8, -9
 KVX_TIER_CREATE, KVX_TIER_NO_PIN = 0x1, 0x2
@@ -57,7 +56,7 @@ class KvxError(RuntimeError):
 class kvx_opts(ctypes.Structure):
     _fields_ = [("store_mode", ctypes.c_int32), ("load_mode", ctypes.c_int32),
                 ("staging_slots", ctypes.c_int32), ("staging_slot_bytes", ctypes.c_int64),
-                ("max_ctas", ctypes.c_int32), ("flags", ctypes.c_uint32)]
+                ("max_ctas", ctypes.c_int32), ("flags", ctypes.c_uint32), ("wait_cycles", ctypes.c_int64)]
 
 
 class kvx_pool(ctypes.Structure):
@@ -112,9 +111,6 @@ def _declare(lib):
         "kv_last_error_message": (ctypes.c_char_p, []),
         "kv_status_string": (ctypes.c_char_p, [ctypes.c_int]),
         "kv_abi_version": (ctypes.c_int, []),
-        "kvx_probe_delayed_fill": (st, [vp, i64, i32, i64, vp]),
-        "kvx_probe_delayed_copy": (st, [vp, vp, i64, i64, vp]),
-        "kvx_probe_copy": (st, [vp, vp, i64, i32, vp]),
         "kv_store_noalloc": (st, [P(kvx_pool), vp, i64, i64, i64, i32, P(vp), i64, vp, vp]),
         "kv_host_alloc": (st, [i64, P(vp)]),
         "kv_host_free": (None, [vp]),
@@ -140,6 +136,7 @@ def _declare(lib):
         "kv_tier_prefix_hits": (st, [vp, P(ctypes.c_uint64), i64, P(i64)]),
         "kv_tier_stats": (st, [vp, P(kvx_tier_stats)]),
         "kv_fault_inject": (st, [ctypes.c_char_p, i32]),
+        "kv_host_touch": (st, [P(vp), P(i64), i64]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -257,8 +254,8 @@ class KvPool:
 
 def kv_ctx_create(device: int = 0, store_mode: int = KVX_MODE_AUTO, load_mode: int = KVX_MODE_AUTO,
                   staging_slots: int = 0, staging_slot_bytes: int = 0, max_ctas: int = 0,
-                  flags: int = 0) -> int:
-    opts = kvx_opts(store_mode, load_mode, staging_slots, staging_slot_bytes, max_ctas, flags)
+                  flags: int = 0, wait_cycles: int = 0) -> int:
+    opts = kvx_opts(store_mode, load_mode, staging_slots, staging_slot_bytes, max_ctas, flags, wait_cycles)
     out = ctypes.c_void_p()
     _check(_lib.kv_ctx_create(device, ctypes.byref(opts), ctypes.byref(out)), "kv_ctx_create")
     return out.value
@@ -403,6 +400,25 @@ def kv_host_free(ptr: int) -> None:
     _lib.kv_host_free(ptr)
 
 
+def kv_host_touch(buffers) -> None:
+    """Read one byte of every host page of each buffer (tensors, numpy arrays, or
+    (pointer, bytes) pairs) on the library's touch threads; see kvxfer.h."""
+    ptrs, sizes = [], []
+    for b in buffers:
+        if isinstance(b, tuple):
+            p, n = b
+        elif hasattr(b, "data_ptr"):
+            _check_tensor(b, "buffer")
+            p, n = b.data_ptr(), _nbytes(b)
+        else:
+            p, n = b.ctypes.data, b.nbytes
+        ptrs.append(p)
+        sizes.append(n)
+    arr = (ctypes.c_void_p * max(1, len(ptrs)))(*ptrs)
+    sz = (ctypes.c_int64 * max(1, len(sizes)))(*sizes)
+    _check(_lib.kv_host_touch(arr, sz, len(ptrs)), "kv_host_touch")
+
+
 class HostBuffer:
     """A kv_host_alloc allocation with a uint8 CPU tensor view (``.tensor``) over it.
 
@@ -493,23 +509,6 @@ def kv_abi_version() -> int:
 
 def kv_status_string(status: int) -> str:
     return _lib.kv_status_string(status).decode()
-
-
-# ---------------------------------------------------------------- ordering probes
-
-
-def kvx_probe_delayed_fill(dev, nbytes: int, value: int, cycles: int, stream=None) -> None:
-    _check(_lib.kvx_probe_delayed_fill(_ptr(dev), nbytes, value, cycles, _stream_handle(stream)),
-           "kvx_probe_delayed_fill")
-
-
-def kvx_probe_delayed_copy(dst, src, nbytes: int, cycles: int, stream=None) -> None:
-    _check(_lib.kvx_probe_delayed_copy(_ptr(dst), _ptr(src), nbytes, cycles, _stream_handle(stream)),
-           "kvx_probe_delayed_copy")
-
-
-def kvx_probe_copy(dst, src, nbytes: int, how: int, stream=None) -> None:
-    _check(_lib.kvx_probe_copy(_ptr(dst), _ptr(src), nbytes, how, _stream_handle(stream)), "kvx_probe_copy")
 
 
 # ---------------------------------------------------------------- convenience

@@ -3,6 +3,7 @@ its host-only logic (chunk geometry, argument checks) behaves as documented."""
 import ctypes
 import os
 import re
+import time
 
 import pytest
 
@@ -19,10 +20,10 @@ def k():
     return kvxfer
 
 
-def declared_functions():
+def declared_functions(header=None):
     names = set()
     for h in os.listdir(os.path.join(ROOT, "include")):
-        if not h.endswith(".h"):
+        if not h.endswith(".h") or (header and h != header):
             continue
         text = open(os.path.join(ROOT, "include", h)).read()
         text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
@@ -32,12 +33,26 @@ def declared_functions():
 
 
 def test_exports_every_declared_symbol(k):
-    declared = declared_functions()
-    assert "kv_store" in declared and "kvx_probe_copy" in declared
+    declared = declared_functions("kvxfer.h")
+    assert "kv_store" in declared and "kv_store_noalloc" in declared
     lib = ctypes.CDLL(k.library_path())
     missing = [n for n in sorted(declared) if not hasattr(lib, n)]
     assert not missing, missing
     assert set(k.EXPORTED) == declared
+
+
+def test_probe_library_exports_its_header_and_the_transfer_library_no_probe(k):
+    """The measuring probes live in libkvxfer_probe.so only."""
+    from paper_2609_15021_gb300 import probe
+    declared = declared_functions("kvxfer_probe.h")
+    assert "kvx_probe_copy" in declared and "kvx_probe_stream_copy" in declared
+    lib = ctypes.CDLL(probe.library_path())
+    missing = [n for n in sorted(declared) if not hasattr(lib, n)]
+    assert not missing, missing
+    assert set(probe.EXPORTED) == declared
+    product = ctypes.CDLL(k.library_path())
+    assert not [n for n in declared if hasattr(product, n)]
+    assert declared_functions() == declared | set(k.EXPORTED)
 
 
 def declared_constants():
@@ -57,20 +72,24 @@ def declared_constants():
 
 
 def test_binding_constants_match_headers(k):
+    from paper_2609_15021_gb300 import probe
     declared = declared_constants()
     for name in ("KVX_OK", "KVX_ETIMEOUT", "KVX_FLAG_DEVICE_LSU", "KVX_FLAGS_ALL", "KVX_PROBE_MAX_CYCLES",
                  "KVX_NOALLOC_SCRATCH_BYTES", "KVX_TIER_NO_PIN", "KVX_MODE_ZEROCOPY"):
         assert name in declared, name
-    mismatched = {n: (v, getattr(k, n)) for n, v in declared.items() if hasattr(k, n) and getattr(k, n) != v}
+    def binding(n):
+        return probe if n.startswith("KVX_PROBE_") else k
+    mismatched = {n: (v, getattr(binding(n), n)) for n, v in declared.items()
+                  if hasattr(binding(n), n) and getattr(binding(n), n) != v}
     assert not mismatched, mismatched
-    missing = sorted(n for n in declared if not hasattr(k, n) and n not in ("KVX_ABI_VERSION",))
+    missing = sorted(n for n in declared if not hasattr(binding(n), n) and n not in ("KVX_ABI_VERSION",))
     assert not missing, missing
     flags = [v for n, v in declared.items() if n.startswith("KVX_FLAG_")]
     assert declared["KVX_FLAGS_ALL"] == sum(flags) and all(v & (v - 1) == 0 for v in flags)
 
 
 def test_abi_version_and_strings(k):
-    assert k.kv_abi_version() == 2
+    assert k.kv_abi_version() == 3
     assert k.kv_status_string(k.KVX_ENOTPINNED) == "host buffer is not page-locked"
     assert k.kv_status_string(123) == "unknown status"
 
@@ -251,3 +270,46 @@ def test_malformed_fault_environment_is_reported_and_ignored(k, value):
     res, err = _run_with_fault_env(value)
     assert "ignoring KVX_FAULT" in err
     assert not any("injected" in msg for _, msg in res)
+
+
+def test_host_touch_reads_ranges_and_checks_arguments(k):
+    """kv_host_touch on the CPU: any readable host memory, several ranges (one
+    empty), repeated calls; argument errors return KVX_EINVAL before any read."""
+    import numpy as np
+    bufs = [np.ones(5 << 20, np.uint8), np.zeros(0, np.uint8), np.full(12345, 7, np.uint8)]
+    for _ in range(3):
+        k.kv_host_touch(bufs)
+    k.kv_host_touch([])
+    lib = k._lib
+    ptrs = (ctypes.c_void_p * 2)(bufs[0].ctypes.data, None)
+    assert lib.kv_host_touch(ptrs, (ctypes.c_int64 * 2)(16, 0), 2) == k.KVX_OK       # null with size 0: skipped
+    assert lib.kv_host_touch(ptrs, (ctypes.c_int64 * 2)(16, 16), 2) == k.KVX_EINVAL  # null with a size
+    assert lib.kv_host_touch(ptrs, (ctypes.c_int64 * 2)(-1, 0), 2) == k.KVX_EINVAL
+    assert lib.kv_host_touch(ptrs, (ctypes.c_int64 * 2)(16, 0), -1) == k.KVX_EINVAL
+    assert lib.kv_host_touch(None, None, 0) == k.KVX_OK
+
+
+@pytest.mark.filterwarnings("ignore:This process .* is multi-threaded")
+def test_host_touch_in_a_forked_child(k):
+    """A child forked after the touch threads started inherits none of them; its
+    calls read the pages on the calling thread and return."""
+    import numpy as np
+    buf = np.ones(8 << 20, np.uint8)
+    k.kv_host_touch([buf])          # the parent's threads exist from here on
+    pid = os.fork()
+    if pid == 0:
+        code = 1
+        try:
+            for _ in range(3):
+                k.kv_host_touch([buf])
+            code = 0
+        finally:
+            os._exit(code)
+    deadline = time.time() + 60
+    while True:
+        done, status = os.waitpid(pid, os.WNOHANG)
+        if done:
+            break
+        assert time.time() < deadline, "forked child did not finish its touch"
+        time.sleep(0.05)
+    assert os.waitstatus_to_exitcode(status) == 0

@@ -23,7 +23,7 @@ import torch
 import oracle
 from gpu_util import (POISON, device_pool, first_mismatch, gather_pages, host_layers, kvx, np_of, oracle_load,
                       oracle_store)
-from paper_2609_15021_gb300 import synth
+from paper_2609_15021_gb300 import probe, synth
 
 pytestmark = pytest.mark.gpu
 
@@ -38,9 +38,9 @@ def _copy(k, how, dst, src, n, stream):
         with torch.cuda.stream(stream):
             dst.copy_(src, non_blocking=True)
         return
-    code = {"raw": k.KVX_PROBE_RAW, "wait_then_copy": k.KVX_PROBE_WAIT_THEN_COPY,
-            "async_on_stream": k.KVX_PROBE_ASYNC_ON_STREAM}[how]
-    k.kvx_probe_copy(dst, src, n, code, stream)
+    code = {"raw": probe.KVX_PROBE_RAW, "wait_then_copy": probe.KVX_PROBE_WAIT_THEN_COPY,
+            "async_on_stream": probe.KVX_PROBE_ASYNC_ON_STREAM}[how]
+    probe.kvx_probe_copy(dst, src, n, code, stream)
 
 
 def _d2h_mismatches(k, how, n, delay):
@@ -48,7 +48,7 @@ def _d2h_mismatches(k, how, n, delay):
     dev = torch.zeros(n, dtype=torch.uint8, device="cuda")
     host = torch.zeros(n, dtype=torch.uint8).pin_memory()
     torch.cuda.synchronize()
-    k.kvx_probe_delayed_fill(dev, n, 37, delay, stream)   # producer: delayed write of 37
+    probe.kvx_probe_delayed_fill(dev, n, 37, delay, stream)   # producer: delayed write of 37
     _copy(k, how, host, dev, n, stream)
     stream.synchronize()                                   # host completion before consumption
     return int((host != 37).sum())
@@ -60,7 +60,7 @@ def _h2d_mismatches(k, how, n, delay):
     readout = torch.full((n,), 1, dtype=torch.uint8, device="cuda")
     src = torch.full((n,), 53, dtype=torch.uint8).pin_memory()
     torch.cuda.synchronize()
-    k.kvx_probe_delayed_copy(readout, buf, n, delay, stream)  # consumer: delayed read of the old value
+    probe.kvx_probe_delayed_copy(readout, buf, n, delay, stream)  # consumer: delayed read of the old value
     _copy(k, how, buf, src, n, stream)                        # then overwrite with 53
     stream.synchronize()
     torch.cuda.synchronize()
@@ -178,7 +178,7 @@ def test_store_after_delayed_producer(orc, ctxs, n_bytes):
                 host = [torch.full((n_bytes,), POISON, dtype=torch.uint8).pin_memory()]
                 stream = torch.cuda.Stream()
                 torch.cuda.synchronize()
-                k.kvx_probe_delayed_copy(pool.layers[0], final_dev, spec.layer_bytes, delay, stream)
+                probe.kvx_probe_delayed_copy(pool.layers[0], final_dev, spec.layer_bytes, delay, stream)
                 k.kv_store(ctx, pool, table_d, 0, C, C, host, stream=stream)
                 stream.synchronize()
                 got = np_of(host[0])
@@ -209,9 +209,9 @@ def test_load_after_delayed_consumer(orc, ctxs, n_bytes):
                 after = torch.full((spec.layer_bytes,), POISON, dtype=torch.uint8, device="cuda")
                 stream = torch.cuda.Stream()
                 torch.cuda.synchronize()
-                k.kvx_probe_delayed_copy(readout, pool.layers[0], spec.layer_bytes, delay, stream)
+                probe.kvx_probe_delayed_copy(readout, pool.layers[0], spec.layer_bytes, delay, stream)
                 k.kv_load(ctx, pool, table_d, 0, C, C, host, stream=stream)
-                k.kvx_probe_delayed_copy(after, pool.layers[0], spec.layer_bytes, 0, stream)
+                probe.kvx_probe_delayed_copy(after, pool.layers[0], spec.layer_bytes, 0, stream)
                 stream.synchronize()
                 assert first_mismatch(np_of(pool.layers[0]), loaded[0]) is None, (name, delay, trial)
                 # a consumer enqueued after kv_load sees the loaded pages
@@ -256,7 +256,7 @@ def test_injected_delay_at_full_32k_size(orc):
                 stream = torch.cuda.Stream()
                 torch.cuda.synchronize()
                 for l in range(L):
-                    k.kvx_probe_delayed_copy(pool_layers[l], final[l], spec.layer_bytes, DELAY if l == 0 else 0,
+                    probe.kvx_probe_delayed_copy(pool_layers[l], final[l], spec.layer_bytes, DELAY if l == 0 else 0,
                                              stream)
                 k.kv_store(ctx, pool, table_d, 0, T, C, chunks, stream=stream)
                 stream.synchronize()

@@ -415,3 +415,50 @@ def test_calls_after_idle_time(orc, touch):
     loaded, _ = oracle_load(orc, spec, [np.full(spec.layer_bytes, POISON, np.uint8)] * 4, tb, 0, T, C, want)
     for l in range(4):
         assert first_mismatch(np_of(dst.layers[l]), loaded[l]) is None, l
+
+
+@pytest.mark.parametrize("mode", list(MODES))
+def test_tok_end_limit_with_logical_blocks(orc, ctxs, mode):
+    """The range rule of kvxfer.h: tok_end <= table_len * P * B with P pages per
+    logical block.  Exactly at the limit a store, a restore and the allocation-free
+    store move every token bit-exactly; one token beyond it each returns KVX_ERANGE
+    and leaves the chunks and the pool untouched."""
+    k = kvx()
+    P, B, C, n_log = 4, 16, 128, 17
+    spec = oracle.PoolSpec(2, P * 20, B, 2, 64, 2, HND, P)
+    src_np = host_layers(spec, seed=515)
+    src = device_pool(spec, src_np)
+    ta = synth.permuted_table(20, n_log, seed=516)
+    tb = synth.permuted_table(20, n_log, seed=517)
+    ta_d, tb_d = torch.from_numpy(ta).cuda(), torch.from_numpy(tb).cuda()
+    limit = n_log * P * B
+    ctx = ctxs(MODES[mode])
+    # one token beyond: rejected before anything is enqueued
+    full = oracle.chunk_tokens_of(0, limit + 1, C)
+    host = [torch.full((orc.chunk_bytes(spec, n),), POISON, dtype=torch.uint8).pin_memory() for n in full]
+    dst = device_pool(spec)
+    for call in (lambda: k.kv_store(ctx, src, ta_d, 0, limit + 1, C, host),
+                 lambda: k.kv_load(ctx, dst, tb_d, 0, limit + 1, C, host),
+                 lambda: k.kv_store_noalloc(src, ta_d, 0, limit + 1, C, host)):
+        with pytest.raises(k.KvxError) as ex:
+            call()
+        assert ex.value.status == k.KVX_ERANGE
+    torch.cuda.synchronize()
+    assert all(np.all(np_of(h) == POISON) for h in host)
+    assert all(np.all(np_of(l) == POISON) for l in dst.layers)
+    # exactly at the limit
+    want, _ = oracle_store(orc, spec, src_np, ta, 0, limit, C)
+    for store in (lambda h: k.kv_store(ctx, src, ta_d, 0, limit, C, h),
+                  lambda h: k.kv_store_noalloc(src, ta_d, 0, limit, C, h)):
+        got = pinned_chunks(orc, spec, 0, limit, C)
+        store(got)
+        torch.cuda.synchronize()
+        for g, w in zip(got, want):
+            assert first_mismatch(np_of(g), w) is None
+    k.kv_load(ctx, dst, tb_d, 0, limit, C, got)
+    torch.cuda.synchronize()
+    poisoned = [np.full(spec.layer_bytes, POISON, np.uint8) for _ in range(2)]
+    want_l, _ = oracle_load(orc, spec, poisoned, tb, 0, limit, C, want)
+    for l in range(2):
+        assert first_mismatch(np_of(dst.layers[l]), want_l[l]) is None
+    assert k.kv_get_device_error(ctx) == -1

@@ -11,7 +11,7 @@ import torch
 
 import oracle
 from gpu_util import POISON, device_pool, first_mismatch, host_layers, kvx, np_of, oracle_load, oracle_store
-from paper_2609_15021_gb300 import synth
+from paper_2609_15021_gb300 import probe, synth
 
 pytestmark = pytest.mark.gpu
 
@@ -44,7 +44,7 @@ def test_store_then_restore_across_streams_through_the_tier(orc, commit):
         torch.cuda.synchronize()
         # replica A: delayed producer writes the final KV, then each chunk is stored into a slot
         for l in range(spec.num_layers):
-            k.kvx_probe_delayed_copy(pool_a.layers[l], final_dev[l], spec.layer_bytes, DELAY if l == 0 else 0, s_a)
+            probe.kvx_probe_delayed_copy(pool_a.layers[l], final_dev[l], spec.layer_bytes, DELAY if l == 0 else 0, s_a)
         ta_d = torch.from_numpy(ta).cuda()
         if commit == "many":
             slots = tier.reserve_many(keys)
@@ -106,7 +106,7 @@ def test_slots_in_use_by_the_gpu_are_not_evicted(orc):
             tier.commit(key, stream=s)
         s.synchronize()
         # readers enqueue restores behind a long delay and release at once (host side)
-        k.kvx_probe_delayed_copy(busy, busy, busy.numel(), DELAY, s)
+        probe.kvx_probe_delayed_copy(busy, busy, busy.numel(), DELAY, s)
         for key, c in ((101, 0), (102, 1)):
             slot = tier.acquire(key, stream=s)
             k.kv_load(ctx, dst, table, c * C, (c + 1) * C, C, [slot], stream=s)

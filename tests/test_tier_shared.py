@@ -21,6 +21,8 @@ import sys
 import numpy as np
 import pytest
 
+from paper_2609_15021_gb300 import probe
+
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 
@@ -303,7 +305,7 @@ def test_shared_tier_store_in_one_process_restore_in_another(commit):
         torch.cuda.synchronize()
         assert q_out.get(timeout=300) == "ready"  # the other process waits for the keys from here on
         for l in range(4):   # the producer finishes writing the KV ~2*10^9 cycles (~1 s) later
-            k.kvx_probe_delayed_copy(pool.layers[l], final_dev[l], spec.layer_bytes, 2 * 10 ** 9 if l == 0 else 0, s)
+            probe.kvx_probe_delayed_copy(pool.layers[l], final_dev[l], spec.layer_bytes, 2 * 10 ** 9 if l == 0 else 0, s)
         if commit == "many":                    # one store, one publication launch for both chunks
             slots = tier.reserve_many(keys)
             k.kv_store(ctx, pool, ta_d, 0, T, C, slots, stream=s)
@@ -348,7 +350,7 @@ def _child_commits_then_dies(name, q_out):
     t.reserve(503)                   # a reservation left unfinished
     scratch = torch.empty(4096, dtype=torch.uint8, device="cuda")
     torch.cuda.synchronize()
-    k.kvx_probe_delayed_fill(scratch, 4096, 0, 4 * 10 ** 8, s)   # the stores start ~0.2 s from now
+    probe.kvx_probe_delayed_fill(scratch, 4096, 0, 4 * 10 ** 8, s)   # the stores start ~0.2 s from now
     for c, key in enumerate([501, 502]):
         slot = t.reserve(key)
         k.kv_store(ctx, pool, ta_d, c * C, (c + 1) * C, C, [slot], stream=s)
