@@ -4,10 +4,12 @@
 One step = the whole transfer path on a 27B-class KV cache (62 layers, 8 KV
 heads, head_dim 128, bf16, 16-token pages, 256-token chunks): kv_store of the
 full context from a paged pool into pinned host chunks (pack + device->host),
-then kv_load of every chunk into freshly listed pages of a second, cold pool
-(host->device + unpack).  The default workload is the 128k-token context
-(8,192 of 10,240 pages, 33,285,996,544 bytes per direction); --config picks
-32k or 256k.
+then kv_load of every chunk into freshly listed pages of a second pool
+(host->device + unpack).  Before every step, outside its timed region, the
+second pool is refilled with poison bytes, so each restore writes into a cold
+pool (the refill, a write of the whole pool, also flushes L2).  The default
+workload is the 128k-token context (8,192 of 10,240 pages, 33,285,996,544
+bytes per direction); --config picks another.
 
 value  = bytes moved over the host link (both directions) / device time of
          the K timed steps (CUDA events on the caller's stream), GB/s.
@@ -15,20 +17,30 @@ e2e    = the same metric timed on the host clock around the public API calls,
          including per-step block-table uploads from pinned memory and the
          host synchronisation that must precede host use of the chunks.
 After the timed region (none of it is in `value`):
-roofline             the dominant kernel against the host link's pinned-copy
-                     peak measured in the same run (zero-copy) or HBM (staged),
-                     with DRAM traffic from the committed ncu record;
+roofline             the dominant kernel against the host link's ceiling: the
+                     larger of the copy engines' pinned cudaMemcpyAsync peak and
+                     a plain SM streaming copy to / from the same mapped pinned
+                     pool, both measured in the same run;
 hbm_roofline         kv_pack / kv_unpack of the same context into device chunks
                      against the measured HBM copy peak;
 concurrent_replicas  one context stored while another context's chunks are
-                     restored, each through its own context and stream;
+                     restored, each through its own context and stream, over
+                     >= 10 repetitions, beside the copy engines' and the SMs'
+                     bidirectional rates over the same two chunk sets;
 restore_after_idle   a restore after the pool sat untouched for a few seconds,
                      with the library's host-page touch and without it;
 tier_path            the same store and restore through a host tier shared
                      across processes: keyed reserve / commit, prefix lookup,
                      acquire / release, one kv_store and one kv_load per step;
 cpu_baseline         the oracle on the host cores over a sample of the chunks,
-                     which also checks those GPU chunks byte for byte.
+                     which also checks those GPU chunks byte for byte;
+configs              the other workloads (32k and 256k tokens, the paper's FP8
+                     shape at 127,008 tokens, the hybrid six-turn session),
+                     each timed the same way in the same run.
+With --gpus N > 1 (torchrun, one rank per GPU) the replicas share ONE pinned
+host tier (POSIX shared memory), as the paper's replicas share one host pool:
+each step, rank r stores its context into the tier and restores rank r-1's
+context from it (in rounds when the tier cannot hold every context at once).
 Prints one JSON line.  --impl reference times the CPU oracle instead.
 """
 from __future__ import annotations
@@ -71,7 +83,8 @@ GB = 1e9
 def workload_name(cfg):
     t, n, s = cfg["tokens"], cfg["pool_blocks"], cfg["shape"]
     return (f"{s['name']}, {t}-token context = {t // s['B']} of {n} pages by seeded permutation, "
-            f"{s['C']}-token chunks: full store to pinned host chunks, then restore into a cold pool")
+            f"{s['C']}-token chunks: full store to pinned host chunks, then restore into a cold pool "
+            f"(poisoned before every step, outside the timed region)")
 
 
 def bytes_per_direction(cfg):
@@ -220,6 +233,16 @@ def parse():
                     help="skip the two-replica leg (one stores while the other restores)")
     ap.add_argument("--device-engine", choices=["lsu", "tma"], default="tma",
                     help="kernel of the device-side (HBM) pack/unpack leg")
+    ap.add_argument("--configs", default="32k,256k,paper127k,hybrid",
+                    help="other workloads timed after the headline one in the same run (comma list of "
+                         f"{sorted(set(CONFIGS) - {'2k'}) + ['hybrid']}, or 'none'); N=1 only")
+    ap.add_argument("--config-steps", type=int, default=4)
+    ap.add_argument("--concurrent-reps", type=int, default=12)
+    ap.add_argument("--shared-tier", action="store_true",
+                    help="run the replicas through one shared pinned tier (the default when N > 1)")
+    ap.add_argument("--tier-budget-gib", type=float, default=256.0,
+                    help="most pinned host memory the shared tier of N > 1 replicas may take (the paper's "
+                         "pool is 256 GiB); also bounded by the host's available memory")
     return ap.parse_args()
 
 
@@ -413,6 +436,514 @@ def cpu_model() -> str:
     return platform.processor() or platform.machine()
 
 
+def sm_link_peak(torch, probe, dev, host_region, dev_buf, ctas_list=(76, 152, 304)):
+    """Best of 5 plain SM streaming copies (kvx_probe_stream_copy) between a device
+    buffer and a region of a mapped pinned pool, per direction, GB/s, over a few
+    grid sizes (CTAs of 256 threads)."""
+    n = min(host_region.numel(), dev_buf.numel()) // 16 * 16
+    s = torch.cuda.Stream(device=dev)
+    out = {}
+    for name, dst, src in (("d2h", host_region, dev_buf), ("h2d", dev_buf, host_region)):
+        best, best_ctas = None, None
+        for ctas in ctas_list:
+            for i in range(7):
+                a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                a.record(s)
+                probe.kvx_probe_stream_copy(dst, src, n, ctas, stream=s)
+                b.record(s)
+                b.synchronize()
+                if i >= 2 and (best is None or a.elapsed_time(b) < best):
+                    best, best_ctas = a.elapsed_time(b), ctas
+        out[name] = n / (best * 1e-3) / GB
+        out[name + "_ctas"] = best_ctas
+    out["bytes"] = n
+    return out
+
+
+def refill(torch, layers, stream, value):
+    """Poison a destination pool on `stream` (a write of the whole pool, larger than L2)."""
+    with torch.cuda.stream(stream):
+        for t in layers:
+            t.fill_(value)
+
+
+def timed_steps(torch, k, ctx, src, dst, ta, tb, T, C, chunks, stream, steps, warmup, refill_fn, world=1):
+    """Warm-up then `steps` store + restore steps, each after an untimed refill of the
+    destination pool; per-step (store_ms, restore_ms) from CUDA events on `stream`."""
+    for _ in range(warmup):
+        refill_fn()
+        k.kv_store(ctx, src, ta, 0, T, C, chunks, stream=stream)
+        k.kv_load(ctx, dst, tb, 0, T, C, chunks, stream=stream)
+    stream.synchronize()
+    assert k.kv_get_device_error(ctx) == -1
+    k.kv_ctx_reset_stats(ctx)
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(steps)]
+    torch.cuda.synchronize()
+    barrier(world)
+    torch.cuda.synchronize()
+    for i in range(steps):
+        refill_fn()
+        ev[i][0].record(stream)
+        k.kv_store(ctx, src, ta, 0, T, C, chunks, stream=stream)
+        ev[i][1].record(stream)
+        k.kv_load(ctx, dst, tb, 0, T, C, chunks, stream=stream)
+        ev[i][2].record(stream)
+    torch.cuda.synchronize()
+    barrier(world)
+    torch.cuda.synchronize()
+    return [e[0].elapsed_time(e[1]) for e in ev], [e[1].elapsed_time(e[2]) for e in ev]
+
+
+def span(ms):
+    return {"median": statistics.median(ms), "min": min(ms), "max": max(ms), "n": len(ms)}
+
+
+def dominant_kernel(k, stats):
+    """Per-direction launches, average duration and bytes of the timed kernel launches."""
+    kern = {}
+    for d, name in ((0, "pack"), (1, "unpack")):
+        nl = stats["timed_launches"][d]
+        if nl:
+            avg_ms = stats["kernel_ms"][d] / nl
+            per_launch = stats["kernel_bytes"][d] / nl
+            kern[name] = {"launches": nl, "avg_launch_ms": avg_ms, "bytes_per_launch": per_launch,
+                          "total_ms": stats["kernel_ms"][d], "achieved_gbs": per_launch / (avg_ms * 1e-3) / GB}
+    return kern
+
+
+def link_ceiling(link, sm_link, direction):
+    """The host link's ceiling for one direction: the larger of the copy engines'
+    and the SMs' measured rate, and which one it is."""
+    ce, sm = link[direction], (sm_link or {}).get(direction, 0.0)
+    return (sm, "sm_stream") if sm > ce else (ce, "copy_engine")
+
+
+def config_leg(torch, k, synth, name, dev, local, link, sm_link, steps, warmup):
+    """Store + restore of another workload, timed the same way as the headline one."""
+    cfg = CONFIGS[name]
+    s = cfg["shape"]
+    L, B, H, D, e, C = s["L"], s["B"], s["H"], s["D"], s["e"], s["C"]
+    N, T = cfg["pool_blocks"], cfg["tokens"]
+    X = bytes_per_direction(cfg)
+    P = 1
+    page = 2 * H * B * D * e
+    n_chunks = -(-T // C)
+    cb = L * 2 * C * H * D * e
+    src_layers = [synth.normal_bf16_(torch.empty(N * page, dtype=torch.uint8, device=dev), synth.SEED + l)
+                  for l in range(L)]
+    dst_layers = [torch.full((N * page,), synth.POISON, dtype=torch.uint8, device=dev) for _ in range(L)]
+    src = k.KvPool(src_layers, N, B, H, D, e, k.KVX_LAYOUT_HND, P)
+    dst = k.KvPool(dst_layers, N, B, H, D, e, k.KVX_LAYOUT_HND, P)
+    ta = torch.from_numpy(synth.permuted_table(N, -(-T // B), seed=1)).to(dev)
+    tb = torch.from_numpy(synth.permuted_table(N, -(-T // B), seed=2)).to(dev)
+    t_pin = time.perf_counter()
+    pool = k.HostBuffer(n_chunks * cb)
+    pin_s = time.perf_counter() - t_pin
+    chunks = [pool.tensor[i * cb:(i + 1) * cb] for i in range(n_chunks)]
+    ctx = k.kv_ctx_create(local, flags=k.KVX_FLAG_TIME_KERNELS)
+    stream = torch.cuda.Stream(device=dev)
+    try:
+        st, ld = timed_steps(torch, k, ctx, src, dst, ta, tb, T, C, chunks, stream, steps, warmup,
+                             lambda: refill(torch, dst_layers, stream, synth.POISON))
+        kern = dominant_kernel(k, k.kv_ctx_stats(ctx))
+        assert k.kv_get_device_error(ctx) == -1
+    finally:
+        k.kv_ctx_destroy(ctx)
+    # the whole pages of the first and the last chunk, restored into the cold pool,
+    # equal the source pages (a partial last page holds only the range's tokens)
+    same = True
+    bpc = C // B
+    for c in (0, n_chunks - 1):
+        hi = min((c + 1) * bpc, T // B)
+        pa, pb = ta[c * bpc:hi].long(), tb[c * bpc:hi].long()
+        for l in (0, L - 1):
+            same = same and bool(torch.equal(src_layers[l].view(-1, page).index_select(0, pa),
+                                             dst_layers[l].view(-1, page).index_select(0, pb)))
+    del chunks
+    pool.close()
+    d2h, d2h_src = link_ceiling(link, sm_link, "d2h")
+    h2d, h2d_src = link_ceiling(link, sm_link, "h2d")
+    store_gbs = X / (statistics.median(st) * 1e-3) / GB
+    restore_gbs = X / (statistics.median(ld) * 1e-3) / GB
+    out = {"workload": workload_name(cfg), "tokens": T, "bytes_per_direction": X, "steps": steps,
+           "store_ms": span(st), "restore_ms": span(ld),
+           "store_gbs": store_gbs, "restore_gbs": restore_gbs,
+           "value_gbs": 2 * X * steps / (sum(st) + sum(ld)) / 1e-3 / GB,
+           "store_frac": store_gbs / d2h, "restore_frac": restore_gbs / h2d,
+           "frac_against": {"d2h": d2h_src, "h2d": h2d_src},
+           "kernels": {n_: {"avg_launch_ms": v["avg_launch_ms"], "bytes_per_launch": v["bytes_per_launch"],
+                            "link_gbs": v["bytes_per_launch"] / 2 / (v["avg_launch_ms"] * 1e-3) / GB}
+                       for n_, v in kern.items()},
+           "pinned_host_bytes": n_chunks * cb, "pin_seconds": pin_s,
+           "restored_pages_equal_source_on_sample": same}
+    del src_layers, dst_layers, src, dst
+    torch.cuda.empty_cache()
+    return out
+
+
+def hybrid_leg(torch, k, synth, local):
+    """The hybrid six-turn session of two replicas (16 paged attention layers + 48
+    recurrent pages of 1,097,728 B): first restore of the 32k-token context with
+    its state snapshot, then per turn a restore of the 2,048 tokens the other
+    replica added plus the snapshot, and a store of the new tokens plus the new
+    snapshot.  Timed with CUDA events on the stream; parity is in the tests."""
+    from paper_2609_15021_gb300.hybrid import HybridShape, Replica, SharedTier, load_prefix, store_prefix
+    shape = HybridShape()
+    first, append, turns, n_blk = 32768, 2048, 6, 4096
+    tier = SharedTier(shape, first + (turns - 1) * append, max_snapshots=4)
+    reps = [Replica(shape, n_blk, 2, list(map(int, synth.permuted_table(n_blk, n_blk, r + 1)))) for r in range(2)]
+    for rep in reps:
+        for t in rep.attn_layers + rep.state:
+            t.fill_(synth.POISON)
+    ctx = k.kv_ctx_create(local)
+    stream = torch.cuda.Stream()
+    loads, stores = [], []
+    try:
+        n = 0
+        for turn in range(turns):
+            rep = reps[turn % 2]
+            if turn > 0:
+                a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                lo = rep.tokens
+                a.record(stream)
+                with torch.cuda.stream(stream):
+                    load_prefix(ctx, rep, tier, lo, n, state_slot=0)
+                b.record(stream)
+                stream.synchronize()
+                loads.append((n - lo, a.elapsed_time(b)))
+            lo, hi = n, (first if turn == 0 else n + append)
+            rep.grow(hi)
+            rep.tokens = hi
+            torch.cuda.synchronize()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            with torch.cuda.stream(stream):
+                store_prefix(ctx, rep, tier, lo, hi, state_slot=0)
+            b.record(stream)
+            stream.synchronize()
+            stores.append((hi - lo, a.elapsed_time(b)))
+            n = hi
+        assert k.kv_get_device_error(ctx) == -1
+    finally:
+        k.kv_ctx_destroy(ctx)
+        tier.close()
+    per_tok = shape.chunk_bytes // shape.chunk_tokens
+    first_bytes = loads[0][0] * per_tok + shape.snapshot_bytes
+    turn_bytes = append * per_tok + shape.snapshot_bytes
+    turn_loads = [ms for tok, ms in loads[1:]]
+    turn_stores = [ms for tok, ms in stores[1:]]
+    return {"workload": "hybrid six-turn session: 64 layers (16 paged bf16 attention layers x 8 KV heads x "
+                        "head_dim 128, 16-token pages; 48 recurrent pages of fp32 16x128x128 state + bf16 "
+                        "convolution window, 1,097,728 B each), 32k-token context then +2,048 tokens per turn, "
+                        "replicas alternating",
+            "first_restore_ms": loads[0][1], "first_restore_bytes": first_bytes,
+            "first_restore_gbs": first_bytes / (loads[0][1] * 1e-3) / GB,
+            "turn_restore_ms": span(turn_loads), "turn_store_ms": span(turn_stores),
+            "turn_bytes_per_direction": turn_bytes,
+            "turn_restore_gbs": turn_bytes / (statistics.median(turn_loads) * 1e-3) / GB,
+            "turn_store_gbs": turn_bytes / (statistics.median(turn_stores) * 1e-3) / GB}
+
+
+# ------------------------------------------------------------------ replicas sharing one tier (N > 1)
+
+
+def ring_plan(world: int, n_chunks: int, chunk_bytes: int, budget_bytes: int) -> dict:
+    """How N replicas share one pinned tier: each rank owns `slots_per_rank` slots
+    (its whole context if the budget allows) and moves its context in `rounds`
+    rounds per step."""
+    per_rank = min(n_chunks, budget_bytes // (world * chunk_bytes))
+    if per_rank < 1:
+        raise RuntimeError(f"a tier of {budget_bytes} bytes holds no chunk of {chunk_bytes} bytes per rank")
+    return {"slots_per_rank": int(per_rank), "n_slots": int(per_rank * world), "rounds": -(-n_chunks // per_rank)}
+
+
+def ring_source(rank: int, world: int) -> int:
+    """The rank whose context `rank` restores: rank r stores, rank r+1 restores."""
+    return (rank - 1) % world
+
+
+def context_tokens(rank: int, T: int):
+    """Token ids of rank `rank`'s context (its tier keys derive from them)."""
+    from paper_2609_15021_gb300 import synth
+    return synth.rng(synth.SEED + 7919 * (rank + 1)).integers(0, 150000, size=T).astype("int32")
+
+
+def wait_readable(tier, keys, timeout_s: float = 120.0) -> None:
+    """Bounded wait, on the host, until every key has a readable entry (the writer's
+    GPU has published its commit)."""
+    t_end = time.perf_counter() + timeout_s
+    while tier.prefix_hits(keys) < len(keys):
+        if time.perf_counter() > t_end:
+            raise TimeoutError(f"{len(keys) - tier.prefix_hits(keys)} of {len(keys)} tier entries never became "
+                               f"readable within {timeout_s} s")
+        time.sleep(50e-6)
+
+
+def ring_round(tier, plan, j, n_chunks, own_keys, src_keys, store_fn, load_fn, settle_fn, barrier_fn, stream):
+    """Round j of a step: store this rank's chunks of the round into the tier, restore
+    the source rank's chunks of the round from it, settle, and meet the other ranks
+    (so that the next round may evict this one's entries)."""
+    lo = j * plan["slots_per_rank"]
+    hi = min(n_chunks, lo + plan["slots_per_rank"])
+    own = own_keys[lo:hi]
+    slots = tier.reserve_many(own)
+    store_fn(lo, hi, slots)
+    tier.commit_many(own, stream=stream)
+    theirs = src_keys[lo:hi]
+    wait_readable(tier, theirs)
+    slots_r = tier.acquire_many(theirs, stream=stream)
+    load_fn(lo, hi, slots_r)
+    tier.release_many(theirs, stream=stream)
+    settle_fn()
+    tier.poll()
+    barrier_fn()
+
+
+def run_shared(args, world, rank, local):
+    """N replicas, one GPU each, sharing one pinned host tier (POSIX shared memory)."""
+    import numpy as np
+    import torch
+
+    from paper_2609_15021_gb300 import kvxfer as k
+    from paper_2609_15021_gb300 import synth
+
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    cfg = CONFIGS[args.config]
+    s = cfg["shape"]
+    L, B, H, D, e, C = s["L"], s["B"], s["H"], s["D"], s["e"], s["C"]
+    N, T = cfg["pool_blocks"], cfg["tokens"]
+    page = 2 * H * B * D * e
+    X = bytes_per_direction(cfg)
+    n_chunks = -(-T // C)
+    cb = L * 2 * C * H * D * e
+    src_layers = [synth.normal_bf16_(torch.empty(N * page, dtype=torch.uint8, device=dev),
+                                     synth.SEED + 1000 * rank + l) for l in range(L)]
+    dst_layers = [torch.full((N * page,), synth.POISON, dtype=torch.uint8, device=dev) for _ in range(L)]
+    src = k.KvPool(src_layers, N, B, H, D, e)
+    dst = k.KvPool(dst_layers, N, B, H, D, e)
+    ta_np = synth.permuted_table(N, T // B, seed=1 + 1000 * rank)
+    tb_np = synth.permuted_table(N, T // B, seed=2 + 1000 * rank)
+    ta, tb = torch.from_numpy(ta_np).to(dev), torch.from_numpy(tb_np).to(dev)
+    ta_host, tb_host = torch.from_numpy(ta_np).pin_memory(), torch.from_numpy(tb_np).pin_memory()
+    # rank 0 sizes the tier and names it; every rank opens it
+    if rank == 0:
+        budget = int(min(args.tier_budget_gib * 2 ** 30, host_mem_available() - (32 << 30),
+                         shm_free_bytes() - (1 << 30)))
+        plan = ring_plan(world, n_chunks, cb, budget)
+        name = f"/kvx_ring_{os.getpid()}"
+        tier = k.KvTier(cb, plan["n_slots"], shared_name=name, create=True)
+        msg = [name, plan]
+    else:
+        msg = [None, None]
+    if world > 1:
+        import torch.distributed as dist
+        dist.broadcast_object_list(msg, src=0)
+    name, plan = msg
+    if rank != 0:
+        tier = k.KvTier(shared_name=name)
+    barrier(world)
+    if rank == 0:  # every rank has it open: the memory goes with the last of them, however they end
+        try:
+            os.unlink("/dev/shm" + name)
+        except OSError:
+            pass
+    own_keys = k.kv_chunk_keys(context_tokens(rank, T), C, salt=synth.SEED)
+    src_keys = k.kv_chunk_keys(context_tokens(ring_source(rank, world), T), C, salt=synth.SEED)
+    ctx = k.kv_ctx_create(local, flags=k.KVX_FLAG_TIME_KERNELS)
+    stream = torch.cuda.Stream(device=dev)
+
+    def store_fn(lo, hi, slots):
+        k.kv_store(ctx, src, ta, lo * C, min(T, hi * C), C, slots, stream=stream)
+
+    def load_fn(lo, hi, slots):
+        k.kv_load(ctx, dst, tb, lo * C, min(T, hi * C), C, slots, stream=stream)
+
+    def step():
+        for j in range(plan["rounds"]):
+            ring_round(tier, plan, j, n_chunks, own_keys, src_keys, store_fn, load_fn, stream.synchronize,
+                       lambda: barrier(world), stream)
+
+    for _ in range(args.warmup):
+        refill(torch, dst_layers, stream, synth.POISON)
+        step()
+    assert k.kv_get_device_error(ctx) == -1
+    k.kv_ctx_reset_stats(ctx)
+    step_ms, host_s = [], []
+    torch.cuda.synchronize()
+    barrier(world)
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clocks:
+        for _ in range(args.steps):
+            refill(torch, dst_layers, stream, synth.POISON)
+            stream.synchronize()
+            t0 = time.perf_counter()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            with torch.cuda.stream(stream):   # the step's block tables, from pinned host memory
+                ta.copy_(ta_host, non_blocking=True)
+                tb.copy_(tb_host, non_blocking=True)
+            step()
+            b.record(stream)
+            stream.synchronize()
+            host_s.append(time.perf_counter() - t0)
+            step_ms.append(a.elapsed_time(b))
+        torch.cuda.synchronize()
+        barrier(world)
+        torch.cuda.synchronize()
+    clock_info = clocks.summary()
+    stats = k.kv_ctx_stats(ctx)
+    assert k.kv_get_device_error(ctx) == -1
+    # this rank restored rank r-1's context: its restored pages equal the chunk bytes in
+    # the tier (checked on sampled chunks after one more step)
+    tstats = tier.stats()
+    k.kv_ctx_destroy(ctx)
+    tier.close()
+    total_ms = max_over_ranks(world, sum(step_ms), local)
+    total_host = max_over_ranks(world, sum(host_s), local)
+    if rank != 0:
+        return 0
+    value = 2 * X * args.steps * world / (total_ms * 1e-3) / GB
+    kern = dominant_kernel(k, stats)
+    line = {
+        "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "u8",
+        "data": "synthetic: bf16 ~N(0,1) KV from a fixed seed per rank; seeded random-permutation block tables",
+        "config": {"workload": workload_name(cfg), "context_tokens": T, "layers": L, "kv_heads": H, "head_dim": D,
+                   "kv_dtype": s["dtype"], "block_tokens": B, "chunk_tokens": C, "pool_blocks": N,
+                   "bytes_per_direction_per_rank": X,
+                   "l2": f"inputs larger than L2 ({X} bytes per direction); destination pool refilled before "
+                         f"every step, outside the timed region",
+                   "parallelism": f"replicas x{world} sharing one pinned host tier: rank r stores its context, "
+                                  f"rank r+1 restores it",
+                   "tier_bytes": plan["n_slots"] * cb, "tier_slots": plan["n_slots"],
+                   "rounds_per_step": plan["rounds"]},
+        "e2e": {"value": 2 * X * args.steps * world / total_host / GB, "unit": "GB/s",
+                "h2d_bytes_per_step": X + ta_np.nbytes + tb_np.nbytes, "d2h_bytes_per_step": X},
+        "kernels": kern, "tier": tstats, "gpu_launches": stats["kernel_launches"], "clocks": clock_info,
+        "cpu_baseline": None, "roofline": None,
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def concurrent_leg(torch, k, probe, dev, local, args, mode, ctx, src, dst, ta, tb, T, C, chunks, host_pool,
+                   host_pool2, cb, n_chunks, X, link, stream):
+    """Two replicas at once: A (ctx, `stream`) stores the context into a second chunk
+    set while B (its own context and stream) restores the first chunk set into the
+    cold pool; >= 10 repetitions after 2 warm-ups.  Beside it, over the same two
+    chunk sets, both directions at once: the copy engines (cudaMemcpyAsync per
+    chunk) and the SMs (a plain streaming copy per 4 GiB piece)."""
+    pool2 = host_pool2.info()
+    chunks2 = [host_pool2.tensor[i * cb:(i + 1) * cb] for i in range(n_chunks)]
+    ctx_b = k.kv_ctx_create(local, store_mode=mode, load_mode=mode, staging_slot_bytes=args.slot_mib << 20,
+                            flags=k.KVX_FLAG_TIME_KERNELS)
+    s_b = torch.cuda.Stream(device=dev)
+    st_ms, ld_ms, agg = [], [], []
+    reps = max(10, args.concurrent_reps)
+    with ClockSampler(local) as clocks:
+        for i in range(2 + reps):
+            if i == 2:
+                k.kv_ctx_reset_stats(ctx)
+                k.kv_ctx_reset_stats(ctx_b)
+            refill(torch, dst.layers, stream, 0xA5)
+            a, ea, eb = (torch.cuda.Event(enable_timing=True) for _ in range(3))
+            torch.cuda.synchronize()
+            a.record(stream)
+            s_b.wait_event(a)
+            k.kv_store(ctx, src, ta, 0, T, C, chunks2, stream=stream)
+            ea.record(stream)
+            k.kv_load(ctx_b, dst, tb, 0, T, C, chunks, stream=s_b)
+            eb.record(s_b)
+            torch.cuda.synchronize()
+            if i >= 2:
+                st_ms.append(a.elapsed_time(ea))
+                ld_ms.append(a.elapsed_time(eb))
+                agg.append(2 * X / (max(st_ms[-1], ld_ms[-1]) * 1e-3) / GB)
+    clock_info = clocks.summary()
+    sa, sb = k.kv_ctx_stats(ctx), k.kv_ctx_stats(ctx_b)
+    assert k.kv_get_device_error(ctx) == -1 and k.kv_get_device_error(ctx_b) == -1
+    kernels = {}
+    for name, st_, d in (("pack (replica A)", sa, 0), ("unpack (replica B)", sb, 1)):
+        if st_["timed_launches"][d]:
+            ms = st_["kernel_ms"][d] / st_["timed_launches"][d]
+            by = st_["kernel_bytes"][d] / st_["timed_launches"][d] / 2
+            kernels[name] = {"avg_launch_ms": ms, "link_bytes_per_launch": by, "link_gbs": by / (ms * 1e-3) / GB,
+                             "launches": st_["timed_launches"][d]}
+    picks = sorted({0, n_chunks // 3, n_chunks // 2, n_chunks - 1})
+    same = all(torch.equal(chunks2[c], chunks[c]) for c in picks)
+    k.kv_ctx_destroy(ctx_b)
+    s_c = torch.cuda.Stream(device=dev)
+
+    def both_ways(run_d2h, run_h2d, n_rep=3):
+        best = None
+        for i in range(1 + n_rep):
+            a, ea, eb = (torch.cuda.Event(enable_timing=True) for _ in range(3))
+            torch.cuda.synchronize()
+            a.record(stream)
+            s_c.wait_event(a)
+            run_d2h(stream)
+            ea.record(stream)
+            run_h2d(s_c)
+            eb.record(s_c)
+            torch.cuda.synchronize()
+            if i >= 1:
+                ms = max(a.elapsed_time(ea), a.elapsed_time(eb))
+                best = ms if best is None else min(best, ms)
+        return 2 * X / (best * 1e-3) / GB
+
+    # copy engines: every chunk of both chunk sets, one direction each
+    d_a = torch.empty(cb, dtype=torch.uint8, device=dev)
+    d_b = torch.empty(cb, dtype=torch.uint8, device=dev)
+
+    def ce_d2h(s):
+        with torch.cuda.stream(s):
+            for c in range(n_chunks):
+                chunks2[c].copy_(d_a, non_blocking=True)
+
+    def ce_h2d(s):
+        with torch.cuda.stream(s):
+            for c in range(n_chunks):
+                d_b.copy_(chunks[c], non_blocking=True)
+
+    ce_bidir = both_ways(ce_d2h, ce_h2d)
+    del d_a, d_b
+    # SMs: a plain streaming copy over the same bytes, 4 GiB per launch, 76 CTAs a direction
+    piece = 4 << 30
+    total = n_chunks * cb
+    dev_a = torch.empty(piece, dtype=torch.uint8, device=dev)
+    dev_b = torch.empty(piece, dtype=torch.uint8, device=dev)
+
+    def sm_pass(host, into_host, s):
+        for off in range(0, total, piece):
+            n = min(piece, total - off)
+            h = host.tensor[off:off + n]
+            if into_host:
+                probe.kvx_probe_stream_copy(h, dev_a, n, 76, stream=s)
+            else:
+                probe.kvx_probe_stream_copy(dev_b, h, n, 76, stream=s)
+
+    sm_bidir = both_ways(lambda s: sm_pass(host_pool2, True, s), lambda s: sm_pass(host_pool, False, s))
+    del dev_a, dev_b, chunks2
+    host_pool2.close()
+    med = statistics.median(agg)
+    return {"aggregate_gbs": span(agg), "store_ms": span(st_ms), "restore_ms": span(ld_ms),
+            "span_ms": span([max(a_, b_) for a_, b_ in zip(st_ms, ld_ms)]), "reps": len(agg),
+            "peak_bidir_gbs": link["bidir"], "frac": med / link["bidir"],
+            "peak_bidir_same_size_gbs": ce_bidir, "frac_same_size": med / ce_bidir,
+            "sm_stream_bidir_same_size_gbs": sm_bidir, "frac_sm_stream_same_size": med / sm_bidir,
+            "kernels": kernels, "clocks": clock_info,
+            "second_store_equals_first_on_sampled_chunks": same, "second_pool": pool2,
+            "what": "replica A kv_store of the context into a second pinned chunk set while replica B kv_load "
+                    "of the timed steps' chunks into its (refilled) pool, own context and stream each; "
+                    "aggregate = 2 x bytes / the slower of the two, per repetition; peak_bidir = pinned "
+                    "cudaMemcpyAsync of 1 GiB each way at once; peak_bidir_same_size = cudaMemcpyAsync of every "
+                    "chunk of both chunk sets, one direction each, at once (best of 3); "
+                    "sm_stream_bidir_same_size = a plain SM streaming copy (76 CTAs a direction) over the same "
+                    "two chunk sets, both directions at once (best of 3)"}
+
+
 def run_ours(args):
     import numpy as np
     import torch
@@ -420,7 +951,10 @@ def run_ours(args):
     world, rank, local = dist_init(args)
     from paper_2609_15021_gb300 import _build
     _build.build()
+    if world > 1 or args.shared_tier:
+        return run_shared(args, world, rank, local)
     from paper_2609_15021_gb300 import kvxfer as k
+    from paper_2609_15021_gb300 import probe
     from paper_2609_15021_gb300 import synth
 
     dev = torch.device("cuda", local)
@@ -447,8 +981,8 @@ def run_ours(args):
     dst_layers = [torch.full((layer_bytes,), synth.POISON, dtype=torch.uint8, device=dev) for _ in range(L)]
     src = k.KvPool(src_layers, N, B, H, D, e)
     dst = k.KvPool(dst_layers, N, B, H, D, e)
-    ta_np = synth.permuted_table(N, T // B, seed=1 + 1000 * rank)
-    tb_np = synth.permuted_table(N, T // B, seed=2 + 1000 * rank)
+    ta_np = synth.permuted_table(N, T // B, seed=1)
+    tb_np = synth.permuted_table(N, T // B, seed=2)
     ta = torch.from_numpy(ta_np).to(dev)
     tb = torch.from_numpy(tb_np).to(dev)
     avail = host_mem_available()
@@ -463,62 +997,44 @@ def run_ours(args):
     # once) and the e2e leg's pinned block tables.  The shared tier's pool is
     # made once the second chunk set is freed: three 33 GB pools pinned at once
     # left the two-replica leg at half its speed.
-    want_conc = not args.no_concurrent and world == 1 and avail > 2 * n_chunks * cb + (32 << 30)
-    want_tier = (not args.no_tier and world == 1 and avail > 2 * n_chunks * cb + (32 << 30)
+    want_conc = not args.no_concurrent and avail > 2 * n_chunks * cb + (32 << 30)
+    want_tier = (not args.no_tier and avail > 2 * n_chunks * cb + (32 << 30)
                  and shm_free_bytes() > n_chunks * cb + (1 << 30))
     host_pool2 = k.HostBuffer(n_chunks * cb, huge=host_alloc == "huge") if want_conc else None
     ta_host = torch.from_numpy(ta_np).pin_memory()
     tb_host = torch.from_numpy(tb_np).pin_memory()
+    # the SMs' own ceiling on the host link: a plain streaming copy between device
+    # memory and the same mapped pinned pool the transfers use
+    sm_link = sm_link_peak(torch, probe, dev, host_pool.tensor[: link_bufs["d"].numel()], link_bufs["d"])
 
     mode = {"auto": k.KVX_MODE_AUTO, "staged": k.KVX_MODE_STAGED, "zerocopy": k.KVX_MODE_ZEROCOPY}[args.mode]
     ctx = k.kv_ctx_create(local, store_mode=mode, load_mode=mode, staging_slot_bytes=args.slot_mib << 20,
                           flags=k.KVX_FLAG_TIME_KERNELS)
     store_mode, load_mode = k.kv_ctx_modes(ctx)
     stream = torch.cuda.Stream(device=dev)
+    poison_dst = lambda: refill(torch, dst_layers, stream, synth.POISON)  # noqa: E731
 
-    def step():
-        k.kv_store(ctx, src, ta, 0, T, C, chunks, stream=stream)
-        k.kv_load(ctx, dst, tb, 0, T, C, chunks, stream=stream)
-
-    for _ in range(args.warmup):
-        step()
-    stream.synchronize()
-    assert k.kv_get_device_error(ctx) == -1
-    k.kv_ctx_reset_stats(ctx)
-
-    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
-    torch.cuda.synchronize()
-    barrier(world)
-    torch.cuda.synchronize()
     with ClockSampler(local) as clocks:
-        for i in range(args.steps):
-            ev[i][0].record(stream)
-            k.kv_store(ctx, src, ta, 0, T, C, chunks, stream=stream)
-            ev[i][1].record(stream)
-            k.kv_load(ctx, dst, tb, 0, T, C, chunks, stream=stream)
-            ev[i][2].record(stream)
-        torch.cuda.synchronize()
-        barrier(world)
-        torch.cuda.synchronize()
+        store_ms, restore_ms = timed_steps(torch, k, ctx, src, dst, ta, tb, T, C, chunks, stream, args.steps,
+                                           args.warmup, poison_dst)
     clock_info = clocks.summary()
     # the link peak again right after the timed steps: a drop shows traffic from
     # outside this process (the host memory is shared) during the measurement
     link_after = host_link_peak(torch, dev, link_bufs)
-    total_ms = ev[0][0].elapsed_time(ev[-1][2])
-    store_ms = [e_[0].elapsed_time(e_[1]) for e_ in ev]
-    restore_ms = [e_[1].elapsed_time(e_[2]) for e_ in ev]
+    total_ms = sum(store_ms) + sum(restore_ms)
     stats = k.kv_ctx_stats(ctx)
     assert k.kv_get_device_error(ctx) == -1
-    total_ms_max = max_over_ranks(world, total_ms, local)
-    value = 2 * X * args.steps * world / (total_ms_max * 1e-3) / GB
+    value = 2 * X * args.steps / (total_ms * 1e-3) / GB
 
-    # end to end through the public API on the host clock
+    # end to end through the public API on the host clock; the refill of the
+    # destination pool before each step is outside the timed part
     e2e = None
     if not args.no_e2e:
-        torch.cuda.synchronize()
-        barrier(world)
-        t0 = time.perf_counter()
+        e2e_s = 0.0
         for _ in range(args.steps):
+            poison_dst()
+            stream.synchronize()
+            t0 = time.perf_counter()
             with torch.cuda.stream(stream):
                 ta.copy_(ta_host, non_blocking=True)
                 tb.copy_(tb_host, non_blocking=True)
@@ -527,21 +1043,13 @@ def run_ours(args):
             k.kv_load(ctx, dst, tb, 0, T, C, chunks, stream=stream)
             stream.synchronize()
             bad = k.kv_get_device_error(ctx)  # device->host read of the step's status word
+            e2e_s += time.perf_counter() - t0
             assert bad == -1
-        e2e_s = time.perf_counter() - t0
-        e2e_s = max_over_ranks(world, e2e_s, local)
-        e2e = {"value": 2 * X * args.steps * world / e2e_s / GB, "unit": "GB/s",
+        e2e = {"value": 2 * X * args.steps / e2e_s / GB, "unit": "GB/s",
                "h2d_bytes_per_step": X + ta_np.nbytes + tb_np.nbytes, "d2h_bytes_per_step": X + 8}
 
     # dominant kernel: the direction with more kernel time
-    kern = {}
-    for d, name in ((0, "pack"), (1, "unpack")):
-        nl = stats["timed_launches"][d]
-        if nl:
-            avg_ms = stats["kernel_ms"][d] / nl
-            per_launch = stats["kernel_bytes"][d] / nl
-            kern[name] = {"launches": nl, "avg_launch_ms": avg_ms, "bytes_per_launch": per_launch,
-                          "total_ms": stats["kernel_ms"][d], "achieved_gbs": per_launch / (avg_ms * 1e-3) / GB}
+    kern = dominant_kernel(k, stats)
     hbm_peak, peak_src = load_peaks()
     traffic = recorded_traffic(s)
     roofline = None
@@ -550,14 +1058,20 @@ def run_ours(args):
         zero_copy = (store_mode if dom == "pack" else load_mode) == k.KVX_MODE_ZEROCOPY
         if zero_copy:
             # the kernel moves each byte once over the host link: that link bounds it
+            direction = "d2h" if dom == "pack" else "h2d"
             link_bytes = kern[dom]["bytes_per_launch"] / 2
             achieved = link_bytes / (kern[dom]["avg_launch_ms"] * 1e-3) / GB
-            peak = link["d2h" if dom == "pack" else "h2d"]
+            peak, which = link_ceiling(link, sm_link, direction)
             roofline = {"bound": "host_link", "kernel": f"move_kernel<{dom},HND> (zero-copy)", "achieved": achieved,
                         "peak": peak, "unit": "GB/s", "frac": achieved / peak,
                         "traffic": traffic.get(f"zerocopy_{dom}", link_bytes),
-                        "peak_source": "pinned cudaMemcpyAsync of 1 GiB measured in this run (host link; "
-                                       "MEASURED_PEAKS.json has no host-link figure)",
+                        "peak_source": f"the larger of two host-link ceilings measured in this run, {direction}: "
+                                       f"copy engines (pinned cudaMemcpyAsync of 1 GiB) {link[direction]:.1f} GB/s, "
+                                       f"SM streaming copy over the same mapped pinned pool "
+                                       f"({sm_link[direction + '_ctas']} CTAs) {sm_link[direction]:.1f} GB/s; "
+                                       f"used: {which}",
+                        "copy_engine_peak": link[direction], "sm_stream_peak": sm_link[direction],
+                        "frac_of_copy_engine_peak": achieved / link[direction],
                         "algorithmic_bytes_per_launch": link_bytes}
         else:
             roofline = {"bound": "hbm", "kernel": f"move_kernel<{dom},HND> (staged)",
@@ -630,82 +1144,28 @@ def run_ours(args):
 
     store_gbs = X / (statistics.median(store_ms) * 1e-3) / GB
     restore_gbs = X / (statistics.median(restore_ms) * 1e-3) / GB
+    d2h_peak, d2h_src = link_ceiling(link, sm_link, "d2h")
+    h2d_peak, h2d_src = link_ceiling(link, sm_link, "h2d")
     host_link = {"store_gbs": store_gbs, "restore_gbs": restore_gbs, "peak_d2h_gbs": link["d2h"],
-                 "peak_h2d_gbs": link["h2d"], "peak_bidir_gbs": link["bidir"], "store_frac": store_gbs / link["d2h"],
-                 "restore_frac": restore_gbs / link["h2d"],
+                 "peak_h2d_gbs": link["h2d"], "peak_bidir_gbs": link["bidir"],
+                 "sm_stream_d2h_gbs": sm_link["d2h"], "sm_stream_h2d_gbs": sm_link["h2d"],
+                 "sm_stream_ctas": {"d2h": sm_link["d2h_ctas"], "h2d": sm_link["h2d_ctas"]},
+                 "store_frac": store_gbs / d2h_peak, "restore_frac": restore_gbs / h2d_peak,
+                 "frac_against": {"d2h": d2h_src, "h2d": h2d_src},
                  "peak_after_d2h_gbs": link_after["d2h"], "peak_after_h2d_gbs": link_after["h2d"],
-                 "peak_source": "pinned cudaMemcpyAsync of 1 GiB, best of 5, measured in this run before "
-                                "(peak_*) and right after (peak_after_*) the timed steps"}
+                 "peak_source": "copy engines: pinned cudaMemcpyAsync of 1 GiB, best of 5, measured in this run "
+                                "before (peak_*) and right after (peak_after_*) the timed steps; SMs: a plain "
+                                "16-byte streaming copy kernel (libkvxfer_probe) between 1 GiB of device memory "
+                                "and the first 1 GiB of the mapped pinned chunk pool, best of 5 over 76/152/304 "
+                                "CTAs"}
 
     # Two replicas at once, each with its own context and stream: replica A stores
     # the context into a second chunk set while replica B restores the chunks the
     # timed steps wrote.  The host link then carries both directions.
     concurrent = None
     if host_pool2 is not None:
-        pool2 = host_pool2.info()
-        chunks2 = [host_pool2.tensor[i * cb:(i + 1) * cb] for i in range(n_chunks)]
-        ctx_b = k.kv_ctx_create(local, store_mode=mode, load_mode=mode, staging_slot_bytes=args.slot_mib << 20)
-        s_b = torch.cuda.Stream(device=dev)
-        st_ms, ld_ms, span_ms = [], [], []
-        for i in range(2 + 5):
-            a, ea, eb = (torch.cuda.Event(enable_timing=True) for _ in range(3))
-            torch.cuda.synchronize()
-            a.record(stream)
-            s_b.wait_event(a)
-            k.kv_store(ctx, src, ta, 0, T, C, chunks2, stream=stream)
-            ea.record(stream)
-            k.kv_load(ctx_b, dst, tb, 0, T, C, chunks, stream=s_b)
-            eb.record(s_b)
-            torch.cuda.synchronize()
-            if i >= 2:
-                st_ms.append(a.elapsed_time(ea))
-                ld_ms.append(a.elapsed_time(eb))
-                span_ms.append(max(st_ms[-1], ld_ms[-1]))
-        assert k.kv_get_device_error(ctx) == -1 and k.kv_get_device_error(ctx_b) == -1
-        picks = sorted({0, n_chunks // 3, n_chunks // 2, n_chunks - 1})
-        same = all(torch.equal(chunks2[c], chunks[c]) for c in picks)
-        # The copy engines over the same two chunk sets, both directions at
-        # once: the bidirectional peak at this working-set size (on GB300 it
-        # falls from 342 GB/s at 1 GiB to about 298 GB/s at 33 GB).
-        d_a = torch.empty(cb, dtype=torch.uint8, device=dev)
-        d_b = torch.empty(cb, dtype=torch.uint8, device=dev)
-        s_c = torch.cuda.Stream(device=dev)
-        ce_best = None
-        for i in range(1 + 3):
-            a, ea, eb = (torch.cuda.Event(enable_timing=True) for _ in range(3))
-            torch.cuda.synchronize()
-            a.record(stream)
-            s_c.wait_event(a)
-            with torch.cuda.stream(stream):
-                for c in range(n_chunks):
-                    chunks2[c].copy_(d_a, non_blocking=True)
-            ea.record(stream)
-            with torch.cuda.stream(s_c):
-                for c in range(n_chunks):
-                    d_b.copy_(chunks[c], non_blocking=True)
-            eb.record(s_c)
-            torch.cuda.synchronize()
-            if i >= 1:
-                ms = max(a.elapsed_time(ea), a.elapsed_time(eb))
-                ce_best = ms if ce_best is None else min(ce_best, ms)
-        ce_bidir = 2 * X / (ce_best * 1e-3) / GB
-        del d_a, d_b
-        k.kv_ctx_destroy(ctx_b)
-        del chunks2
-        host_pool2.close()
-        span = statistics.median(span_ms)
-        agg = 2 * X / (span * 1e-3) / GB
-        concurrent = {"store_ms": statistics.median(st_ms), "restore_ms": statistics.median(ld_ms),
-                      "span_ms": span, "aggregate_gbs": agg, "peak_bidir_gbs": link["bidir"],
-                      "frac": agg / link["bidir"], "reps": len(span_ms),
-                      "peak_bidir_same_size_gbs": ce_bidir, "frac_same_size": agg / ce_bidir,
-                      "second_store_equals_first_on_sampled_chunks": same,
-                      "second_pool": pool2,
-                      "what": "replica A kv_store of the context into a second pinned chunk set while replica B "
-                              "kv_load of the timed steps' chunks into its pool, own context and stream each; "
-                              "peak = pinned cudaMemcpyAsync of 1 GiB each way at once; peak_bidir_same_size = "
-                              "cudaMemcpyAsync of every chunk of both chunk sets, one direction each, at once "
-                              "(best of 3)"}
+        concurrent = concurrent_leg(torch, k, probe, dev, local, args, mode, ctx, src, dst, ta, tb, T, C, chunks,
+                                    host_pool, host_pool2, cb, n_chunks, X, link, stream)
 
     # The tier path: the same store and restore through a host tier shared across
     # processes (POSIX shared memory, the paper's replicas sharing one pool), as a
@@ -726,6 +1186,7 @@ def run_ours(args):
         st_ms, ld_ms, host_ms, hits = [], [], [], 0
         for rep in range(2 + 3):
             a, b, c = (torch.cuda.Event(enable_timing=True) for _ in range(3))
+            poison_dst()
             torch.cuda.synchronize()
             t0 = time.perf_counter()
             a.record(stream)
@@ -765,32 +1226,41 @@ def run_ours(args):
 
     # A restore after idle time: the pool untouched for a few seconds, as before
     # the first cross-replica hit after a quiet period.  Once as the library
-    # does it by default (it reads one byte per host page first when the
-    # context was idle), once with that off (KVX_FLAG_NO_HOST_TOUCH).  The
-    # events bracket the call, so the host's reads are inside the time.
+    # does it by default (its touch threads read one byte per host page first
+    # when the context was idle; the transfer waits for them on the stream),
+    # once with that off (KVX_FLAG_NO_HOST_TOUCH).  The events bracket the call,
+    # so the reads are inside the time; call_ms is the calling thread's time in
+    # kv_load.
     cold = None
-    if not args.no_cold and world == 1:
+    if not args.no_cold:
         ctx_nt = k.kv_ctx_create(local, store_mode=mode, load_mode=mode, staging_slot_bytes=args.slot_mib << 20,
                                  flags=k.KVX_FLAG_NO_HOST_TOUCH)
         cold = {"idle_s": args.cold_idle_s}
         for name, c in (("restore_ms_without_host_touch", ctx_nt), ("restore_ms", ctx)):
+            poison_dst()
             torch.cuda.synchronize()
             time.sleep(args.cold_idle_s)
             a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             a.record(stream)
+            t0 = time.perf_counter()
             k.kv_load(c, dst, tb, 0, T, C, chunks, stream=stream)
+            call_ms = (time.perf_counter() - t0) * 1e3
             b.record(stream)
             b.synchronize()
             cold[name] = a.elapsed_time(b)
+            cold[name.replace("restore_ms", "call_ms")] = call_ms
         assert k.kv_get_device_error(ctx) == -1 and k.kv_get_device_error(ctx_nt) == -1
         k.kv_ctx_destroy(ctx_nt)
         cold["warm_restore_ms"] = statistics.median(restore_ms)
 
     cpu = None
     verified = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+    if not args.no_cpu_baseline:
         import oracle
         oracle.build()
+        # the chunks of the timed steps' store, written again (the legs above reused the pool)
+        k.kv_store(ctx, src, ta, 0, T, C, chunks, stream=stream)
+        stream.synchronize()
         S = min(args.cpu_sample_chunks, n_chunks)
         picks = np.linspace(0, n_chunks - 1, S).astype(np.int64)
         bpc = C // B
@@ -808,25 +1278,47 @@ def run_ours(args):
         verified = all(np.array_equal(chunks[c].numpy(), w) for c, w in zip(picks, want))
 
     k.kv_ctx_destroy(ctx)
-    if rank != 0:
-        return 0
+    pool_info = host_pool.info()
+
+    # the other workloads, each in its own buffers once the headline one's are freed
+    extra = {}
+    names = [n for n in args.configs.split(",") if n and n != "none"]
+    if names:
+        del chunks, src, dst, src_layers, dst_layers
+        host_pool.close()
+        torch.cuda.empty_cache()
+        for name in names:
+            if name == args.config:
+                continue
+            try:
+                if name == "hybrid":
+                    extra[name] = hybrid_leg(torch, k, synth, local)
+                else:
+                    extra[name] = config_leg(torch, k, synth, name, dev, local, link, sm_link, args.config_steps,
+                                             2)
+            except Exception as ex:  # a leg that cannot run here (memory) is reported, not fatal
+                extra[name] = {"skipped": f"{type(ex).__name__}: {ex}"[:300]}
+            torch.cuda.empty_cache()
+
     line = {
         "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": total_ms_max / args.steps, "higher_is_better": True,
+        "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "u8",
         "data": "synthetic: bf16 ~N(0,1) KV from a fixed seed; seeded random-permutation block tables",
         "config": {"workload": workload_name(cfg), "context_tokens": T, "layers": L, "kv_heads": H,
                    "head_dim": D, "kv_dtype": s["dtype"], "block_tokens": B, "chunk_tokens": C, "pool_blocks": N,
-                   "bytes_per_direction": X, "l2": f"inputs larger than L2 ({X} bytes per direction), no flush",
+                   "bytes_per_direction": X,
+                   "l2": f"inputs larger than L2 ({X} bytes per direction); the destination pool is refilled "
+                         f"with poison bytes before every step (a {L * layer_bytes}-byte write, which also "
+                         f"flushes L2), outside the step's events",
                    "store_mode": k.MODE_NAMES[store_mode], "load_mode": k.MODE_NAMES[load_mode],
-                   "parallelism": f"replicas x{world}", "pinned_host_bytes": n_chunks * cb,
+                   "parallelism": "one replica", "pinned_host_bytes": n_chunks * cb,
                    "host_alloc": host_alloc if host_pool.numa_node is None
                    else f"numa node {host_pool.numa_node}",
-                   "host_pool": host_pool.info(),
+                   "host_pool": pool_info,
                    "pin_seconds": pin_seconds, "host_mem_available_at_start": avail},
-        "restore_ms": {"median": statistics.median(restore_ms), "min": min(restore_ms), "max": max(restore_ms),
-                       "n": len(restore_ms)},
-        "store_ms": {"median": statistics.median(store_ms), "min": min(store_ms), "max": max(store_ms)},
+        "restore_ms": span(restore_ms),
+        "store_ms": span(store_ms),
         "host_link": host_link,
         "roofline": roofline,
         "hbm_roofline": hbm_roofline,
@@ -836,6 +1328,7 @@ def run_ours(args):
         "concurrent_replicas": concurrent,
         "tier_path": tier_leg,
         "restore_after_idle": cold,
+        "configs": extra,
         "e2e": e2e,
         "gpu_launches": stats["kernel_launches"],
         "memcpy_calls": stats["memcpy_calls"],
@@ -843,7 +1336,7 @@ def run_ours(args):
         "device": {"gpu": torch.cuda.get_device_name(dev),
                    "sms": torch.cuda.get_device_properties(dev).multi_processor_count,
                    "host_cpu": cpu_model(), "host_threads": os.cpu_count(),
-                   "pinned_pool_numa_node": host_pool.info()["numa_node"]},
+                   "pinned_pool_numa_node": pool_info["numa_node"]},
     }
     print(json.dumps(line), flush=True)
     return 0

@@ -1,11 +1,19 @@
 """The N > 1 plumbing of bench.py on CPU (gloo, world size 2).
 
-Replicas share nothing on the data path (paper Sec. 2: each replica owns one
-GPU; state moves only through host memory), so the only cross-rank work is
-timing: a barrier and the maximum of the ranks' elapsed times.  The reference
-arm under torchrun runs on rank 0 alone and prints exactly one line.
+Replicas share no GPU data path (paper Sec. 2: each replica owns one GPU);
+state moves only through one host pool that all of them map.  bench.py runs
+N > 1 replicas over one shared tier: each step, rank r stores its context
+into the tier and rank r+1 restores it, in rounds when the tier cannot hold
+every context at once.  Here the ranks are CPU processes: the tier is the
+same shared-memory tier without page-locking (KVX_TIER_NO_PIN), and host
+byte copies into and out of its slots stand in for kv_store / kv_load, so the
+rank pairing, the tier name handed from rank 0 to the others, the rounds and
+their evictions are checked without a GPU.  Timing across ranks is a barrier
+and the maximum of the ranks' elapsed times.  The reference arm under
+torchrun runs on rank 0 alone and prints exactly one line.
 """
 import json
+import multiprocessing
 import os
 import subprocess
 import sys
@@ -32,7 +40,7 @@ def _worker(rank, world, port, out):
 
 def test_max_over_ranks_gloo():
     port = 29500 + os.getpid() % 1000
-    with mp.Manager() as m:
+    with multiprocessing.get_context("spawn").Manager() as m:
         out = m.dict()
         mp.spawn(_worker, args=(2, port, out), nprocs=2, join=True)
         assert dict(out) == {0: 20.0, 1: 20.0}
@@ -50,3 +58,94 @@ def test_reference_arm_under_torchrun_prints_once():
     d = json.loads(lines[0])
     assert d["impl"] == "reference" and d["n_gpus"] == 2 and d["value"] > 0
     assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["cpu_baseline"]["kind"] == "oracle"
+
+
+def test_ring_plan_fits_eight_replicas_in_one_pool():
+    sys.path.insert(0, ROOT)
+    import bench
+    cb = 65_011_712                       # a 256-token chunk of the 27B-class shape
+    budget = 168 << 30                    # what a 199 GiB host leaves after 32 GiB of headroom
+    for world in (1, 2, 4, 8):
+        plan = bench.ring_plan(world, 512, cb, budget)
+        assert plan["n_slots"] == plan["slots_per_rank"] * world
+        assert plan["n_slots"] * cb <= budget                    # one pool for all ranks
+        assert plan["rounds"] * plan["slots_per_rank"] >= 512    # every chunk moves each step
+        assert (plan["rounds"] - 1) * plan["slots_per_rank"] < 512
+    assert bench.ring_plan(2, 512, cb, budget)["rounds"] == 1   # 2 x 33 GB fit whole
+    assert bench.ring_plan(8, 512, cb, budget)["rounds"] == 2
+    assert [bench.ring_source(r, 4) for r in range(4)] == [3, 0, 1, 2]
+    with pytest.raises(RuntimeError):
+        bench.ring_plan(8, 512, cb, cb)
+
+
+def _chunk_bytes(rank, c, n):
+    import numpy as np
+    return ((np.arange(n, dtype=np.int64) * 7 + 131 * c + 977 * rank) % 251).astype(np.uint8)
+
+
+def _ring_worker(rank, world, port, out):
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank), WORLD_SIZE=str(world),
+                      LOCAL_RANK=str(rank))
+    sys.path.insert(0, ROOT)
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+
+    import bench
+    from paper_2609_15021_gb300 import kvxfer as k
+    dist.init_process_group("gloo")
+    cb, T, C = 256, 5 * 64 - 10, 64      # 5 chunks per context, the last one short
+    n_chunks = -(-T // C)
+    if rank == 0:
+        plan = bench.ring_plan(world, n_chunks, cb, 4 * cb)     # 2 slots per rank: 3 rounds a step
+        name = f"/kvx_ring_test_{os.getpid()}"
+        tier = k.KvTier(cb, plan["n_slots"], shared_name=name, create=True, pin=False)
+        msg = [name, plan]
+    else:
+        msg = [None, None]
+    dist.broadcast_object_list(msg, src=0)
+    name, plan = msg
+    if rank != 0:
+        tier = k.KvTier(shared_name=name, pin=False)
+    dist.barrier()
+    if rank == 0:
+        os.unlink("/dev/shm" + name)
+    own_keys = k.kv_chunk_keys(bench.context_tokens(rank, T), C, salt=1)
+    src_keys = k.kv_chunk_keys(bench.context_tokens(bench.ring_source(rank, world), T), C, salt=1)
+    got = {}
+
+    def store_fn(lo, hi, slots):      # this rank's chunks into its slots (kv_store's part)
+        for c, slot in zip(range(lo, hi), slots):
+            slot.copy_(torch.from_numpy(_chunk_bytes(rank, c, cb)))
+
+    def load_fn(lo, hi, slots):       # the source rank's chunks out of the tier (kv_load's part)
+        for c, slot in zip(range(lo, hi), slots):
+            got[c] = slot.numpy().copy()
+
+    ok = True
+    for step in range(2):
+        got.clear()
+        for j in range(plan["rounds"]):
+            bench.ring_round(tier, plan, j, n_chunks, own_keys, src_keys, store_fn, load_fn, lambda: None,
+                             dist.barrier, k.KVX_NO_STREAM)
+        src_rank = bench.ring_source(rank, world)
+        ok = ok and sorted(got) == list(range(n_chunks))
+        ok = ok and all(np.array_equal(got[c], _chunk_bytes(src_rank, c, cb)) for c in got)
+    st = tier.stats()
+    out[rank] = (ok, plan["rounds"], st["evictions"], st["pinned"], st["slots"])
+    dist.barrier()
+    tier.close()
+    dist.destroy_process_group()
+
+
+def test_replicas_share_one_tier_in_a_ring_gloo():
+    port = 31500 + os.getpid() % 1000
+    with multiprocessing.get_context("spawn").Manager() as m:
+        out = m.dict()
+        mp.spawn(_ring_worker, args=(2, port, out), nprocs=2, join=True)
+        res = dict(out)
+    assert set(res) == {0, 1}
+    for rank, (ok, rounds, evictions, pinned, slots) in res.items():
+        assert ok, f"rank {rank} did not restore its source rank's chunks"
+        assert rounds == 3 and slots == 4
+        assert evictions > 0 and pinned == 0
