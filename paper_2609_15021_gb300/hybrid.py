@@ -70,10 +70,11 @@ class SharedTier:
         self.present: set[int] = set()              # chunk indices stored
         self.snapshot_slot: dict[int, int] = {}      # boundary token -> slot, oldest first
         self._free_snaps = list(range(max_snapshots))
+        cb = shape.chunk_bytes
+        self._chunk_views = [self.chunks.tensor[c * cb:(c + 1) * cb] for c in range(self.max_chunks)]
 
     def chunk(self, c: int):
-        cb = self.shape.chunk_bytes
-        return self.chunks.tensor[c * cb:(c + 1) * cb]
+        return self._chunk_views[c]
 
     def snapshot(self, boundary: int):
         sb = self.shape.snapshot_bytes
@@ -96,6 +97,7 @@ class SharedTier:
         return chunks and t1 in self.snapshot_slot
 
     def close(self):
+        self._chunk_views = []
         self.chunks.close()
         self.snaps.close()
 
@@ -121,20 +123,32 @@ class Replica:
                              s.elem_bytes)
         self.state = [torch.empty(self.state_slots * s.state_bytes, dtype=torch.uint8, device=self.device)
                       for _ in range(s.state_layers)]
-        self._table_dev = None
+        # The block table only grows (pages are appended), so it lives on the
+        # device at its largest size and each new entry is uploaded once, on the
+        # caller's stream, from a pinned staging copy written once.
+        self._table_dev = torch.empty(self.num_blocks, dtype=torch.int32, device=self.device)
+        self._table_pinned = torch.empty(self.num_blocks, dtype=torch.int32).pin_memory()
+        self._uploaded = 0
 
     def grow(self, n_tokens: int):
         """Allocate fresh pages so the table covers n_tokens."""
         need = -(-n_tokens // self.shape.block_tokens)
         while len(self.table) < need:
             self.table.append(self.free_pages.pop(0))
-        self._table_dev = None
 
-    def table_tensor(self):
+    def table_tensor(self, stream=None):
+        """Device view of the table; entries added since the last call are copied up
+        on `stream` (default: the current stream), ahead of the work that uses them."""
         import torch
-        if self._table_dev is None:
-            self._table_dev = torch.tensor(self.table, dtype=torch.int32, device=self.device)
-        return self._table_dev
+        n = len(self.table)
+        if self._uploaded < n:
+            a = self._uploaded
+            self._table_pinned[a:n] = torch.tensor(self.table[a:n], dtype=torch.int32)
+            s = stream if stream is not None else torch.cuda.current_stream(self._table_dev.device)
+            with torch.cuda.stream(s):
+                self._table_dev[a:n].copy_(self._table_pinned[a:n], non_blocking=True)
+            self._uploaded = n
+        return self._table_dev[:n]
 
 
 def store_prefix(ctx, rep: Replica, tier: SharedTier, t0: int, t1: int, state_slot: int, stream=None):
@@ -142,7 +156,7 @@ def store_prefix(ctx, rep: Replica, tier: SharedTier, t0: int, t1: int, state_sl
     s = tier.shape
     C = s.chunk_tokens
     chunks = [tier.chunk(c) for c in range(t0 // C, -(-t1 // C))]
-    k.kv_store(ctx, rep.pool, rep.table_tensor(), t0, t1, C, chunks, stream=stream)
+    k.kv_store(ctx, rep.pool, rep.table_tensor(stream), t0, t1, C, chunks, stream=stream)
     snap = tier.reserve_snapshot(t1)
     k.kv_state_store(ctx, rep.state, rep.state_slots, s.state_bytes, state_slot, snap, stream=stream)
     tier.present.update(range(t0 // C, -(-t1 // C)))
@@ -159,6 +173,6 @@ def load_prefix(ctx, rep: Replica, tier: SharedTier, t0: int, t1: int, state_slo
     C = s.chunk_tokens
     rep.grow(t1)
     chunks = [tier.chunk(c) for c in range(t0 // C, -(-t1 // C))]
-    k.kv_load(ctx, rep.pool, rep.table_tensor(), t0, t1, C, chunks, stream=stream)
+    k.kv_load(ctx, rep.pool, rep.table_tensor(stream), t0, t1, C, chunks, stream=stream)
     k.kv_state_load(ctx, rep.state, rep.state_slots, s.state_bytes, state_slot, tier.snapshot(t1), stream=stream)
     rep.tokens = t1
