@@ -21,6 +21,7 @@ All data movement is in libkvxfer; this module only keeps the bookkeeping.
 from __future__ import annotations
 
 from dataclasses import dataclass, field
+from typing import Sequence
 
 from . import kvxfer as k
 
@@ -109,14 +110,17 @@ class Replica:
     shape: HybridShape
     num_blocks: int
     state_slots: int
-    free_pages: list[int]                      # allocation order (seeded by the caller)
+    free_pages: Sequence[int]                  # allocation order (seeded by the caller)
     device: str = "cuda"
     table: list[int] = field(default_factory=list)
     tokens: int = 0                            # context length held locally
 
     def __post_init__(self):
+        import collections
+
         import torch
         s = self.shape
+        self.free_pages = collections.deque(self.free_pages)  # taken from the front, O(1) each
         self.attn_layers = [torch.empty(self.num_blocks * s.page_bytes, dtype=torch.uint8, device=self.device)
                             for _ in range(s.attn_layers)]
         self.pool = k.KvPool(self.attn_layers, self.num_blocks, s.block_tokens, s.kv_heads, s.head_dim,
@@ -134,7 +138,7 @@ class Replica:
         """Allocate fresh pages so the table covers n_tokens."""
         need = -(-n_tokens // self.shape.block_tokens)
         while len(self.table) < need:
-            self.table.append(self.free_pages.pop(0))
+            self.table.append(self.free_pages.popleft())
 
     def table_tensor(self, stream=None):
         """Device view of the table; entries added since the last call are copied up
