@@ -668,6 +668,22 @@ def context_tokens(rank: int, T: int):
     return synth.rng(synth.SEED + 7919 * (rank + 1)).integers(0, 150000, size=T).astype("int32")
 
 
+def step_salt(step: int) -> int:
+    """Salt of the tier keys of step `step`.  Every step stores its contexts under
+    keys of their own (a new namespace, as for a new request): with the same keys
+    every step, a reader would find the previous step's entry still readable,
+    pin it and restore it before the writer had stored this step's bytes, and the
+    writer's reservation of that key would then fail as busy."""
+    return (314159 + 1000003 * step) & (2 ** 64 - 1)
+
+
+def ring_keys(k, rank: int, world: int, T: int, C: int, step: int):
+    """(this rank's keys, the keys of the rank it restores) for one step."""
+    own = k.kv_chunk_keys(context_tokens(rank, T), C, salt=step_salt(step))
+    src = k.kv_chunk_keys(context_tokens(ring_source(rank, world), T), C, salt=step_salt(step))
+    return own, src
+
+
 def wait_readable(tier, keys, timeout_s: float = 120.0, interval_s: float = 200e-6) -> None:
     """Bounded wait, on the host, until every key has a readable entry (the writer's
     GPU has published its commit).  The writer commits a round's keys together
@@ -760,8 +776,7 @@ def run_shared(args, world, rank, local):
             os.unlink("/dev/shm" + name)
         except OSError:
             pass
-    own_keys = k.kv_chunk_keys(context_tokens(rank, T), C, salt=synth.SEED)
-    src_keys = k.kv_chunk_keys(context_tokens(ring_source(rank, world), T), C, salt=synth.SEED)
+    step_keys = [ring_keys(k, rank, world, T, C, i) for i in range(args.warmup + args.steps)]
     ctx = k.kv_ctx_create(local, flags=k.KVX_FLAG_TIME_KERNELS)
     stream = torch.cuda.Stream(device=dev)
 
@@ -771,14 +786,15 @@ def run_shared(args, world, rank, local):
     def load_fn(lo, hi, slots):
         k.kv_load(ctx, dst, tb, lo * C, min(T, hi * C), C, slots, stream=stream)
 
-    def step():
+    def step(i):
+        own_keys, src_keys = step_keys[i]
         for j in range(plan["rounds"]):
             ring_round(tier, plan, j, n_chunks, own_keys, src_keys, store_fn, load_fn, stream.synchronize,
                        lambda: barrier(world), stream)
 
-    for _ in range(args.warmup):
+    for i in range(args.warmup):
         refill(torch, dst_layers, stream, synth.POISON)
-        step()
+        step(i)
     assert k.kv_get_device_error(ctx) == -1
     k.kv_ctx_reset_stats(ctx)
     step_ms, host_s = [], []
@@ -786,7 +802,7 @@ def run_shared(args, world, rank, local):
     barrier(world)
     torch.cuda.synchronize()
     with ClockSampler(local) as clocks:
-        for _ in range(args.steps):
+        for i in range(args.steps):
             refill(torch, dst_layers, stream, synth.POISON)
             stream.synchronize()
             t0 = time.perf_counter()
@@ -795,7 +811,7 @@ def run_shared(args, world, rank, local):
             with torch.cuda.stream(stream):   # the step's block tables, from pinned host memory
                 ta.copy_(ta_host, non_blocking=True)
                 tb.copy_(tb_host, non_blocking=True)
-            step()
+            step(args.warmup + i)
             b.record(stream)
             stream.synchronize()
             host_s.append(time.perf_counter() - t0)

@@ -78,12 +78,12 @@ def test_ring_plan_fits_eight_replicas_in_one_pool():
         bench.ring_plan(8, 512, cb, cb)
 
 
-def _chunk_bytes(rank, c, n):
+def _chunk_bytes(rank, c, n, step):
     import numpy as np
-    return ((np.arange(n, dtype=np.int64) * 7 + 131 * c + 977 * rank) % 251).astype(np.uint8)
+    return ((np.arange(n, dtype=np.int64) * 7 + 131 * c + 977 * rank + 61 * step) % 251).astype(np.uint8)
 
 
-def _ring_worker(rank, world, port, out):
+def _ring_worker(rank, world, port, out, slots_per_rank):
     os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank), WORLD_SIZE=str(world),
                       LOCAL_RANK=str(rank))
     sys.path.insert(0, ROOT)
@@ -97,7 +97,7 @@ def _ring_worker(rank, world, port, out):
     cb, T, C = 256, 5 * 64 - 10, 64      # 5 chunks per context, the last one short
     n_chunks = -(-T // C)
     if rank == 0:
-        plan = bench.ring_plan(world, n_chunks, cb, 4 * cb)     # 2 slots per rank: 3 rounds a step
+        plan = bench.ring_plan(world, n_chunks, cb, world * slots_per_rank * cb)
         name = f"/kvx_ring_test_{os.getpid()}"
         tier = k.KvTier(cb, plan["n_slots"], shared_name=name, create=True, pin=False)
         msg = [name, plan]
@@ -110,27 +110,27 @@ def _ring_worker(rank, world, port, out):
     dist.barrier()
     if rank == 0:
         os.unlink("/dev/shm" + name)
-    own_keys = k.kv_chunk_keys(bench.context_tokens(rank, T), C, salt=1)
-    src_keys = k.kv_chunk_keys(bench.context_tokens(bench.ring_source(rank, world), T), C, salt=1)
     got = {}
+    step = 0
 
     def store_fn(lo, hi, slots):      # this rank's chunks into its slots (kv_store's part)
         for c, slot in zip(range(lo, hi), slots):
-            slot.copy_(torch.from_numpy(_chunk_bytes(rank, c, cb)))
+            slot.copy_(torch.from_numpy(_chunk_bytes(rank, c, cb, step)))
 
     def load_fn(lo, hi, slots):       # the source rank's chunks out of the tier (kv_load's part)
         for c, slot in zip(range(lo, hi), slots):
             got[c] = slot.numpy().copy()
 
     ok = True
-    for step in range(2):
+    for step in range(3):             # each step's bytes differ: a stale read would show
         got.clear()
+        own_keys, src_keys = bench.ring_keys(k, rank, world, T, C, step)
         for j in range(plan["rounds"]):
             bench.ring_round(tier, plan, j, n_chunks, own_keys, src_keys, store_fn, load_fn, lambda: None,
                              dist.barrier, k.KVX_NO_STREAM)
         src_rank = bench.ring_source(rank, world)
         ok = ok and sorted(got) == list(range(n_chunks))
-        ok = ok and all(np.array_equal(got[c], _chunk_bytes(src_rank, c, cb)) for c in got)
+        ok = ok and all(np.array_equal(got[c], _chunk_bytes(src_rank, c, cb, step)) for c in got)
     st = tier.stats()
     out[rank] = (ok, plan["rounds"], st["evictions"], st["pinned"], st["slots"])
     dist.barrier()
@@ -138,14 +138,19 @@ def _ring_worker(rank, world, port, out):
     dist.destroy_process_group()
 
 
-def test_replicas_share_one_tier_in_a_ring_gloo():
-    port = 31500 + os.getpid() % 1000
+@pytest.mark.parametrize("slots_per_rank,rounds", [(2, 3), (5, 1)])
+def test_replicas_share_one_tier_in_a_ring_gloo(slots_per_rank, rounds):
+    """Two slots per rank: three rounds a step, each evicting the last.  Five:
+    whole contexts, so the previous step's entries are still in the tier when
+    the next step starts; each step's own keys keep a reader from taking them
+    for this step's (their bytes differ, and the test would see them)."""
+    port = 31500 + os.getpid() % 1000 + slots_per_rank
     with multiprocessing.get_context("spawn").Manager() as m:
         out = m.dict()
-        mp.spawn(_ring_worker, args=(2, port, out), nprocs=2, join=True)
+        mp.spawn(_ring_worker, args=(2, port, out, slots_per_rank), nprocs=2, join=True)
         res = dict(out)
     assert set(res) == {0, 1}
-    for rank, (ok, rounds, evictions, pinned, slots) in res.items():
+    for rank, (ok, got_rounds, evictions, pinned, slots) in res.items():
         assert ok, f"rank {rank} did not restore its source rank's chunks"
-        assert rounds == 3 and slots == 4
+        assert got_rounds == rounds and slots == 2 * slots_per_rank
         assert evictions > 0 and pinned == 0

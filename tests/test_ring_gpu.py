@@ -8,8 +8,9 @@ context into the tier (kv_store, commit on its stream: the GPU publishes the
 commits) and restores the other rank's context from it (host wait until the
 keys are readable, acquire on its stream, kv_load, release).  The tier holds
 half a context per rank, so each step runs in two rounds whose entries the
-next round evicts.  Each rank checks its restored pages against the oracle's
-restore of the other rank's chunks.  No kernel waits on another process:
+next round evicts.  Every step stores new bytes under keys of its own; each
+rank checks its restored pages against the oracle's restore of the other
+rank's chunks of that step.  No kernel waits on another process:
 only the host polls the tier.
 """
 import multiprocessing
@@ -44,14 +45,14 @@ def _rank(rank, world, port, out):
         n_chunks = -(-T // C)
         cb = orc.chunk_bytes(spec, C)
 
-        def src_np_of(r):
-            return host_layers(spec, 5000 + 17 * r)
+        def src_np_of(r, step):     # every step's context bytes differ: a stale restore would show
+            return host_layers(spec, 5000 + 17 * r + 101 * step)
 
         def ta_of(r):
             return synth.permuted_table(96, n_used, 6000 + r)
 
         tb = synth.permuted_table(96, n_used, 7000 + rank)
-        src = device_pool(spec, src_np_of(rank))
+        src = device_pool(spec, src_np_of(rank, 0))
         dst = device_pool(spec)
         ta_d, tb_d = torch.from_numpy(ta_of(rank)).cuda(), torch.from_numpy(tb).cuda()
         if rank == 0:
@@ -68,8 +69,6 @@ def _rank(rank, world, port, out):
         dist.barrier()
         if rank == 0:
             os.unlink("/dev/shm" + name)
-        own_keys = k.kv_chunk_keys(bench.context_tokens(rank, T), C, salt=9)
-        src_keys = k.kv_chunk_keys(bench.context_tokens(bench.ring_source(rank, world), T), C, salt=9)
         ctx = k.kv_ctx_create(0)
         stream = torch.cuda.Stream()
 
@@ -80,16 +79,19 @@ def _rank(rank, world, port, out):
             k.kv_load(ctx, dst, tb_d, lo * C, min(T, hi * C), C, slots, stream=stream)
 
         ok = []
-        for step in range(2):
+        for step in range(3):
+            for l, a in zip(src.layers, src_np_of(rank, step)):
+                l.copy_(torch.from_numpy(a))
             for l in dst.layers:
                 l.fill_(POISON)
             torch.cuda.synchronize()
+            own_keys, src_keys = bench.ring_keys(k, rank, world, T, C, step)
             for j in range(plan["rounds"]):
                 bench.ring_round(tier, plan, j, n_chunks, own_keys, src_keys, store_fn, load_fn, stream.synchronize,
                                  dist.barrier, stream)
             assert k.kv_get_device_error(ctx) == -1
             s_rank = bench.ring_source(rank, world)
-            chunks, _ = oracle_store(orc, spec, src_np_of(s_rank), ta_of(s_rank), 0, T, C)
+            chunks, _ = oracle_store(orc, spec, src_np_of(s_rank, step), ta_of(s_rank), 0, T, C)
             want, _ = oracle_load(orc, spec, [np.full(spec.layer_bytes, POISON, np.uint8)] * spec.num_layers,
                                   tb, 0, T, C, chunks)
             ok.append(all(first_mismatch(np_of(dst.layers[l]), want[l]) is None for l in range(spec.num_layers)))
@@ -120,5 +122,5 @@ def test_two_replicas_share_one_tier_in_a_ring():
     for rank, r in res.items():
         assert not isinstance(r, str), f"rank {rank}: {r}"
         ok, rounds, evictions, pinned = r
-        assert ok == [True, True], f"rank {rank} restored bytes differ from the oracle: {ok}"
+        assert ok == [True, True, True], f"rank {rank} restored bytes differ from the oracle: {ok}"
         assert rounds == 2 and evictions > 0 and pinned == 0
