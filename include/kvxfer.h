@@ -122,8 +122,8 @@ typedef enum {
    159 ms.  So when a context has begun no transfer for more than 1 s,
    kv_store and kv_load read one byte of every host page of the chunks they
    are given before moving them.  The reads run on a pool of up to 16
-   persistent library threads (started once per process), not on the calling
-   thread: the call enqueues on `stream`, ahead of its transfer, a host
+   persistent library threads (started once per process, by the first
+   kv_ctx_create), not on the calling thread: the call enqueues on `stream`, ahead of its transfer, a host
    function (cudaLaunchHostFunc) that waits until the pages have been read
    (2-4 ms for 33 GB on GB300), so the transfer follows the reads, the call
    itself returns without waiting, and `stream` completes only after the last

@@ -743,8 +743,9 @@ void wait_touch(TouchJob& j) {
   }
 }
 
-// The persistent threads.  Made once, in the process that first needs them;
-// a forked child (which inherits no threads) touches on its calling thread.
+// The persistent threads.  Made once per process, by the first kv_ctx_create
+// (or the first kv_host_touch); a forked child (which inherits no threads)
+// touches on its calling thread.
 struct TouchPool {
   std::mutex mu;
   std::condition_variable cv;
@@ -1128,6 +1129,9 @@ kvx_status kv_ctx_create(int device, const kvx_opts* opts, kvx_ctx** out) {
       for (int l = 0; l < 2; ++l) ctx->move_occ[d][l] = move_ctas_per_sm(d, l);
     ctx->seg_occ = segment_ctas_per_sm();
     if ((e = prepare_tma_kernels()) != cudaSuccess) return fail(e);
+    // the host-page touch threads, once per process, at set-up rather than
+    // inside a transfer call
+    if (!(o.flags & KVX_FLAG_NO_HOST_TOUCH)) touch_pool();
     if (ctx->store_mode == KVX_MODE_STAGED || ctx->load_mode == KVX_MODE_STAGED) {
       kvx_status st = ensure_staging(ctx);
       if (st != KVX_OK) {

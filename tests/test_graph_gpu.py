@@ -107,3 +107,53 @@ def test_tier_calls_during_a_capture(orc):
     finally:
         k.kv_ctx_destroy(ctx)
         tier.close()
+
+
+def test_first_calls_of_a_context_inside_a_capture(orc):
+    """A context's first transfer, or its first after more than 1 s, is when the
+    library reads the chunks' host pages behind a host function on the stream.
+    Made on a capturing stream, that read is skipped: nothing of it enters the
+    graph (a replayed host function would wait on a job that no longer exists).
+    The capture below is the new context's very first call, and a second one
+    follows 1.1 s later; both graphs replay twice bit-exactly."""
+    import time
+    k = kvx()
+    spec = oracle.PoolSpec(4, 64, 16, 8, 128, 2, oracle.HND)
+    C, n_used = 256, 40
+    T = n_used * 16 - 7
+    src = device_pool(spec, host_layers(spec, 21))
+    dst = device_pool(spec)
+    ta = synth.permuted_table(64, n_used, 22)
+    tb = synth.permuted_table(64, n_used, 23)
+    ta_d, tb_d = torch.from_numpy(ta).cuda(), torch.from_numpy(tb).cuda()
+    host = pinned_chunks(orc, spec, 0, T, C)
+    ctx = k.kv_ctx_create(0)
+    try:
+        s = torch.cuda.Stream()
+        torch.cuda.synchronize()
+        graphs = []
+        for pause in (0.0, 1.1):
+            time.sleep(pause)
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=s):   # global capture mode
+                k.kv_store(ctx, src, ta_d, 0, T, C, host)
+                k.kv_load(ctx, dst, tb_d, 0, T, C, host)
+            graphs.append(g)
+        for i, g in enumerate(graphs * 2):
+            new = host_layers(spec, 30 + i)
+            for l, a in enumerate(new):
+                src.layers[l].copy_(torch.from_numpy(a))
+            for t in dst.layers:
+                t.fill_(POISON)
+            torch.cuda.synchronize()
+            g.replay()
+            torch.cuda.synchronize()
+            want, _ = oracle_store(orc, spec, new, ta, 0, T, C)
+            for h, w in zip(host, want):
+                assert first_mismatch(np_of(h), w) is None, i
+            loaded, _ = oracle_load(orc, spec, [np.full(spec.layer_bytes, POISON, np.uint8)] * 4, tb, 0, T, C, want)
+            for l in range(4):
+                assert first_mismatch(np_of(dst.layers[l]), loaded[l]) is None, (i, l)
+        assert k.kv_get_device_error(ctx) == -1
+    finally:
+        k.kv_ctx_destroy(ctx)
