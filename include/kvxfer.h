@@ -123,11 +123,11 @@ typedef enum {
    kv_store and kv_load read one byte of every host page of the chunks they
    are given before moving them.  The reads run on a pool of up to 16
    persistent library threads (started once per process, by the first
-   kv_ctx_create), not on the calling thread: the call enqueues on `stream`, ahead of its transfer, a host
-   function (cudaLaunchHostFunc) that waits until the pages have been read
-   (2-4 ms for 33 GB on GB300), so the transfer follows the reads, the call
-   itself returns without waiting, and `stream` completes only after the last
-   read.  It is skipped while `stream` is being captured.  If the library
+   kv_ctx_create), not on the calling thread: the call enqueues on `stream`,
+   ahead of its transfer, a host function (cudaLaunchHostFunc) that waits
+   until the pages have been read (2-4 ms for 33 GB on GB300), so the transfer
+   follows the reads, the call itself returns without waiting, and `stream`
+   completes only after the last read.  It is skipped while `stream` is being captured.  If the library
    cannot start threads (or in a forked child, which inherits none) the
    calling thread reads the pages itself before it enqueues.  kv_host_touch
    does the same reads on request.  This flag turns the idle-time touch off. */

@@ -141,7 +141,8 @@ extern "C" kvx_status kv_store_noalloc(const kvx_pool* pool, const int32_t* bloc
     st = check_transfer(device, pool, block_table, table_len, tok_begin, tok_end, chunk_tokens, host_chunks,
                         n_chunks, stream, kHostChunks, KVX_MODE_STAGED, &g, &n, nullptr);
     if (st != KVX_OK || n == 0) return st;
-    const int64_t layer_bytes_max = 2ll * std::min<int64_t>(chunk_tokens, tok_end - tok_begin) * pool->num_heads * g.row;
+    const int64_t layer_bytes_max =
+        2ll * std::min<int64_t>(chunk_tokens, tok_end - tok_begin) * pool->num_heads * g.row;
     if (layer_bytes_max > KVX_NOALLOC_SCRATCH_BYTES) {
       char msg[160];
       snprintf(msg, sizeof(msg), "one layer of one chunk needs %lld bytes; the static staging array holds %lld",
@@ -173,7 +174,9 @@ extern "C" kvx_status kv_store_noalloc(const kvx_pool* pool, const int32_t* bloc
     } batch[kMaxJobs];
     int nb = 0;
     int64_t used = 0;
-    auto tokens_of = [&](int64_t i) { return std::min<int64_t>(chunk_tokens, tok_end - (first_chunk + i) * chunk_tokens); };
+    auto tokens_of = [&](int64_t i) {
+      return std::min<int64_t>(chunk_tokens, tok_end - (first_chunk + i) * chunk_tokens);
+    };
     auto layer_bytes = [&](int64_t i) { return 2ll * tokens_of(i) * pool->num_heads * g.row; };
     auto flush = [&]() -> kvx_status {
       if (nb == 0) return KVX_OK;
