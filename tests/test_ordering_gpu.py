@@ -276,3 +276,34 @@ def test_injected_delay_at_full_32k_size(orc):
     finally:
         del chunks
         host.close()
+
+
+def test_stream_copy_probe_moves_the_bytes():
+    """The SM streaming copy that bench.py times as the host link's SM-side
+    ceiling moves exactly the bytes asked, both ways over mapped pinned memory
+    and at every grid size it is timed with; misaligned or pageable arguments
+    are refused before any launch."""
+    k = kvx()
+    n = 64 << 20
+    src = torch.from_numpy(synth.splitmix64_bytes(n + 4096, 77)).cuda()
+    host = torch.full((n + 4096,), POISON, dtype=torch.uint8).pin_memory()
+    back = torch.full((n + 4096,), POISON, dtype=torch.uint8, device="cuda")
+    s = torch.cuda.Stream()
+    for ctas in (1, 76, 152, 304):
+        host.fill_(POISON)
+        back.fill_(POISON)
+        torch.cuda.synchronize()
+        probe.kvx_probe_stream_copy(host, src, n, ctas, stream=s)   # device -> mapped host
+        probe.kvx_probe_stream_copy(back, host, n, ctas, stream=s)  # mapped host -> device
+        s.synchronize()
+        assert torch.equal(host[:n], src[:n].cpu()), ctas
+        assert torch.equal(back[:n], src[:n]), ctas
+        assert bool((host[n:] == POISON).all()) and bool((back[n:] == POISON).all()), ctas
+    for bad, status in (((host[1:], src, 4096), k.KVX_EALIGN), ((host, src, 4095), k.KVX_EALIGN),
+                        ((torch.empty(4096, dtype=torch.uint8), src, 4096), k.KVX_ENOTPINNED)):
+        with pytest.raises(k.KvxError) as e:
+            probe.kvx_probe_stream_copy(*bad, 76, stream=s)
+        assert e.value.status == status
+    with pytest.raises(k.KvxError) as e:
+        probe.kvx_probe_stream_copy(host, src, 4096, 0, stream=s)
+    assert e.value.status == k.KVX_EINVAL
