@@ -83,3 +83,67 @@ def test_random_case(orc, ctxs, seed):
     for l in range(spec.num_layers):
         assert first_mismatch(np_of(dst.layers[l]), want_l[l]) is None, (spec, C, t0, t1, which, l)
     assert k.kv_get_device_error(ctx) == -1
+
+
+N_ENGINE_CASES = 36
+
+
+@pytest.mark.parametrize("seed", range(N_ENGINE_CASES))
+def test_random_case_engines_and_grids(orc, seed):
+    """The same random shapes through every engine and launch shape: device
+    pack/unpack with the default engine, TMA row/flat copies
+    (KVX_FLAG_DEVICE_TMA) or 16-byte loads/stores (KVX_FLAG_DEVICE_LSU); a CTA
+    cap drawn at random (a persistent grid; a ring of stages for TMA); staged
+    mode with slots of one to four layers of a chunk (batches that split
+    chunks by layers); zero-copy with a random cap; and kv_store_noalloc."""
+    k = kvx()
+    spec, used, C, t0, t1 = draw(7000 + seed)
+    r = synth.rng(9000 + seed)
+    P = spec.pages_per_block
+    src_np = host_layers(spec, 11000 + seed)
+    src = device_pool(spec, src_np)
+    ta = synth.permuted_table(spec.num_blocks // P, used, 13 + seed)
+    tb = synth.permuted_table(spec.num_blocks // P, used, 14 + seed)
+    want, _ = oracle_store(orc, spec, src_np, ta, t0, t1, C)
+    want_l, _ = oracle_load(orc, spec, [np.full(spec.layer_bytes, POISON, np.uint8)] * spec.num_layers,
+                            tb, t0, t1, C, want)
+    which = ("device", "staged", "zerocopy", "noalloc")[seed % 4]
+    max_ctas = int(r.choice([0, 1, 3, 7, 19, 64]))
+    flags = 0
+    slot_bytes = 0
+    mode = 2
+    if which == "device":
+        flags = int(r.choice([0, k.KVX_FLAG_DEVICE_TMA, k.KVX_FLAG_DEVICE_LSU]))
+    elif which == "staged":
+        mode = 1
+        layer = 2 * min(C, t1 - t0) * spec.num_heads * spec.head_dim * spec.elem_bytes
+        slot_bytes = (layer * int(r.integers(1, 5)) + 15) // 16 * 16
+    ctx = None if which == "noalloc" else k.kv_ctx_create(0, store_mode=mode, load_mode=mode, max_ctas=max_ctas,
+                                                         flags=flags, staging_slot_bytes=slot_bytes)
+    try:
+        ta_d, tb_d = torch.from_numpy(ta).cuda(), torch.from_numpy(tb).cuda()
+        if which == "device":
+            chunks = device_chunks(orc, spec, t0, t1, C)
+            k.kv_pack(ctx, src, ta_d, t0, t1, C, chunks)
+        else:
+            chunks = pinned_chunks(orc, spec, t0, t1, C)
+            if which == "noalloc":
+                k.kv_store_noalloc(src, ta_d, t0, t1, C, chunks)
+            else:
+                k.kv_store(ctx, src, ta_d, t0, t1, C, chunks)
+        torch.cuda.synchronize()
+        what = (spec, C, t0, t1, which, max_ctas, flags, slot_bytes)
+        for i, (c, w) in enumerate(zip(chunks, want)):
+            assert first_mismatch(np_of(c), w) is None, (what, i)
+        if which == "noalloc":
+            return
+        dst = device_pool(spec)
+        fn = k.kv_unpack if which == "device" else k.kv_load
+        fn(ctx, dst, tb_d, t0, t1, C, chunks)
+        torch.cuda.synchronize()
+        for l in range(spec.num_layers):
+            assert first_mismatch(np_of(dst.layers[l]), want_l[l]) is None, (what, l)
+        assert k.kv_get_device_error(ctx) == -1
+    finally:
+        if ctx is not None:
+            k.kv_ctx_destroy(ctx)
