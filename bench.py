@@ -684,19 +684,11 @@ def ring_keys(k, rank: int, world: int, T: int, C: int, step: int):
     return own, src
 
 
-def wait_readable(tier, keys, timeout_s: float = 120.0, interval_s: float = 200e-6) -> None:
+def wait_readable(tier, keys, timeout_s: float = 120.0) -> None:
     """Bounded wait, on the host, until every key has a readable entry (the writer's
-    GPU has published its commit).  The writer commits a round's keys together
-    (one publication launch), so the wait polls the last key alone, which holds
-    the tier's process-shared lock only briefly while N ranks poll, then checks
-    the whole round once."""
-    t_end = time.perf_counter() + timeout_s
-    for probe_keys in (keys[-1:], keys):
-        while tier.prefix_hits(probe_keys) < len(probe_keys):
-            if time.perf_counter() > t_end:
-                raise TimeoutError(f"{len(keys) - tier.prefix_hits(keys)} of {len(keys)} tier entries never "
-                                   f"became readable within {timeout_s} s")
-            time.sleep(interval_s)
+    GPU has published its commit): kv_tier_wait, which polls with a growing sleep
+    and holds the tier's process-shared lock only while it checks."""
+    tier.wait(keys, timeout_s)
 
 
 def ring_round(tier, plan, j, n_chunks, own_keys, src_keys, store_fn, load_fn, settle_fn, barrier_fn, stream):

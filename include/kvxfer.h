@@ -79,8 +79,9 @@ typedef enum {
   KVX_EDEVICE = -7,    /* a device pointer is not device memory of ctx's GPU    */
   KVX_ENOENT = -8,     /* tier: no committed entry for the key                  */
   KVX_EBUSY = -9,      /* tier: the entry is still in use and cannot be rewritten */
-  KVX_ETIMEOUT = -10   /* a bounded wait inside a kernel expired; the kernel
-                          returned early and its output is incomplete          */
+  KVX_ETIMEOUT = -10   /* a bounded wait expired: inside a kernel (the kernel
+                          returned early and its output is incomplete), or
+                          kv_tier_wait's host wait                             */
 } kvx_status;
 
 typedef enum { KVX_LAYOUT_HND = 0, KVX_LAYOUT_NHD = 1 } kvx_layout;
@@ -570,6 +571,18 @@ kvx_status kv_tier_release_many(kvx_tier* tier, const uint64_t* keys, int64_t n,
 kvx_status kv_tier_reclaim(kvx_tier* tier, int64_t* reclaimed);
 /* Number of leading keys with committed entries (the cached prefix). */
 kvx_status kv_tier_prefix_hits(kvx_tier* tier, const uint64_t* keys, int64_t n, int64_t* hits);
+/*
+ * Waits on the host until all n keys have readable entries -- committed, and
+ * for another process's commits published by the GPU -- or until timeout_ns
+ * has passed (Fig. 1: a replica restores what another replica stored only once
+ * the store is complete).  It checks the keys, then sleeps 20 us, doubling to
+ * at most 1 ms, holding the tier's lock only while it checks, so many waiting
+ * replicas do not hold up the writers.  KVX_OK when every key is readable;
+ * KVX_ETIMEOUT when the limit passed first.  *hits (may be NULL) receives the
+ * number of leading keys readable at the last check.  Nothing is pinned: the
+ * caller acquires the entries afterwards (an entry can be evicted in between).
+ */
+kvx_status kv_tier_wait(kvx_tier* tier, const uint64_t* keys, int64_t n, int64_t timeout_ns, int64_t* hits);
 kvx_status kv_tier_stats(kvx_tier* tier, kvx_tier_stats* out);
 
 /*

@@ -1061,7 +1061,7 @@ const char* kv_status_string(kvx_status s) {
     case KVX_EDEVICE: return "pointer is not device memory of the context's GPU";
     case KVX_ENOENT: return "no committed tier entry for the key";
     case KVX_EBUSY: return "tier entry still in use";
-    case KVX_ETIMEOUT: return "a bounded wait in a kernel expired";
+    case KVX_ETIMEOUT: return "a bounded wait expired";
   }
   return "unknown status";
 }

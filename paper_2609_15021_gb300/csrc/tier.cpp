@@ -993,6 +993,46 @@ kvx_status kv_tier_prefix_hits(kvx_tier* t, const uint64_t* keys, int64_t n, int
   });
 }
 
+kvx_status kv_tier_wait(kvx_tier* t, const uint64_t* keys, int64_t n, int64_t timeout_ns, int64_t* hits) {
+  return guarded([&]() -> kvx_status {
+    if (!t || n < 0 || (n > 0 && !keys) || timeout_ns < 0) return KVX_EINVAL;
+    auto now = [] {
+      timespec ts;
+      clock_gettime(CLOCK_MONOTONIC, &ts);
+      return (int64_t)ts.tv_sec * 1000000000ll + ts.tv_nsec;
+    };
+    const int64_t deadline = now() + timeout_ns;
+    int64_t pause_ns = 20000, h = 0;
+    for (;;) {
+      {
+        TierLock lock(t);
+        poll_locked(t, kFront);
+        // Entries become readable in any order, and one can be evicted again
+        // before it is pinned: count the readable prefix from the start each
+        // time, a lookup per key.
+        h = 0;
+        while (h < n) {
+          const int64_t i = find_slot(t, keys[h]);
+          if (i < 0) break;
+          const SlotMeta& m = t->meta[i];
+          if (!(m.state == kReady || (m.state == kCommitting && m.writer_pid == t->pid))) break;
+          ++h;
+        }
+      }
+      if (h == n || now() >= deadline) break;
+      const int64_t left = deadline - now();
+      const int64_t d = std::max<int64_t>(0, std::min(pause_ns, left));
+      timespec ts{(time_t)(d / 1000000000ll), (long)(d % 1000000000ll)};
+      nanosleep(&ts, nullptr);
+      pause_ns = std::min<int64_t>(pause_ns * 2, 1000000);
+    }
+    if (hits) *hits = h;
+    if (h == n) return KVX_OK;
+    set_error_text("tier entries did not become readable before the wait's limit");
+    return KVX_ETIMEOUT;
+  });
+}
+
 kvx_status kv_tier_stats(kvx_tier* t, kvx_tier_stats* out) {
   return guarded([&]() -> kvx_status {
     if (!t || !out) return KVX_EINVAL;

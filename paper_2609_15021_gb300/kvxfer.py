@@ -40,7 +40,7 @@ EXPORTED = (
     "kv_chunk_keys", "kv_tier_create", "kv_tier_create_on", "kv_tier_destroy", "kv_tier_reserve", "kv_tier_reserve_many", "kv_tier_commit", "kv_tier_commit_many",
     "kv_tier_acquire", "kv_tier_release", "kv_tier_acquire_many", "kv_tier_release_many", "kv_tier_prefix_hits", "kv_tier_stats", "kv_fault_inject",
     "kv_tier_open_shared", "kv_tier_poll", "kv_tier_reclaim", "kv_host_alloc_numa", "kv_host_alloc_ex",
-    "kv_host_pool_info", "kv_host_touch",
+    "kv_host_pool_info", "kv_host_touch", "kv_tier_wait",
 )
 KVX_ENOENT, KVX_EBUSY = -8, -9
 KVX_TIER_CREATE, KVX_TIER_NO_PIN = 0x1, 0x2
@@ -134,6 +134,7 @@ def _declare(lib):
         "kv_tier_acquire_many": (st, [vp, P(ctypes.c_uint64), i64, vp, P(vp)]),
         "kv_tier_release_many": (st, [vp, P(ctypes.c_uint64), i64, vp]),
         "kv_tier_prefix_hits": (st, [vp, P(ctypes.c_uint64), i64, P(i64)]),
+        "kv_tier_wait": (st, [vp, P(ctypes.c_uint64), i64, i64, P(i64)]),
         "kv_tier_stats": (st, [vp, P(kvx_tier_stats)]),
         "kv_fault_inject": (st, [ctypes.c_char_p, i32]),
         "kv_host_touch": (st, [P(vp), P(i64), i64]),
@@ -630,6 +631,19 @@ class KvTier:
         arr = (ctypes.c_uint64 * max(1, len(keys)))(*keys)
         out = ctypes.c_int64()
         _check(_lib.kv_tier_prefix_hits(self.handle, arr, len(keys), ctypes.byref(out)), "kv_tier_prefix_hits")
+        return out.value
+
+    def wait(self, keys, timeout_s: float = 60.0) -> int:
+        """Wait until every key is readable (see kv_tier_wait); returns len(keys), or
+        raises KvxError (KVX_ETIMEOUT) with `.hits`, the readable prefix at the end."""
+        arr = (ctypes.c_uint64 * max(1, len(keys)))(*keys)
+        out = ctypes.c_int64()
+        status = _lib.kv_tier_wait(self.handle, arr, len(keys), int(timeout_s * 1e9), ctypes.byref(out))
+        try:
+            _check(status, "kv_tier_wait")
+        except KvxError as e:
+            e.hits = out.value
+            raise
         return out.value
 
     def reclaim(self) -> int:

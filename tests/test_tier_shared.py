@@ -415,3 +415,58 @@ def test_published_entries_of_a_dead_writer_stay_readable():
             assert first_mismatch(np_of(dst.layers[l]), loaded[l]) is None, f"layer {l}"
     finally:
         tier.close()
+
+
+def _late_writer(name, keys, delay_s, q):
+    sys.path.insert(0, ROOT)
+    import time
+    from paper_2609_15021_gb300 import kvxfer as k
+    t = k.KvTier(shared_name=name, pin=False)
+    q.put("open")
+    time.sleep(delay_s)
+    for key in keys:
+        t.reserve(key).fill_(key % 251)
+        t.commit(key, -1)
+    q.put("committed")
+    t.close()
+
+
+def test_tier_wait_across_processes():
+    """kv_tier_wait returns at once for readable keys, runs out (KVX_ETIMEOUT,
+    the readable prefix reported) when one is missing, and returns soon after
+    another process commits the keys it waits for, well inside its limit."""
+    import time
+    sys.path.insert(0, ROOT)
+    from paper_2609_15021_gb300 import kvxfer as k
+    name = _name("wait")
+    t = k.KvTier(64, 8, shared_name=name, create=True, pin=False)
+    try:
+        for key in (1, 2):
+            t.reserve(key)
+            t.commit(key, -1)
+        assert t.wait([1, 2], timeout_s=0.0) == 2
+        t0 = time.perf_counter()
+        with pytest.raises(k.KvxError) as e:
+            t.wait([1, 2, 3], timeout_s=0.05)
+        waited = time.perf_counter() - t0
+        assert e.value.status == k.KVX_ETIMEOUT and e.value.hits == 2
+        assert 0.04 < waited < 2.0
+        lib = k._lib
+        keys = (__import__("ctypes").c_uint64 * 1)(1)
+        assert lib.kv_tier_wait(t.handle, keys, 1, -1, None) == k.KVX_EINVAL
+        assert lib.kv_tier_wait(t.handle, keys, -1, 0, None) == k.KVX_EINVAL
+        ctx = mp.get_context("spawn")
+        q = ctx.Queue()
+        p = ctx.Process(target=_late_writer, args=(name, [11, 12, 13], 0.3, q))
+        p.start()
+        assert q.get(timeout=60) == "open"
+        t0 = time.perf_counter()
+        assert t.wait([11, 12, 13], timeout_s=30.0) == 3
+        waited = time.perf_counter() - t0
+        assert q.get(timeout=60) == "committed"
+        p.join(timeout=60)
+        assert 0.25 < waited < 10.0
+        assert int(t.acquire(12, -1)[0]) == 12
+        t.release(12, -1)
+    finally:
+        t.close()
