@@ -78,17 +78,12 @@ def _reader_on_gpu1(name, keys, q):
     """Child process on device 1: wait for the keys, acquire them on its stream,
     restore into its own pool, and send the pool bytes back."""
     try:  # a spawned child gets the parent's sys.path, so this module and its helpers import here
-        import time
-
         import torch
 
         from paper_2609_15021_gb300 import kvxfer as k
         torch.cuda.set_device(1)
         tier = k.KvTier(shared_name=name)
-        t_end = time.time() + 120
-        while tier.prefix_hits(keys) < len(keys):
-            assert time.time() < t_end, "entries never became readable"
-            time.sleep(0.001)
+        tier.wait(keys, timeout_s=120)   # until the other GPU has published the commits
         ctx = k.kv_ctx_create(1)
         dst = _pool_on(1)
         s = torch.cuda.Stream(device=1)
