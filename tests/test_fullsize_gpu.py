@@ -377,3 +377,63 @@ def test_fullsize_every_chunk_and_page_vs_torch(mode):
             host.close()
         del src_layers, dst_layers, src, dst
         torch.cuda.empty_cache()
+
+
+def test_fullsize_paper_shape_logical_blocks(orc):
+    """The paper's own KV at full size (Table 1, Sec. 3.1-3.2): 16 attention layers x
+    4 KV heads x head_dim 256 in FP8 (1 byte), 32-token kernel pages packed 49 to a
+    1,568-token logical block, the 127,008-token cross-replica hit = 81 chunks of
+    one logical block each, stored and restored through the default context into
+    a pool of 100 logical blocks.  Sampled chunks against the oracle (packed
+    view, P = 49), their restored pages against the oracle's restore, and the
+    pages of logical blocks outside the load table untouched."""
+    k = kvx()
+    Lp, Bp, Hp, Dp, Ep, P, Cp, T = 16, 32, 4, 256, 1, 49, 1568, 127008
+    n_log = 100
+    spec = oracle.PoolSpec(Lp, n_log * P, Bp, Hp, Dp, Ep, oracle.HND, P)
+    n_chunks = T // Cp
+    cb = orc.chunk_bytes(spec, Cp)
+    assert n_chunks == 81 and cb == 51_380_224
+    host_pool = k.HostBuffer(n_chunks * cb)
+    try:
+        chunks = [host_pool.tensor[i * cb:(i + 1) * cb] for i in range(n_chunks)]
+        src_layers = [synth.normal_bf16_(torch.empty(spec.layer_bytes, dtype=torch.uint8, device="cuda"), 880 + l)
+                      for l in range(Lp)]
+        dst_layers = [torch.full((spec.layer_bytes,), POISON, dtype=torch.uint8, device="cuda") for _ in range(Lp)]
+        src = k.KvPool(src_layers, spec.num_blocks, Bp, Hp, Dp, Ep, k.KVX_LAYOUT_HND, P)
+        dst = k.KvPool(dst_layers, spec.num_blocks, Bp, Hp, Dp, Ep, k.KVX_LAYOUT_HND, P)
+        ta = synth.permuted_table(n_log, n_chunks, seed=31)
+        tb = synth.permuted_table(n_log, n_chunks, seed=32)
+        ctx = k.kv_ctx_create(0)
+        torch.cuda.synchronize()
+        try:
+            stream = torch.cuda.Stream()
+            with torch.cuda.stream(stream):
+                k.kv_store(ctx, src, torch.from_numpy(ta).cuda(), 0, T, Cp, chunks)
+                k.kv_load(ctx, dst, torch.from_numpy(tb).cuda(), 0, T, Cp, chunks)
+            stream.synchronize()
+            assert k.kv_get_device_error(ctx) == -1
+        finally:
+            k.kv_ctx_destroy(ctx)
+        mini = oracle.PoolSpec(Lp, P, Bp, Hp, Dp, Ep, oracle.HND, P)   # one logical block
+        ident = np.zeros(1, dtype=np.int32)
+        pages_of = lambda blk: [int(blk) * P + j for j in range(P)]      # noqa: E731
+        for c in sorted({0, 1, 40, n_chunks - 1, *map(int, synth.rng(33).integers(0, n_chunks, 3))}):
+            pool_np = [gather_pages(t, spec.page_bytes, pages_of(ta[c])) for t in src_layers]
+            want = [np.full(cb, POISON, np.uint8)]
+            assert orc.store(mini, pool_np, ident, 0, Cp, Cp, want)[0] == 0
+            got = np_of(chunks[c])
+            assert sha(got) == sha(want[0]), (c, first_mismatch(got, want[0]))
+            loaded = [np.full(mini.layer_bytes, POISON, np.uint8) for _ in range(Lp)]
+            assert orc.load(mini, loaded, ident, 0, Cp, Cp, want)[0] == 0
+            for l in (0, 7, Lp - 1):
+                got_pages = gather_pages(dst_layers[l], spec.page_bytes, pages_of(tb[c]))
+                assert first_mismatch(got_pages, loaded[l]) is None, (c, l)
+        unused = np.setdiff1d(np.arange(n_log), tb)
+        for l in (0, Lp - 1):
+            for blk in unused[:4]:
+                assert np.all(gather_pages(dst_layers[l], spec.page_bytes, pages_of(blk)) == POISON), (l, blk)
+        del src_layers, dst_layers, src, dst, chunks
+        torch.cuda.empty_cache()
+    finally:
+        host_pool.close()
