@@ -32,6 +32,9 @@ restore_after_idle   a restore after the pool sat untouched for a few seconds,
 tier_path            the same store and restore through a host tier shared
                      across processes: keyed reserve / commit, prefix lookup,
                      acquire / release, one kv_store and one kv_load per step;
+streamed_cross_replica  replica B restores, group by group, what replica A is
+                     storing through a shared tier, each group as soon as it is
+                     committed (time from A's first store to B's last restore);
 cpu_baseline         the oracle on the host cores over a sample of the chunks,
                      which also checks those GPU chunks byte for byte;
 configs              the other workloads (32k and 256k tokens, the paper's FP8
@@ -1260,6 +1263,65 @@ def run_ours(args):
                     "transfer_calls_per_direction": 1,
                     "slots_equal_timed_chunks_on_sample": same, "evictions": tstats["evictions"]}
 
+    # The same two replicas, but B restores what A is storing, group by group, as
+    # soon as each group is stored: A commits every group of chunks on its stream
+    # as it goes, and B's acquire of a group makes B's stream wait for that
+    # group's commit.  The time from A's first store to B's last restore is a
+    # cross-replica hit that arrives while the context is still being stored.
+    streamed = None
+    if want_tier:
+        shm_name = f"/kvx_stream_{os.getpid()}"
+        tier_s = k.KvTier(cb, n_chunks, shared_name=shm_name, create=True)
+        try:
+            os.unlink("/dev/shm" + shm_name)
+        except OSError:
+            pass
+        token_ids = synth.rng(synth.SEED + 1).integers(0, 150000, size=T).astype(np.int32)
+        skeys = k.kv_chunk_keys(token_ids, C, salt=synth.SEED + 1)
+        ctx_b = k.kv_ctx_create(local)
+        s_b = torch.cuda.Stream(device=dev)
+        group = 64
+        groups = [(g, min(n_chunks, g + group)) for g in range(0, n_chunks, group)]
+        tot_ms, st_ms = [], []
+        for rep in range(2 + 3):
+            poison_dst()
+            torch.cuda.synchronize()
+            a, ea, eb = (torch.cuda.Event(enable_timing=True) for _ in range(3))
+            a.record(stream)
+            s_b.wait_event(a)
+            for g0, g1 in groups:
+                slots = tier_s.reserve_many(skeys[g0:g1])
+                k.kv_store(ctx, src, ta, g0 * C, min(T, g1 * C), C, slots, stream=stream)
+                tier_s.commit_many(skeys[g0:g1], stream=stream)
+            ea.record(stream)
+            for g0, g1 in groups:
+                slots = tier_s.acquire_many(skeys[g0:g1], stream=s_b)
+                k.kv_load(ctx_b, dst, tb, g0 * C, min(T, g1 * C), C, slots, stream=s_b)
+                tier_s.release_many(skeys[g0:g1], stream=s_b)
+            eb.record(s_b)
+            torch.cuda.synchronize()
+            tier_s.poll()
+            if rep >= 2:
+                tot_ms.append(a.elapsed_time(eb))
+                st_ms.append(a.elapsed_time(ea))
+        assert k.kv_get_device_error(ctx) == -1 and k.kv_get_device_error(ctx_b) == -1
+        bpc = C // B
+        same = all(bool(torch.equal(src_layers[l].view(-1, page).index_select(0, ta[c * bpc:(c + 1) * bpc].long()),
+                                    dst_layers[l].view(-1, page).index_select(0, tb[c * bpc:(c + 1) * bpc].long())))
+                   for c in (0, n_chunks // 2, n_chunks - 1) for l in (0, L - 1))
+        k.kv_ctx_destroy(ctx_b)
+        tier_s.close()
+        seq_ms = statistics.median(store_ms) + statistics.median(restore_ms)
+        streamed = {"group_chunks": group, "groups": len(groups), "total_ms": span(tot_ms),
+                    "store_ms": statistics.median(st_ms),
+                    "sequential_ms": seq_ms, "speedup_vs_sequential": seq_ms / statistics.median(tot_ms),
+                    "aggregate_gbs": 2 * X / (statistics.median(tot_ms) * 1e-3) / GB,
+                    "restored_pages_equal_source_on_sample": same,
+                    "what": "replica A stores the context into a shared tier in groups of chunks, committing "
+                            "each group on its stream; replica B (own context and stream) acquires each group "
+                            "on its stream, which waits for that group's commit, and restores it; total = A's "
+                            "first store to B's last restore; sequential = the timed steps' store + restore"}
+
     # A restore after idle time: the pool untouched for a few seconds, as before
     # the first cross-replica hit after a quiet period.  Once as the library
     # does it by default (its touch threads read one byte per host page first
@@ -1363,6 +1425,7 @@ def run_ours(args):
         "verified_sample_vs_oracle": verified,
         "concurrent_replicas": concurrent,
         "tier_path": tier_leg,
+        "streamed_cross_replica": streamed,
         "restore_after_idle": cold,
         "configs": extra,
         "e2e": e2e,
