@@ -32,3 +32,18 @@ def test_cross_replica_128k_example():
     assert r.returncode == 0, r.stdout + r.stderr
     print("\n" + r.stdout.strip())
     assert "bit-exact" in r.stdout
+
+
+def test_streamed_cross_replica_example():
+    """B restores each group of 64 chunks as soon as A's GPU has published it,
+    across two processes, and the sampled pages of every run are bit-exact."""
+    import torch
+    free, _ = torch.cuda.mem_get_info()
+    st = os.statvfs("/dev/shm")
+    if free < (130 << 30) or st.f_bavail * st.f_frsize < (34 << 30):
+        pytest.skip("needs ~130 GB of device memory and 34 GB of /dev/shm")
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "examples", "streamed_cross_replica.py")], cwd=ROOT,
+                       capture_output=True, text=True, timeout=900)
+    assert r.returncode == 0, r.stdout + r.stderr
+    print("\n" + r.stdout.strip())
+    assert "bit-exact" in r.stdout
