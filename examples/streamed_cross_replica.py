@@ -8,9 +8,14 @@ of 64 chunks, committing each group on its stream: the GPU publishes a
 group's entries in the tier as soon as its bytes are stored.  Replica B (this
 process) waits for each group with kv_tier_wait, acquires it on its own
 stream, restores it into freshly listed pages of its own pool, and releases
-it; so B restores group g while A stores group g+1.  Both replicas use the one
-GPU here, so A's stores and B's restores share its host link (both
-directions at once).
+it; so B can restore group g while A stores group g+1.  With each replica on
+its own GPU (the paper's setting), the two overlap.  With both processes on
+one GPU, as here without MPS, the GPU time-slices the two processes' contexts,
+so their kernels do not run at the same time and the streamed restore ends
+about when a store followed by a restore would; what the run shows then is
+that every group is published, found and restored intact.  (Two replicas in
+one process, on two streams of one context, do overlap: bench.py's
+streamed_cross_replica leg.)
 
 Prints A's store time, when B's last restore ended relative to the start of
 A's store (host clocks of the two processes), the same for a store followed
