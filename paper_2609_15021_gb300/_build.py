@@ -17,7 +17,7 @@ LIB = os.path.join(PKG, "_lib", "libkvxfer.so")
 PROBE_LIB = os.path.join(PKG, "_lib", "libkvxfer_probe.so")
 
 SOURCES = ["pack_kernels.cu", "segment_kernels.cu", "tma_kernels.cu", "kvxfer.cu", "no_alloc.cu", "tier.cpp",
-           "tier_kernels.cu", "host_alloc.cpp"]
+           "tier_kernels.cu", "host_alloc.cpp", "host_touch.cpp"]
 PROBE_SOURCES = ["probe.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC,-O2,-Wall,-Wextra", f"-I{INCLUDE}"]

@@ -5,6 +5,7 @@
 #include <stdint.h>
 
 #include <new>
+#include <vector>
 
 #include "kvxfer.h"
 
@@ -130,6 +131,17 @@ struct TierPublish {
 cudaError_t launch_tier_publish(const TierPublish& b, cudaStream_t s);
 // Loads the publication kernel (at tier open, never inside a commit).
 cudaError_t prepare_tier_kernels();
+
+// Host-page touch (host_touch.cpp).  start_touch_threads starts the
+// process-wide reading threads once (kv_ctx_create); touch_before_transfer
+// reads one byte per host page of the chunks of a transfer on those threads
+// and enqueues on `stream` a host function that waits for the reads, so the
+// transfer behind it follows them (nothing while `stream` is capturing; on the
+// calling thread where no threads or host function are to be had).  Neither
+// throws: the touch is only a speed-up.
+void start_touch_threads();
+void touch_before_transfer(void* const* chunks, const std::vector<int32_t>& tokens, const kvx_pool* P,
+                           const Geometry& g, cudaStream_t stream);
 
 // Records the last CUDA error seen by this thread (kv_last_cuda_error).
 void set_last_cuda_error(int e);
