@@ -14,7 +14,7 @@
 //   peak from both kinds of pool in a quiet process.  In the benchmark, whose
 //   process also pins and frees other buffers and starts a subprocess,
 //   cudaHostAlloc pools held the peak in every run of an interleaved A/B on
-//   one box (200.5-201.8 GB/s), while the library's huge-page pools fell to
+//   one machine (200.5-201.8 GB/s), while the library's huge-page pools fell to
 //   146-194 GB/s in the same runs: their zero-copy accesses stalled for
 //   hundreds of milliseconds after memory-management events in the process.
 // * The copy engines (cudaMemcpyAsync, KVX_MODE_STAGED) moved 6-18 GB/s from a
