@@ -8,9 +8,9 @@
  * chunks (Table 1: 1,568-token chunks in a 256 GiB RAM pool).  Storing a
  * prefix gathers its pages into packed chunks in pinned host memory; loading
  * it on another replica scatters the chunks into freshly allocated pages
- * (Sec. 3.2, "gather/scatter dependencies").  Every copy is ordered on the
- * caller's current CUDA stream: the paper's diagnosed corruption (Sec. 3.2,
- * Fig. 2) is a copy that omits exactly this dependency.
+ * (Sec. 3.2).  Every copy is ordered on the caller's current CUDA stream:
+ * the paper's diagnosed corruption (Sec. 3.2, Fig. 2) is a copy that omits
+ * exactly this dependency.
  *
  * Data layout (all sizes in bytes unless stated; row = head_dim * elem_bytes):
  *   pool layer l   : num_blocks pages, page = [2 (K,V)][H][B][row] for
