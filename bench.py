@@ -1113,11 +1113,15 @@ def run_ours(args):
                         "frac_of_copy_engine_peak": achieved / link[direction],
                         "algorithmic_bytes_per_launch": link_bytes}
         else:
-            roofline = {"bound": "hbm", "kernel": f"move_kernel<{dom},HND> (staged)",
+            roofline = {"bound": "hbm", "kernel": f"tmap_move_kernel<{dom}> (staged: one staging slot per launch)",
                         "achieved": kern[dom]["achieved_gbs"], "peak": hbm_peak, "unit": "GB/s",
                         "frac": kern[dom]["achieved_gbs"] / hbm_peak,
                         "traffic": traffic.get(f"staged_{dom}", kern[dom]["bytes_per_launch"]), "peak_source": peak_src,
-                        "algorithmic_bytes_per_launch": kern[dom]["bytes_per_launch"]}
+                        "algorithmic_bytes_per_launch": kern[dom]["bytes_per_launch"],
+                        "note": "in staged mode the copy engines' cudaMemcpyAsync over the host link bound the "
+                                "transfer, not this kernel: each launch packs one staging slot in tens of "
+                                "microseconds, so launch and tail time weigh on its rate; host_link.store_frac and "
+                                "restore_frac give the transfer against the link"}
 
     # device-side pack / unpack of the same context into device chunks: the
     # HBM-bound form of the kernels (staged mode, kv_pack / kv_unpack)
