@@ -313,3 +313,23 @@ def test_host_touch_in_a_forked_child(k):
         assert time.time() < deadline, "forked child did not finish its touch"
         time.sleep(0.05)
     assert os.waitstatus_to_exitcode(status) == 0
+
+
+def test_ctx_options_checked_before_any_device_call(k):
+    """Bad options are refused (KVX_EINVAL) before the library looks for a GPU,
+    including a negative limit for the kernels' bounded waits."""
+    for kw in ({"wait_cycles": -1}, {"max_ctas": -1}, {"flags": 0x80}, {"staging_slot_bytes": 17},
+               {"flags": k.KVX_FLAG_DEVICE_TMA | k.KVX_FLAG_DEVICE_LSU}):
+        with pytest.raises(k.KvxError) as e:
+            k.kv_ctx_create(0, **kw)
+        assert e.value.status == k.KVX_EINVAL, kw
+
+
+def test_tier_wait_with_no_keys_returns_at_once(k):
+    t = k.KvTier(64, 2, shared_name=f"/kvx_wait0_{os.getpid()}", create=True, pin=False)
+    try:
+        t0 = time.perf_counter()
+        assert t.wait([], timeout_s=5.0) == 0
+        assert time.perf_counter() - t0 < 1.0
+    finally:
+        t.close()
