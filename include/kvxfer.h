@@ -106,13 +106,16 @@ typedef enum {
                                       paper's missing dependency (Sec. 3.2).
                                       Results are then undefined.             */
 /* Device-side moves (kv_pack, kv_unpack, staged mode) use, by default, the
-   TMA tensor-map kernel for HND pools whose K or V page half is at most
-   48 KiB (one TMA box per page half, staged through shared memory; measured
-   faster than the load/store kernel on GB300), and the 16-byte load/store
-   kernel otherwise.  Zero-copy moves always use the load/store kernel.  The
-   flags below force one of them for device-side moves.                      */
+   TMA kernel when a K or V page half is at most 48 KiB: one tensor-map box
+   per page half for HND pools, one bulk copy per side for NHD pools (whose
+   page halves are contiguous), staged through shared memory; both measured
+   faster than the load/store kernel on GB300.  HND pools that no tensor map
+   describes use the 16-byte load/store kernel.  Zero-copy moves always use
+   the load/store kernel.  The flags below force one of them for device-side
+   moves.                                                                     */
 #define KVX_FLAG_DEVICE_TMA 0x4u   /* TMA everywhere it fits, with one bulk
-                                      copy per row where no tensor map does  */
+                                      copy per row of HND pages no tensor map
+                                      describes                              */
 #define KVX_FLAG_DEVICE_LSU 0x8u   /* the 16-byte load/store kernel always   */
 /* Host memory after idle time.  Measured on GB300 (Grace host): after the
    pinned pool had sat untouched for 10 s, a 128k-token restore through it took
