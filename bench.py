@@ -1111,6 +1111,7 @@ def run_ours(args):
                                        f"used: {which}",
                         "copy_engine_peak": link[direction], "sm_stream_peak": sm_link[direction],
                         "frac_of_copy_engine_peak": achieved / link[direction],
+                        "frac_of_sm_stream_peak": achieved / sm_link[direction],
                         "algorithmic_bytes_per_launch": link_bytes}
         else:
             roofline = {"bound": "hbm", "kernel": f"tmap_move_kernel<{dom}> (staged: one staging slot per launch)",
