@@ -52,10 +52,10 @@ def up_to_date() -> bool:
 def build(force: bool = False, verbose: bool = False, ptxas_report: str | None = None) -> str:
     """Compile every CUDA source in parallel and link both shared libraries;
     returns the path of libkvxfer.so."""
+    if not force and up_to_date():
+        return LIB
     todo = [(lib, srcs) for lib, srcs in ((LIB, SOURCES), (PROBE_LIB, PROBE_SOURCES))
             if force or not _fresh(lib, srcs)]
-    if not todo:
-        return LIB
     os.makedirs(BUILD, exist_ok=True)
     os.makedirs(os.path.dirname(LIB), exist_ok=True)
     nvcc = _nvcc()
