@@ -138,19 +138,20 @@ def _ring_worker(rank, world, port, out, slots_per_rank):
     dist.destroy_process_group()
 
 
-@pytest.mark.parametrize("slots_per_rank,rounds", [(2, 3), (5, 1)])
-def test_replicas_share_one_tier_in_a_ring_gloo(slots_per_rank, rounds):
+@pytest.mark.parametrize("world,slots_per_rank,rounds", [(2, 2, 3), (2, 5, 1), (3, 2, 3)])
+def test_replicas_share_one_tier_in_a_ring_gloo(world, slots_per_rank, rounds):
     """Two slots per rank: three rounds a step, each evicting the last.  Five:
     whole contexts, so the previous step's entries are still in the tier when
     the next step starts; each step's own keys keep a reader from taking them
-    for this step's (their bytes differ, and the test would see them)."""
-    port = 31500 + os.getpid() % 1000 + slots_per_rank
+    for this step's (their bytes differ, and the test would see them).  Three
+    ranks: each restores the one before it, not the one after."""
+    port = 31500 + os.getpid() % 1000 + 10 * world + slots_per_rank
     with multiprocessing.get_context("spawn").Manager() as m:
         out = m.dict()
-        mp.spawn(_ring_worker, args=(2, port, out, slots_per_rank), nprocs=2, join=True)
+        mp.spawn(_ring_worker, args=(world, port, out, slots_per_rank), nprocs=world, join=True)
         res = dict(out)
-    assert set(res) == {0, 1}
+    assert set(res) == set(range(world))
     for rank, (ok, got_rounds, evictions, pinned, slots) in res.items():
         assert ok, f"rank {rank} did not restore its source rank's chunks"
-        assert got_rounds == rounds and slots == 2 * slots_per_rank
+        assert got_rounds == rounds and slots == world * slots_per_rank
         assert evictions > 0 and pinned == 0
