@@ -83,9 +83,10 @@ FALLBACK_HBM_GBS = 6800.0
 GB = 1e9
 
 
-def workload_name(cfg):
+def workload_name(cfg, layout="hnd"):
     t, n, s = cfg["tokens"], cfg["pool_blocks"], cfg["shape"]
-    return (f"{s['name']}, {t}-token context = {t // s['B']} of {n} pages by seeded permutation, "
+    pages = "pages" if layout == "hnd" else "NHD pages ([K|V][token][head][row])"
+    return (f"{s['name']}, {t}-token context = {t // s['B']} of {n} {pages} by seeded permutation, "
             f"{s['C']}-token chunks: full store to pinned host chunks, then restore into a cold pool "
             f"(poisoned before every step, outside the timed region)")
 
@@ -117,8 +118,9 @@ def kernel_source_hash(source="pack_kernels.cu"):
     return h.hexdigest()[:16]
 
 
-def shape_key(s):
-    return f"L{s['L']} H{s['H']} D{s['D']} e{s['e']} B{s['B']} C{s['C']}"
+def shape_key(s, layout="hnd"):
+    key = f"L{s['L']} H{s['H']} D{s['D']} e{s['e']} B{s['B']} C{s['C']}"
+    return key if layout == "hnd" else key + " NHD"
 
 
 class Traffic:
@@ -136,7 +138,7 @@ class Traffic:
         return traffic * alg_bytes / captured_alg
 
 
-def recorded_traffic(shape, source="pack_kernels.cu"):
+def recorded_traffic(shape, source="pack_kernels.cu", layout="hnd"):
     """Traffic record from profiles/ for this kernel source file (as it is now)
     and KV shape; a record with no entries if none matches."""
     pdir = os.path.join(ROOT, "profiles")
@@ -152,7 +154,7 @@ def recorded_traffic(shape, source="pack_kernels.cu"):
                 if m:
                     d = json.loads(m.group(1))
                     if (d.get("kernel_sha256") == want and d.get("source", "pack_kernels.cu") == source
-                            and d.get("shape") == shape_key(shape)):
+                            and d.get("shape") == shape_key(shape, layout)):
                         return Traffic(d)
     return Traffic(None)
 
@@ -236,6 +238,9 @@ def parse():
                     help="skip the two-replica leg (one stores while the other restores)")
     ap.add_argument("--device-engine", choices=["lsu", "tma"], default="tma",
                     help="kernel of the device-side (HBM) pack/unpack leg")
+    ap.add_argument("--layout", choices=["hnd", "nhd"], default="hnd",
+                    help="page layout of the headline workload's pools (HND: [K|V][head][token][row], the "
+                         "paper's; NHD: [K|V][token][head][row])")
     ap.add_argument("--configs", default="32k,256k,paper127k,hybrid",
                     help="other workloads timed after the headline one in the same run (comma list of "
                          f"{sorted(set(CONFIGS) - {'2k'}) + ['hybrid']}, or 'none'); N=1 only")
@@ -284,7 +289,7 @@ def max_over_ranks(world, value: float, local: int) -> float:
 # ------------------------------------------------------------------ CPU oracle legs
 
 
-def oracle_sample(cfg, n_chunks_sample, pool_pages_np=None):
+def oracle_sample(cfg, n_chunks_sample, pool_pages_np=None, layout="hnd"):
     """Mini-workload for the oracle: n_chunks_sample full chunks whose pages are given
     (or random), as a pool of exactly those pages under an identity table."""
     import numpy as np
@@ -293,7 +298,8 @@ def oracle_sample(cfg, n_chunks_sample, pool_pages_np=None):
     from paper_2609_15021_gb300 import synth
     s = cfg["shape"]
     bpc = s["C"] // s["B"]
-    spec = oracle.PoolSpec(s["L"], n_chunks_sample * bpc, s["B"], s["H"], s["D"], s["e"], oracle.HND)
+    spec = oracle.PoolSpec(s["L"], n_chunks_sample * bpc, s["B"], s["H"], s["D"], s["e"],
+                           oracle.NHD if layout == "nhd" else oracle.HND)
     if pool_pages_np is None:
         pool_pages_np = [synth.random_bytes(spec.layer_bytes, 100 + l) for l in range(s["L"])]
     ident = np.arange(n_chunks_sample * bpc, dtype=np.int32)
@@ -332,7 +338,7 @@ def run_reference(args):
     cfg = CONFIGS[args.config]
     threads = os.cpu_count() or 1
     S = args.cpu_sample_chunks
-    spec, layers, ident = oracle_sample(cfg, S)
+    spec, layers, ident = oracle_sample(cfg, S, layout=args.layout)
     step_times = []
     moved = None
     for i in range(args.warmup + args.steps):
@@ -349,7 +355,8 @@ def run_reference(args):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total / len(step_times),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u8",
         "data": "synthetic random bytes in the workload's shape",
-        "config": {"workload": workload_name(cfg), "context_tokens": cfg["tokens"]},
+        "config": {"workload": workload_name(cfg, args.layout), "context_tokens": cfg["tokens"],
+                   "page_layout": args.layout.upper()},
         "cpu_baseline": {"value": value, "unit": "GB/s", "cores": min(threads, S), "kind": "oracle", "sample": sample},
         "e2e": {"value": value, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
@@ -1018,8 +1025,10 @@ def run_ours(args):
     src_layers = [synth.normal_bf16_(torch.empty(layer_bytes, dtype=torch.uint8, device=dev), synth.SEED + l)
                   for l in range(L)]
     dst_layers = [torch.full((layer_bytes,), synth.POISON, dtype=torch.uint8, device=dev) for _ in range(L)]
-    src = k.KvPool(src_layers, N, B, H, D, e)
-    dst = k.KvPool(dst_layers, N, B, H, D, e)
+    lay = k.KVX_LAYOUT_NHD if args.layout == "nhd" else k.KVX_LAYOUT_HND
+    LAY = args.layout.upper()
+    src = k.KvPool(src_layers, N, B, H, D, e, lay)
+    dst = k.KvPool(dst_layers, N, B, H, D, e, lay)
     ta_np = synth.permuted_table(N, T // B, seed=1)
     tb_np = synth.permuted_table(N, T // B, seed=2)
     ta = torch.from_numpy(ta_np).to(dev)
@@ -1090,7 +1099,7 @@ def run_ours(args):
     # dominant kernel: the direction with more kernel time
     kern = dominant_kernel(k, stats)
     hbm_peak, peak_src = load_peaks()
-    traffic = recorded_traffic(s)
+    traffic = recorded_traffic(s, layout=args.layout)
     roofline = None
     if kern:
         dom = max(kern, key=lambda n: kern[n]["total_ms"])
@@ -1101,7 +1110,7 @@ def run_ours(args):
             link_bytes = kern[dom]["bytes_per_launch"] / 2
             achieved = link_bytes / (kern[dom]["avg_launch_ms"] * 1e-3) / GB
             peak, which = link_ceiling(link, sm_link, direction)
-            roofline = {"bound": "host_link", "kernel": f"move_kernel<{dom},HND> (zero-copy)", "achieved": achieved,
+            roofline = {"bound": "host_link", "kernel": f"move_kernel<{dom},{LAY}> (zero-copy)", "achieved": achieved,
                         "peak": peak, "unit": "GB/s", "frac": achieved / peak,
                         "traffic": traffic.get(f"zerocopy_{dom}", link_bytes),
                         "peak_source": f"the larger of two host-link ceilings measured in this run, {direction}: "
@@ -1151,14 +1160,16 @@ def run_ours(args):
 
         tma = args.device_engine == "tma"
         legs = {tma: device_leg(tma), not tma: device_leg(not tma)}  # the chosen engine and the other one
-        dev_traffic = recorded_traffic(s, "tma_kernels.cu") if tma else traffic
+        dev_traffic = recorded_traffic(s, "tma_kernels.cu", args.layout) if tma else traffic
+        tma_engine = ("TMA tensor-map boxes (tmap_move_kernel)" if args.layout == "hnd" else
+                      "TMA bulk copies, one per side of a unit (tma_move_kernel)")
         hbm_roofline = {"bound": "hbm", "peak": hbm_peak, "unit": "GB/s", "peak_source": peak_src,
-                        "engine": "TMA tensor-map boxes (tmap_move_kernel)" if tma else
-                                  "16-byte loads/stores (move_kernel)"}
+                        "engine": tma_engine if tma else "16-byte loads/stores (move_kernel)"}
         for d, name in ((0, "pack"), (1, "unpack")):
             nl, per_launch, ms = legs[tma][d]
             achieved = per_launch / (ms * 1e-3) / GB
-            kname = f"tmap_move_kernel<{name}>" if tma else f"move_kernel<{name},HND>"
+            kname = ((f"tmap_move_kernel<{name}>" if args.layout == "hnd" else f"tma_move_kernel<{name},NHD>")
+                     if tma else f"move_kernel<{name},{LAY}>")
             hbm_roofline[name] = {"kernel": f"{kname} (device chunks)", "achieved": achieved,
                                   "frac": achieved / hbm_peak, "launches": nl,
                                   "algorithmic_bytes_per_launch": per_launch, "avg_launch_ms": ms,
@@ -1180,7 +1191,7 @@ def run_ours(args):
         del a, b
         other = legs[not tma]
         hbm_roofline["other_engine"] = {
-            "engine": "16-byte loads/stores (move_kernel)" if tma else "TMA tensor-map boxes (tmap_move_kernel)",
+            "engine": "16-byte loads/stores (move_kernel)" if tma else tma_engine,
             **{name: {"achieved": other[d][1] / (other[d][2] * 1e-3) / GB,
                       "frac": other[d][1] / (other[d][2] * 1e-3) / GB / hbm_peak, "avg_launch_ms": other[d][2]}
                for d, name in ((0, "pack"), (1, "unpack"))}}
@@ -1370,7 +1381,7 @@ def run_ours(args):
         pages = np.concatenate([ta_np[c * bpc:(c + 1) * bpc] for c in picks]).astype(np.int64)
         idx = torch.from_numpy(pages).to(dev)
         pool_np = [t.view(-1, page).index_select(0, idx).cpu().numpy().reshape(-1) for t in src_layers]
-        spec, layers_np, ident = oracle_sample(cfg, S, pool_np)
+        spec, layers_np, ident = oracle_sample(cfg, S, pool_np, args.layout)
         threads = os.cpu_count() or 1
         reps, el, want, moved = time_oracle(spec, layers_np, ident, S, args.cpu_seconds, threads, C)
         reps1, el1, _, _ = time_oracle(spec, layers_np, ident, S, args.cpu_seconds / 2, 1, C)
@@ -1408,8 +1419,9 @@ def run_ours(args):
         "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "u8",
         "data": "synthetic: bf16 ~N(0,1) KV from a fixed seed; seeded random-permutation block tables",
-        "config": {"workload": workload_name(cfg), "context_tokens": T, "layers": L, "kv_heads": H,
+        "config": {"workload": workload_name(cfg, args.layout), "context_tokens": T, "layers": L, "kv_heads": H,
                    "head_dim": D, "kv_dtype": s["dtype"], "block_tokens": B, "chunk_tokens": C, "pool_blocks": N,
+                   "page_layout": LAY,
                    "bytes_per_direction": X,
                    "l2": f"inputs larger than L2 ({X} bytes per direction); the destination pool is refilled "
                          f"with poison bytes before every step (a {L * layer_bytes}-byte write, which also "
