@@ -880,13 +880,56 @@ def concurrent_leg(torch, k, probe, dev, local, args, mode, ctx, src, dst, ta, t
     set while B (its own context and stream) restores the first chunk set into the
     cold pool; >= 10 repetitions after 2 warm-ups.  Beside it, over the same two
     chunk sets, both directions at once: the copy engines (cudaMemcpyAsync per
-    chunk) and the SMs (a plain streaming copy per 4 GiB piece)."""
+    chunk) and the SMs (a plain streaming copy per 4 GiB piece).  The two probes
+    run inside every repetition, right after the replicas, so each repetition
+    compares the replicas with the link's both-ways rate at that moment (the host
+    link's both-ways rate varies from one second to the next on a shared host)."""
     pool2 = host_pool2.info()
     chunks2 = [host_pool2.tensor[i * cb:(i + 1) * cb] for i in range(n_chunks)]
     ctx_b = k.kv_ctx_create(local, store_mode=mode, load_mode=mode, staging_slot_bytes=args.slot_mib << 20,
                             flags=k.KVX_FLAG_TIME_KERNELS)
     s_b = torch.cuda.Stream(device=dev)
-    st_ms, ld_ms, agg = [], [], []
+    s_c = torch.cuda.Stream(device=dev)
+    piece = 4 << 30
+    total = n_chunks * cb
+    d_a = torch.empty(cb, dtype=torch.uint8, device=dev)
+    d_b = torch.empty(cb, dtype=torch.uint8, device=dev)
+    dev_a = torch.empty(piece, dtype=torch.uint8, device=dev)
+    dev_b = torch.empty(piece, dtype=torch.uint8, device=dev)
+
+    def both_ways(run_d2h, run_h2d):
+        """(ms of the D2H side, ms of the H2D side), both started together."""
+        a, ea, eb = (torch.cuda.Event(enable_timing=True) for _ in range(3))
+        torch.cuda.synchronize()
+        a.record(stream)
+        s_c.wait_event(a)
+        run_d2h(stream)
+        ea.record(stream)
+        run_h2d(s_c)
+        eb.record(s_c)
+        torch.cuda.synchronize()
+        return a.elapsed_time(ea), a.elapsed_time(eb)
+
+    def ce_d2h(s):   # copy engines: every chunk of both chunk sets, one direction each
+        with torch.cuda.stream(s):
+            for c in range(n_chunks):
+                chunks2[c].copy_(d_a, non_blocking=True)
+
+    def ce_h2d(s):
+        with torch.cuda.stream(s):
+            for c in range(n_chunks):
+                d_b.copy_(chunks[c], non_blocking=True)
+
+    def sm_pass(host, into_host, s):  # SMs: a plain streaming copy, 4 GiB per launch, 76 CTAs a direction
+        for off in range(0, total, piece):
+            n = min(piece, total - off)
+            h = host.tensor[off:off + n]
+            if into_host:
+                probe.kvx_probe_stream_copy(h, dev_a, n, 76, stream=s)
+            else:
+                probe.kvx_probe_stream_copy(dev_b, h, n, 76, stream=s)
+
+    st_ms, ld_ms, agg, sm_agg, ce_agg = [], [], [], [], []
     reps = max(10, args.concurrent_reps)
     with ClockSampler(local) as clocks:
         for i in range(2 + reps):
@@ -903,10 +946,14 @@ def concurrent_leg(torch, k, probe, dev, local, args, mode, ctx, src, dst, ta, t
             k.kv_load(ctx_b, dst, tb, 0, T, C, chunks, stream=s_b)
             eb.record(s_b)
             torch.cuda.synchronize()
+            sm = max(both_ways(lambda s: sm_pass(host_pool2, True, s), lambda s: sm_pass(host_pool, False, s)))
+            ce = max(both_ways(ce_d2h, ce_h2d))
             if i >= 2:
                 st_ms.append(a.elapsed_time(ea))
                 ld_ms.append(a.elapsed_time(eb))
                 agg.append(2 * X / (max(st_ms[-1], ld_ms[-1]) * 1e-3) / GB)
+                sm_agg.append(2 * X / (sm * 1e-3) / GB)
+                ce_agg.append(2 * X / (ce * 1e-3) / GB)
     clock_info = clocks.summary()
     sa, sb = k.kv_ctx_stats(ctx), k.kv_ctx_stats(ctx_b)
     assert k.kv_get_device_error(ctx) == -1 and k.kv_get_device_error(ctx_b) == -1
@@ -920,74 +967,28 @@ def concurrent_leg(torch, k, probe, dev, local, args, mode, ctx, src, dst, ta, t
     picks = sorted({0, n_chunks // 3, n_chunks // 2, n_chunks - 1})
     same = all(torch.equal(chunks2[c], chunks[c]) for c in picks)
     k.kv_ctx_destroy(ctx_b)
-    s_c = torch.cuda.Stream(device=dev)
-
-    def both_ways(run_d2h, run_h2d, n_rep=3):
-        best = None
-        for i in range(1 + n_rep):
-            a, ea, eb = (torch.cuda.Event(enable_timing=True) for _ in range(3))
-            torch.cuda.synchronize()
-            a.record(stream)
-            s_c.wait_event(a)
-            run_d2h(stream)
-            ea.record(stream)
-            run_h2d(s_c)
-            eb.record(s_c)
-            torch.cuda.synchronize()
-            if i >= 1:
-                ms = max(a.elapsed_time(ea), a.elapsed_time(eb))
-                best = ms if best is None else min(best, ms)
-        return 2 * X / (best * 1e-3) / GB
-
-    # copy engines: every chunk of both chunk sets, one direction each
-    d_a = torch.empty(cb, dtype=torch.uint8, device=dev)
-    d_b = torch.empty(cb, dtype=torch.uint8, device=dev)
-
-    def ce_d2h(s):
-        with torch.cuda.stream(s):
-            for c in range(n_chunks):
-                chunks2[c].copy_(d_a, non_blocking=True)
-
-    def ce_h2d(s):
-        with torch.cuda.stream(s):
-            for c in range(n_chunks):
-                d_b.copy_(chunks[c], non_blocking=True)
-
-    ce_bidir = both_ways(ce_d2h, ce_h2d)
-    del d_a, d_b
-    # SMs: a plain streaming copy over the same bytes, 4 GiB per launch, 76 CTAs a direction
-    piece = 4 << 30
-    total = n_chunks * cb
-    dev_a = torch.empty(piece, dtype=torch.uint8, device=dev)
-    dev_b = torch.empty(piece, dtype=torch.uint8, device=dev)
-
-    def sm_pass(host, into_host, s):
-        for off in range(0, total, piece):
-            n = min(piece, total - off)
-            h = host.tensor[off:off + n]
-            if into_host:
-                probe.kvx_probe_stream_copy(h, dev_a, n, 76, stream=s)
-            else:
-                probe.kvx_probe_stream_copy(dev_b, h, n, 76, stream=s)
-
-    sm_bidir = both_ways(lambda s: sm_pass(host_pool2, True, s), lambda s: sm_pass(host_pool, False, s))
-    del dev_a, dev_b, chunks2
+    del d_a, d_b, dev_a, dev_b, chunks2
     host_pool2.close()
     med = statistics.median(agg)
+    sm_med, ce_med = statistics.median(sm_agg), statistics.median(ce_agg)
     return {"aggregate_gbs": span(agg), "store_ms": span(st_ms), "restore_ms": span(ld_ms),
             "span_ms": span([max(a_, b_) for a_, b_ in zip(st_ms, ld_ms)]), "reps": len(agg),
             "peak_bidir_gbs": link["bidir"], "frac": med / link["bidir"],
-            "peak_bidir_same_size_gbs": ce_bidir, "frac_same_size": med / ce_bidir,
-            "sm_stream_bidir_same_size_gbs": sm_bidir, "frac_sm_stream_same_size": med / sm_bidir,
+            "peak_bidir_same_size_gbs": ce_med, "frac_same_size": med / ce_med,
+            "sm_stream_bidir_same_size_gbs": sm_med, "frac_sm_stream_same_size": med / sm_med,
+            "per_rep": {"sm_stream_gbs": span(sm_agg), "copy_engine_gbs": span(ce_agg),
+                        "frac_sm_stream": span([r / p for r, p in zip(agg, sm_agg)]),
+                        "frac_copy_engine": span([r / p for r, p in zip(agg, ce_agg)])},
             "kernels": kernels, "clocks": clock_info,
             "second_store_equals_first_on_sampled_chunks": same, "second_pool": pool2,
             "what": "replica A kv_store of the context into a second pinned chunk set while replica B kv_load "
                     "of the timed steps' chunks into its (refilled) pool, own context and stream each; "
                     "aggregate = 2 x bytes / the slower of the two, per repetition; peak_bidir = pinned "
-                    "cudaMemcpyAsync of 1 GiB each way at once; peak_bidir_same_size = cudaMemcpyAsync of every "
-                    "chunk of both chunk sets, one direction each, at once (best of 3); "
-                    "sm_stream_bidir_same_size = a plain SM streaming copy (76 CTAs a direction) over the same "
-                    "two chunk sets, both directions at once (best of 3)"}
+                    "cudaMemcpyAsync of 1 GiB each way at once; in every repetition, right after the replicas, "
+                    "over the same two chunk sets, both directions at once: cudaMemcpyAsync of every chunk "
+                    "(peak_bidir_same_size, median over the repetitions) and a plain SM streaming copy, 76 CTAs "
+                    "a direction (sm_stream_bidir_same_size, median); per_rep.frac_* = the replicas' rate over "
+                    "the probe's in the same repetition"}
 
 
 def run_ours(args):
