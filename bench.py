@@ -931,6 +931,8 @@ def concurrent_leg(torch, k, probe, dev, local, args, mode, ctx, src, dst, ta, t
 
     st_ms, ld_ms, agg, sm_agg, ce_agg = [], [], [], [], []
     reps = max(10, args.concurrent_reps)
+    picks = sorted({0, n_chunks // 3, n_chunks // 2, n_chunks - 1})
+    same = False
     with ClockSampler(local) as clocks:
         for i in range(2 + reps):
             if i == 2:
@@ -946,6 +948,8 @@ def concurrent_leg(torch, k, probe, dev, local, args, mode, ctx, src, dst, ta, t
             k.kv_load(ctx_b, dst, tb, 0, T, C, chunks, stream=s_b)
             eb.record(s_b)
             torch.cuda.synchronize()
+            if i == 1 + reps:  # A's chunks, before the probes below write over that chunk set
+                same = all(torch.equal(chunks2[c], chunks[c]) for c in picks)
             sm = max(both_ways(lambda s: sm_pass(host_pool2, True, s), lambda s: sm_pass(host_pool, False, s)))
             ce = max(both_ways(ce_d2h, ce_h2d))
             if i >= 2:
@@ -964,8 +968,6 @@ def concurrent_leg(torch, k, probe, dev, local, args, mode, ctx, src, dst, ta, t
             by = st_["kernel_bytes"][d] / st_["timed_launches"][d] / 2
             kernels[name] = {"avg_launch_ms": ms, "link_bytes_per_launch": by, "link_gbs": by / (ms * 1e-3) / GB,
                              "launches": st_["timed_launches"][d]}
-    picks = sorted({0, n_chunks // 3, n_chunks // 2, n_chunks - 1})
-    same = all(torch.equal(chunks2[c], chunks[c]) for c in picks)
     k.kv_ctx_destroy(ctx_b)
     del d_a, d_b, dev_a, dev_b, chunks2
     host_pool2.close()

@@ -73,9 +73,16 @@ class SharedTier:
         self._free_snaps = list(range(max_snapshots))
         cb = shape.chunk_bytes
         self._chunk_views = [self.chunks.tensor[c * cb:(c + 1) * cb] for c in range(self.max_chunks)]
+        # Raw addresses of the slots, each exactly one chunk long (the library still
+        # checks that every chunk it is given is pinned host memory).
+        self._chunk_ptrs = [v.data_ptr() for v in self._chunk_views]
 
     def chunk(self, c: int):
         return self._chunk_views[c]
+
+    def chunk_ptrs(self, c0: int, c1: int) -> list[int]:
+        """Host addresses of chunk slots c0 .. c1-1."""
+        return self._chunk_ptrs[c0:c1]
 
     def snapshot(self, boundary: int):
         sb = self.shape.snapshot_bytes
@@ -99,6 +106,7 @@ class SharedTier:
 
     def close(self):
         self._chunk_views = []
+        self._chunk_ptrs = []
         self.chunks.close()
         self.snaps.close()
 
@@ -116,41 +124,54 @@ class Replica:
     tokens: int = 0                            # context length held locally
 
     def __post_init__(self):
-        import collections
-
+        import numpy as np
         import torch
         s = self.shape
-        self.free_pages = collections.deque(self.free_pages)  # taken from the front, O(1) each
+        self._free = np.asarray(self.free_pages, dtype=np.int32)  # taken from the front by a cursor
+        self._next_free = 0
         self.attn_layers = [torch.empty(self.num_blocks * s.page_bytes, dtype=torch.uint8, device=self.device)
                             for _ in range(s.attn_layers)]
         self.pool = k.KvPool(self.attn_layers, self.num_blocks, s.block_tokens, s.kv_heads, s.head_dim,
                              s.elem_bytes)
         self.state = [torch.empty(self.state_slots * s.state_bytes, dtype=torch.uint8, device=self.device)
                       for _ in range(s.state_layers)]
+        self.state_layers = k.StateLayers(self.state)
         # The block table only grows (pages are appended), so it lives on the
         # device at its largest size and each new entry is uploaded once, on the
-        # caller's stream, from a pinned staging copy written once.
+        # caller's stream, from a pinned staging copy written once (when the page
+        # is allocated).
         self._table_dev = torch.empty(self.num_blocks, dtype=torch.int32, device=self.device)
         self._table_pinned = torch.empty(self.num_blocks, dtype=torch.int32).pin_memory()
+        self._table_np = self._table_pinned.numpy()
         self._uploaded = 0
 
     def grow(self, n_tokens: int):
         """Allocate fresh pages so the table covers n_tokens."""
         need = -(-n_tokens // self.shape.block_tokens)
-        while len(self.table) < need:
-            self.table.append(self.free_pages.popleft())
+        have = len(self.table)
+        if need <= have:
+            return
+        take = need - have
+        if self._next_free + take > len(self._free):
+            raise MemoryError(f"replica has {len(self._free) - self._next_free} free pages, needs {take}")
+        new = self._free[self._next_free:self._next_free + take]
+        self._next_free += take
+        self._table_np[have:need] = new
+        self.table.extend(new.tolist())
 
     def table_tensor(self, stream=None):
         """Device view of the table; entries added since the last call are copied up
         on `stream` (default: the current stream), ahead of the work that uses them."""
-        import torch
         n = len(self.table)
         if self._uploaded < n:
             a = self._uploaded
-            self._table_pinned[a:n] = torch.tensor(self.table[a:n], dtype=torch.int32)
-            s = stream if stream is not None else torch.cuda.current_stream(self._table_dev.device)
-            with torch.cuda.stream(s):
-                self._table_dev[a:n].copy_(self._table_pinned[a:n], non_blocking=True)
+            src, dst = self._table_pinned[a:n], self._table_dev[a:n]
+            if stream is None:
+                dst.copy_(src, non_blocking=True)
+            else:
+                import torch
+                with torch.cuda.stream(stream):
+                    dst.copy_(src, non_blocking=True)
             self._uploaded = n
         return self._table_dev[:n]
 
@@ -159,10 +180,10 @@ def store_prefix(ctx, rep: Replica, tier: SharedTier, t0: int, t1: int, state_sl
     """Store tokens [t0, t1) of rep and its state (slot state_slot) as the snapshot at t1."""
     s = tier.shape
     C = s.chunk_tokens
-    chunks = [tier.chunk(c) for c in range(t0 // C, -(-t1 // C))]
+    chunks = tier.chunk_ptrs(t0 // C, -(-t1 // C))
     k.kv_store(ctx, rep.pool, rep.table_tensor(stream), t0, t1, C, chunks, stream=stream)
     snap = tier.reserve_snapshot(t1)
-    k.kv_state_store(ctx, rep.state, rep.state_slots, s.state_bytes, state_slot, snap, stream=stream)
+    k.kv_state_store(ctx, rep.state_layers, rep.state_slots, s.state_bytes, state_slot, snap, stream=stream)
     tier.present.update(range(t0 // C, -(-t1 // C)))
 
 
@@ -176,7 +197,8 @@ def load_prefix(ctx, rep: Replica, tier: SharedTier, t0: int, t1: int, state_slo
     s = tier.shape
     C = s.chunk_tokens
     rep.grow(t1)
-    chunks = [tier.chunk(c) for c in range(t0 // C, -(-t1 // C))]
+    chunks = tier.chunk_ptrs(t0 // C, -(-t1 // C))
     k.kv_load(ctx, rep.pool, rep.table_tensor(stream), t0, t1, C, chunks, stream=stream)
-    k.kv_state_load(ctx, rep.state, rep.state_slots, s.state_bytes, state_slot, tier.snapshot(t1), stream=stream)
+    k.kv_state_load(ctx, rep.state_layers, rep.state_slots, s.state_bytes, state_slot, tier.snapshot(t1),
+                    stream=stream)
     rep.tokens = t1

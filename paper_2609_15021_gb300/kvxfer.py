@@ -172,6 +172,9 @@ def _check(status: int, where: str):
 def _stream_handle(stream) -> int | None:
     if stream is None:
         import torch
+        raw = getattr(torch._C, "_cuda_getCurrentRawStream", None)  # the handle without a Stream object
+        if raw is not None:
+            return raw(torch.cuda.current_device()) or None
         return torch.cuda.current_stream().cuda_stream or None
     if isinstance(stream, int):
         return stream or None
@@ -466,15 +469,30 @@ class HostBuffer:
             pass
 
 
+class StateLayers:
+    """Per-layer recurrent-state buffers (one device tensor, or raw pointer, per layer)
+    with their base pointers marshalled once, for state copies made every turn.
+    kv_state_store / kv_state_load take this or a plain sequence of tensors."""
+
+    def __init__(self, layers):
+        self.layers = list(layers)
+        self._arr = _ptr_array(self.layers)
+
+    def __len__(self) -> int:
+        return len(self.layers)
+
+
+def _layer_array(layers):
+    return layers._arr if isinstance(layers, StateLayers) else _ptr_array(layers)
+
+
 def kv_state_store(ctx, layers, num_slots: int, slot_bytes: int, slot: int, host_obj, stream=None) -> None:
-    arr = _ptr_array(layers)
-    _check(_lib.kv_state_store(ctx, len(layers), arr, num_slots, slot_bytes, slot, _ptr(host_obj),
+    _check(_lib.kv_state_store(ctx, len(layers), _layer_array(layers), num_slots, slot_bytes, slot, _ptr(host_obj),
                                _stream_handle(stream)), "kv_state_store")
 
 
 def kv_state_load(ctx, layers, num_slots: int, slot_bytes: int, slot: int, host_obj, stream=None) -> None:
-    arr = _ptr_array(layers)
-    _check(_lib.kv_state_load(ctx, len(layers), arr, num_slots, slot_bytes, slot, _ptr(host_obj),
+    _check(_lib.kv_state_load(ctx, len(layers), _layer_array(layers), num_slots, slot_bytes, slot, _ptr(host_obj),
                               _stream_handle(stream)), "kv_state_load")
 
 
