@@ -210,6 +210,22 @@ def test_binding_rejects_what_raw_pointers_cannot_show(k):
         k._check_transfer_tensors(pool, table, 0, 43, C, [chunks[0], short])
 
 
+def test_state_layers_marshalled_once(k):
+    """StateLayers builds the layer-pointer array once; the state copies pass it
+    through unchanged (a null context is rejected before any device call)."""
+    ptrs = [0x10000, 0x20000, 0x30000]
+    sl = k.StateLayers(ptrs)
+    assert len(sl) == 3
+    arr = k._layer_array(sl)
+    assert [arr[i] for i in range(3)] == ptrs and k._layer_array(sl) is arr
+    assert [k._layer_array(ptrs)[i] for i in range(3)] == ptrs  # a plain sequence: marshalled per call
+    for fn in (k.kv_state_store, k.kv_state_load):
+        for layers in (sl, ptrs):
+            with pytest.raises(k.KvxError) as e:
+                fn(None, layers, 2, 4096, 0, 0x40000, stream=0)
+            assert e.value.status == k.KVX_EINVAL
+
+
 def test_host_alloc_numa_arguments(k):
     import torch
     out = ctypes.c_void_p()
