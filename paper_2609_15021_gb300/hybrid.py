@@ -180,10 +180,12 @@ def store_prefix(ctx, rep: Replica, tier: SharedTier, t0: int, t1: int, state_sl
     """Store tokens [t0, t1) of rep and its state (slot state_slot) as the snapshot at t1."""
     s = tier.shape
     C = s.chunk_tokens
-    chunks = tier.chunk_ptrs(t0 // C, -(-t1 // C))
-    k.kv_store(ctx, rep.pool, rep.table_tensor(stream), t0, t1, C, chunks, stream=stream)
+    # The snapshot needs no block table, so it is enqueued first: the GPU copies
+    # it while the host prepares the KV store (both on the caller's stream).
     snap = tier.reserve_snapshot(t1)
     k.kv_state_store(ctx, rep.state_layers, rep.state_slots, s.state_bytes, state_slot, snap, stream=stream)
+    chunks = tier.chunk_ptrs(t0 // C, -(-t1 // C))
+    k.kv_store(ctx, rep.pool, rep.table_tensor(stream), t0, t1, C, chunks, stream=stream)
     tier.present.update(range(t0 // C, -(-t1 // C)))
 
 
@@ -196,9 +198,11 @@ def load_prefix(ctx, rep: Replica, tier: SharedTier, t0: int, t1: int, state_slo
         raise LookupError(f"shared tier lacks chunks of [{t0}, {t1}) or the state snapshot at {t1}")
     s = tier.shape
     C = s.chunk_tokens
+    # The snapshot goes first: the GPU copies it while the host allocates the
+    # pages and uploads their table entries for the KV restore behind it.
+    k.kv_state_load(ctx, rep.state_layers, rep.state_slots, s.state_bytes, state_slot, tier.snapshot(t1),
+                    stream=stream)
     rep.grow(t1)
     chunks = tier.chunk_ptrs(t0 // C, -(-t1 // C))
     k.kv_load(ctx, rep.pool, rep.table_tensor(stream), t0, t1, C, chunks, stream=stream)
-    k.kv_state_load(ctx, rep.state_layers, rep.state_slots, s.state_bytes, state_slot, tier.snapshot(t1),
-                    stream=stream)
     rep.tokens = t1
