@@ -40,6 +40,9 @@ CASES = {
     # n_used counts logical blocks, N pages
     "paper_logical_blocks_49": (4, 49 * 6, 32, 4, 256, 1, HND, 5, 1568, 1, 100, 49),
     "logical_blocks_4_nhd_ragged": (3, 4 * 20, 16, 2, 64, 2, NHD, 17, 96, 2, 7, 4),
+    # the most layers a pool description holds (KVX_MAX_LAYERS)
+    "max_layers_128": (128, 24, 16, 2, 64, 2, HND, 20, 64, 1, 5),
+    "max_layers_128_nhd_logical": (128, 2 * 12, 16, 2, 64, 2, NHD, 10, 64, 1, 5, 2),
 }
 
 MODES = {"staged": 1, "zerocopy": 2}
