@@ -25,8 +25,9 @@ hbm_roofline         kv_pack / kv_unpack of the same context into device chunks
                      against the measured HBM copy peak;
 concurrent_replicas  one context stored while another context's chunks are
                      restored, each through its own context and stream, over
-                     >= 10 repetitions, beside the copy engines' and the SMs'
-                     bidirectional rates over the same two chunk sets;
+                     >= 10 repetitions; in every repetition the copy engines'
+                     and the SMs' bidirectional rates over the same two chunk
+                     sets are timed right after the replicas;
 restore_after_idle   a restore after the pool sat untouched for a few seconds,
                      with the library's host-page touch and without it;
 tier_path            the same store and restore through a host tier shared
