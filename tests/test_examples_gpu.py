@@ -47,3 +47,14 @@ def test_streamed_cross_replica_example():
     assert r.returncode == 0, r.stdout + r.stderr
     print("\n" + r.stdout.strip())
     assert "bit-exact" in r.stdout
+
+
+def test_hybrid_session_example():
+    """Two replicas of a hybrid model alternate on one session through a shared
+    tier; their pages for the common tokens agree and each state is its
+    boundary's snapshot."""
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "examples", "hybrid_session.py")], cwd=ROOT,
+                       capture_output=True, text=True, timeout=600)
+    assert r.returncode == 0, r.stdout + r.stderr
+    print("\n" + r.stdout.strip())
+    assert "session bit-exact" in r.stdout
