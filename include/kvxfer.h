@@ -89,8 +89,10 @@ typedef enum { KVX_LAYOUT_HND = 0, KVX_LAYOUT_NHD = 1 } kvx_layout;
 /* How host chunks are filled and read.  Both move exactly the same bytes. */
 typedef enum {
   KVX_MODE_AUTO = 0,     /* library's measured default: ZEROCOPY both ways
-                            (GB300 + Grace: link peak every step; STAGED
-                            alternates between peak and ~25% slower steps)   */
+                            (GB300 + Grace: the link's ceiling every step on
+                            every pool kind measured; STAGED reaches 0.98-0.99
+                            of it only from huge-page pools, KVX_HOST_HUGE,
+                            and varies from step to step on others)           */
   KVX_MODE_STAGED = 1,   /* pack into a device staging ring, then
                             cudaMemcpyAsync over the host link on a side stream,
                             pack of batch i+1 overlapping the copy of batch i  */
