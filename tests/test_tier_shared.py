@@ -470,3 +470,122 @@ def test_tier_wait_across_processes():
         t.release(12, -1)
     finally:
         t.close()
+
+
+def _stress_worker(name, seed, n_ops, n_keys, q_out, start=None):
+    """Random reserve / write / commit (or abandon), acquire / check / hold /
+    release on one shared tier.  Every writer of a key writes the same bytes
+    (the key repeated), so a slot this process holds pinned must always read
+    back as its key: any other bytes mean the slot went to another key, or to
+    a writer, while it was pinned.  Puts (bytes mismatches, counts) on q_out;
+    a call that had to succeed and did not is reported there too."""
+    import collections
+    import ctypes
+    import random
+    import traceback
+    sys.path.insert(0, ROOT)
+    from paper_2609_15021_gb300 import kvxfer as k
+    lib = k._lib
+    t = k.KvTier(shared_name=name, pin=False)
+    nb = t.slot_bytes
+    no = ctypes.c_void_p(k.KVX_NO_STREAM & (2**64 - 1))
+    pattern = {key: key.to_bytes(8, "little") * (nb // 8) for key in range(1, n_keys + 1)}
+    rnd = random.Random(seed)
+    held, counts = [], collections.Counter()
+
+    def check(key, ptr):
+        if ctypes.string_at(ptr, nb) != pattern[key]:
+            counts["bad bytes"] += 1
+
+    def must(status, what):
+        if status != k.KVX_OK:
+            raise RuntimeError(f"{what} returned {status}")
+
+    if start is not None:
+        start.wait(timeout=120)  # every process begins at once
+    try:
+        for _ in range(n_ops):
+            key = rnd.randint(1, n_keys)
+            r = rnd.random()
+            out = ctypes.c_void_p()
+            if r < 0.4:
+                st = lib.kv_tier_reserve(t.handle, key, ctypes.byref(out))
+                if st == k.KVX_OK:
+                    ctypes.memmove(out.value, pattern[key], nb)
+                    if rnd.random() < 0.1:
+                        must(lib.kv_tier_release(t.handle, key, no), "release of a reservation")
+                        counts["abandoned"] += 1
+                    else:
+                        must(lib.kv_tier_commit(t.handle, key, no), "commit")
+                        counts["committed"] += 1
+                elif st in (k.KVX_EBUSY, k.KVX_ENOMEM):
+                    counts[f"reserve {st}"] += 1
+                else:
+                    must(st, "reserve")
+            elif r < 0.85:
+                st = lib.kv_tier_acquire(t.handle, key, no, ctypes.byref(out))
+                if st == k.KVX_OK:
+                    check(key, out.value)
+                    counts["acquired"] += 1
+                    if rnd.random() < 0.3 and len(held) < 3:
+                        held.append((key, out.value))
+                    else:
+                        must(lib.kv_tier_release(t.handle, key, no), "release")
+                elif st in (k.KVX_ENOENT, k.KVX_EBUSY):
+                    counts[f"acquire {st}"] += 1
+                else:
+                    must(st, "acquire")
+            elif held:
+                key, ptr = held.pop(rnd.randrange(len(held)))
+                check(key, ptr)
+                must(lib.kv_tier_release(t.handle, key, no), "release of a held pin")
+        for key, ptr in held:
+            check(key, ptr)
+            must(lib.kv_tier_release(t.handle, key, no), "release of a held pin")
+    except Exception:
+        counts["failed"] += 1
+        counts[traceback.format_exc().strip().splitlines()[-1]] += 1
+    t.close()
+    q_out.put(dict(counts))
+
+
+def test_processes_racing_on_one_tier_never_share_a_pinned_slot():
+    """Three processes make thousands of random tier calls on 8 slots shared by
+    24 keys (constant eviction).  No pinned slot ever changes under its holder,
+    every committed entry reads back as its key, and nothing stays pinned."""
+    sys.path.insert(0, ROOT)
+    from paper_2609_15021_gb300 import _build
+    _build.build()
+    from paper_2609_15021_gb300 import kvxfer as k
+    n_keys, n_ops = 24, 20000
+    name = _name("stress")
+    t = k.KvTier(4096, 8, shared_name=name, create=True, pin=False)
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    start = ctx.Barrier(4)
+    procs = [ctx.Process(target=_stress_worker, args=(name, seed, n_ops, n_keys, q, start)) for seed in (11, 12, 13)]
+    for p in procs:
+        p.start()
+    try:
+        start.wait(timeout=120)
+        results = [q.get(timeout=300) for _ in procs]
+        for p in procs:
+            p.join(timeout=60)
+            assert p.exitcode == 0
+        for counts in results:
+            assert "failed" not in counts and "bad bytes" not in counts, counts
+            assert counts.get("committed", 0) > 1000 and counts.get("acquired", 0) > 1000, counts
+        st = t.stats()
+        assert st["pinned"] == 0 and st["entries"] <= 8 and st["evictions"] > 0, st
+        import ctypes
+        no = ctypes.c_void_p(k.KVX_NO_STREAM & (2**64 - 1))
+        for key in range(1, n_keys + 1):
+            out = ctypes.c_void_p()
+            if k._lib.kv_tier_acquire(t.handle, key, no, ctypes.byref(out)) == k.KVX_OK:
+                assert ctypes.string_at(out.value, 4096) == key.to_bytes(8, "little") * 512
+                assert k._lib.kv_tier_release(t.handle, key, no) == k.KVX_OK
+    finally:
+        for p in procs:
+            if p.is_alive():
+                p.kill()
+        t.close()
