@@ -305,6 +305,32 @@ def test_host_touch_reads_ranges_and_checks_arguments(k):
     assert lib.kv_host_touch(None, None, 0) == k.KVX_OK
 
 
+def test_host_touch_from_many_threads_at_once(k):
+    """Eight host threads touch their own buffers at once through the one pool
+    of touch threads (the ctypes calls release the GIL): every call returns
+    KVX_OK, none waits for another's pages beyond its bound, and a thread's
+    buffer is read, not written."""
+    import threading
+    import numpy as np
+    bufs = [np.full((3 << 20) + 4096 * i, i, np.uint8) for i in range(8)]
+    status, t0 = [None] * 8, time.monotonic()
+
+    def run(i):
+        arr = (ctypes.c_void_p * 1)(bufs[i].ctypes.data)
+        sizes = (ctypes.c_int64 * 1)(bufs[i].nbytes)
+        status[i] = [k._lib.kv_host_touch(arr, sizes, 1) for _ in range(20)]
+
+    threads = [threading.Thread(target=run, args=(i,)) for i in range(8)]
+    for t in threads:
+        t.start()
+    for t in threads:
+        t.join(timeout=60)
+    assert not any(t.is_alive() for t in threads)
+    assert all(st == [k.KVX_OK] * 20 for st in status), status
+    assert time.monotonic() - t0 < 30  # far inside one call's 5 s bound per touch
+    assert all(int(b.min()) == i == int(b.max()) for i, b in enumerate(bufs))
+
+
 @pytest.mark.filterwarnings("ignore:This process .* is multi-threaded")
 def test_host_touch_in_a_forked_child(k):
     """A child forked after the touch threads started inherits none of them; its
