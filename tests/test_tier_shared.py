@@ -589,3 +589,65 @@ def test_processes_racing_on_one_tier_never_share_a_pinned_slot():
             if p.is_alive():
                 p.kill()
         t.close()
+
+
+def _pin_holder(name, q_in, q_out):
+    """Acquires key 1 of a shared tier, reports, and releases it when told."""
+    import ctypes
+    sys.path.insert(0, ROOT)
+    from paper_2609_15021_gb300 import kvxfer as k
+    t = k.KvTier(shared_name=name, pin=False)
+    no = ctypes.c_void_p(k.KVX_NO_STREAM & (2**64 - 1))
+    out = ctypes.c_void_p()
+    q_out.put(k._lib.kv_tier_acquire(t.handle, 1, no, ctypes.byref(out)))
+    assert q_in.get(timeout=120) == "release"
+    q_out.put(k._lib.kv_tier_release(t.handle, 1, no))
+    t.close()
+
+
+def test_at_most_eight_processes_pin_one_entry():
+    """Eight processes hold pins on one entry; a ninth gets KVX_EBUSY, and gets
+    its pin once one of the eight has released (pins are kept per process, so
+    a process's second pin on the entry costs no extra holder)."""
+    import ctypes
+    sys.path.insert(0, ROOT)
+    from paper_2609_15021_gb300 import _build
+    _build.build()
+    from paper_2609_15021_gb300 import kvxfer as k
+    name = _name("holders")
+    t = k.KvTier(64, 2, shared_name=name, create=True, pin=False)
+    no = ctypes.c_void_p(k.KVX_NO_STREAM & (2**64 - 1))
+    out = ctypes.c_void_p()
+    assert k._lib.kv_tier_reserve(t.handle, 1, ctypes.byref(out)) == k.KVX_OK
+    assert k._lib.kv_tier_commit(t.handle, 1, no) == k.KVX_OK
+    ctx = mp.get_context("spawn")
+    q_out = ctx.Queue()
+    holders = [(ctx.Process(target=_pin_holder, args=(name, q_in, q_out)), q_in)
+               for q_in in (ctx.Queue() for _ in range(8))]
+    try:
+        for p, _ in holders:
+            p.start()
+        assert [q_out.get(timeout=120) for _ in holders] == [k.KVX_OK] * 8
+        assert t.stats()["pinned"] == 1
+        assert k._lib.kv_tier_acquire(t.handle, 1, no, ctypes.byref(out)) == k.KVX_EBUSY  # a ninth process
+        assert k._lib.kv_tier_reserve(t.handle, 1, ctypes.byref(out)) == k.KVX_EBUSY      # pinned: no rewrite
+        p0, q0 = holders[0]
+        q0.put("release")
+        assert q_out.get(timeout=120) == k.KVX_OK
+        p0.join(timeout=60)
+        assert k._lib.kv_tier_acquire(t.handle, 1, no, ctypes.byref(out)) == k.KVX_OK
+        assert k._lib.kv_tier_acquire(t.handle, 1, no, ctypes.byref(out)) == k.KVX_OK  # same process, same holder
+        for _ in range(2):
+            assert k._lib.kv_tier_release(t.handle, 1, no) == k.KVX_OK
+        for p, q_in in holders[1:]:
+            q_in.put("release")
+        assert [q_out.get(timeout=120) for _ in holders[1:]] == [k.KVX_OK] * 7
+        for p, _ in holders:
+            p.join(timeout=60)
+            assert p.exitcode == 0
+        assert t.stats()["pinned"] == 0
+    finally:
+        for p, _ in holders:
+            if p.is_alive():
+                p.kill()
+        t.close()
