@@ -112,6 +112,7 @@ def test_tma_wait_runs_out_then_recovery(orc, direction, layout, flags, max_ctas
             chunks = [torch.from_numpy(w).cuda() for w in want]
             dst = device_pool(spec)
             run = lambda: k.kv_unpack(ctx, dst, table_d, 0, T, C, chunks, stream=s)
+        torch.cuda.synchronize()  # buffers above were filled on the default stream
         k.kv_fault_inject("tma_wait", 0)
         run()
         s.synchronize()

@@ -282,6 +282,7 @@ def test_host_alloc_numa_round_trip(orc, node):
         ta, tb = synth.permuted_table(64, n_used, 61), synth.permuted_table(64, n_used, 62)
         ta_d, tb_d = torch.from_numpy(ta).cuda(), torch.from_numpy(tb).cuda()
         ctx = k.kv_ctx_create(0, store_mode=k.KVX_MODE_ZEROCOPY, load_mode=k.KVX_MODE_ZEROCOPY)
+        torch.cuda.synchronize()  # the poisoned pool was filled on the default stream
         try:
             s = torch.cuda.Stream()
             k.kv_store(ctx, src, ta_d, 0, T, Cs, chunks, stream=s)

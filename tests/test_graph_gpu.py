@@ -29,6 +29,7 @@ def test_store_restore_replayed_from_a_cuda_graph(orc):
     ta_d, tb_d = torch.from_numpy(ta).cuda(), torch.from_numpy(tb).cuda()
     host = pinned_chunks(orc, spec, 0, T, C)
     ctx = k.kv_ctx_create(0)
+    torch.cuda.synchronize()  # the poisoned pool was filled on the default stream
     try:
         s = torch.cuda.Stream()
         with torch.cuda.stream(s):  # warm up outside the capture

@@ -260,6 +260,7 @@ def test_back_to_back_calls_reuse_slots(orc, ctxs):
     h1 = pinned_chunks(orc, spec, t0, t1, C)
     h2 = pinned_chunks(orc, spec, t0, t1, C)
     dst = device_pool(spec)
+    torch.cuda.synchronize()  # the poisoned pool was filled on the default stream
     s = torch.cuda.Stream()
     with torch.cuda.stream(s):
         for _ in range(3):
@@ -401,6 +402,7 @@ def test_calls_after_idle_time(orc, touch):
     ta_d, tb_d = torch.from_numpy(ta).cuda(), torch.from_numpy(tb).cuda()
     host = pinned_chunks(orc, spec, 0, T, C)
     ctx = k.kv_ctx_create(0, flags=0 if touch else k.KVX_FLAG_NO_HOST_TOUCH)
+    torch.cuda.synchronize()  # the poisoned pool was filled on the default stream
     try:
         s = torch.cuda.Stream()
         time.sleep(1.1)

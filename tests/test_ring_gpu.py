@@ -70,6 +70,7 @@ def _rank(rank, world, port, out):
         if rank == 0:
             os.unlink("/dev/shm" + name)
         ctx = k.kv_ctx_create(0)
+        torch.cuda.synchronize()  # pools made on the default stream before the side stream uses them
         stream = torch.cuda.Stream()
 
         def store_fn(lo, hi, slots):

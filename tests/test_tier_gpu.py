@@ -97,6 +97,7 @@ def test_slots_in_use_by_the_gpu_are_not_evicted(orc):
     cb = orc.chunk_bytes(spec, C)
     tier = k.KvTier(cb, 2)
     ctx = k.kv_ctx_create(0)
+    torch.cuda.synchronize()  # the poisoned pool was filled on the default stream
     s = torch.cuda.Stream()
     busy = torch.empty(1 << 20, dtype=torch.uint8, device="cuda")
     try:

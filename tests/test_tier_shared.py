@@ -397,6 +397,7 @@ def test_published_entries_of_a_dead_writer_stay_readable():
         tb = synth.permuted_table(64, n_used, 23)
         tb_d = torch.from_numpy(tb).cuda()
         ctx = k.kv_ctx_create(0)
+        torch.cuda.synchronize()  # the poisoned pool was filled on the default stream
         s = torch.cuda.Stream()
         try:
             for c, key in enumerate([501, 502]):
