@@ -553,6 +553,7 @@ def config_leg(torch, k, synth, name, dev, local, link, sm_link, steps, warmup):
     chunks = [pool.tensor[i * cb:(i + 1) * cb] for i in range(n_chunks)]
     ctx = k.kv_ctx_create(local, flags=k.KVX_FLAG_TIME_KERNELS)
     stream = torch.cuda.Stream(device=dev)
+    torch.cuda.synchronize()  # the pools were written on the default stream; the steps run on `stream`
     try:
         st, ld = timed_steps(torch, k, ctx, src, dst, ta, tb, T, C, chunks, stream, steps, warmup,
                              lambda: refill(torch, dst_layers, stream, synth.POISON))
@@ -1065,6 +1066,7 @@ def run_ours(args):
     store_mode, load_mode = k.kv_ctx_modes(ctx)
     stream = torch.cuda.Stream(device=dev)
     poison_dst = lambda: refill(torch, dst_layers, stream, synth.POISON)  # noqa: E731
+    torch.cuda.synchronize()  # the pools were written on the default stream; the steps run on `stream`
 
     with ClockSampler(local) as clocks:
         store_ms, restore_ms = timed_steps(torch, k, ctx, src, dst, ta, tb, T, C, chunks, stream, args.steps,
