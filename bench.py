@@ -783,6 +783,7 @@ def run_shared(args, world, rank, local):
     step_keys = [ring_keys(k, rank, world, T, C, i) for i in range(args.warmup + args.steps)]
     ctx = k.kv_ctx_create(local, flags=k.KVX_FLAG_TIME_KERNELS)
     stream = torch.cuda.Stream(device=dev)
+    torch.cuda.synchronize()  # the pools were written on the default stream; the steps run on `stream`
 
     def store_fn(lo, hi, slots):
         k.kv_store(ctx, src, ta, lo * C, min(T, hi * C), C, slots, stream=stream)
