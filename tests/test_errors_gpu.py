@@ -125,3 +125,53 @@ def test_allocation_free_store_rejects_bad_memory(orc, setup):
              pinned_chunks(orc, SPEC, 0, T, C))
     torch.cuda.synchronize()
     assert all(bool((c == POISON).all()) for c in pageable + on_device)
+
+
+def test_modes_pool_info_and_foreign_pointers(orc):
+    """KVX_MODE_AUTO resolves to zero-copy both ways (the measured default);
+    explicit and mixed modes stay as asked, and the counters show which path
+    ran (copies only in staged mode).  kv_host_pool_info knows the start of a
+    library pool only; kv_host_free ignores NULL and memory it did not
+    allocate."""
+    import ctypes
+    k = kvx()
+    for asked, want in (((0, 0), (2, 2)), ((1, 1), (1, 1)), ((1, 2), (1, 2)), ((2, 1), (2, 1))):
+        ctx = k.kv_ctx_create(0, store_mode=asked[0], load_mode=asked[1])
+        try:
+            assert k.kv_ctx_modes(ctx) == want
+            src_np = host_layers(SPEC, 99)
+            src, dst = device_pool(SPEC, src_np), device_pool(SPEC)
+            tab = torch.from_numpy(synth.permuted_table(SPEC.num_blocks, T // SPEC.block_tokens, 3)).cuda()
+            chunks = pinned_chunks(orc, SPEC, 0, T, C)
+            torch.cuda.synchronize()
+            k.kv_store(ctx, src, tab, 0, T, C, chunks)
+            k.kv_load(ctx, dst, tab, 0, T, C, chunks)
+            torch.cuda.synchronize()
+            st = k.kv_ctx_stats(ctx)
+            assert st["kernel_launches"] >= 2
+            assert (st["memcpy_calls"] > 0) == (1 in want), (asked, st)
+            for l in range(SPEC.num_layers):  # restored through the same table: the pages it names
+                idx = tab.long()
+                page = SPEC.layer_bytes // SPEC.num_blocks
+                assert torch.equal(src.layers[l].view(-1, page)[idx], dst.layers[l].view(-1, page)[idx])
+        finally:
+            k.kv_ctx_destroy(ctx)
+    buf = k.HostBuffer(3 << 20)
+    try:
+        assert buf.info()["bytes"] == 3 << 20
+        with pytest.raises(k.KvxError) as e:
+            k.kv_host_pool_info(buf.ptr + 4096)          # inside a pool, not its start
+        assert e.value.status == k.KVX_ENOENT
+        foreign = torch.full((1 << 20,), 7, dtype=torch.uint8).pin_memory()
+        with pytest.raises(k.KvxError) as e:
+            k.kv_host_pool_info(foreign.data_ptr())      # pinned, but not the library's
+        assert e.value.status == k.KVX_ENOENT
+        k._lib.kv_host_free(None)
+        k._lib.kv_host_free(ctypes.c_void_p(foreign.data_ptr()))   # ignored: not the library's
+        assert int(foreign[-1]) == 7
+        d = torch.empty(1 << 20, dtype=torch.uint8, device="cuda")
+        d.copy_(foreign, non_blocking=True)                       # still pinned and usable
+        torch.cuda.synchronize()
+        assert int(d[0]) == 7
+    finally:
+        buf.close()
