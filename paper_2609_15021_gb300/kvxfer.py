@@ -288,7 +288,68 @@ def kv_pool_view_check(pool: KvPool, tensor) -> None:
     _view_check(pool.c, tensor)
 
 
+class ChunkList:
+    """A fixed sequence of chunks (tensors, or raw addresses) with their
+    addresses marshalled and their sizes read once, for transfers made again and
+    again over the same chunks.  kv_store / kv_load / kv_pack / kv_unpack /
+    kv_store_noalloc take it wherever they take a list of chunks; element i is
+    the call's i-th chunk, as in a list, and a slice is a ChunkList over a run
+    of the same chunks, sharing the marshalled addresses.  Per call only the
+    sizes the range needs are compared (vectorised).  The chunks must keep
+    their storage while the list is in use (it holds references to them)."""
+
+    def __init__(self, chunks, _parent=None, _start=0, _stop=None):
+        import numpy as np
+        if _parent is not None:
+            self._items, self._arr, self._sizes = _parent._items, _parent._arr, _parent._sizes
+            self._start, self._n = _start, _stop - _start
+            return
+        self._items = list(chunks)
+        n = len(self._items)
+        self._arr = (ctypes.c_void_p * max(1, n))(*[_ptr(c) for c in self._items])
+        sizes = np.full(n, np.iinfo(np.int64).max, dtype=np.int64)  # raw addresses: size unknown
+        for i, c in enumerate(self._items):
+            if not isinstance(c, int):
+                _check_tensor(c, f"chunk {i}")
+                sizes[i] = _nbytes(c)
+        self._sizes, self._start, self._n = sizes, 0, n
+
+    def __len__(self) -> int:
+        return self._n
+
+    def __getitem__(self, key):
+        if isinstance(key, slice):
+            a, b, step = key.indices(self._n)
+            if step != 1:
+                raise ValueError("a ChunkList slice must be contiguous")
+            return ChunkList(None, self, self._start + a, self._start + max(a, b))
+        if not -self._n <= key < self._n:
+            raise IndexError(key)
+        return self._items[self._start + key % self._n]
+
+    def _pointer(self):
+        return ctypes.cast(ctypes.byref(self._arr, self._start * ctypes.sizeof(ctypes.c_void_p)),
+                           ctypes.POINTER(ctypes.c_void_p))
+
+    def _check_sizes(self, per_token: int, chunk_tokens: int, tok_begin: int, tok_end: int) -> None:
+        import numpy as np
+        first = tok_begin // chunk_tokens
+        used = min(self._n, -(-tok_end // chunk_tokens) - first)
+        if used <= 0:
+            return
+        need = np.full(used, per_token * chunk_tokens, dtype=np.int64)
+        last = first + used - 1
+        need[-1] = per_token * min(chunk_tokens, tok_end - last * chunk_tokens)
+        sizes = self._sizes[self._start:self._start + used]
+        bad = np.nonzero(sizes < need)[0]
+        if bad.size:
+            i = int(bad[0])
+            raise ValueError(f"chunk {i} holds {int(sizes[i])} bytes, needs {int(need[i])}")
+
+
 def _ptr_array(chunks):
+    if isinstance(chunks, ChunkList):
+        return chunks._pointer()
     return (ctypes.c_void_p * max(1, len(chunks)))(*[_ptr(c) for c in chunks])
 
 
@@ -304,6 +365,9 @@ def _check_transfer_tensors(pool: KvPool, block_table, tok_begin, tok_end, chunk
         return
     first = tok_begin // chunk_tokens
     per_token = pool.c.num_layers * 2 * pool.num_heads * pool.row_bytes
+    if isinstance(chunks, ChunkList):
+        chunks._check_sizes(per_token, chunk_tokens, tok_begin, tok_end)
+        return
     for i, c in enumerate(chunks):
         start = (first + i) * chunk_tokens
         if start >= tok_end:

@@ -226,6 +226,41 @@ def test_state_layers_marshalled_once(k):
             assert e.value.status == k.KVX_EINVAL
 
 
+def test_chunk_list_marshals_once_and_checks_sizes_per_call(k):
+    """A ChunkList checks contiguity once, keeps the chunks' addresses, slices
+    without copying them, and per call rejects a chunk too small for the
+    tokens it must hold, with the same message as a plain list."""
+    import torch
+    L, N, B, H, D, e, C = 2, 8, 16, 2, 64, 2, 32
+    pool = k.KvPool([torch.empty(N * 2 * H * B * D * e, dtype=torch.uint8) for _ in range(L)], N, B, H, D, e)
+    cb = L * 2 * C * H * D * e
+    items = [torch.empty(cb, dtype=torch.uint8) for _ in range(4)] + [torch.empty(cb // 2, dtype=torch.uint8)]
+    cl = k.ChunkList(items)
+    table = torch.zeros(8, dtype=torch.int32)
+    assert len(cl) == 5 and cl[1] is items[1] and cl[-1] is items[4]
+    ptrs = k._ptr_array(cl)
+    assert [ptrs[i] for i in range(5)] == [t.data_ptr() for t in items]
+    k._check_transfer_tensors(pool, table, 0, 4 * C + 16, C, cl)        # a short last chunk: half a chunk
+    for chunks in (cl, items):
+        with pytest.raises(ValueError, match="chunk 4 holds 16384 bytes, needs 17408"):
+            k._check_transfer_tensors(pool, table, 0, 4 * C + 17, C, chunks)
+    sub = cl[1:3]
+    assert len(sub) == 2 and sub[0] is items[1]
+    sp = k._ptr_array(sub)
+    assert (sp[0], sp[1]) == (items[1].data_ptr(), items[2].data_ptr())
+    k._check_transfer_tensors(pool, table, C, 3 * C, C, sub)            # chunks 1 and 2 of the range
+    assert len(cl[4:9]) == 1 and len(cl[3:1]) == 0
+    with pytest.raises(ValueError, match="contiguous"):
+        cl[::2]
+    with pytest.raises(ValueError, match="contiguous"):
+        k.ChunkList([torch.empty(2, cb, dtype=torch.uint8)[:, 0]])
+    raw = k.ChunkList([16 * 1000, 16 * 2000])                           # raw addresses: size unknown, not checked
+    k._check_transfer_tensors(pool, table, 0, 2 * C, C, raw)
+    with pytest.raises(k.KvxError) as ex:                                # reaches the C ABI: no context
+        k.kv_store(None, pool, table, 0, 2 * C, C, cl[:2], stream=0)
+    assert ex.value.status == k.KVX_EINVAL
+
+
 def test_host_alloc_numa_arguments(k):
     import torch
     out = ctypes.c_void_p()

@@ -467,3 +467,42 @@ def test_tok_end_limit_with_logical_blocks(orc, ctxs, mode):
     for l in range(2):
         assert first_mismatch(np_of(dst.layers[l]), want_l[l]) is None
     assert k.kv_get_device_error(ctx) == -1
+
+
+@pytest.mark.parametrize("mode", list(MODES))
+def test_chunk_lists_move_what_lists_move(orc, ctxs, mode):
+    """kv_store / kv_load / kv_pack / kv_unpack / kv_store_noalloc given a
+    ChunkList, or a slice of one for a range that starts at a later chunk,
+    move the same bytes the oracle gives for the whole range."""
+    k = kvx()
+    spec = oracle.PoolSpec(3, 64, 16, 4, 64, 2, HND)
+    C, n_used, c0 = 64, 50, 3
+    T, t0 = n_used * 16 - 5, c0 * C
+    src_np = host_layers(spec, 808)
+    src, dst, dst2 = device_pool(spec, src_np), device_pool(spec), device_pool(spec)
+    ta, tb = synth.permuted_table(64, n_used, 81), synth.permuted_table(64, n_used, 82)
+    ta_d, tb_d = torch.from_numpy(ta).cuda(), torch.from_numpy(tb).cuda()
+    host = k.ChunkList(pinned_chunks(orc, spec, 0, T, C))
+    host2 = k.ChunkList(pinned_chunks(orc, spec, 0, T, C))
+    devc = k.ChunkList(device_chunks(orc, spec, 0, T, C))
+    ctx = ctxs(MODES[mode])
+    torch.cuda.synchronize()
+    k.kv_store(ctx, src, ta_d, 0, t0, C, host[:c0])
+    k.kv_store(ctx, src, ta_d, t0, T, C, host[c0:])
+    k.kv_pack(ctx, src, ta_d, 0, T, C, devc)
+    k.kv_store_noalloc(src, ta_d, 0, T, C, host2)
+    torch.cuda.synchronize()
+    want, _ = oracle_store(orc, spec, src_np, ta, 0, T, C)
+    for i, w in enumerate(want):
+        for name, cl in (("store", host), ("pack", devc), ("noalloc", host2)):
+            assert first_mismatch(np_of(cl[i]), w) is None, (name, i)
+    k.kv_load(ctx, dst, tb_d, t0, T, C, host[c0:])
+    k.kv_load(ctx, dst, tb_d, 0, t0, C, host[:c0])
+    k.kv_unpack(ctx, dst2, tb_d, 0, T, C, devc)
+    torch.cuda.synchronize()
+    want_l, _ = oracle_load(orc, spec, [np.full(spec.layer_bytes, POISON, np.uint8)] * spec.num_layers,
+                            tb, 0, T, C, want)
+    for l in range(spec.num_layers):
+        assert first_mismatch(np_of(dst.layers[l]), want_l[l]) is None, ("load", l)
+        assert first_mismatch(np_of(dst2.layers[l]), want_l[l]) is None, ("unpack", l)
+    assert k.kv_get_device_error(ctx) == -1
