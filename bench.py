@@ -711,12 +711,12 @@ def ring_round(tier, plan, j, n_chunks, own_keys, src_keys, store_fn, load_fn, s
     lo = j * plan["slots_per_rank"]
     hi = min(n_chunks, lo + plan["slots_per_rank"])
     own = own_keys[lo:hi]
-    slots = tier.reserve_many(own)
+    slots = tier.reserve_many(own, as_chunk_list=True)
     store_fn(lo, hi, slots)
     tier.commit_many(own, stream=stream)
     theirs = src_keys[lo:hi]
     wait_readable(tier, theirs)
-    slots_r = tier.acquire_many(theirs, stream=stream)
+    slots_r = tier.acquire_many(theirs, stream=stream, as_chunk_list=True)
     load_fn(lo, hi, slots_r)
     tier.release_many(theirs, stream=stream)
     settle_fn()
@@ -1254,12 +1254,12 @@ def run_ours(args):
             torch.cuda.synchronize()
             t0 = time.perf_counter()
             a.record(stream)
-            slots = tier.reserve_many(keys)
+            slots = tier.reserve_many(keys, as_chunk_list=True)
             k.kv_store(ctx, src, ta, 0, T, C, slots, stream=stream)
             tier.commit_many(keys, stream=stream)
             b.record(stream)
             hits = tier.prefix_hits(keys)
-            slots = tier.acquire_many(keys[:hits], stream=stream)
+            slots = tier.acquire_many(keys[:hits], stream=stream, as_chunk_list=True)
             k.kv_load(ctx, dst, tb, 0, T, C, slots, stream=stream)
             tier.release_many(keys[:hits], stream=stream)
             c.record(stream)
@@ -1315,12 +1315,12 @@ def run_ours(args):
             a.record(stream)
             s_b.wait_event(a)
             for g0, g1 in groups:
-                slots = tier_s.reserve_many(skeys[g0:g1])
+                slots = tier_s.reserve_many(skeys[g0:g1], as_chunk_list=True)
                 k.kv_store(ctx, src, ta, g0 * C, min(T, g1 * C), C, slots, stream=stream)
                 tier_s.commit_many(skeys[g0:g1], stream=stream)
             ea.record(stream)
             for g0, g1 in groups:
-                slots = tier_s.acquire_many(skeys[g0:g1], stream=s_b)
+                slots = tier_s.acquire_many(skeys[g0:g1], stream=s_b, as_chunk_list=True)
                 k.kv_load(ctx_b, dst, tb, g0 * C, min(T, g1 * C), C, slots, stream=s_b)
                 tier_s.release_many(skeys[g0:g1], stream=s_b)
             eb.record(s_b)

@@ -62,7 +62,7 @@ def replica_a(name, q, q_in):
     torch.cuda.synchronize()
     q.put("ready")
     a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    slots = tier.reserve_many(keys)
+    slots = tier.reserve_many(keys, as_chunk_list=True)
     a.record(s)
     k.kv_store(ctx, pool, table, 0, T, C, slots, stream=s)
     b.record(s)
@@ -106,7 +106,7 @@ def main():
             a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             torch.cuda.synchronize()
             a.record(s)
-            slots = tier.acquire_many(keys, stream=s)
+            slots = tier.acquire_many(keys, stream=s, as_chunk_list=True)
             k.kv_load(ctx, dst, tb, 0, T, C, slots, stream=s)
             tier.release_many(keys, stream=s)
             b.record(s)

@@ -78,7 +78,7 @@ def replica_a(name, q, q_in):
         t0 = time.time()
         a.record(s)
         for g0, g1 in (groups() if grouped else [(0, T // C)]):
-            slots = tier.reserve_many(keys[g0:g1])
+            slots = tier.reserve_many(keys[g0:g1], as_chunk_list=True)
             k.kv_store(ctx, pool, table, g0 * C, g1 * C, C, slots, stream=s)
             tier.commit_many(keys[g0:g1], stream=s)
         b.record(s)
@@ -120,7 +120,7 @@ def main():
             torch.cuda.synchronize()
             for g0, g1 in (groups() if grouped else [(0, n_chunks)]):
                 tier.wait(keys[g0:g1], timeout_s=120)     # until A's GPU has published the group
-                slots = tier.acquire_many(keys[g0:g1], stream=s)
+                slots = tier.acquire_many(keys[g0:g1], stream=s, as_chunk_list=True)
                 k.kv_load(ctx, dst, tb, g0 * C, g1 * C, C, slots, stream=s)
                 tier.release_many(keys[g0:g1], stream=s)
             s.synchronize()

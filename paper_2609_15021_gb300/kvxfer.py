@@ -298,16 +298,23 @@ class ChunkList:
     sizes the range needs are compared (vectorised).  The chunks must keep
     their storage while the list is in use (it holds references to them)."""
 
-    def __init__(self, chunks, _parent=None, _start=0, _stop=None):
+    def __init__(self, chunks, nbytes: int | None = None, *, _parent=None, _start=0, _stop=None, _array=None):
+        """chunks: tensors or raw addresses; nbytes: the size of every raw
+        address's chunk, if known (tensors report their own)."""
         import numpy as np
         if _parent is not None:
             self._items, self._arr, self._sizes = _parent._items, _parent._arr, _parent._sizes
             self._start, self._n = _start, _stop - _start
             return
-        self._items = list(chunks)
-        n = len(self._items)
-        self._arr = (ctypes.c_void_p * max(1, n))(*[_ptr(c) for c in self._items])
-        sizes = np.full(n, np.iinfo(np.int64).max, dtype=np.int64)  # raw addresses: size unknown
+        if _array is not None:  # a ctypes address array the library filled in (tier slots)
+            self._arr, n = _array, len(chunks)
+            self._items = list(chunks)
+        else:
+            self._items = list(chunks)
+            n = len(self._items)
+            self._arr = (ctypes.c_void_p * max(1, n))(*[_ptr(c) for c in self._items])
+        unknown = np.iinfo(np.int64).max
+        sizes = np.full(n, unknown if nbytes is None else nbytes, dtype=np.int64)
         for i, c in enumerate(self._items):
             if not isinstance(c, int):
                 _check_tensor(c, f"chunk {i}")
@@ -322,7 +329,7 @@ class ChunkList:
             a, b, step = key.indices(self._n)
             if step != 1:
                 raise ValueError("a ChunkList slice must be contiguous")
-            return ChunkList(None, self, self._start + a, self._start + max(a, b))
+            return ChunkList(None, _parent=self, _start=self._start + a, _stop=self._start + max(a, b))
         if not -self._n <= key < self._n:
             raise IndexError(key)
         return self._items[self._start + key % self._n]
@@ -666,16 +673,23 @@ class KvTier:
         _check(_lib.kv_tier_reserve(self.handle, key, ctypes.byref(out)), "kv_tier_reserve")
         return self._slot_tensor(out.value)
 
-    def reserve_many(self, keys) -> list:
-        """Slots for `keys`, reserved in order under one lock.  If a key cannot be
-        reserved, KvxError is raised with `.reserved`: the slots of the keys
-        before it, which stay reserved (commit or release them)."""
+    def _slots(self, out, n: int, as_chunk_list: bool):
+        if as_chunk_list:
+            return ChunkList([out[j] for j in range(n)], self.slot_bytes, _array=out)
+        return [self._slot_tensor(out[j]) for j in range(n)]
+
+    def reserve_many(self, keys, as_chunk_list: bool = False):
+        """Slots for `keys`, reserved in order under one lock: host tensor views,
+        or with as_chunk_list a ChunkList of the slots' addresses (no tensor per
+        slot; what the transfer calls take).  If a key cannot be reserved,
+        KvxError is raised with `.reserved`: the slots of the keys before it,
+        which stay reserved (commit or release them)."""
         n = len(keys)
         arr = (ctypes.c_uint64 * max(1, n))(*keys)
         out = (ctypes.c_void_p * max(1, n))()
         done = ctypes.c_int64()
         status = _lib.kv_tier_reserve_many(self.handle, arr, n, out, ctypes.byref(done))
-        slots = [self._slot_tensor(out[j]) for j in range(done.value)]
+        slots = self._slots(out, done.value, as_chunk_list)
         try:
             _check(status, "kv_tier_reserve_many")
         except KvxError as e:
@@ -698,12 +712,14 @@ class KvTier:
     def release(self, key: int, stream=None):
         _check(_lib.kv_tier_release(self.handle, key, self._stream(stream)), "kv_tier_release")
 
-    def acquire_many(self, keys, stream=None) -> list:
+    def acquire_many(self, keys, stream=None, as_chunk_list: bool = False):
+        """Slots of committed `keys`, pinned, `stream` waiting for their commits:
+        host tensor views, or with as_chunk_list a ChunkList of their addresses."""
         arr = (ctypes.c_uint64 * max(1, len(keys)))(*keys)
         out = (ctypes.c_void_p * max(1, len(keys)))()
         _check(_lib.kv_tier_acquire_many(self.handle, arr, len(keys), self._stream(stream), out),
                "kv_tier_acquire_many")
-        return [self._slot_tensor(out[j]) for j in range(len(keys))]
+        return self._slots(out, len(keys), as_chunk_list)
 
     def release_many(self, keys, stream=None):
         arr = (ctypes.c_uint64 * max(1, len(keys)))(*keys)

@@ -87,8 +87,9 @@ def _ring_worker(rank, world, port, out, slots_per_rank):
     os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank), WORLD_SIZE=str(world),
                       LOCAL_RANK=str(rank))
     sys.path.insert(0, ROOT)
+    import ctypes
+
     import numpy as np
-    import torch
     import torch.distributed as dist
 
     import bench
@@ -113,13 +114,18 @@ def _ring_worker(rank, world, port, out, slots_per_rank):
     got = {}
     step = 0
 
+    def view(addr):                   # the ring hands the slots over as addresses (a ChunkList)
+        return np.ctypeslib.as_array((ctypes.c_uint8 * cb).from_address(addr))
+
     def store_fn(lo, hi, slots):      # this rank's chunks into its slots (kv_store's part)
-        for c, slot in zip(range(lo, hi), slots):
-            slot.copy_(torch.from_numpy(_chunk_bytes(rank, c, cb, step)))
+        assert len(slots) == hi - lo
+        for i, c in enumerate(range(lo, hi)):
+            view(slots[i])[:] = _chunk_bytes(rank, c, cb, step)
 
     def load_fn(lo, hi, slots):       # the source rank's chunks out of the tier (kv_load's part)
-        for c, slot in zip(range(lo, hi), slots):
-            got[c] = slot.numpy().copy()
+        assert len(slots) == hi - lo
+        for i, c in enumerate(range(lo, hi)):
+            got[c] = view(slots[i]).copy()
 
     ok = True
     for step in range(3):             # each step's bytes differ: a stale read would show
