@@ -336,3 +336,26 @@ def test_absurd_counts_return_enomem_not_a_crash(k):
     tier.reserve(7).fill_(7)
     tier.commit(7, NO)
     assert tier.prefix_hits([7]) == 1
+
+
+def test_batch_slots_as_a_chunk_list(k):
+    """reserve_many / acquire_many with as_chunk_list hand back the slots'
+    addresses (the same ones the tensor form views) with the slot size as each
+    chunk's size, so the transfer calls' size check still applies."""
+    import torch
+    t, buf = _tier(k, 4, 1024)
+    cl = t.reserve_many([5, 6, 7], as_chunk_list=True)
+    assert isinstance(cl, k.ChunkList) and len(cl) == 3
+    assert list(cl._sizes) == [1024] * 3 and len({cl[i] for i in range(3)}) == 3
+    t.commit_many([5, 6, 7], stream=NO)
+    views = t.acquire_many([5, 6, 7], stream=NO)
+    acl = t.acquire_many([6, 7], stream=NO, as_chunk_list=True)
+    assert [acl[i] for i in range(2)] == [v.data_ptr() for v in views[1:]] == [cl[1], cl[2]]
+    t.release_many([5, 6, 7, 6, 7], stream=NO)
+    # a 1024-byte slot holds 16 tokens of a pool with 64 bytes per token, not 17
+    pool = k.KvPool([torch.empty(8 * 2 * 2 * 16 * 16, dtype=torch.uint8)], 8, 16, 2, 8, 2)
+    table = torch.zeros(8, dtype=torch.int32)
+    k._check_transfer_tensors(pool, table, 0, 48, 16, cl)
+    with pytest.raises(ValueError, match="chunk 0 holds 1024 bytes, needs 2048"):
+        k._check_transfer_tensors(pool, table, 0, 64, 32, cl)
+    t.close()
